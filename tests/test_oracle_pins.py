@@ -1,0 +1,344 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test checks one oracle function against something other than itself:
+a closed form, a special case, brute force on a tiny input, an invariant, a
+library routine, or a fact the paper states (tests/golden/paper_facts.json).
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+from oracle import outlets_oracle as O
+from paper_2609_01068_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "paper_facts.json")
+
+
+def _facts():
+    with open(GOLDEN) as fh:
+        return json.load(fh)
+
+
+SMALL = synth.ModelShape("pin-small", 32, 4, 2, 8, 48, (16,), 10000.0, 1e-5, "f32")
+
+
+def _weights(shape=SMALL, seed=0):
+    return synth.make_weights(shape, seed)
+
+
+def _taps(shape, T, seed=0, off=0):
+    return synth.make_taps(shape, T, seed, off)
+
+
+# ---------------------------------------------------------------- golden facts
+def test_tap_layer_indices_match_paper():
+    for c in _facts()["tap_layers"]["cases"]:
+        assert list(synth.tap_layer_indices(c["n_layers"])) == c["layers"]
+
+
+def test_log_space_target_round_trip():
+    # z = log(1 + length) (Sec. 4.2) and the oracle's inverse
+    for c in _facts()["log_space_target"]["cases"]:
+        assert math.isclose(math.log1p(c["length"]), c["z"], rel_tol=0, abs_tol=1e-15)
+        assert O.z_to_length(np.array([c["z"]]))[0] == pytest.approx(c["length"], rel=1e-12, abs=1e-12)
+    assert O.z_to_length(np.array([-3.0]))[0] == 0.0
+
+
+def test_head_parameter_count_consistent_with_paper():
+    fact = _facts()["head_params_d2048"]
+
+    def count(widths):
+        shape = synth.ModelShape("p", widths[0], 1, 1, 2, 2, tuple(widths[1:-1]), 1e4, 1e-5, "f32")
+        n = 0
+        w = {}
+        for i in range(len(widths) - 1):
+            w[f"head_w{i}"] = np.zeros((widths[i + 1], widths[i]))
+            w[f"head_b{i}"] = np.zeros(widths[i + 1])
+        ws, bs = O.head_weights(w)
+        for a, b in zip(ws, bs):
+            n += a.size + b.size
+        return n, shape
+
+    n_ok, _ = count(fact["widths_consistent"])
+    n_bad, _ = count(fact["widths_inconsistent"])
+    assert abs(n_ok - fact["approx_params"]) / fact["approx_params"] < fact["rel_tol"]
+    assert abs(n_bad - fact["approx_params"]) / fact["approx_params"] > fact["rel_tol"]
+
+
+def test_remaining_length_definition():
+    for c in _facts()["static_vs_dynamic"]["cases"]:
+        assert c["L"] - c["t"] == c["r"]
+
+
+# ---------------------------------------------------------------- head
+def test_zero_weight_head_returns_output_bias():
+    w = _weights()
+    h = np.random.default_rng(1).standard_normal((5, SMALL.d))
+    ws, bs = O.head_weights(w)
+    zero_ws = [np.zeros_like(a) for a in ws]
+    z = O.length_head(h, zero_ws, bs)
+    assert np.all(z == np.float64(bs[-1][0]))
+
+
+def test_head_relu_all_active_is_affine():
+    rng = np.random.default_rng(2)
+    W1 = rng.standard_normal((6, 4))
+    W2 = rng.standard_normal((1, 6))
+    b1 = np.full(6, 1e3)     # every pre-activation positive: ReLU is the identity
+    b2 = np.array([0.25])
+    h = rng.standard_normal((7, 4))
+    z = O.length_head(h, [W1, W2], [b1, b2])
+    np.testing.assert_allclose(z, h @ (W2 @ W1).T[:, 0] + (W2 @ b1)[0] + b2[0], rtol=1e-12)
+
+
+def test_head_relu_all_dead_gives_bias():
+    rng = np.random.default_rng(3)
+    W1 = rng.standard_normal((6, 4))
+    W2 = rng.standard_normal((1, 6))
+    z = O.length_head(rng.standard_normal((7, 4)), [W1, W2], [np.full(6, -1e3), np.array([1.5])])
+    assert np.all(z == 1.5)
+
+
+def test_head_relu_brute_force():
+    rng = np.random.default_rng(4)
+    W1, b1 = rng.standard_normal((5, 3)), rng.standard_normal(5)
+    W2, b2 = rng.standard_normal((1, 5)), rng.standard_normal(1)
+    h = rng.standard_normal((4, 3))
+    z = O.length_head(h, [W1, W2], [b1, b2])
+    for r in range(4):
+        acc = b2[0]
+        for j in range(5):
+            pre = b1[j]
+            for i in range(3):
+                pre += W1[j, i] * h[r, i]
+            if pre > 0:
+                acc += W2[0, j] * pre
+        assert z[r] == pytest.approx(acc, rel=1e-12, abs=1e-12)
+
+
+# ---------------------------------------------------------------- Eq. 1
+def test_fc_identity_blocks_select_each_tap():
+    d = 8
+    taps = [np.random.default_rng(i).standard_normal((5, d)) for i in range(3)]
+    for j in range(3):
+        w = np.zeros((d, 3 * d))
+        w[:, j * d:(j + 1) * d] = np.eye(d)
+        np.testing.assert_array_equal(O.fuse_taps(taps, w), taps[j])
+
+
+def test_fc_is_linear_in_each_tap():
+    rng = np.random.default_rng(5)
+    d = 6
+    w = rng.standard_normal((d, 3 * d))
+    t = [rng.standard_normal((3, d)) for _ in range(3)]
+    t2 = [rng.standard_normal((3, d)) for _ in range(3)]
+    lhs = O.fuse_taps([a + 2 * b for a, b in zip(t, t2)], w)
+    np.testing.assert_allclose(lhs, O.fuse_taps(t, w) + 2 * O.fuse_taps(t2, w), rtol=1e-12, atol=1e-12)
+
+
+# ---------------------------------------------------------------- RMSNorm
+def test_rmsnorm_hand_example():
+    # [3, 4]: mean square 12.5
+    y = O.rms_norm(np.array([[3.0, 4.0]]), np.ones(2), 0.0)
+    np.testing.assert_allclose(y, [[3 / math.sqrt(12.5), 4 / math.sqrt(12.5)]], rtol=1e-15)
+
+
+def test_rmsnorm_unit_rms_and_scale_invariance():
+    x = np.random.default_rng(6).standard_normal((9, 64))
+    y = O.rms_norm(x, np.ones(64), 0.0)
+    np.testing.assert_allclose(np.sqrt(np.mean(y * y, axis=1)), 1.0, rtol=1e-12)
+    np.testing.assert_allclose(O.rms_norm(7.5 * x, np.ones(64), 0.0), y, rtol=1e-12)
+    g = np.random.default_rng(7).standard_normal(64)
+    np.testing.assert_allclose(O.rms_norm(x, g, 0.0), y * g, rtol=1e-12)
+
+
+# ---------------------------------------------------------------- RoPE
+def test_rope_position_zero_is_identity_and_isometry():
+    x = np.random.default_rng(8).standard_normal((5, 3, 16))
+    np.testing.assert_array_equal(O.apply_rope(x, np.zeros(5, int), 1e4), x)
+    y = O.apply_rope(x, np.arange(5) * 97, 5e5)
+    np.testing.assert_allclose(np.linalg.norm(y, axis=-1), np.linalg.norm(x, axis=-1), rtol=1e-12)
+
+
+def test_rope_frequency_schedule_closed_form():
+    # Rotate unit vectors e_i at position 1 and read back each pair's angle.
+    hd, theta = 16, 1e4
+    half = hd // 2
+    x = np.zeros((1, half, hd))
+    for i in range(half):
+        x[0, i, i] = 1.0
+    y = O.apply_rope(x, np.array([1]), theta)[0]
+    ang = np.array([math.atan2(y[i, i + half], y[i, i]) for i in range(half)])
+    assert ang[0] == pytest.approx(1.0, abs=1e-15)             # theta^0 = 1 rad per position
+    np.testing.assert_allclose(ang[1:] / ang[:-1], theta ** (-2.0 / hd), rtol=1e-12)
+    # the rest of each rotated vector is zero: the pair is (i, i + hd/2)
+    for i in range(half):
+        rest = np.delete(y[i], [i, i + half])
+        assert np.all(rest == 0)
+
+
+def test_rope_composes_and_is_relative():
+    rng = np.random.default_rng(9)
+    q = rng.standard_normal((1, 1, 32))
+    k = rng.standard_normal((1, 1, 32))
+    theta = 5e5
+    a = O.apply_rope(O.apply_rope(q, np.array([11]), theta), np.array([30]), theta)
+    np.testing.assert_allclose(a, O.apply_rope(q, np.array([41]), theta), rtol=1e-10, atol=1e-12)
+    s1 = np.sum(O.apply_rope(q, np.array([5]), theta) * O.apply_rope(k, np.array([2]), theta))
+    s2 = np.sum(O.apply_rope(q, np.array([1005]), theta) * O.apply_rope(k, np.array([1002]), theta))
+    assert s1 == pytest.approx(s2, rel=1e-9)
+
+
+# ---------------------------------------------------------------- attention
+def _rand_qkv(T, H, KVH, hd, seed):
+    rng = np.random.default_rng(seed)
+    return (rng.standard_normal((T, H, hd)), rng.standard_normal((T, KVH, hd)),
+            rng.standard_normal((T, KVH, hd)))
+
+
+def test_attention_brute_force_loops():
+    H, KVH, hd = 4, 2, 8
+    cu = np.array([0, 3, 8, 9])
+    q, k, v = _rand_qkv(9, H, KVH, hd, 10)
+    out = O.causal_gqa_attention(q, k, v, cu)
+    for b in range(3):
+        for i in range(cu[b], cu[b + 1]):
+            for h in range(H):
+                g = h // (H // KVH)
+                scores = []
+                for j in range(cu[b], i + 1):
+                    scores.append(sum(q[i, h, c] * k[j, g, c] for c in range(hd)) / math.sqrt(hd))
+                mx = max(scores)
+                ex = [math.exp(s - mx) for s in scores]
+                tot = sum(ex)
+                for c in range(hd):
+                    ref = sum(ex[n] / tot * v[cu[b] + n, g, c] for n in range(len(ex)))
+                    assert out[i, h, c] == pytest.approx(ref, rel=1e-10, abs=1e-12)
+
+
+def test_attention_matches_torch_sdpa():
+    torch = pytest.importorskip("torch")
+    H, KVH, hd = 8, 2, 16
+    cu = np.array([0, 5, 6, 30])
+    q, k, v = _rand_qkv(30, H, KVH, hd, 11)
+    out = O.causal_gqa_attention(q, k, v, cu)
+    for b in range(3):
+        s0, s1 = cu[b], cu[b + 1]
+        tq = torch.from_numpy(q[s0:s1]).permute(1, 0, 2)[None]
+        tk = torch.from_numpy(k[s0:s1]).permute(1, 0, 2).repeat_interleave(H // KVH, dim=0)[None]
+        tv = torch.from_numpy(v[s0:s1]).permute(1, 0, 2).repeat_interleave(H // KVH, dim=0)[None]
+        ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv, is_causal=True)
+        np.testing.assert_allclose(out[s0:s1], ref[0].permute(1, 0, 2).numpy(), rtol=1e-10, atol=1e-12)
+
+
+def test_gqa_with_replicated_kv_equals_mha():
+    H, KVH, hd = 4, 2, 8
+    cu = np.array([0, 7, 12])
+    q, k, v = _rand_qkv(12, H, KVH, hd, 12)
+    gqa = O.causal_gqa_attention(q, k, v, cu)
+    mha = O.causal_gqa_attention(q, np.repeat(k, H // KVH, axis=1), np.repeat(v, H // KVH, axis=1), cu)
+    np.testing.assert_allclose(gqa, mha, rtol=1e-13, atol=1e-14)
+
+
+def test_attend_single_is_last_row_of_causal():
+    H, KVH, hd = 4, 2, 8
+    q, k, v = _rand_qkv(6, H, KVH, hd, 13)
+    full = O.causal_gqa_attention(q, k, v, np.array([0, 6]))
+    np.testing.assert_allclose(O.attend_single(q[5], k, v), full[5], rtol=1e-13, atol=1e-14)
+
+
+# ---------------------------------------------------------------- SwiGLU
+def test_silu_against_library_sigmoid():
+    scipy_special = pytest.importorskip("scipy.special")
+    x = np.linspace(-30, 30, 121)
+    np.testing.assert_allclose(O.silu(x), x * scipy_special.expit(x), rtol=1e-13, atol=1e-300)
+    assert O.silu(np.array([0.0]))[0] == 0.0
+
+
+# ---------------------------------------------------------------- whole forward
+def _prefill(w, shape, lengths, seed=0, off=0, **kw):
+    cu = synth.cu_seqlens(lengths)
+    taps = _taps(shape, int(cu[-1]), seed, off)
+    return O.predict_prefill(w, shape, taps, cu, **kw), taps, cu
+
+
+def test_zero_out_projections_make_layer_identity():
+    w = dict(_weights())
+    w["w_o"] = np.zeros_like(w["w_o"])
+    w["w_down"] = np.zeros_like(w["w_down"])
+    out, _, _ = _prefill(w, SMALL, [3, 5])
+    np.testing.assert_array_equal(out["y"], out["f"])
+
+
+def test_causal_prefix_invariance():
+    w = _weights()
+    out, taps, cu = _prefill(w, SMALL, [9], all_tokens=True)
+    for kpos in (0, 3, 8):
+        trunc = O.predict_prefill(w, SMALL, [t[:kpos + 1] for t in taps], np.array([0, kpos + 1]))
+        assert trunc["z"][0] == pytest.approx(out["z"][kpos], rel=1e-12, abs=1e-12)
+
+
+def test_batch_permutation_and_padding_invariance():
+    w = _weights()
+    lengths = [4, 7, 2]
+    out, taps, cu = _prefill(w, SMALL, lengths)
+    perm = [2, 0, 1]
+    ptaps = [np.concatenate([t[cu[b]:cu[b + 1]] for b in perm]) for t in taps]
+    pout = O.predict_prefill(w, SMALL, ptaps, synth.cu_seqlens([lengths[b] for b in perm]))
+    np.testing.assert_allclose(pout["z"], out["z"][perm], rtol=1e-12, atol=1e-12)
+    # an extra sequence in the pack changes nothing for the others
+    extra = _taps(SMALL, 5, seed=3)
+    xtaps = [np.concatenate([t, e]) for t, e in zip(taps, extra)]
+    xout = O.predict_prefill(w, SMALL, xtaps, synth.cu_seqlens(lengths + [5]))
+    np.testing.assert_allclose(xout["z"][:3], out["z"], rtol=1e-12, atol=1e-12)
+
+
+def test_prefill_equals_prefix_then_steps():
+    w = _weights()
+    lengths = [6, 4]
+    full, taps, cu = _prefill(w, SMALL, lengths, all_tokens=True)
+    kpre = [2, 1]
+    pre_taps = [np.concatenate([t[cu[b]:cu[b] + kpre[b]] for b in range(2)]) for t in taps]
+    pre_cu = synth.cu_seqlens(kpre)
+    pre = O.predict_prefill(w, SMALL, pre_taps, pre_cu)
+    caches = O.caches_from_prefill(pre, pre_cu)
+    for step in range(3):
+        rows = [cu[b] + kpre[b] + step for b in range(2)]
+        st = O.predict_step(w, SMALL, [t[rows] for t in taps], caches)
+        np.testing.assert_allclose(st["z"], full["z"][rows], rtol=1e-11, atol=1e-11)
+        caches = st["caches"]
+
+
+def test_sampled_rows_equal_full_batch():
+    w = _weights()
+    lengths = [5, 2, 7, 1]
+    out, taps, cu = _prefill(w, SMALL, lengths)
+    sub = O.sample_prefill_rows(w, SMALL, taps, cu, [3, 1])
+    np.testing.assert_allclose(sub["z"], out["z"][[3, 1]], rtol=1e-12, atol=1e-12)
+
+
+# ---------------------------------------------------------------- generator
+def test_bf16_rounding_matches_torch():
+    torch = pytest.importorskip("torch")
+    x = np.random.default_rng(14).standard_normal(10000).astype(np.float32) * 3
+    ours = synth.round_bf16(x)
+    ref = torch.from_numpy(x).to(torch.bfloat16).float().numpy()
+    np.testing.assert_array_equal(ours, ref)
+    bits = synth.bf16_bits(ours)
+    back = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).float().numpy()
+    np.testing.assert_array_equal(back, ours)
+
+
+def test_generator_is_seeded_and_shaped():
+    a = synth.lengths_8b_prefill(0)
+    assert len(a) == 64 and a.min() >= 16 and a.max() <= 2048
+    np.testing.assert_array_equal(a, synth.lengths_8b_prefill(0))
+    c = synth.lengths_8b_step_cache(0)
+    assert len(c) == 256 and c.min() >= 1 and c.max() <= 4096
+    s = synth.lengths_sweep(0)
+    assert len(s) == 1024 and s.max() <= 8192
+    cu = synth.cu_seqlens([3, 4])
+    assert cu.tolist() == [0, 3, 7] and cu.dtype == np.int32

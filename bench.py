@@ -1,0 +1,377 @@
+#!/usr/bin/env python
+"""Benchmark of OUTLETS length prediction on GB300.
+
+Workload (the headline): static prediction (Sec. 3.2) with a Llama-3.1-8B-shaped
+EAGLE-3 draft backbone (d=4096, 32/8 heads, hd 128, SwiGLU 14336, head
+4096->1024->1), bf16, over 64 ragged prompts (lognormal median 256, clipped to
+[16, 2048], packed varlen).  One step = one outlets_predict_prefill call: tap
+fusion, the draft decoder layer over every token, and the length head.
+
+Also reported: dynamic prediction (one outlets_predict_step over 256 live
+requests with lognormal cache lengths, median 512, <= 4096), the CPU oracle on
+a bounded sample, and the end-to-end number through the C ABI with host
+buffers.  `--impl reference` times the CPU oracle alone (the reference arm).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Under torchrun each rank runs an independent replica (weak scaling).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "length predictions/s and draft tokens/s on 1 GB300; % bf16 tensor peak / % HBM BW"
+WORKLOAD = ("static length prediction, Llama-3.1-8B-shaped EAGLE-3 draft layer + length head, "
+            "64 ragged prompts (lognormal median 256, clipped 16-2048), packed varlen")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-step-mode", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as fh:
+            j = json.load(fh)
+        return {"hbm_gbs": j["hbm_gbs"], "bf16": j["bf16_tflops"], "bf16_sus": j["bf16_tflops_sustained"],
+                "src": "of measured"}
+    return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sus": 1700.0, "src": "of fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "100",
+                 "-i", str(self.index)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, power, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm), "power_w_max": max(power) if power else None}
+
+
+def prefill_flops(shape, lengths, n_out):
+    """Algorithmic FLOPs of one static-prediction pass (dense GEMMs + causal attention + head)."""
+    d, H, KVH, hd, F = shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
+    T = int(np.sum(lengths))
+    per_tok = 2 * (3 * d * d + d * (H + 2 * KVH) * hd + H * hd * d + 3 * d * F)
+    attn = 4 * H * hd * float(np.sum(lengths * (lengths + 1) / 2))
+    widths = (d,) + tuple(shape.head_widths) + (1,)
+    head = 2 * sum(widths[i] * widths[i + 1] for i in range(len(widths) - 1)) * n_out
+    return per_tok * T + attn + head
+
+
+def cpu_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("internal_api") in ("openblas", "mkl")]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count()
+
+
+def oracle_sample(shape, w, taps, cu, lengths, budget_tokens):
+    """Oracle on whole prompts taken in order until the token budget is used."""
+    from oracle import outlets_oracle as OR
+    picks, tot = [], 0
+    for b in np.argsort(np.abs(lengths - np.median(lengths))):
+        if tot + lengths[b] > budget_tokens and picks:
+            break
+        picks.append(int(b))
+        tot += int(lengths[b])
+    t0 = time.perf_counter()
+    OR.sample_prefill_rows(w, shape, taps, cu, picks)
+    dt = time.perf_counter() - t0
+    return len(picks), tot, dt
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2609_01068_gb300 import synth
+    shape = synth.LLAMA8B
+    w = synth.make_weights(shape, 0)
+    lengths = synth.lengths_8b_prefill(0)
+    cu = synth.cu_seqlens(lengths)
+    taps = synth.make_taps(shape, int(cu[-1]), 0)
+    budget = 400
+    for _ in range(args.warmup):
+        oracle_sample(shape, w, taps, cu, lengths, budget)
+    n_pred, n_tok, secs = 0, 0, 0.0
+    for _ in range(args.steps):
+        p, t, dt = oracle_sample(shape, w, taps, cu, lengths, budget)
+        n_pred, n_tok, secs = n_pred + p, n_tok + t, secs + dt
+    value = n_pred / secs
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "predictions/s", "n_gpus": args.gpus,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * secs / args.steps,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "draft_tokens_per_s": n_tok / secs,
+           "config": {"workload": WORKLOAD, "sample": f"~{budget} prompt tokens per step (whole prompts)"},
+           "cpu_baseline": {"value": value, "unit": "predictions/s", "cores": cpu_threads(), "kind": "oracle",
+                            "sample": f"{n_pred} prompts / {n_tok} tokens over {args.steps} steps"},
+           "e2e": {"value": value, "unit": "predictions/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_01068_gb300 import build as B
+    from paper_2609_01068_gb300 import outlets, synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    B.build()
+    peaks = load_peaks()
+    shape = synth.LLAMA8B
+    w = synth.make_weights(shape, 0)
+    lengths = synth.lengths_8b_prefill(0)
+    cu = synth.cu_seqlens(lengths)
+    T, Bq = int(cu[-1]), len(lengths)
+    taps = synth.make_taps(shape, T, 0, rank)
+
+    def dev(a):
+        return torch.from_numpy(synth.bf16_bits(a).view(np.int16)).view(torch.bfloat16).cuda()
+
+    taps_d = [dev(t) for t in taps]
+    step_B = 256
+    pred = outlets.Predictor(shape, w, max_tokens=32768, max_batch=step_B, max_position=8192, device=local)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    # ---------------- device-timed static prediction
+    z = torch.empty(Bq, dtype=torch.float32, device="cuda")
+    ln = torch.empty(Bq, dtype=torch.float32, device="cuda")
+    for _ in range(args.warmup):
+        pred.prefill(taps_d, cu, z_out=z, len_out=ln)
+    pred.check()
+    pred.profile(True)
+    launches0 = pred.launch_count
+    sampler = ClockSampler(local)
+    sampler.start()
+    barrier()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        pred.prefill(taps_d, cu, z_out=z, len_out=ln)
+    ev1.record(stream)
+    ev1.synchronize()
+    barrier()
+    clocks = sampler.stop()
+    ms = max_over_ranks(ev0.elapsed_time(ev1))
+    launches = pred.launch_count - launches0
+    prof = pred.profile_read()
+    pred.profile(False)
+    pred.check()
+    ms_step = ms / args.steps
+    value = world * Bq * args.steps / (ms / 1e3)
+    flops = prefill_flops(shape, lengths, Bq)
+    gu_ms, gu_n = prof["gateup_swiglu_gemm"]
+    gu_flops = 2.0 * T * (2 * shape.ffn) * shape.d
+    gu_tflops = gu_flops / (gu_ms / gu_n / 1e3) / 1e12
+    roofline = {"bound": "tensor", "kernel": "gateup_swiglu_gemm (k_gemm_tc<256, SWIGLU>)",
+                "achieved": gu_tflops, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
+                "frac": gu_tflops / peaks["bf16_sus"], "peak_kind": f"bf16 sustained {peaks['src']}",
+                "traffic": None,
+                "algorithmic_per_launch": f"{gu_flops:.4g} FLOP = 2*T*(2F)*d, T={T}"}
+    stages = {k: {"ms_per_step": v[0] / max(args.steps, 1), "share": v[0] / max(sum(x[0] for x in prof.values()), 1e-9)}
+              for k, v in prof.items() if v[1]}
+
+    # ---------------- end to end through the C ABI with host buffers
+    host_taps = [t.cpu().pin_memory() for t in taps_d]
+    zh = torch.empty(Bq, dtype=torch.float32).pin_memory()
+    lh = torch.empty(Bq, dtype=torch.float32).pin_memory()
+    for _ in range(max(2, args.warmup // 2)):
+        pred.prefill(host_taps, cu, z_out=zh, len_out=lh)
+        stream.synchronize()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        pred.prefill(host_taps, cu, z_out=zh, len_out=lh)
+        stream.synchronize()
+    e2e_s = max_over_ranks(time.perf_counter() - t0)
+    e2e = {"value": world * Bq * args.steps / e2e_s, "unit": "predictions/s",
+           "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps)),
+           "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4)}
+
+    # ---------------- dynamic prediction (per-step path)
+    step_mode = None
+    if not args.no_step_mode:
+        step_mode = run_step_mode(args, pred, shape, peaks, step_B, world, barrier, max_over_ranks, stream)
+
+    out = {"metric": METRIC, "value": value, "unit": "predictions/s", "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+           "config": {"workload": WORKLOAD, "prompts_per_gpu": Bq, "tokens_per_gpu": T,
+                      "l2": "inputs larger than L2 (taps 3x[T,4096] bf16 = %.0f MB, weights 545 MB)"
+                            % (3 * T * 4096 * 2 / 1e6),
+                      "parallelism": f"replicas x{world}"},
+           "draft_tokens_per_s": world * T * args.steps / (ms / 1e3),
+           "tflops_per_s": flops * args.steps / (ms / 1e3) / 1e12,
+           "tensor_peak_frac_step": flops * args.steps / (ms / 1e3) / 1e12 / peaks["bf16_sus"],
+           "roofline": roofline, "stages": stages, "clocks": clocks, "e2e": e2e,
+           "gpu_launches": launches, "step_mode": step_mode}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n_pred, n_tok, secs = oracle_sample(shape, w, taps, cu, lengths, 1200)
+        out["cpu_baseline"] = {"value": n_pred / secs, "unit": "predictions/s", "cores": cpu_threads(),
+                               "kind": "oracle",
+                               "sample": f"{n_pred} whole prompts ({n_tok} tokens) of the same workload, {secs:.1f} s"}
+    if rank == 0:
+        print(json.dumps(out))
+    pred.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, stream):
+    import torch
+
+    from paper_2609_01068_gb300 import outlets, synth
+    lens = synth.lengths_8b_step_cache(0, B)
+    n_steps = args.steps + args.warmup
+    kv = outlets.KVCache(pred, max_slots=B, max_tokens_total=int(lens.sum()) + (n_steps + 64) * B)
+    gen = torch.Generator(device="cuda").manual_seed(1)
+    b = 0
+    while b < B:   # fill the draft cache (untimed set-up)
+        e, tot = b, 0
+        while e < B and tot + lens[e] <= 32768:
+            tot += int(lens[e])
+            e += 1
+        taps = [torch.randn(tot, shape.d, device="cuda", generator=gen).to(torch.bfloat16) for _ in range(3)]
+        pred.prefill(taps, synth.cu_seqlens(lens[b:e]), kv=kv, slots=np.arange(b, e, dtype=np.int32))
+        b = e
+    slots = np.arange(B, dtype=np.int32)
+    st_taps = [torch.randn(B, shape.d, device="cuda", generator=gen).to(torch.bfloat16) for _ in range(3)]
+    z = torch.empty(B, dtype=torch.float32, device="cuda")
+    ln = torch.empty(B, dtype=torch.float32, device="cuda")
+    for _ in range(args.warmup):
+        pred.step(st_taps, kv, slots, z_out=z, len_out=ln)
+    pred.check()
+    cache0 = sum(kv.slot_length(int(s)) for s in slots)
+    pred.profile(True)
+    barrier()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        pred.step(st_taps, kv, slots, z_out=z, len_out=ln)
+    ev1.record(stream)
+    ev1.synchronize()
+    barrier()
+    ms = max_over_ranks(ev0.elapsed_time(ev1))
+    prof = pred.profile_read()
+    pred.profile(False)
+    pred.check()
+    d, KVH, hd, F = shape.d, shape.n_kv_heads, shape.head_dim, shape.ffn
+    # keys read per step: every cached position plus the new one, K and V, bf16
+    keys_avg = cache0 + B * (args.steps + 1) / 2.0
+    kv_bytes = keys_avg * KVH * hd * 2 * 2
+    widths = (d,) + tuple(shape.head_widths) + (1,)
+    w_bytes = 2 * (3 * d * d + d * shape.qkv_out + shape.n_heads * hd * d + 3 * d * F + widths[0] * widths[1])
+    step_bytes = kv_bytes + w_bytes + 3 * B * d * 2
+    at_ms, at_n = prof["attention"]
+    at_gbs = kv_bytes / (at_ms / at_n / 1e3) / 1e9
+    ms_step = ms / args.steps
+    kv.close()
+    return {"workload": "dynamic prediction, 256 live requests x 1 new token, cache lengths lognormal "
+                        "median 512 clipped 1-4096 (sum %d)" % int(lens.sum()),
+            "value": world * B * args.steps / (ms / 1e3), "unit": "predictions/s", "ms_per_step": ms_step,
+            "hbm_frac_step": step_bytes / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"],
+            "algorithmic_bytes_per_step": step_bytes,
+            "roofline": {"bound": "hbm", "kernel": "decode attention (k_attn_decode_bf16 + combine)",
+                         "achieved": at_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": at_gbs / peaks["hbm_gbs"], "traffic": None,
+                         "algorithmic_per_launch": f"{kv_bytes:.4g} B of K/V (cached + new)"},
+            "stages": {k: v[0] / max(args.steps, 1) for k, v in prof.items() if v[1]}}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

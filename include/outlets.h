@@ -1,0 +1,238 @@
+/*
+ * OUTLETS length prediction on one GB300 (sm_103a): the C ABI.
+ *
+ * The library computes the batched length-prediction forward of OUTLETS
+ * ("Output-Length Prediction from Speculative Decoding Backbones"):
+ *
+ *   Eq. 1, Sec. 4.1    f_ctx = W_proj . Concat(h^(2), h^(floor(N/2)), h^(N-2))
+ *   Sec. 4.1           one draft decoder layer (pre-norm: RMSNorm, RoPE causal
+ *                      GQA self-attention, residual, RMSNorm, SwiGLU MLP, residual)
+ *   Sec. 4.2           final RMSNorm -> h^draft; z_hat = MLP_len(h^draft)
+ *                      (Linear/ReLU/.../Linear); z = log(1 + length), so the
+ *                      returned length is max(0, exp(z_hat) - 1)
+ *   Sec. 3.2           static prediction r_hat_0 after prefill (last prompt
+ *                      position); dynamic prediction r_hat_t at decode step t,
+ *                      one new token per request against the draft KV cache.
+ *
+ * The returned length is the REMAINING length r_hat_t (Sec. 3.1); a scheduler
+ * forms the projected total t + r_hat_t itself.
+ *
+ * Conventions
+ *  - Every entry point returns an outlets_status.  Argument errors are found
+ *    on the host before anything is launched; the context's last-error string
+ *    (outlets_last_error) then says what was wrong.  No C++ exception crosses
+ *    the ABI.
+ *  - Prediction calls are asynchronous on the caller's CUDA stream (a
+ *    cudaStream_t passed as void*, NULL = legacy default stream).  Calls on
+ *    one context are ordered: a call on a different stream waits for the
+ *    previous call of the same context.
+ *  - Tensors: "device or host" arguments may be device memory or host memory
+ *    (pageable or pinned); the library detects which.  Host inputs are copied
+ *    to the device inside the call; host outputs are written by an
+ *    asynchronous copy, so synchronize the stream before reading them.
+ *    Small index arrays (cu_seqlens, slots) are always host memory.
+ *  - The library owns its device copy of the weights, its workspace and the
+ *    KV pools; inputs and outputs stay owned by the caller and are only
+ *    borrowed for the duration of the call's work on the stream.
+ *  - Kernels never trap.  Bounded waits that run out, or indices a kernel
+ *    refuses, set a device error word; outlets_check() synchronizes and
+ *    reports it (OUTLETS_ETIMEOUT / OUTLETS_EDEVICE).
+ */
+#ifndef OUTLETS_H_
+#define OUTLETS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum outlets_status {
+  OUTLETS_OK = 0,
+  OUTLETS_EINVAL = 1,        /* invalid argument; nothing was launched or changed */
+  OUTLETS_ENOMEM = 2,        /* device or pinned-host allocation failed */
+  OUTLETS_ECUDA = 3,         /* a CUDA runtime/driver call failed */
+  OUTLETS_EUNSUPPORTED = 4,  /* shape this build does not implement */
+  OUTLETS_ECAPACITY = 5,     /* KV cache or workspace too small; nothing changed */
+  OUTLETS_ETIMEOUT = 6,      /* a kernel's bounded wait ran out (from outlets_check) */
+  OUTLETS_EDEVICE = 7        /* a kernel refused an index (from outlets_check) */
+} outlets_status;
+
+typedef enum outlets_dtype {
+  OUTLETS_F32 = 0,   /* f32 weights/activations, CUDA-core kernels */
+  OUTLETS_BF16 = 1   /* bf16 weights/activations, f32 accumulation, tensor cores */
+} outlets_dtype;
+
+#define OUTLETS_MAX_HEAD_HIDDEN 7
+
+/* Shape of the draft backbone and of the length head, plus workspace limits. */
+typedef struct outlets_config {
+  int32_t d_model;        /* d: width of each tap, of f_ctx and of the draft state */
+  int32_t n_heads;        /* H query heads */
+  int32_t n_kv_heads;     /* KVH key/value heads; H % KVH == 0 */
+  int32_t head_dim;       /* hd (even; 64 or 128 on the bf16 path) */
+  int32_t ffn_dim;        /* F: SwiGLU inner width */
+  int32_t n_head_hidden;  /* hidden Linear+ReLU layers of MLP_len (1 .. OUTLETS_MAX_HEAD_HIDDEN) */
+  int32_t head_hidden[OUTLETS_MAX_HEAD_HIDDEN];  /* their widths; the last Linear maps to 1 */
+  float rope_theta;       /* RoPE base */
+  float rms_eps;          /* RMSNorm epsilon */
+  int32_t dtype;          /* outlets_dtype */
+  int32_t max_tokens;     /* most packed rows in one prefill call */
+  int32_t max_batch;      /* most sequences per prefill call / requests per step call */
+  int32_t max_position;   /* positions 0 .. max_position-1 are supported (RoPE table) */
+  int32_t device;         /* CUDA device ordinal */
+} outlets_config;
+
+/* Host pointers to f32 weights, nn.Linear layout [out, in], row-major.
+ * On the bf16 path every value is rounded to bf16 (nearest even) on upload.
+ *   w_proj [d, 3d]           the FC of Eq. 1 (taps concatenated low, mid, high)
+ *   w_q [H*hd, d], w_k [KVH*hd, d], w_v [KVH*hd, d], w_o [d, H*hd]
+ *   g_in, g_post, g_final [d] RMSNorm gains (input, post-attention, final)
+ *   w_gate [F, d], w_up [F, d], w_down [d, F]
+ *   head_w[i] [w_{i+1}, w_i], head_b[i] [w_{i+1}] for i = 0 .. n_head_hidden,
+ *   widths w_0 = d, w_1.. = head_hidden, last = 1.
+ * The library copies everything during outlets_create; the caller may free
+ * its arrays afterwards. */
+typedef struct outlets_weights {
+  const float* w_proj;
+  const float* w_q;
+  const float* w_k;
+  const float* w_v;
+  const float* w_o;
+  const float* g_in;
+  const float* g_post;
+  const float* g_final;
+  const float* w_gate;
+  const float* w_up;
+  const float* w_down;
+  const float* head_w[OUTLETS_MAX_HEAD_HIDDEN + 1];
+  const float* head_b[OUTLETS_MAX_HEAD_HIDDEN + 1];
+} outlets_weights;
+
+typedef struct outlets_ctx outlets_ctx;
+typedef struct outlets_kv outlets_kv;
+
+/* Validates cfg, uploads the weights (re-laid out for the kernels), builds the
+ * RoPE table in fp64 on the host and allocates the workspace for max_tokens
+ * rows.  Synchronous.  On failure *out is NULL and no memory is held. */
+outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* w, outlets_ctx** out);
+
+/* Frees everything the context owns (after synchronizing its device). */
+void outlets_destroy(outlets_ctx* ctx);
+
+/* Details of the last failed call on ctx ("" if none); valid until the next call. */
+const char* outlets_last_error(const outlets_ctx* ctx);
+
+/* Number of bytes the context holds on the device (weights + workspace). */
+size_t outlets_device_bytes(const outlets_ctx* ctx);
+
+/* Draft KV cache: post-RoPE keys and values of every cached position, bf16 or
+ * f32 like the context, in pages of 64 positions; pools [pages][KVH][64][hd].
+ * Slots 0 .. max_slots-1 each hold one request; max_tokens_total bounds the
+ * positions cached over all slots together.  Needed by the dynamic prediction
+ * of Sec. 3.2. */
+outlets_status outlets_kv_create(outlets_ctx* ctx, int32_t max_slots, int32_t max_tokens_total,
+                                 outlets_kv** out);
+void outlets_kv_destroy(outlets_kv* kv);
+/* Empties one slot (host bookkeeping only; ordered after earlier calls). */
+outlets_status outlets_kv_reset_slot(outlets_kv* kv, int32_t slot);
+/* Cached positions of a slot, or -1 for an invalid slot. */
+int32_t outlets_kv_slot_length(const outlets_kv* kv, int32_t slot);
+/* Pages not held by any slot. */
+int32_t outlets_kv_free_pages(const outlets_kv* kv);
+
+#define OUTLETS_ALL_TOKENS 1u /* prefill flag: predict at every packed row, not only each sequence's last */
+
+/* Static prediction over a packed varlen batch (Sec. 3.2, t = 0).
+ *   taps[3]     device or host, [T, d] each (bf16 or f32 like the context),
+ *               row-major, 16-byte aligned: hidden states of target layers
+ *               2, floor(N/2), N-2 for every prompt token (Eq. 1).
+ *   cu_seqlens  host int32 [B+1]: cu[0] = 0, strictly increasing, cu[B] = T.
+ *   kv, slots   optional (both or neither): slots is host int32 [B], distinct;
+ *               each slot is reset and then holds its sequence's post-RoPE
+ *               keys/values, ready for outlets_predict_step.
+ *   flags       0 or OUTLETS_ALL_TOKENS.
+ *   z_out, len_out  device or host f32 [B] (or [T] with OUTLETS_ALL_TOKENS):
+ *               z_hat and max(0, expm1(z_hat)) = predicted remaining length.
+ *               len_out may be NULL.
+ * Errors: EINVAL (shapes, pointers, cu_seqlens), ECAPACITY (T > max_tokens,
+ * B > max_batch, a position >= max_position, or too few free KV pages). */
+outlets_status outlets_predict_prefill(outlets_ctx* ctx, const void* const taps[3], const int32_t* cu_seqlens,
+                                       int32_t B, int32_t T, outlets_kv* kv, const int32_t* slots, uint32_t flags,
+                                       float* z_out, float* len_out, void* stream);
+
+/* Dynamic prediction for one new token per request (Sec. 3.2, t >= 1).
+ *   taps[3]   device or host [B, d] each: the new token's tapped hidden states.
+ *   slots     host int32 [B], distinct.  The new token takes position
+ *             L = outlets_kv_slot_length(slot), attends to the slot's L cached
+ *             positions and itself, and is appended (slot length L + 1).
+ *   z_out, len_out  device or host f32 [B].
+ * Errors: EINVAL, ECAPACITY (no free page / position >= max_position / B >
+ * max_batch); on error no slot changes. */
+outlets_status outlets_predict_step(outlets_ctx* ctx, const void* const taps[3], int32_t B, outlets_kv* kv,
+                                    const int32_t* slots, float* z_out, float* len_out, void* stream);
+
+/* Synchronizes the stream, then reports (and clears) the device error word. */
+outlets_status outlets_check(outlets_ctx* ctx, void* stream);
+
+/* Intermediates of the last prediction call, for parity testing. */
+typedef enum outlets_tensor {
+  OUTLETS_T_FCTX = 0,   /* f_ctx [rows, d] f32 (Eq. 1) */
+  OUTLETS_T_XIN = 1,    /* input-normed x [rows, d] act */
+  OUTLETS_T_Q = 2,      /* post-RoPE q [rows, H, hd] act */
+  OUTLETS_T_ATTN = 3,   /* attention output [rows, H*hd] act */
+  OUTLETS_T_A = 4,      /* after attention residual [rows, d] f32 */
+  OUTLETS_T_Y = 5,      /* layer output [rows, d] f32 */
+  OUTLETS_T_HDRAFT = 6  /* final-normed draft state h^draft [out_rows, d] act */
+} outlets_tensor;
+
+typedef struct outlets_tensor_info {
+  int32_t dtype;  /* outlets_dtype of the stored values */
+  int32_t rows;
+  int32_t cols;
+} outlets_tensor_info;
+
+/* Describes intermediate `which` of the last call in *info and, if dst is not
+ * NULL, copies it (rows * cols elements, row-major) to dst (device or host,
+ * dst_bytes large enough) on the stream. */
+outlets_status outlets_get_intermediate(outlets_ctx* ctx, int32_t which, void* dst, size_t dst_bytes,
+                                        outlets_tensor_info* info, void* stream);
+
+/* Per-stage device timing.  While enabled, every prediction call records a
+ * CUDA event pair around each stage on the call's stream (a stage is one
+ * kernel, or the two kernels of split-KV decode attention). */
+typedef enum outlets_stage {
+  OUTLETS_S_FC = 0,          /* Eq. 1 tap-fusion GEMM */
+  OUTLETS_S_NORM_IN = 1,     /* input RMSNorm */
+  OUTLETS_S_QKV = 2,         /* QKV projection GEMM */
+  OUTLETS_S_ROPE = 3,        /* RoPE + q / K / V scatter (cache append) */
+  OUTLETS_S_ATTN = 4,        /* varlen causal attention or decode attention */
+  OUTLETS_S_O = 5,           /* O projection GEMM + residual */
+  OUTLETS_S_NORM_POST = 6,   /* post-attention RMSNorm */
+  OUTLETS_S_GATEUP = 7,      /* gate/up GEMM with SwiGLU */
+  OUTLETS_S_DOWN = 8,        /* down projection GEMM + residual */
+  OUTLETS_S_FINAL_NORM = 9,  /* final RMSNorm of the predicted rows (h^draft) */
+  OUTLETS_S_HEAD = 10,       /* length head (Sec. 4.2): Linear+ReLU layers and output row */
+  OUTLETS_N_STAGES = 11
+} outlets_stage;
+
+/* Turns stage timing on (1) or off (0) for later calls; clears recorded times. */
+outlets_status outlets_profile_enable(outlets_ctx* ctx, int32_t enable);
+
+/* Waits for the recorded events, then writes for each stage the summed
+ * duration in milliseconds (ms[OUTLETS_N_STAGES]) and how many times it ran
+ * (count[OUTLETS_N_STAGES], may be NULL), and clears the records. */
+outlets_status outlets_profile_read(outlets_ctx* ctx, double* ms, int32_t* count);
+
+/* Static name of a stage ("fc_gemm", ...), or "" for an invalid id. */
+const char* outlets_stage_name(int32_t stage);
+
+/* Number of kernels this context has launched for prediction calls so far. */
+uint64_t outlets_launch_count(const outlets_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OUTLETS_H_ */

@@ -1,0 +1,337 @@
+// tcgen05 GEMM for sm_103a: C[M, N] = A[M, K] * B[N, K]^T, bf16 in, f32 accumulate.
+//
+// Persistent, one CTA per SM, 6 warps:
+//   warp 0      TMA producer (one thread): A and B K-blocks into a smem ring
+//   warp 1      MMA issuer (one thread): tcgen05.mma 128 x BN x 16 into TMEM;
+//               also owns the TMEM allocation
+//   warps 2..5  epilogue: tcgen05.ld the accumulator, fuse the epilogue op,
+//               store to global.  Warp w reads TMEM lanes 32*(w%4) .. +31.
+// Two TMEM accumulators (2 * BN columns) let the epilogue of tile i overlap
+// the main loop of tile i+1.  Every mbarrier wait is bounded.
+//
+// Used for Eq. 1 (three-tap fusion: A is split along K over the three taps),
+// the QKV / O / gate-up / down projections of the draft decoder layer, and
+// the first Linear of the length head (Sec. 4.2).
+#include "common.cuh"
+#include "kernels.h"
+
+namespace outlets {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;  // one 128-byte swizzle row of bf16
+
+template <int BN>
+struct TcCfg {
+  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
+  static constexpr uint32_t A_BYTES = BM * BK * 2;
+  static constexpr uint32_t B_BYTES = BN * BK * 2;
+  static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;
+  static constexpr size_t SMEM = 1024 + STAGES * STAGE_BYTES + 256;
+};
+
+struct Tile {
+  int m_blk, n_blk, kb0, kb1;
+};
+
+__device__ __forceinline__ Tile decode_tile(int t, int num_m, int num_n, int group_m, int kb_total, int kb_per) {
+  const int per_split = num_m * num_n;
+  const int split = t / per_split;
+  const int r = t - split * per_split;
+  const int width = group_m * num_n;
+  const int group = r / width;
+  const int first_m = group * group_m;
+  const int gm = min(num_m - first_m, group_m);
+  const int rr = r - group * width;
+  Tile tl;
+  tl.m_blk = first_m + rr % gm;
+  tl.n_blk = rr / gm;
+  tl.kb0 = split * kb_per;
+  tl.kb1 = min(kb_total, tl.kb0 + kb_per);
+  return tl;
+}
+
+__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + __expf(-x)); }
+
+template <typename T>
+__device__ __forceinline__ void store_row32(T* dst, const float* v, int valid);
+
+template <>
+__device__ __forceinline__ void store_row32<float>(float* dst, const float* v, int valid) {
+  if (valid >= 32) {
+#pragma unroll
+    for (int j = 0; j < 32; j += 4)
+      *reinterpret_cast<float4*>(dst + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+  } else {
+    for (int j = 0; j < valid; ++j) dst[j] = v[j];
+  }
+}
+
+template <>
+__device__ __forceinline__ void store_row32<bf16>(bf16* dst, const float* v, int valid) {
+  if (valid >= 32) {
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) {
+      uint4 p;
+      p.x = pack_bf16x2(v[j], v[j + 1]);
+      p.y = pack_bf16x2(v[j + 2], v[j + 3]);
+      p.z = pack_bf16x2(v[j + 4], v[j + 5]);
+      p.w = pack_bf16x2(v[j + 6], v[j + 7]);
+      *reinterpret_cast<uint4*>(dst + j) = p;
+    }
+  } else {
+    for (int j = 0; j < valid; ++j) dst[j] = __float2bfloat16_rn(v[j]);
+  }
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(192, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_a1,
+              const __grid_constant__ CUtensorMap map_a2, const __grid_constant__ CUtensorMap map_b,
+              const GemmArgs p) {
+  using C = TcCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* tfull = empty + C::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 128);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&map_a0);
+    tma_prefetch_map(&map_a1);
+    tma_prefetch_map(&map_a2);
+    tma_prefetch_map(&map_b);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int num_m = (p.M + BM - 1) / BM;
+  const int num_n = (p.N + BN - 1) / BN;
+  const int kb_total = (p.K + BK - 1) / BK;
+  const int kb_per = (kb_total + p.splits - 1) / p.splits;
+  const int num_tiles = num_m * num_n * p.splits;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
+        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
+        for (int kb = tl.kb0; kb < tl.kb1; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.err)) goto producer_done;
+          uint8_t* sa = smem + stage * C::STAGE_BYTES;
+          uint8_t* sb = sa + C::A_BYTES;
+          mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
+          const int kg = kb * BK;
+          const int piece = kg / p.k_per_map;
+          const int kl = kg - piece * p.k_per_map;
+          const CUtensorMap* am = piece == 0 ? &map_a0 : (piece == 1 ? &map_a1 : &map_a2);
+          tma_load_2d(sa, am, &full[stage], kl, tl.m_blk * BM);
+          tma_load_2d(sb, &map_b, &full[stage], kg, tl.n_blk * BN);
+          if (++stage == C::STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+    producer_done:;
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
+        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, p.err)) goto mma_done;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+        for (int kb = tl.kb0; kb < tl.kb1; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, p.err)) goto mma_done;
+          tc_fence_after();
+          const uint32_t a_addr = smem_u32(smem + stage * C::STAGE_BYTES);
+          const uint32_t b_addr = a_addr + C::A_BYTES;
+          const uint64_t adesc = sw128_kmajor_desc(a_addr);
+          const uint64_t bdesc = sw128_kmajor_desc(b_addr);
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            // advance 16 elements (32 bytes = 2 units of 16 bytes) along K
+            tc_mma_bf16(d_tmem, adesc + 2u * kk, bdesc + 2u * kk, idesc, (kb > tl.kb0 || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(&empty[stage]);
+          if (++stage == C::STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        tc_commit(&tfull[acc]);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+    mma_done:;
+    }
+  } else {
+    // epilogue warps 2..5
+    const int quarter = warp & 3;
+    const int row_in_tile = quarter * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
+      const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
+      if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err)) break;
+      tc_fence_after();
+      const int m = tl.m_blk * BM + row_in_tile;
+      const bool row_ok = m < p.M;
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      if constexpr (EPI == EPI_SWIGLU) {
+        // tile columns [0, BN/2) are gate, [BN/2, BN) are up, for the same outputs
+        constexpr int HALF = BN / 2;
+        const int n_out = p.N / 2;
+        for (int c = 0; c < HALF; c += 32) {
+          uint32_t g[32], u[32];
+          tmem_ld_32x32b_x32(tbase + c, g);
+          tmem_ld_32x32b_x32(tbase + HALF + c, u);
+          tmem_ld_wait();
+          const int n0 = tl.n_blk * HALF + c;
+          if (row_ok && n0 < n_out) {
+            float v[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = silu_f(__uint_as_float(g[j])) * __uint_as_float(u[j]);
+            store_row32(reinterpret_cast<bf16*>(p.out) + (long long)m * p.ldo + n0, v, min(32, n_out - n0));
+          }
+        }
+      } else {
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tbase + c, r);
+          tmem_ld_wait();
+          const int n0 = tl.n_blk * BN + c;
+          if (row_ok && n0 < p.N) {
+            const int valid = min(32, p.N - n0);
+            float v[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+            if constexpr (EPI == EPI_F32) {
+              if (p.residual) {
+                const float* res = p.residual + (long long)m * p.ldr + n0;
+                if (valid >= 32) {
+#pragma unroll
+                  for (int j = 0; j < 32; j += 4) {
+                    const float4 q = *reinterpret_cast<const float4*>(res + j);
+                    v[j] += q.x;
+                    v[j + 1] += q.y;
+                    v[j + 2] += q.z;
+                    v[j + 3] += q.w;
+                  }
+                } else {
+                  for (int j = 0; j < valid; ++j) v[j] += res[j];
+                }
+              }
+              store_row32(reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n0, v, valid);
+            } else if constexpr (EPI == EPI_ACT) {
+              store_row32(reinterpret_cast<bf16*>(p.out) + (long long)m * p.ldo + n0, v, valid);
+            } else if constexpr (EPI == EPI_BIAS_RELU) {
+              for (int j = 0; j < valid; ++j) v[j] = fmaxf(v[j] + p.bias[n0 + j], 0.0f);
+              store_row32(reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n0, v, valid);
+            } else {  // EPI_ATOMIC
+              float* dst = reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n0;
+              if (valid >= 32) {
+#pragma unroll
+                for (int j = 0; j < 32; j += 4)
+                  atomicAdd(reinterpret_cast<float4*>(dst + j), make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]));
+              } else {
+                for (int j = 0; j < valid; ++j) atomicAdd(dst + j, v[j]);
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&tempty[acc]);
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+template <int BN, int EPI>
+cudaError_t launch_one(const CUtensorMap a_maps[3], const CUtensorMap& b_map, const GemmArgs& args, int num_sms,
+                       cudaStream_t stream) {
+  using C = TcCfg<BN>;
+  auto kern = k_gemm_tc<BN, EPI>;
+  static bool attr_set = false;  // per (BN, EPI) instantiation
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const long long tiles = (long long)((args.M + BM - 1) / BM) * ((args.N + BN - 1) / BN) * args.splits;
+  const int grid = (int)(tiles < num_sms ? tiles : num_sms);
+  if (grid <= 0) return cudaSuccess;
+  kern<<<grid, 192, C::SMEM, stream>>>(a_maps[0], a_maps[1], a_maps[2], b_map, args);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], const CUtensorMap& b_map, int bn, int epi,
+                           const GemmArgs& args, int num_sms, cudaStream_t stream) {
+#define OUTLETS_TC_CASE(BNV, EV) \
+  if (bn == BNV && epi == EV) return launch_one<BNV, EV>(a_maps, b_map, args, num_sms, stream);
+  OUTLETS_TC_CASE(256, EPI_F32)
+  OUTLETS_TC_CASE(256, EPI_ACT)
+  OUTLETS_TC_CASE(256, EPI_SWIGLU)
+  OUTLETS_TC_CASE(256, EPI_BIAS_RELU)
+  OUTLETS_TC_CASE(256, EPI_ATOMIC)
+  OUTLETS_TC_CASE(128, EPI_F32)
+  OUTLETS_TC_CASE(128, EPI_ACT)
+  OUTLETS_TC_CASE(128, EPI_BIAS_RELU)
+  OUTLETS_TC_CASE(128, EPI_ATOMIC)
+  OUTLETS_TC_CASE(64, EPI_F32)
+  OUTLETS_TC_CASE(64, EPI_ACT)
+  OUTLETS_TC_CASE(64, EPI_BIAS_RELU)
+  OUTLETS_TC_CASE(64, EPI_ATOMIC)
+#undef OUTLETS_TC_CASE
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace outlets

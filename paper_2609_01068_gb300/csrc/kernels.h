@@ -1,0 +1,143 @@
+// Internal launch interface between the C-ABI runtime (outlets.cu) and the
+// kernels.  Nothing here is part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace outlets {
+
+typedef __nv_bfloat16 bf16;
+
+// Error bits written by kernels into the context's device error word.
+enum : int {
+  ERR_TIMEOUT = 1,    // a bounded wait ran out (an mbarrier phase never completed)
+  ERR_BAD_INDEX = 2,  // a kernel met an index it refused to use
+};
+
+// GEMM: C[M, N] = A[M, K] * B[N, K]^T, A optionally split along K across up to
+// three separately addressed row-major matrices (the three taps of Eq. 1).
+enum Epi : int {
+  EPI_F32 = 0,        // out f32 = acc (+ residual f32)
+  EPI_ACT = 1,        // out act (bf16 on the tensor-core path, f32 on the CUDA-core path) = acc
+  EPI_SWIGLU = 2,     // B rows interleaved in blocks of 128 [gate | up]; out act = silu(g) * u
+  EPI_BIAS_RELU = 3,  // out f32 = max(acc + bias, 0)
+  EPI_ATOMIC = 4,     // out f32 += acc (split-K partial sums)
+};
+
+struct GemmArgs {
+  int M, N, K;
+  int k_per_map;          // K extent of each A piece (multiple of 64 when pieces > 1)
+  int splits;             // split-K factor (> 1 only with EPI_ATOMIC); every split non-empty
+  int group_m;            // tile raster: M blocks per group
+  void* out;
+  long long ldo;          // elements
+  const float* residual;  // EPI_F32 only, may be null
+  long long ldr;
+  const float* bias;      // EPI_BIAS_RELU
+  int* err;
+};
+
+// tcgen05 path (bf16 operands).  a_maps: 3 tensor maps over the A pieces (box
+// 64 x 128), b_map: tensor map over B (box 64 x bn).  grid = min(tiles, num_sms).
+cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], const CUtensorMap& b_map, int bn, int epi,
+                           const GemmArgs& args, int num_sms, cudaStream_t stream);
+
+// CUDA-core path of the f32 configuration.  a[0..2]: A pieces with row stride k_per_map.
+cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int epi, const GemmArgs& args,
+                                 cudaStream_t stream);
+
+// ---------------------------------------------------------------- elementwise
+// y[r] = x[r] * g * rsqrt(mean(x[r]^2) + eps); optionally copy x[r] into copy_out[r].
+template <typename Act>
+cudaError_t rmsnorm_launch(const float* x, const float* g, Act* y, float* copy_out, int rows, int d, float eps,
+                           cudaStream_t stream);
+
+// y[i] = norm(x[row_index[i]]).
+template <typename Act>
+cudaError_t rmsnorm_gather_launch(const float* x, const int* row_index, const float* g, Act* y, int rows, int d,
+                                  float eps, cudaStream_t stream);
+
+struct RopeArgs {
+  int T;                 // rows of this call
+  int H, KVH, hd;
+  const int* cu;         // prefill: sequence offsets [B+1] (position = row - cu[b]); else null
+  int B;
+  const int* pos;        // step: position of each row; else null
+  const float* cos_tab;  // [max_pos, hd/2]
+  const float* sin_tab;
+  int max_pos;
+  void* q_out;           // [T, H, hd]
+  void* k_out;           // head-major [KVH, kv_ld_rows, hd] or null
+  void* v_out;
+  long long kv_ld_rows;
+  void* k_pool;          // paged cache [pages][KVH][page_tokens][hd] or null
+  void* v_pool;
+  const int* page_list;  // pages of each sequence/request, concatenated
+  const int* page_off;   // [B+1] (prefill: per sequence; step: per row)
+  int page_tokens;
+  int* err;
+};
+template <typename In, typename Act>
+cudaError_t rope_scatter_launch(const In* qkv, const RopeArgs& a, cudaStream_t stream);
+
+// u[r, j] = silu(gu[r, gate(j)]) * gu[r, up(j)], gu interleaved in blocks of 128.
+template <typename Act>
+cudaError_t swiglu_launch(const float* gu, Act* u, int rows, int f_pad, cudaStream_t stream);
+
+// z[r] = w_last . a(h[r]) + b_last, a(x) = relu(x + b_prev) (identity if b_prev is null);
+// len[r] = max(0, expm1(z[r])).
+cudaError_t head_tail_launch(const float* h_pre, const float* b_prev, const float* w_last, const float* b_last,
+                             int rows, int width, float* z, float* len, cudaStream_t stream);
+
+// dst[map(r)][c] = src[r][c] (f32 -> Act); row_mode 0: row_base + r, 1: gate rows, 2: up rows
+// of the [gate | up] interleave (blocks of 128).
+template <typename Act>
+cudaError_t convert_rows_launch(const float* src, Act* dst, int rows, int cols, long long dst_ld, int row_mode,
+                                int row_base, cudaStream_t stream);
+
+// ---------------------------------------------------------------- attention
+struct AttnTile {
+  int q_start;    // first query row (packed index)
+  int q_len;      // rows in this tile (<= 64)
+  int seq_start;  // first row of the sequence
+  int seq_len;    // rows of the sequence
+};
+
+// k/v head-major [KVH, kv_ld, hd]; q/out [n_rows, H, hd].
+template <typename Act>
+cudaError_t attn_prefill_simt_launch(const Act* q, const Act* k, const Act* v, const int* cu, int B, int n_rows,
+                                     int kv_ld, int H, int KVH, int hd, Act* out, cudaStream_t stream);
+
+// bf16 flash attention; q_map over [rows, H*hd] (box 64 x 64), k/v maps over
+// head-major [KVH * kv_ld, hd] (box 64 x 64); kv_ld passed as T.
+cudaError_t attn_prefill_bf16_launch(const CUtensorMap& q_map, const CUtensorMap& k_map, const CUtensorMap& v_map,
+                                     const AttnTile* tiles, int n_tiles, int T, int H, int KVH, int hd, void* out,
+                                     int* err, cudaStream_t stream);
+
+struct DecodeArgs {
+  int B, H, KVH, hd;
+  const void* q;          // [B, H, hd]
+  const void* k_pool;     // [pages][KVH][page_tokens][hd]
+  const void* v_pool;
+  int page_tokens;
+  const int* page_list;   // concatenated page ids of every request
+  const int* page_off;    // [B+1] offsets into page_list
+  const int* seq_len;     // [B] keys per request (cached + the new token)
+  const int* work;        // [n_work] pairs (request, split), grouped by request
+  const int* work_off;    // [B+1] first work item of each request
+  int n_work;
+  int split_len;          // keys per split (multiple of page_tokens)
+  float* part_o;          // [n_work, H, hd] normalized partial outputs
+  float* part_ml;         // [n_work, H, 2] (max in log2 units, sum)
+  void* out;              // [B, H, hd]
+  int* err;
+};
+cudaError_t attn_decode_bf16_launch(const CUtensorMap& k_map, const CUtensorMap& v_map, const DecodeArgs& a,
+                                    cudaStream_t stream);
+template <typename Act>
+cudaError_t attn_decode_simt_launch(const DecodeArgs& a, cudaStream_t stream);
+
+}  // namespace outlets

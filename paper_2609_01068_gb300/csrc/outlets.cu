@@ -1,0 +1,1096 @@
+// Host runtime behind the C ABI of include/outlets.h: argument validation,
+// weight upload and re-layout, the paged draft KV cache, per-call metadata
+// staging and the launch sequences of static (prefill) and dynamic (step)
+// prediction (Sec. 3.2).
+//
+// Launch sequence of one prediction call, on the caller's stream:
+//   FC (Eq. 1, tcgen05 GEMM over the three taps) -> RMSNorm ->
+//   QKV GEMM -> RoPE + K/V scatter (workspace and/or paged cache) ->
+//   attention (varlen causal flash attention, or paged split-KV decode) ->
+//   O GEMM + residual -> RMSNorm -> gate/up GEMM with fused SwiGLU ->
+//   down GEMM + residual -> final RMSNorm of the predicted rows (h^draft) ->
+//   head Linear+ReLU (GEMM) ... -> head output row + expm1 (Sec. 4.2).
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "kernels.h"
+#include "outlets.h"
+
+using namespace outlets;
+
+namespace {
+
+constexpr int kPageTokens = 64;
+constexpr int kSplitLen = 512;
+constexpr int kRing = 4;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// 2D bf16 tensor map: rows x cols (cols contiguous, row stride ld elements),
+// box box_rows x 64 columns, 128-byte swizzle, zero fill outside the tensor.
+bool make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld, uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || rows == 0 || cols == 0) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+inline long long cdiv(long long a, long long b) { return (a + b - 1) / b; }
+
+}  // namespace
+
+struct outlets_ctx {
+  outlets_config cfg{};
+  std::string err;
+  int num_sms = 0;
+  bool bf16 = true;
+  size_t esz = 2;
+  int d = 0, H = 0, KVH = 0, hd = 0, F = 0, Fp = 0, qkv_n = 0, attn_w = 0, max_rows = 0;
+  std::vector<int> head_dims;  // d, hidden..., 1
+  std::vector<void*> allocs;
+  size_t dev_bytes = 0;
+
+  void *w_proj = nullptr, *w_qkv = nullptr, *w_o = nullptr, *w_gu = nullptr, *w_down = nullptr,
+       *head_w0 = nullptr;
+  float *g_in = nullptr, *g_post = nullptr, *g_final = nullptr;
+  std::vector<float*> head_wf, head_b;
+  float *rope_cos = nullptr, *rope_sin = nullptr;
+
+  float *f = nullptr, *a = nullptr, *y = nullptr, *h1a = nullptr, *h1b = nullptr, *z = nullptr, *len = nullptr,
+        *gu32 = nullptr;
+  void *xhat = nullptr, *ahat = nullptr, *qkv = nullptr, *q = nullptr, *kh = nullptr, *vh = nullptr,
+       *attn = nullptr, *u = nullptr, *hn = nullptr;
+  void* taps_stage[3] = {nullptr, nullptr, nullptr};
+  int* err_dev = nullptr;
+  int* meta_dev = nullptr;
+  size_t meta_cap = 0;  // ints
+
+  struct Pin {
+    int* h = nullptr;
+    size_t cap = 0;
+    cudaEvent_t ev = nullptr;
+    bool used = false;
+  } ring[kRing];
+  int ring_i = 0;
+  cudaEvent_t done_ev = nullptr;
+  bool have_prev = false;
+
+  int last_rows = 0, last_out_rows = 0;
+  bool oom = false;
+
+  // stage timing and launch accounting
+  struct ProfRec {
+    int stage;
+    cudaEvent_t a, b;
+  };
+  bool prof = false;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  std::vector<ProfRec> recs;
+  unsigned long long launches = 0;
+  cudaStream_t cur_stream = nullptr;
+
+  cudaEvent_t next_event() {
+    if (ev_used == ev_pool.size()) {
+      cudaEvent_t e = nullptr;
+      if (cudaEventCreate(&e) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+      }
+      ev_pool.push_back(e);
+    }
+    return ev_pool[ev_used++];
+  }
+  void stage_begin(int stage) {
+    if (!prof) return;
+    ProfRec r{stage, next_event(), next_event()};
+    if (!r.a || !r.b) return;
+    cudaEventRecord(r.a, cur_stream);
+    recs.push_back(r);
+  }
+  void stage_end(int n_kernels) {
+    launches += (unsigned long long)n_kernels;
+    if (!prof || recs.empty()) return;
+    cudaEventRecord(recs.back().b, cur_stream);
+  }
+
+  outlets_status fail(outlets_status st, const std::string& msg) {
+    err = msg;
+    return st;
+  }
+  outlets_status cuda_fail(cudaError_t e, const char* what) {
+    err = std::string(what) + ": " + cudaGetErrorString(e);
+    return OUTLETS_ECUDA;
+  }
+  void* alloc(size_t bytes) {
+    if (bytes == 0) bytes = 16;
+    void* p = nullptr;
+    if (cudaMalloc(&p, bytes) != cudaSuccess) {
+      cudaGetLastError();
+      oom = true;
+      return nullptr;
+    }
+    cudaMemset(p, 0, bytes);
+    allocs.push_back(p);
+    dev_bytes += bytes;
+    return p;
+  }
+};
+
+struct outlets_kv {
+  outlets_ctx* ctx = nullptr;
+  int device = 0;
+  int max_slots = 0, num_pages = 0, max_pages_per_slot = 0;
+  void *k_pool = nullptr, *v_pool = nullptr;
+  float *part_o = nullptr, *part_ml = nullptr;
+  size_t part_items = 0;
+  std::vector<int> len;
+  std::vector<std::vector<int>> pages;
+  std::vector<int> free_list;
+  std::vector<void*> allocs;
+};
+
+#define OUT_CK(ctx, ...)                                         \
+  do {                                                            \
+    cudaError_t e_ = (__VA_ARGS__);                               \
+    if (e_ != cudaSuccess) return (ctx)->cuda_fail(e_, #__VA_ARGS__); \
+  } while (0)
+
+namespace {
+
+// Uploads a host f32 matrix [rows, cols] through a device staging buffer and
+// converts it (f32 -> act) into dst with the given row mapping.
+outlets_status upload_rows(outlets_ctx* c, const float* src, int rows, int cols, void* dst, long long dst_ld,
+                           int row_mode, int row_base, float* stage, size_t stage_floats) {
+  const int chunk = (int)std::max<size_t>(1, stage_floats / (size_t)cols);
+  for (int r0 = 0; r0 < rows; r0 += chunk) {
+    const int n = std::min(chunk, rows - r0);
+    OUT_CK(c, cudaMemcpy(stage, src + (size_t)r0 * cols, (size_t)n * cols * 4, cudaMemcpyHostToDevice));
+    // rows r0.. map like global rows: shift the mapping by r0
+    cudaError_t e;
+    if (row_mode == 0) {
+      e = c->bf16 ? convert_rows_launch<bf16>(stage, (bf16*)dst, n, cols, dst_ld, 0, row_base + r0, 0)
+                  : convert_rows_launch<float>(stage, (float*)dst, n, cols, dst_ld, 0, row_base + r0, 0);
+    } else {
+      // chunk boundaries are multiples of 128 rows (see caller) so the interleave maps locally
+      const long long off = (long long)(r0 >> 7) * 256 * dst_ld;
+      e = c->bf16 ? convert_rows_launch<bf16>(stage, (bf16*)dst + off, n, cols, dst_ld, row_mode, 0, 0)
+                  : convert_rows_launch<float>(stage, (float*)dst + off, n, cols, dst_ld, row_mode, 0, 0);
+    }
+    OUT_CK(c, e);
+    OUT_CK(c, cudaDeviceSynchronize());
+  }
+  return OUTLETS_OK;
+}
+
+outlets_status validate_config(const outlets_config* cfg, std::string& why) {
+  auto bad = [&](const char* m) {
+    why = m;
+    return OUTLETS_EINVAL;
+  };
+  if (cfg->dtype != OUTLETS_F32 && cfg->dtype != OUTLETS_BF16) return bad("dtype must be OUTLETS_F32 or OUTLETS_BF16");
+  if (cfg->d_model <= 0 || cfg->d_model % 64) return bad("d_model must be a positive multiple of 64");
+  if (cfg->n_heads <= 0 || cfg->n_kv_heads <= 0 || cfg->n_heads % cfg->n_kv_heads)
+    return bad("n_heads must be a positive multiple of n_kv_heads");
+  if (cfg->head_dim <= 0 || cfg->head_dim % 2) return bad("head_dim must be positive and even");
+  if ((cfg->n_heads * cfg->head_dim) % 64) return bad("n_heads * head_dim must be a multiple of 64");
+  if (cfg->ffn_dim <= 0) return bad("ffn_dim must be positive");
+  if (cfg->n_head_hidden < 1 || cfg->n_head_hidden > OUTLETS_MAX_HEAD_HIDDEN)
+    return bad("n_head_hidden must be in 1..OUTLETS_MAX_HEAD_HIDDEN");
+  for (int i = 0; i < cfg->n_head_hidden; ++i)
+    if (cfg->head_hidden[i] <= 0 || cfg->head_hidden[i] % 4) return bad("head widths must be positive multiples of 4");
+  if (!(cfg->rope_theta > 1.0f)) return bad("rope_theta must be > 1");
+  if (!(cfg->rms_eps >= 0.0f)) return bad("rms_eps must be >= 0");
+  if (cfg->max_tokens <= 0 || cfg->max_batch <= 0 || cfg->max_position <= 0)
+    return bad("max_tokens, max_batch and max_position must be positive");
+  if (cfg->dtype == OUTLETS_BF16) {
+    if (cfg->head_dim != 64 && cfg->head_dim != 128) return bad("bf16 path supports head_dim 64 or 128");
+    if (cfg->n_heads / cfg->n_kv_heads > 16) return bad("bf16 path supports at most 16 query heads per kv head");
+  } else {
+    if (cfg->head_dim > 256) return bad("f32 path supports head_dim <= 256");
+  }
+  return OUTLETS_OK;
+}
+
+// Pinned staging of one call's index metadata, then one H2D copy.
+outlets_status upload_meta(outlets_ctx* c, const std::vector<int>& meta, cudaStream_t s) {
+  if (meta.empty()) return OUTLETS_OK;
+  if (meta.size() > c->meta_cap) {
+    if (c->meta_dev) {
+      OUT_CK(c, cudaStreamSynchronize(s));
+      cudaFree(c->meta_dev);
+      c->meta_dev = nullptr;
+    }
+    size_t cap = std::max<size_t>(meta.size() * 2, 1 << 16);
+    if (cudaMalloc(&c->meta_dev, cap * sizeof(int)) != cudaSuccess) {
+      cudaGetLastError();
+      c->meta_cap = 0;
+      return c->fail(OUTLETS_ENOMEM, "metadata buffer allocation failed");
+    }
+    c->meta_cap = cap;
+  }
+  outlets_ctx::Pin& p = c->ring[c->ring_i];
+  c->ring_i = (c->ring_i + 1) % kRing;
+  if (p.used) OUT_CK(c, cudaEventSynchronize(p.ev));
+  if (meta.size() > p.cap) {
+    if (p.h) cudaFreeHost(p.h);
+    p.h = nullptr;
+    size_t cap = std::max<size_t>(meta.size() * 2, 1 << 16);
+    if (cudaMallocHost(&p.h, cap * sizeof(int)) != cudaSuccess) {
+      cudaGetLastError();
+      p.cap = 0;
+      return c->fail(OUTLETS_ENOMEM, "pinned metadata buffer allocation failed");
+    }
+    p.cap = cap;
+  }
+  std::memcpy(p.h, meta.data(), meta.size() * sizeof(int));
+  OUT_CK(c, cudaMemcpyAsync(c->meta_dev, p.h, meta.size() * sizeof(int), cudaMemcpyHostToDevice, s));
+  OUT_CK(c, cudaEventRecord(p.ev, s));
+  p.used = true;
+  return OUTLETS_OK;
+}
+
+struct MetaBuilder {
+  std::vector<int> v;
+  size_t put(const int* src, size_t n) {
+    while (v.size() % 4) v.push_back(0);
+    size_t off = v.size();
+    v.insert(v.end(), src, src + n);
+    return off;
+  }
+  size_t put(const std::vector<int>& x) { return put(x.data(), x.size()); }
+};
+
+// bf16 GEMM through tcgen05.  A pieces: row-major [M, k_piece] with row stride lda.
+outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
+                       const void* b, int N, int K, int epi, void* out, long long ldo, const float* residual,
+                       long long ldr, const float* bias, cudaStream_t s) {
+  if (M == 0) return OUTLETS_OK;
+  int bn = 256;
+  if (epi != EPI_SWIGLU) {
+    auto tiles = [&](int bnv) { return cdiv(M, 128) * cdiv(N, bnv); };
+    if (tiles(256) >= c->num_sms) bn = 256;
+    else if (tiles(128) >= c->num_sms) bn = 128;
+    else bn = 64;
+  }
+  CUtensorMap am[3], bm;
+  for (int i = 0; i < 3; ++i) {
+    const void* base = a[i < n_pieces ? i : 0];
+    if (!make_map(&am[i], base, (uint64_t)k_piece, (uint64_t)M, (uint64_t)lda, 128))
+      return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for a GEMM A operand");
+  }
+  if (!make_map(&bm, b, (uint64_t)K, (uint64_t)N, (uint64_t)K, (uint32_t)bn))
+    return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for a GEMM B operand");
+  GemmArgs g{};
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.k_per_map = k_piece;
+  g.splits = 1;
+  g.group_m = 16;
+  g.out = out;
+  g.ldo = ldo;
+  g.residual = residual;
+  g.ldr = ldr;
+  g.bias = bias;
+  g.err = c->err_dev;
+  OUT_CK(c, gemm_tc_launch(am, bm, bn, epi, g, c->num_sms, s));
+  return OUTLETS_OK;
+}
+
+outlets_status gemm_f32(outlets_ctx* c, const void* const* a, int k_piece, int M, const void* b, int N, int K,
+                        int epi, void* out, long long ldo, const float* residual, long long ldr, const float* bias,
+                        cudaStream_t s) {
+  const float* ap[3] = {(const float*)a[0], (const float*)a[1], (const float*)a[2]};
+  GemmArgs g{};
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.k_per_map = k_piece;
+  g.splits = 1;
+  g.group_m = 1;
+  g.out = out;
+  g.ldo = ldo;
+  g.residual = residual;
+  g.ldr = ldr;
+  g.bias = bias;
+  g.err = c->err_dev;
+  OUT_CK(c, gemm_simt_f32_launch(ap, (const float*)b, epi, g, s));
+  return OUTLETS_OK;
+}
+
+#define OUT_TRY(expr)                      \
+  do {                                     \
+    outlets_status st_ = (expr);           \
+    if (st_ != OUTLETS_OK) return st_;     \
+  } while (0)
+
+// Everything after attention: O projection + residual, post-attention norm,
+// SwiGLU MLP + residual, final norm of the predicted rows, length head.
+outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_row_idx_dev, float* z_dev,
+                        float* len_dev, cudaStream_t s) {
+  const int d = c->d;
+  // O projection + residual: a = f + attn W_o^T
+  c->stage_begin(OUTLETS_S_O);
+  {
+    const void* a1[3] = {c->attn, c->attn, c->attn};
+    if (c->bf16)
+      OUT_TRY(gemm_tc(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d,
+                      nullptr, s));
+    else
+      OUT_TRY(gemm_f32(c, a1, c->attn_w, rows, c->w_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d, nullptr, s));
+  }
+  c->stage_end(1);
+  // post-attention RMSNorm
+  c->stage_begin(OUTLETS_S_NORM_POST);
+  if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->a, c->g_post, (bf16*)c->ahat, nullptr, rows, d, c->cfg.rms_eps, s));
+  else OUT_CK(c, rmsnorm_launch<float>(c->a, c->g_post, (float*)c->ahat, nullptr, rows, d, c->cfg.rms_eps, s));
+  c->stage_end(1);
+  // gate/up + SwiGLU
+  c->stage_begin(OUTLETS_S_GATEUP);
+  {
+    const void* a1[3] = {c->ahat, c->ahat, c->ahat};
+    if (c->bf16) {
+      OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_gu, 2 * c->Fp, d, EPI_SWIGLU, c->u, c->Fp, nullptr, 0, nullptr, s));
+    } else {
+      OUT_TRY(gemm_f32(c, a1, d, rows, c->w_gu, 2 * c->Fp, d, EPI_F32, c->gu32, 2 * c->Fp, nullptr, 0, nullptr, s));
+      OUT_CK(c, swiglu_launch<float>(c->gu32, (float*)c->u, rows, c->Fp, s));
+      c->launches += 1;
+    }
+  }
+  c->stage_end(1);
+  // down + residual: y = a + u W_down^T
+  c->stage_begin(OUTLETS_S_DOWN);
+  {
+    const void* a1[3] = {c->u, c->u, c->u};
+    if (c->bf16)
+      OUT_TRY(gemm_tc(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, d, c->Fp, EPI_F32, c->y, d, c->a, d, nullptr, s));
+    else
+      OUT_TRY(gemm_f32(c, a1, c->Fp, rows, c->w_down, d, c->Fp, EPI_F32, c->y, d, c->a, d, nullptr, s));
+  }
+  c->stage_end(1);
+  // final RMSNorm of the predicted rows -> h^draft
+  c->stage_begin(OUTLETS_S_FINAL_NORM);
+  if (c->bf16)
+    OUT_CK(c, rmsnorm_gather_launch<bf16>(c->y, out_row_idx_dev, c->g_final, (bf16*)c->hn, out_rows, d,
+                                          c->cfg.rms_eps, s));
+  else
+    OUT_CK(c, rmsnorm_gather_launch<float>(c->y, out_row_idx_dev, c->g_final, (float*)c->hn, out_rows, d,
+                                           c->cfg.rms_eps, s));
+  c->stage_end(1);
+  // length head: Linear+ReLU layers, then the output row
+  c->stage_begin(OUTLETS_S_HEAD);
+  const int nl = (int)c->head_dims.size() - 1;
+  float* cur = c->h1a;
+  {
+    const void* a1[3] = {c->hn, c->hn, c->hn};
+    const int w1 = c->head_dims[1];
+    if (c->bf16)
+      OUT_TRY(gemm_tc(c, a1, 1, d, d, out_rows, c->head_w0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0,
+                      c->head_b[0], s));
+    else
+      OUT_TRY(gemm_f32(c, a1, d, out_rows, c->head_w0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0, c->head_b[0], s));
+  }
+  for (int i = 1; i < nl - 1; ++i) {
+    float* nxt = (cur == c->h1a) ? c->h1b : c->h1a;
+    const void* a1[3] = {cur, cur, cur};
+    OUT_TRY(gemm_f32(c, a1, c->head_dims[i], out_rows, c->head_wf[i], c->head_dims[i + 1], c->head_dims[i],
+                     EPI_BIAS_RELU, nxt, c->head_dims[i + 1], nullptr, 0, c->head_b[i], s));
+    cur = nxt;
+  }
+  OUT_CK(c, head_tail_launch(cur, nullptr, c->head_wf[nl - 1], c->head_b[nl - 1], out_rows, c->head_dims[nl - 1],
+                             z_dev, len_dev, s));
+  c->stage_end(nl);
+  return OUTLETS_OK;
+}
+
+// Stages host taps (or passes device taps through); checks alignment.
+outlets_status prepare_taps(outlets_ctx* c, const void* const taps[3], int rows, const void* out[3],
+                            cudaStream_t s) {
+  for (int i = 0; i < 3; ++i) {
+    if (!taps[i]) return c->fail(OUTLETS_EINVAL, "taps[i] is NULL");
+    if (is_device_ptr(taps[i])) {
+      if (reinterpret_cast<uintptr_t>(taps[i]) % 16) return c->fail(OUTLETS_EINVAL, "device taps must be 16-byte aligned");
+      out[i] = taps[i];
+    } else {
+      if (!c->taps_stage[i]) {
+        c->taps_stage[i] = c->alloc((size_t)c->max_rows * c->d * c->esz);
+        if (!c->taps_stage[i]) return c->fail(OUTLETS_ENOMEM, "tap staging allocation failed");
+      }
+      OUT_CK(c, cudaMemcpyAsync(c->taps_stage[i], taps[i], (size_t)rows * c->d * c->esz, cudaMemcpyHostToDevice, s));
+      out[i] = c->taps_stage[i];
+    }
+  }
+  return OUTLETS_OK;
+}
+
+outlets_status begin_call(outlets_ctx* c, cudaStream_t s) {
+  OUT_CK(c, cudaSetDevice(c->cfg.device));
+  c->cur_stream = s;
+  if (c->have_prev) OUT_CK(c, cudaStreamWaitEvent(s, c->done_ev, 0));
+  return OUTLETS_OK;
+}
+
+outlets_status end_call(outlets_ctx* c, int out_rows, float* z_out, float* len_out, cudaStream_t s) {
+  if (z_out != c->z) OUT_CK(c, cudaMemcpyAsync(z_out, c->z, (size_t)out_rows * 4, cudaMemcpyDefault, s));
+  if (len_out && len_out != c->len)
+    OUT_CK(c, cudaMemcpyAsync(len_out, c->len, (size_t)out_rows * 4, cudaMemcpyDefault, s));
+  OUT_CK(c, cudaEventRecord(c->done_ev, s));
+  c->have_prev = true;
+  return OUTLETS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* w, outlets_ctx** out) {
+  if (!out) return OUTLETS_EINVAL;
+  *out = nullptr;
+  if (!cfg || !w) return OUTLETS_EINVAL;
+  std::string why;
+  if (validate_config(cfg, why) != OUTLETS_OK) {
+    std::fprintf(stderr, "outlets_create: %s\n", why.c_str());
+    return OUTLETS_EINVAL;
+  }
+  const float* req[] = {w->w_proj, w->w_q, w->w_k, w->w_v, w->w_o, w->g_in, w->g_post, w->g_final,
+                        w->w_gate, w->w_up, w->w_down};
+  for (const float* p : req)
+    if (!p) return OUTLETS_EINVAL;
+  for (int i = 0; i <= cfg->n_head_hidden; ++i)
+    if (!w->head_w[i] || !w->head_b[i]) return OUTLETS_EINVAL;
+  if (cudaSetDevice(cfg->device) != cudaSuccess) {
+    cudaGetLastError();
+    return OUTLETS_ECUDA;
+  }
+  int major = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, cfg->device);
+  if (cfg->dtype == OUTLETS_BF16 && (major < 10 || !encode_fn())) return OUTLETS_EUNSUPPORTED;
+
+  outlets_ctx* c = new outlets_ctx();
+  c->cfg = *cfg;
+  c->bf16 = cfg->dtype == OUTLETS_BF16;
+  c->esz = c->bf16 ? 2 : 4;
+  c->d = cfg->d_model;
+  c->H = cfg->n_heads;
+  c->KVH = cfg->n_kv_heads;
+  c->hd = cfg->head_dim;
+  c->F = cfg->ffn_dim;
+  c->Fp = (int)cdiv(c->F, 128) * 128;
+  c->qkv_n = (c->H + 2 * c->KVH) * c->hd;
+  c->attn_w = c->H * c->hd;
+  c->max_rows = std::max(cfg->max_tokens, cfg->max_batch);
+  c->head_dims.push_back(c->d);
+  for (int i = 0; i < cfg->n_head_hidden; ++i) c->head_dims.push_back(cfg->head_hidden[i]);
+  c->head_dims.push_back(1);
+  cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, cfg->device);
+
+  auto cleanup_fail = [&](outlets_status st) {
+    outlets_destroy(c);
+    return st;
+  };
+  const int d = c->d;
+  const size_t es = c->esz;
+  // ---- weights
+  c->w_proj = c->alloc((size_t)d * 3 * d * es);
+  c->w_qkv = c->alloc((size_t)c->qkv_n * d * es);
+  c->w_o = c->alloc((size_t)d * c->attn_w * es);
+  c->w_gu = c->alloc((size_t)2 * c->Fp * d * es);
+  c->w_down = c->alloc((size_t)d * c->Fp * es);
+  c->g_in = (float*)c->alloc((size_t)d * 4);
+  c->g_post = (float*)c->alloc((size_t)d * 4);
+  c->g_final = (float*)c->alloc((size_t)d * 4);
+  const int nl = (int)c->head_dims.size() - 1;
+  c->head_wf.assign(nl, nullptr);
+  c->head_b.assign(nl, nullptr);
+  c->head_w0 = c->alloc((size_t)c->head_dims[1] * d * es);
+  for (int i = 1; i < nl; ++i) c->head_wf[i] = (float*)c->alloc((size_t)c->head_dims[i + 1] * c->head_dims[i] * 4);
+  for (int i = 0; i < nl; ++i) c->head_b[i] = (float*)c->alloc((size_t)c->head_dims[i + 1] * 4);
+  c->rope_cos = (float*)c->alloc((size_t)cfg->max_position * (c->hd / 2) * 4);
+  c->rope_sin = (float*)c->alloc((size_t)cfg->max_position * (c->hd / 2) * 4);
+  // ---- workspace
+  const size_t R = (size_t)c->max_rows;
+  c->f = (float*)c->alloc(R * d * 4);
+  c->a = (float*)c->alloc(R * d * 4);
+  c->y = (float*)c->alloc(R * d * 4);
+  c->xhat = c->alloc(R * d * es);
+  c->ahat = c->alloc(R * d * es);
+  c->hn = c->alloc(R * d * es);
+  c->qkv = c->alloc(R * c->qkv_n * es);
+  c->q = c->alloc(R * c->attn_w * es);
+  c->attn = c->alloc(R * c->attn_w * es);
+  c->kh = c->alloc((size_t)c->KVH * cfg->max_tokens * c->hd * es);
+  c->vh = c->alloc((size_t)c->KVH * cfg->max_tokens * c->hd * es);
+  c->u = c->alloc(R * c->Fp * es);
+  if (!c->bf16) c->gu32 = (float*)c->alloc(R * 2 * c->Fp * 4);
+  int hmax = 1;
+  for (size_t i = 1; i < c->head_dims.size(); ++i) hmax = std::max(hmax, c->head_dims[i]);
+  c->h1a = (float*)c->alloc(R * hmax * 4);
+  c->h1b = (float*)c->alloc(R * hmax * 4);
+  c->z = (float*)c->alloc(R * 4);
+  c->len = (float*)c->alloc(R * 4);
+  c->err_dev = (int*)c->alloc(16);
+  if (c->oom) return cleanup_fail(OUTLETS_ENOMEM);
+  for (auto& p : c->ring)
+    if (cudaEventCreateWithFlags(&p.ev, cudaEventDisableTiming) != cudaSuccess) return cleanup_fail(OUTLETS_ECUDA);
+  if (cudaEventCreateWithFlags(&c->done_ev, cudaEventDisableTiming) != cudaSuccess) return cleanup_fail(OUTLETS_ECUDA);
+
+  // ---- upload
+  size_t stage_floats = (size_t)16 << 20;  // 64 MB staging
+  float* stage = nullptr;
+  if (cudaMalloc(&stage, stage_floats * 4) != cudaSuccess) {
+    cudaGetLastError();
+    return cleanup_fail(OUTLETS_ENOMEM);
+  }
+  // keep interleaved uploads chunked on 128-row boundaries
+  const size_t il_floats = std::max<size_t>((stage_floats / d) / 128 * 128, 128) * d;
+  outlets_status st = OUTLETS_OK;
+  auto up = [&](const float* src, int rows, int cols, void* dst, long long ld, int mode, int base) {
+    if (st == OUTLETS_OK)
+      st = upload_rows(c, src, rows, cols, dst, ld, mode, base, stage, mode == 0 ? stage_floats : il_floats);
+  };
+  up(w->w_proj, d, 3 * d, c->w_proj, 3 * d, 0, 0);
+  up(w->w_q, c->H * c->hd, d, c->w_qkv, d, 0, 0);
+  up(w->w_k, c->KVH * c->hd, d, c->w_qkv, d, 0, c->H * c->hd);
+  up(w->w_v, c->KVH * c->hd, d, c->w_qkv, d, 0, (c->H + c->KVH) * c->hd);
+  up(w->w_o, d, c->attn_w, c->w_o, c->attn_w, 0, 0);
+  up(w->w_gate, c->F, d, c->w_gu, d, 1, 0);
+  up(w->w_up, c->F, d, c->w_gu, d, 2, 0);
+  up(w->w_down, d, c->F, c->w_down, c->Fp, 0, 0);
+  up(w->head_w[0], c->head_dims[1], d, c->head_w0, d, 0, 0);
+  cudaFree(stage);
+  if (st != OUTLETS_OK) return cleanup_fail(st);
+  auto h2d = [&](void* dst, const void* src, size_t bytes) {
+    if (st == OUTLETS_OK && cudaMemcpy(dst, src, bytes, cudaMemcpyHostToDevice) != cudaSuccess) st = OUTLETS_ECUDA;
+  };
+  h2d(c->g_in, w->g_in, (size_t)d * 4);
+  h2d(c->g_post, w->g_post, (size_t)d * 4);
+  h2d(c->g_final, w->g_final, (size_t)d * 4);
+  for (int i = 1; i < nl; ++i) h2d(c->head_wf[i], w->head_w[i], (size_t)c->head_dims[i + 1] * c->head_dims[i] * 4);
+  for (int i = 0; i < nl; ++i) h2d(c->head_b[i], w->head_b[i], (size_t)c->head_dims[i + 1] * 4);
+  // RoPE table, angles in fp64: pos * theta^(-2i/hd)
+  {
+    const int half = c->hd / 2;
+    std::vector<float> cs((size_t)cfg->max_position * half), sn((size_t)cfg->max_position * half);
+    for (int i = 0; i < half; ++i) {
+      const double inv = std::pow((double)cfg->rope_theta, -2.0 * i / c->hd);
+      for (int p = 0; p < cfg->max_position; ++p) {
+        const double ang = (double)p * inv;
+        cs[(size_t)p * half + i] = (float)std::cos(ang);
+        sn[(size_t)p * half + i] = (float)std::sin(ang);
+      }
+    }
+    h2d(c->rope_cos, cs.data(), cs.size() * 4);
+    h2d(c->rope_sin, sn.data(), sn.size() * 4);
+  }
+  if (st != OUTLETS_OK) return cleanup_fail(st);
+  if (cudaDeviceSynchronize() != cudaSuccess) {
+    cudaGetLastError();
+    return cleanup_fail(OUTLETS_ECUDA);
+  }
+  *out = c;
+  return OUTLETS_OK;
+}
+
+void outlets_destroy(outlets_ctx* c) {
+  if (!c) return;
+  cudaSetDevice(c->cfg.device);
+  cudaDeviceSynchronize();
+  for (void* p : c->allocs)
+    if (p) cudaFree(p);
+  if (c->meta_dev) cudaFree(c->meta_dev);
+  for (auto& p : c->ring) {
+    if (p.h) cudaFreeHost(p.h);
+    if (p.ev) cudaEventDestroy(p.ev);
+  }
+  if (c->done_ev) cudaEventDestroy(c->done_ev);
+  for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
+  delete c;
+}
+
+outlets_status outlets_profile_enable(outlets_ctx* c, int32_t enable) {
+  if (!c) return OUTLETS_EINVAL;
+  OUT_CK(c, cudaSetDevice(c->cfg.device));
+  OUT_CK(c, cudaDeviceSynchronize());
+  c->prof = enable != 0;
+  c->recs.clear();
+  c->ev_used = 0;
+  return OUTLETS_OK;
+}
+
+outlets_status outlets_profile_read(outlets_ctx* c, double* ms, int32_t* count) {
+  if (!c || !ms) return OUTLETS_EINVAL;
+  OUT_CK(c, cudaSetDevice(c->cfg.device));
+  for (int i = 0; i < OUTLETS_N_STAGES; ++i) {
+    ms[i] = 0.0;
+    if (count) count[i] = 0;
+  }
+  for (const auto& r : c->recs) {
+    OUT_CK(c, cudaEventSynchronize(r.b));
+    float t = 0.f;
+    OUT_CK(c, cudaEventElapsedTime(&t, r.a, r.b));
+    ms[r.stage] += t;
+    if (count) count[r.stage] += 1;
+  }
+  c->recs.clear();
+  c->ev_used = 0;
+  return OUTLETS_OK;
+}
+
+const char* outlets_stage_name(int32_t s) {
+  static const char* names[OUTLETS_N_STAGES] = {"fc_gemm",      "rmsnorm_in",     "qkv_gemm",    "rope_scatter",
+                                                "attention",    "o_gemm",         "rmsnorm_post", "gateup_swiglu_gemm",
+                                                "down_gemm",    "final_rmsnorm",  "length_head"};
+  return (s >= 0 && s < OUTLETS_N_STAGES) ? names[s] : "";
+}
+
+uint64_t outlets_launch_count(const outlets_ctx* c) { return c ? (uint64_t)c->launches : 0; }
+
+const char* outlets_last_error(const outlets_ctx* c) { return c ? c->err.c_str() : "null context"; }
+
+size_t outlets_device_bytes(const outlets_ctx* c) { return c ? c->dev_bytes : 0; }
+
+outlets_status outlets_kv_create(outlets_ctx* c, int32_t max_slots, int32_t max_tokens_total, outlets_kv** out) {
+  if (!out) return OUTLETS_EINVAL;
+  *out = nullptr;
+  if (!c) return OUTLETS_EINVAL;
+  if (max_slots <= 0 || max_tokens_total <= 0) return c->fail(OUTLETS_EINVAL, "max_slots and max_tokens_total must be positive");
+  OUT_CK(c, cudaSetDevice(c->cfg.device));
+  outlets_kv* kv = new outlets_kv();
+  kv->ctx = c;
+  kv->device = c->cfg.device;
+  kv->max_slots = max_slots;
+  kv->num_pages = (int)cdiv(max_tokens_total, kPageTokens) + max_slots;
+  kv->max_pages_per_slot = (int)cdiv(c->cfg.max_position, kPageTokens);
+  const size_t pool = (size_t)kv->num_pages * c->KVH * kPageTokens * c->hd * c->esz;
+  kv->part_items = (size_t)c->cfg.max_batch + kv->num_pages;
+  auto a = [&](size_t bytes) -> void* {
+    void* p = nullptr;
+    if (cudaMalloc(&p, bytes) != cudaSuccess) {
+      cudaGetLastError();
+      return nullptr;
+    }
+    cudaMemset(p, 0, bytes);
+    kv->allocs.push_back(p);
+    return p;
+  };
+  kv->k_pool = a(pool);
+  kv->v_pool = a(pool);
+  kv->part_o = (float*)a(kv->part_items * c->H * c->hd * 4);
+  kv->part_ml = (float*)a(kv->part_items * c->H * 2 * 4);
+  if (!kv->k_pool || !kv->v_pool || !kv->part_o || !kv->part_ml) {
+    outlets_kv_destroy(kv);
+    return c->fail(OUTLETS_ENOMEM, "KV pool allocation failed");
+  }
+  kv->len.assign(max_slots, 0);
+  kv->pages.assign(max_slots, {});
+  kv->free_list.reserve(kv->num_pages);
+  for (int p = kv->num_pages - 1; p >= 0; --p) kv->free_list.push_back(p);
+  *out = kv;
+  return OUTLETS_OK;
+}
+
+void outlets_kv_destroy(outlets_kv* kv) {
+  if (!kv) return;
+  cudaSetDevice(kv->device);
+  cudaDeviceSynchronize();
+  for (void* p : kv->allocs) cudaFree(p);
+  delete kv;
+}
+
+outlets_status outlets_kv_reset_slot(outlets_kv* kv, int32_t slot) {
+  if (!kv || slot < 0 || slot >= kv->max_slots) return OUTLETS_EINVAL;
+  for (int p : kv->pages[slot]) kv->free_list.push_back(p);
+  kv->pages[slot].clear();
+  kv->len[slot] = 0;
+  return OUTLETS_OK;
+}
+
+int32_t outlets_kv_slot_length(const outlets_kv* kv, int32_t slot) {
+  if (!kv || slot < 0 || slot >= kv->max_slots) return -1;
+  return kv->len[slot];
+}
+
+int32_t outlets_kv_free_pages(const outlets_kv* kv) { return kv ? (int32_t)kv->free_list.size() : -1; }
+
+outlets_status outlets_check(outlets_ctx* c, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  OUT_CK(c, cudaSetDevice(c->cfg.device));
+  OUT_CK(c, cudaStreamSynchronize((cudaStream_t)stream));
+  int e = 0;
+  OUT_CK(c, cudaMemcpy(&e, c->err_dev, sizeof(int), cudaMemcpyDeviceToHost));
+  if (e) {
+    OUT_CK(c, cudaMemset(c->err_dev, 0, sizeof(int)));
+    if (e & ERR_TIMEOUT) return c->fail(OUTLETS_ETIMEOUT, "a kernel's bounded wait ran out");
+    return c->fail(OUTLETS_EDEVICE, "a kernel refused an out-of-range index");
+  }
+  return OUTLETS_OK;
+}
+
+outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3], const int32_t* cu, int32_t B,
+                                       int32_t T, outlets_kv* kv, const int32_t* slots, uint32_t flags,
+                                       float* z_out, float* len_out, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  cudaStream_t s = (cudaStream_t)stream;
+  if (!taps || !cu || !z_out) return c->fail(OUTLETS_EINVAL, "taps, cu_seqlens and z_out must not be NULL");
+  if (flags & ~OUTLETS_ALL_TOKENS) return c->fail(OUTLETS_EINVAL, "unknown flag");
+  if (B < 0 || T < 0) return c->fail(OUTLETS_EINVAL, "B and T must be >= 0");
+  if ((kv == nullptr) != (slots == nullptr)) return c->fail(OUTLETS_EINVAL, "kv and slots go together");
+  if (kv && kv->ctx != c) return c->fail(OUTLETS_EINVAL, "kv belongs to another context");
+  if (B == 0) {
+    if (T != 0) return c->fail(OUTLETS_EINVAL, "T must be 0 when B is 0");
+    return OUTLETS_OK;
+  }
+  if (cu[0] != 0) return c->fail(OUTLETS_EINVAL, "cu_seqlens[0] must be 0");
+  int max_len = 0;
+  for (int b = 0; b < B; ++b) {
+    if (cu[b + 1] <= cu[b]) return c->fail(OUTLETS_EINVAL, "cu_seqlens must be strictly increasing (every sequence non-empty)");
+    max_len = std::max(max_len, cu[b + 1] - cu[b]);
+  }
+  if (cu[B] != T) return c->fail(OUTLETS_EINVAL, "cu_seqlens[B] must equal T");
+  if (T > c->cfg.max_tokens) return c->fail(OUTLETS_ECAPACITY, "T exceeds max_tokens");
+  if (B > c->cfg.max_batch) return c->fail(OUTLETS_ECAPACITY, "B exceeds max_batch");
+  if (max_len > c->cfg.max_position) return c->fail(OUTLETS_ECAPACITY, "a sequence is longer than max_position");
+  if (kv) {
+    std::vector<char> seen(kv->max_slots, 0);
+    long long need = 0, freed = 0;
+    for (int b = 0; b < B; ++b) {
+      const int sl = slots[b];
+      if (sl < 0 || sl >= kv->max_slots) return c->fail(OUTLETS_EINVAL, "slot out of range");
+      if (seen[sl]) return c->fail(OUTLETS_EINVAL, "slots must be distinct");
+      seen[sl] = 1;
+      need += cdiv(cu[b + 1] - cu[b], kPageTokens);
+      freed += (long long)kv->pages[sl].size();
+    }
+    if (need > (long long)kv->free_list.size() + freed) return c->fail(OUTLETS_ECAPACITY, "not enough free KV pages");
+  }
+  const bool all_tokens = flags & OUTLETS_ALL_TOKENS;
+  const int out_rows = all_tokens ? T : B;
+
+  OUT_TRY(begin_call(c, s));
+  const void* tp[3];
+  OUT_TRY(prepare_taps(c, taps, T, tp, s));
+
+  // ---- host metadata
+  MetaBuilder mb;
+  const size_t off_cu = mb.put(cu, B + 1);
+  std::vector<int> last(B);
+  for (int b = 0; b < B; ++b) last[b] = cu[b + 1] - 1;
+  const size_t off_last = mb.put(last);
+  size_t off_tiles = 0;
+  int n_tiles = 0;
+  if (c->bf16) {
+    std::vector<int> tiles;
+    std::vector<std::pair<int, int>> order;  // (key tiles, tile id): longest first
+    for (int b = 0; b < B; ++b) {
+      const int L = cu[b + 1] - cu[b];
+      for (int i = 0; i * 64 < L; ++i) {
+        order.push_back({i + 1, (int)(tiles.size() / 4)});
+        tiles.push_back(cu[b] + 64 * i);
+        tiles.push_back(std::min(64, L - 64 * i));
+        tiles.push_back(cu[b]);
+        tiles.push_back(L);
+      }
+    }
+    std::stable_sort(order.begin(), order.end(), [](const auto& x, const auto& y) { return x.first > y.first; });
+    std::vector<int> sorted;
+    sorted.reserve(tiles.size());
+    for (auto& o : order) sorted.insert(sorted.end(), tiles.begin() + 4 * o.second, tiles.begin() + 4 * o.second + 4);
+    n_tiles = (int)order.size();
+    off_tiles = mb.put(sorted);
+  }
+  size_t off_pl = 0, off_po = 0;
+  if (kv) {
+    // commit the cache change: reset every slot of the batch, then allocate its pages
+    for (int b = 0; b < B; ++b) outlets_kv_reset_slot(kv, slots[b]);
+    std::vector<int> pl, po(B + 1, 0);
+    for (int b = 0; b < B; ++b) {
+      const int L = cu[b + 1] - cu[b];
+      const int np = (int)cdiv(L, kPageTokens);
+      for (int i = 0; i < np; ++i) {
+        const int p = kv->free_list.back();
+        kv->free_list.pop_back();
+        kv->pages[slots[b]].push_back(p);
+        pl.push_back(p);
+      }
+      kv->len[slots[b]] = L;
+      po[b + 1] = (int)pl.size();
+    }
+    off_pl = mb.put(pl);
+    off_po = mb.put(po);
+  }
+  OUT_TRY(upload_meta(c, mb.v, s));
+  const int* m = c->meta_dev;
+  const int* cu_dev = m + off_cu;
+
+  const int d = c->d;
+  // ---- FC (Eq. 1): f = [tap0 | tap1 | tap2] W_proj^T
+  c->stage_begin(OUTLETS_S_FC);
+  if (c->bf16) OUT_TRY(gemm_tc(c, tp, 3, d, d, T, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
+  else OUT_TRY(gemm_f32(c, tp, d, T, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
+  c->stage_end(1);
+  // ---- input RMSNorm
+  c->stage_begin(OUTLETS_S_NORM_IN);
+  if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xhat, nullptr, T, d, c->cfg.rms_eps, s));
+  else OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, T, d, c->cfg.rms_eps, s));
+  c->stage_end(1);
+  // ---- QKV
+  c->stage_begin(OUTLETS_S_QKV);
+  {
+    const void* a1[3] = {c->xhat, c->xhat, c->xhat};
+    if (c->bf16) OUT_TRY(gemm_tc(c, a1, 1, d, d, T, c->w_qkv, c->qkv_n, d, EPI_ACT, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
+    else OUT_TRY(gemm_f32(c, a1, d, T, c->w_qkv, c->qkv_n, d, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
+  }
+  c->stage_end(1);
+  // ---- RoPE, q, head-major k/v, cache
+  c->stage_begin(OUTLETS_S_ROPE);
+  {
+    RopeArgs ra{};
+    ra.T = T;
+    ra.H = c->H;
+    ra.KVH = c->KVH;
+    ra.hd = c->hd;
+    ra.cu = cu_dev;
+    ra.B = B;
+    ra.cos_tab = c->rope_cos;
+    ra.sin_tab = c->rope_sin;
+    ra.max_pos = c->cfg.max_position;
+    ra.q_out = c->q;
+    ra.k_out = c->kh;
+    ra.v_out = c->vh;
+    ra.kv_ld_rows = c->cfg.max_tokens;
+    if (kv) {
+      ra.k_pool = kv->k_pool;
+      ra.v_pool = kv->v_pool;
+      ra.page_list = m + off_pl;
+      ra.page_off = m + off_po;
+      ra.page_tokens = kPageTokens;
+    }
+    ra.err = c->err_dev;
+    if (c->bf16) OUT_CK(c, rope_scatter_launch<bf16, bf16>((const bf16*)c->qkv, ra, s));
+    else OUT_CK(c, rope_scatter_launch<float, float>((const float*)c->qkv, ra, s));
+  }
+  c->stage_end(1);
+  // ---- attention
+  c->stage_begin(OUTLETS_S_ATTN);
+  if (c->bf16) {
+    CUtensorMap qm, km, vm;
+    const uint64_t kv_rows = (uint64_t)c->KVH * c->cfg.max_tokens;
+    if (!make_map(&qm, c->q, c->attn_w, T, c->attn_w, 64) || !make_map(&km, c->kh, c->hd, kv_rows, c->hd, 64) ||
+        !make_map(&vm, c->vh, c->hd, kv_rows, c->hd, 64))
+      return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for attention");
+    OUT_CK(c, attn_prefill_bf16_launch(qm, km, vm, reinterpret_cast<const AttnTile*>(m + off_tiles), n_tiles,
+                                       c->cfg.max_tokens, c->H, c->KVH, c->hd, c->attn, c->err_dev, s));
+  } else {
+    OUT_CK(c, attn_prefill_simt_launch<float>((const float*)c->q, (const float*)c->kh, (const float*)c->vh, cu_dev,
+                                              B, T, c->cfg.max_tokens, c->H, c->KVH, c->hd, (float*)c->attn, s));
+  }
+  c->stage_end(1);
+  OUT_TRY(run_tail(c, T, out_rows, all_tokens ? nullptr : m + off_last, c->z, c->len, s));
+  c->last_rows = T;
+  c->last_out_rows = out_rows;
+  return end_call(c, out_rows, z_out, len_out, s);
+}
+
+outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], int32_t B, outlets_kv* kv,
+                                    const int32_t* slots, float* z_out, float* len_out, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  cudaStream_t s = (cudaStream_t)stream;
+  if (!taps || !kv || !slots || !z_out) return c->fail(OUTLETS_EINVAL, "taps, kv, slots and z_out must not be NULL");
+  if (kv->ctx != c) return c->fail(OUTLETS_EINVAL, "kv belongs to another context");
+  if (B < 0) return c->fail(OUTLETS_EINVAL, "B must be >= 0");
+  if (B == 0) return OUTLETS_OK;
+  if (B > c->cfg.max_batch) return c->fail(OUTLETS_ECAPACITY, "B exceeds max_batch");
+  std::vector<char> seen(kv->max_slots, 0);
+  int need = 0;
+  for (int b = 0; b < B; ++b) {
+    const int sl = slots[b];
+    if (sl < 0 || sl >= kv->max_slots) return c->fail(OUTLETS_EINVAL, "slot out of range");
+    if (seen[sl]) return c->fail(OUTLETS_EINVAL, "slots must be distinct");
+    seen[sl] = 1;
+    if (kv->len[sl] >= c->cfg.max_position) return c->fail(OUTLETS_ECAPACITY, "slot reached max_position");
+    if (kv->len[sl] % kPageTokens == 0) ++need;
+  }
+  if (need > (int)kv->free_list.size()) return c->fail(OUTLETS_ECAPACITY, "not enough free KV pages");
+
+  OUT_TRY(begin_call(c, s));
+  const void* tp[3];
+  OUT_TRY(prepare_taps(c, taps, B, tp, s));
+
+  // ---- commit the append and build metadata
+  std::vector<int> pos(B), seq_len(B), po(B + 1, 0), pl, work, work_off(B + 1, 0);
+  for (int b = 0; b < B; ++b) {
+    const int sl = slots[b];
+    if (kv->len[sl] % kPageTokens == 0) {
+      kv->pages[sl].push_back(kv->free_list.back());
+      kv->free_list.pop_back();
+    }
+    pos[b] = kv->len[sl];
+    kv->len[sl] += 1;
+    seq_len[b] = kv->len[sl];
+    pl.insert(pl.end(), kv->pages[sl].begin(), kv->pages[sl].end());
+    po[b + 1] = (int)pl.size();
+    const int ns = (int)cdiv(seq_len[b], kSplitLen);
+    for (int sp = 0; sp < ns; ++sp) {
+      work.push_back(b);
+      work.push_back(sp);
+    }
+    work_off[b + 1] = (int)(work.size() / 2);
+  }
+  const int n_work = work_off[B];
+  MetaBuilder mb;
+  const size_t off_pos = mb.put(pos);
+  const size_t off_sl = mb.put(seq_len);
+  const size_t off_po = mb.put(po);
+  const size_t off_pl = mb.put(pl);
+  const size_t off_w = mb.put(work);
+  const size_t off_wo = mb.put(work_off);
+  OUT_TRY(upload_meta(c, mb.v, s));
+  const int* m = c->meta_dev;
+  const int d = c->d;
+
+  c->stage_begin(OUTLETS_S_FC);
+  if (c->bf16) OUT_TRY(gemm_tc(c, tp, 3, d, d, B, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
+  else OUT_TRY(gemm_f32(c, tp, d, B, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
+  c->stage_end(1);
+  c->stage_begin(OUTLETS_S_NORM_IN);
+  if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xhat, nullptr, B, d, c->cfg.rms_eps, s));
+  else OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, B, d, c->cfg.rms_eps, s));
+  c->stage_end(1);
+  c->stage_begin(OUTLETS_S_QKV);
+  {
+    const void* a1[3] = {c->xhat, c->xhat, c->xhat};
+    if (c->bf16) OUT_TRY(gemm_tc(c, a1, 1, d, d, B, c->w_qkv, c->qkv_n, d, EPI_ACT, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
+    else OUT_TRY(gemm_f32(c, a1, d, B, c->w_qkv, c->qkv_n, d, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
+  }
+  c->stage_end(1);
+  c->stage_begin(OUTLETS_S_ROPE);
+  {
+    RopeArgs ra{};
+    ra.T = B;
+    ra.H = c->H;
+    ra.KVH = c->KVH;
+    ra.hd = c->hd;
+    ra.B = B;
+    ra.pos = m + off_pos;
+    ra.cos_tab = c->rope_cos;
+    ra.sin_tab = c->rope_sin;
+    ra.max_pos = c->cfg.max_position;
+    ra.q_out = c->q;
+    ra.k_pool = kv->k_pool;
+    ra.v_pool = kv->v_pool;
+    ra.page_list = m + off_pl;
+    ra.page_off = m + off_po;
+    ra.page_tokens = kPageTokens;
+    ra.err = c->err_dev;
+    if (c->bf16) OUT_CK(c, rope_scatter_launch<bf16, bf16>((const bf16*)c->qkv, ra, s));
+    else OUT_CK(c, rope_scatter_launch<float, float>((const float*)c->qkv, ra, s));
+  }
+  c->stage_end(1);
+  c->stage_begin(OUTLETS_S_ATTN);
+  {
+    DecodeArgs da{};
+    da.B = B;
+    da.H = c->H;
+    da.KVH = c->KVH;
+    da.hd = c->hd;
+    da.q = c->q;
+    da.k_pool = kv->k_pool;
+    da.v_pool = kv->v_pool;
+    da.page_tokens = kPageTokens;
+    da.page_list = m + off_pl;
+    da.page_off = m + off_po;
+    da.seq_len = m + off_sl;
+    da.work = m + off_w;
+    da.work_off = m + off_wo;
+    da.n_work = n_work;
+    da.split_len = kSplitLen;
+    da.part_o = kv->part_o;
+    da.part_ml = kv->part_ml;
+    da.out = c->attn;
+    da.err = c->err_dev;
+    if ((size_t)n_work > kv->part_items) return c->fail(OUTLETS_ECAPACITY, "split-KV partial buffer too small");
+    if (c->bf16) {
+      CUtensorMap km, vm;
+      const uint64_t rows = (uint64_t)kv->num_pages * c->KVH * kPageTokens;
+      if (!make_map(&km, kv->k_pool, c->hd, rows, c->hd, 64) || !make_map(&vm, kv->v_pool, c->hd, rows, c->hd, 64))
+        return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for the KV pools");
+      OUT_CK(c, attn_decode_bf16_launch(km, vm, da, s));
+      c->stage_end(2);
+    } else {
+      OUT_CK(c, attn_decode_simt_launch<float>(da, s));
+      c->stage_end(1);
+    }
+  }
+  OUT_TRY(run_tail(c, B, B, nullptr, c->z, c->len, s));
+  c->last_rows = B;
+  c->last_out_rows = B;
+  return end_call(c, B, z_out, len_out, s);
+}
+
+outlets_status outlets_get_intermediate(outlets_ctx* c, int32_t which, void* dst, size_t dst_bytes,
+                                        outlets_tensor_info* info, void* stream) {
+  if (!c || !info) return OUTLETS_EINVAL;
+  const int act = c->bf16 ? OUTLETS_BF16 : OUTLETS_F32;
+  const void* src = nullptr;
+  outlets_tensor_info ti{};
+  switch (which) {
+    case OUTLETS_T_FCTX: ti = {OUTLETS_F32, c->last_rows, c->d}; src = c->f; break;
+    case OUTLETS_T_XIN: ti = {act, c->last_rows, c->d}; src = c->xhat; break;
+    case OUTLETS_T_Q: ti = {act, c->last_rows, c->attn_w}; src = c->q; break;
+    case OUTLETS_T_ATTN: ti = {act, c->last_rows, c->attn_w}; src = c->attn; break;
+    case OUTLETS_T_A: ti = {OUTLETS_F32, c->last_rows, c->d}; src = c->a; break;
+    case OUTLETS_T_Y: ti = {OUTLETS_F32, c->last_rows, c->d}; src = c->y; break;
+    case OUTLETS_T_HDRAFT: ti = {act, c->last_out_rows, c->d}; src = c->hn; break;
+    default: return c->fail(OUTLETS_EINVAL, "unknown intermediate");
+  }
+  *info = ti;
+  if (!dst) return OUTLETS_OK;
+  const size_t bytes = (size_t)ti.rows * ti.cols * (ti.dtype == OUTLETS_BF16 ? 2 : 4);
+  if (dst_bytes < bytes) return c->fail(OUTLETS_EINVAL, "dst too small");
+  OUT_CK(c, cudaSetDevice(c->cfg.device));
+  OUT_CK(c, cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, (cudaStream_t)stream));
+  return OUTLETS_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,281 @@
+"""Thin ctypes binding of the OUTLETS C ABI (include/outlets.h).
+
+Argument marshalling only: every step of the forward runs in the CUDA library.
+PyTorch supplies device memory and streams.  If the library is missing the
+binding raises; there is no other code path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "liboutlets_gb300.so")
+MAX_HEAD_HIDDEN = 7
+
+OK, EINVAL, ENOMEM, ECUDA, EUNSUPPORTED, ECAPACITY, ETIMEOUT, EDEVICE = range(8)
+STATUS_NAMES = ["OK", "EINVAL", "ENOMEM", "ECUDA", "EUNSUPPORTED", "ECAPACITY", "ETIMEOUT", "EDEVICE"]
+F32, BF16 = 0, 1
+ALL_TOKENS = 1
+T_FCTX, T_XIN, T_Q, T_ATTN, T_A, T_Y, T_HDRAFT = range(7)
+N_STAGES = 11
+
+c_i32, c_f32, c_vp = ctypes.c_int32, ctypes.c_float, ctypes.c_void_p
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("d_model", c_i32), ("n_heads", c_i32), ("n_kv_heads", c_i32), ("head_dim", c_i32),
+                ("ffn_dim", c_i32), ("n_head_hidden", c_i32), ("head_hidden", c_i32 * MAX_HEAD_HIDDEN),
+                ("rope_theta", c_f32), ("rms_eps", c_f32), ("dtype", c_i32), ("max_tokens", c_i32),
+                ("max_batch", c_i32), ("max_position", c_i32), ("device", c_i32)]
+
+
+_WNAMES = ["w_proj", "w_q", "w_k", "w_v", "w_o", "g_in", "g_post", "g_final", "w_gate", "w_up", "w_down"]
+
+
+class Weights(ctypes.Structure):
+    _fields_ = [(n, c_vp) for n in _WNAMES] + [("head_w", c_vp * (MAX_HEAD_HIDDEN + 1)),
+                                               ("head_b", c_vp * (MAX_HEAD_HIDDEN + 1))]
+
+
+class TensorInfo(ctypes.Structure):
+    _fields_ = [("dtype", c_i32), ("rows", c_i32), ("cols", c_i32)]
+
+
+class OutletsError(RuntimeError):
+    def __init__(self, status, msg):
+        self.status = status
+        super().__init__(f"{STATUS_NAMES[status] if 0 <= status < 8 else status}: {msg}")
+
+
+_lib = None
+
+
+def load():
+    """Load the CUDA library (built by ``paper_2609_01068_gb300.build``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: run `python -m paper_2609_01068_gb300.build` first")
+    lib = ctypes.CDLL(LIB_PATH)
+    P = ctypes.POINTER
+    sig = {
+        "outlets_create": (c_i32, [P(Config), P(Weights), P(c_vp)]),
+        "outlets_destroy": (None, [c_vp]),
+        "outlets_last_error": (ctypes.c_char_p, [c_vp]),
+        "outlets_device_bytes": (ctypes.c_size_t, [c_vp]),
+        "outlets_kv_create": (c_i32, [c_vp, c_i32, c_i32, P(c_vp)]),
+        "outlets_kv_destroy": (None, [c_vp]),
+        "outlets_kv_reset_slot": (c_i32, [c_vp, c_i32]),
+        "outlets_kv_slot_length": (c_i32, [c_vp, c_i32]),
+        "outlets_kv_free_pages": (c_i32, [c_vp]),
+        "outlets_predict_prefill": (c_i32, [c_vp, P(c_vp), c_vp, c_i32, c_i32, c_vp, c_vp, ctypes.c_uint32,
+                                            c_vp, c_vp, c_vp]),
+        "outlets_predict_step": (c_i32, [c_vp, P(c_vp), c_i32, c_vp, c_vp, c_vp, c_vp, c_vp]),
+        "outlets_check": (c_i32, [c_vp, c_vp]),
+        "outlets_get_intermediate": (c_i32, [c_vp, c_i32, c_vp, ctypes.c_size_t, P(TensorInfo), c_vp]),
+        "outlets_profile_enable": (c_i32, [c_vp, c_i32]),
+        "outlets_profile_read": (c_i32, [c_vp, P(ctypes.c_double), P(c_i32)]),
+        "outlets_stage_name": (ctypes.c_char_p, [c_i32]),
+        "outlets_launch_count": (ctypes.c_uint64, [c_vp]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _ptr(x):
+    """Address of a torch tensor or a numpy array (None -> NULL)."""
+    if x is None:
+        return None
+    if isinstance(x, np.ndarray):
+        if not x.flags["C_CONTIGUOUS"]:
+            raise ValueError("arrays must be C-contiguous")
+        return x.ctypes.data
+    if not x.is_contiguous():
+        raise ValueError("tensors must be contiguous")
+    return x.data_ptr()
+
+
+def _stream_handle(stream):
+    import torch
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream if torch.cuda.is_available() else 0
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+class Predictor:
+    """One OUTLETS draft backbone + length head resident on a GPU."""
+
+    def __init__(self, shape, weights: dict, max_tokens: int, max_batch: int, max_position: int = 16384,
+                 device: int = 0):
+        self.lib = load()
+        self.shape = shape
+        cfg = Config()
+        cfg.d_model, cfg.n_heads, cfg.n_kv_heads = shape.d, shape.n_heads, shape.n_kv_heads
+        cfg.head_dim, cfg.ffn_dim = shape.head_dim, shape.ffn
+        cfg.n_head_hidden = len(shape.head_widths)
+        for i, wdt in enumerate(shape.head_widths):
+            cfg.head_hidden[i] = wdt
+        cfg.rope_theta, cfg.rms_eps = shape.rope_theta, shape.rms_eps
+        cfg.dtype = BF16 if shape.dtype == "bf16" else F32
+        cfg.max_tokens, cfg.max_batch, cfg.max_position, cfg.device = max_tokens, max_batch, max_position, device
+        self.cfg = cfg
+        self.device = device
+        keep = {}
+        w = Weights()
+        for n in _WNAMES:
+            a = np.ascontiguousarray(weights[n], dtype=np.float32)
+            keep[n] = a
+            setattr(w, n, a.ctypes.data)
+        for i in range(len(shape.head_widths) + 1):
+            wa = np.ascontiguousarray(weights[f"head_w{i}"], dtype=np.float32)
+            ba = np.ascontiguousarray(weights[f"head_b{i}"], dtype=np.float32)
+            keep[f"hw{i}"], keep[f"hb{i}"] = wa, ba
+            w.head_w[i] = wa.ctypes.data
+            w.head_b[i] = ba.ctypes.data
+        h = c_vp()
+        st = self.lib.outlets_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h))
+        if st != OK:
+            raise OutletsError(st, "outlets_create failed")
+        self.h = h
+
+    # -- helpers
+    def _raise(self, st):
+        msg = self.lib.outlets_last_error(self.h)
+        raise OutletsError(st, msg.decode() if msg else "")
+
+    def close(self):
+        if getattr(self, "h", None):
+            self.lib.outlets_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @property
+    def device_bytes(self):
+        return self.lib.outlets_device_bytes(self.h)
+
+    def _outputs(self, n, like, z_out, len_out):
+        import torch
+        if z_out is None:
+            dev = like.device if hasattr(like, "device") else torch.device("cpu")
+            z_out = torch.empty(n, dtype=torch.float32, device=dev)
+            len_out = torch.empty(n, dtype=torch.float32, device=dev)
+        return z_out, len_out
+
+    # -- prediction
+    def prefill(self, taps, cu_seqlens, kv=None, slots=None, all_tokens=False, z_out=None, len_out=None,
+                stream=None):
+        """Static prediction (z_hat, length_hat) for a packed varlen batch."""
+        cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+        B, T = len(cu) - 1, int(cu[-1]) if len(cu) else 0
+        n_out = T if all_tokens else B
+        z_out, len_out = self._outputs(n_out, taps[0], z_out, len_out)
+        tp = (c_vp * 3)(*[_ptr(t) for t in taps])
+        sl = None if slots is None else np.ascontiguousarray(slots, dtype=np.int32)
+        st = self.lib.outlets_predict_prefill(self.h, tp, cu.ctypes.data, B, T, kv.h if kv else None,
+                                              None if sl is None else sl.ctypes.data,
+                                              ALL_TOKENS if all_tokens else 0, _ptr(z_out), _ptr(len_out),
+                                              _stream_handle(stream))
+        if st != OK:
+            self._raise(st)
+        return z_out, len_out
+
+    def step(self, taps, kv, slots, z_out=None, len_out=None, stream=None):
+        """Dynamic prediction for one new token per request."""
+        sl = np.ascontiguousarray(slots, dtype=np.int32)
+        B = len(sl)
+        z_out, len_out = self._outputs(B, taps[0], z_out, len_out)
+        tp = (c_vp * 3)(*[_ptr(t) for t in taps])
+        st = self.lib.outlets_predict_step(self.h, tp, B, kv.h, sl.ctypes.data, _ptr(z_out), _ptr(len_out),
+                                           _stream_handle(stream))
+        if st != OK:
+            self._raise(st)
+        return z_out, len_out
+
+    def check(self, stream=None):
+        st = self.lib.outlets_check(self.h, _stream_handle(stream))
+        if st != OK:
+            self._raise(st)
+
+    def profile(self, enable: bool):
+        st = self.lib.outlets_profile_enable(self.h, 1 if enable else 0)
+        if st != OK:
+            self._raise(st)
+
+    def profile_read(self):
+        """{stage name: (total ms, runs)} of the calls since profiling was enabled / last read."""
+        ms = (ctypes.c_double * N_STAGES)()
+        cnt = (c_i32 * N_STAGES)()
+        st = self.lib.outlets_profile_read(self.h, ms, cnt)
+        if st != OK:
+            self._raise(st)
+        return {self.lib.outlets_stage_name(i).decode(): (ms[i], cnt[i]) for i in range(N_STAGES)}
+
+    @property
+    def launch_count(self):
+        return int(self.lib.outlets_launch_count(self.h))
+
+    def intermediate(self, which, stream=None):
+        """Copy of an intermediate of the last call as a CUDA tensor (f32 or bf16)."""
+        import torch
+        info = TensorInfo()
+        st = self.lib.outlets_get_intermediate(self.h, which, None, 0, ctypes.byref(info), None)
+        if st != OK:
+            self._raise(st)
+        dt = torch.bfloat16 if info.dtype == BF16 else torch.float32
+        out = torch.empty((info.rows, info.cols), dtype=dt, device=f"cuda:{self.device}")
+        st = self.lib.outlets_get_intermediate(self.h, which, out.data_ptr(), out.numel() * out.element_size(),
+                                               ctypes.byref(info), _stream_handle(stream))
+        if st != OK:
+            self._raise(st)
+        return out
+
+
+class KVCache:
+    """Paged draft KV cache bound to one Predictor."""
+
+    def __init__(self, pred: Predictor, max_slots: int, max_tokens_total: int):
+        self.pred = pred
+        self.lib = pred.lib
+        h = c_vp()
+        st = self.lib.outlets_kv_create(pred.h, max_slots, max_tokens_total, ctypes.byref(h))
+        if st != OK:
+            pred._raise(st)
+        self.h = h
+
+    def reset_slot(self, slot):
+        st = self.lib.outlets_kv_reset_slot(self.h, slot)
+        if st != OK:
+            raise OutletsError(st, "bad slot")
+
+    def slot_length(self, slot):
+        return self.lib.outlets_kv_slot_length(self.h, slot)
+
+    @property
+    def free_pages(self):
+        return self.lib.outlets_kv_free_pages(self.h)
+
+    def close(self):
+        if getattr(self, "h", None):
+            self.lib.outlets_kv_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

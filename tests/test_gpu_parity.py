@@ -1,0 +1,272 @@
+"""CUDA path vs the CPU oracle, element by element, through the C ABI.
+
+Small cases span several tiles and ragged tails (every intermediate checked);
+the full-size configurations check sampled outputs the oracle computes one
+sequence / request at a time (sequences never interact, Sec. 3.2).
+"""
+import numpy as np
+import pytest
+
+from oracle import outlets_oracle as OR
+from paper_2609_01068_gb300 import synth
+from _util import HIDDEN_TOL, check_hidden, check_z_len, maxrel, to_device, to_np
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+MID128 = synth.ModelShape("mid-bf16-hd128", 1024, 8, 2, 128, 2816, (256,), 500000.0, 1e-5, "bf16")
+MID64 = synth.ModelShape("mid-bf16-hd64", 512, 8, 4, 64, 1000, (128, 64), 10000.0, 1e-5, "bf16")
+SHAPES = {"tiny-f32": synth.TINY, "mid128": MID128, "mid64": MID64}
+PREFILL_LENGTHS = {
+    "tiny-f32": [16, 32, 48, 64],
+    "mid128": [1, 5, 63, 64, 65, 130, 200, 333],
+    "mid64": [2, 64, 129, 71, 1],
+}
+STEP_PREFIX = {
+    "tiny-f32": [1, 15, 63, 64, 65],
+    "mid128": [1, 63, 64, 65, 511, 512, 513, 700],
+    "mid64": [3, 64, 600, 1100],
+}
+
+_cache = {}
+
+
+def predictor(name, max_tokens=4096, max_batch=64):
+    from paper_2609_01068_gb300 import outlets
+    key = (name, max_tokens, max_batch)
+    if key not in _cache:
+        shape = SHAPES[name]
+        w = synth.make_weights(shape, 0)
+        _cache[key] = (outlets.Predictor(shape, w, max_tokens=max_tokens, max_batch=max_batch, max_position=8192), w)
+    return _cache[key]
+
+
+def _taps(shape, T, off=0):
+    return synth.make_taps(shape, T, 0, off)
+
+
+@pytest.mark.parametrize("name", list(SHAPES))
+def test_prefill_matches_oracle_every_intermediate(name):
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = SHAPES[name]
+    pred, w = predictor(name)
+    cu = synth.cu_seqlens(PREFILL_LENGTHS[name])
+    taps = _taps(shape, int(cu[-1]))
+    ref = OR.predict_prefill(w, shape, taps, cu)
+    z, ln = pred.prefill([to_device(t, shape.dtype) for t in taps], cu)
+    torch.cuda.synchronize()
+    pred.check()
+    T = int(cu[-1])
+    pairs = [(OT.T_FCTX, ref["f"], "f_ctx"), (OT.T_XIN, ref["x"], "x_in"),
+             (OT.T_Q, ref["q"].reshape(T, -1), "q"), (OT.T_ATTN, ref["attn"], "attn"),
+             (OT.T_A, ref["a"], "a"), (OT.T_Y, ref["y"], "y"), (OT.T_HDRAFT, ref["h_draft"], "h_draft")]
+    for which, r, what in pairs:
+        check_hidden(pred.intermediate(which), r, shape.dtype, f"{name} {what}")
+    check_z_len(z, ln, ref["z"], ref["length"], shape.dtype, name)
+
+
+@pytest.mark.parametrize("name", ["tiny-f32", "mid128"])
+def test_all_tokens_mode_and_causal_prefix(name):
+    shape = SHAPES[name]
+    pred, w = predictor(name)
+    cu = synth.cu_seqlens(PREFILL_LENGTHS[name][-3:])
+    taps = _taps(shape, int(cu[-1]), off=1)
+    ref = OR.predict_prefill(w, shape, taps, cu, all_tokens=True)
+    z, ln = pred.prefill([to_device(t, shape.dtype) for t in taps], cu, all_tokens=True)
+    check_z_len(z, ln, ref["z"], ref["length"], shape.dtype, name)
+    # the per-token prediction at row k equals the prediction of the prompt cut after k
+    zall = to_np(z)
+    for b in range(len(cu) - 1):
+        k = int(cu[b]) + (int(cu[b + 1]) - int(cu[b])) // 2
+        sub = [t[int(cu[b]):k + 1] for t in taps]
+        zk, _ = pred.prefill([to_device(t, shape.dtype) for t in sub], np.array([0, len(sub[0])], np.int32))
+        assert abs(to_np(zk)[0] - zall[k]) <= (1e-5 if shape.dtype == "f32" else 2e-3)
+
+
+@pytest.mark.parametrize("name", list(SHAPES))
+def test_steps_match_oracle(name):
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = SHAPES[name]
+    pred, w = predictor(name)
+    pref = STEP_PREFIX[name]
+    n_steps = 3
+    B = len(pref)
+    kv = OT.KVCache(pred, max_slots=B + 3, max_tokens_total=sum(pref) + B * (n_steps + 64))
+    slots = np.arange(3, 3 + B, dtype=np.int32)[::-1].copy()
+    cu = synth.cu_seqlens(pref)
+    taps = _taps(shape, int(cu[-1]), off=2)
+    free0 = kv.free_pages
+    pred.prefill([to_device(t, shape.dtype) for t in taps], cu, kv=kv, slots=slots)
+    assert [kv.slot_length(int(s)) for s in slots] == pref
+    assert kv.free_pages == free0 - sum((L + 63) // 64 for L in pref)
+    ref_pre = OR.predict_prefill(w, shape, taps, cu)
+    caches = OR.caches_from_prefill(ref_pre, cu)
+    for step in range(n_steps):
+        st_taps = _taps(shape, B, off=10 + step)
+        z, ln = pred.step([to_device(t, shape.dtype) for t in st_taps], kv, slots)
+        torch.cuda.synchronize()
+        pred.check()
+        ref = OR.predict_step(w, shape, st_taps, caches)
+        caches = ref["caches"]
+        check_hidden(pred.intermediate(OT.T_ATTN), ref["attn"], shape.dtype, f"{name} step {step} attn")
+        check_hidden(pred.intermediate(OT.T_HDRAFT), ref["h_draft"], shape.dtype, f"{name} step {step} h_draft")
+        check_z_len(z, ln, ref["z"], ref["length"], shape.dtype, f"{name} step {step}")
+    assert [kv.slot_length(int(s)) for s in slots] == [L + n_steps for L in pref]
+    kv.close()
+
+
+@pytest.mark.parametrize("name", ["tiny-f32", "mid128"])
+def test_prefill_then_steps_equals_all_tokens_on_gpu(name):
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = SHAPES[name]
+    pred, w = predictor(name)
+    lengths = [70, 9, 130]
+    cu = synth.cu_seqlens(lengths)
+    taps = _taps(shape, int(cu[-1]), off=3)
+    z_all, _ = pred.prefill([to_device(t, shape.dtype) for t in taps], cu, all_tokens=True)
+    z_all = to_np(z_all)
+    kpre = [64, 1, 126]
+    kv = OT.KVCache(pred, max_slots=3, max_tokens_total=1024)
+    pre = [np.concatenate([t[cu[b]:cu[b] + kpre[b]] for b in range(3)]) for t in taps]
+    pred.prefill([to_device(t, shape.dtype) for t in pre], synth.cu_seqlens(kpre), kv=kv, slots=[0, 1, 2])
+    tol = 1e-5 if shape.dtype == "f32" else 5e-3
+    for s in range(4):
+        rows = [int(cu[b]) + kpre[b] + s for b in range(3)]
+        z, _ = pred.step([to_device(t[rows], shape.dtype) for t in taps], kv, [0, 1, 2])
+        assert np.max(np.abs(to_np(z) - z_all[rows])) <= tol
+    kv.close()
+
+
+def test_batch_permutation_invariance_gpu():
+    shape = MID128
+    pred, w = predictor("mid128")
+    lengths = [40, 200, 3, 129]
+    cu = synth.cu_seqlens(lengths)
+    taps = _taps(shape, int(cu[-1]), off=4)
+    z, _ = pred.prefill([to_device(t, "bf16") for t in taps], cu)
+    z = to_np(z)
+    perm = [3, 1, 0, 2]
+    ptaps = [np.concatenate([t[cu[b]:cu[b + 1]] for b in perm]) for t in taps]
+    zp, _ = pred.prefill([to_device(t, "bf16") for t in ptaps], synth.cu_seqlens([lengths[b] for b in perm]))
+    np.testing.assert_allclose(to_np(zp), z[perm], rtol=0, atol=1e-5)
+
+
+def test_host_buffers_match_device_buffers():
+    shape = MID128
+    pred, w = predictor("mid128")
+    cu = synth.cu_seqlens([17, 90])
+    taps = _taps(shape, int(cu[-1]), off=5)
+    dev = [to_device(t, "bf16") for t in taps]
+    z_d, l_d = pred.prefill(dev, cu)
+    host = [t.cpu() for t in dev]
+    z_h = torch.empty(2, dtype=torch.float32)
+    l_h = torch.empty(2, dtype=torch.float32)
+    pred.prefill(host, cu, z_out=z_h, len_out=l_h)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(z_h.numpy(), z_d.cpu().numpy())
+    np.testing.assert_array_equal(l_h.numpy(), l_d.cpu().numpy())
+
+
+def test_argument_errors_change_nothing():
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = MID128
+    pred, w = predictor("mid128")
+    kv = OT.KVCache(pred, max_slots=4, max_tokens_total=128)
+    taps = [to_device(t, "bf16") for t in _taps(shape, 40, off=6)]
+    with pytest.raises(OT.OutletsError) as e:
+        pred.prefill(taps, np.array([0, 30, 20, 40], np.int32))       # not increasing
+    assert e.value.status == OT.EINVAL
+    with pytest.raises(OT.OutletsError) as e:
+        pred.prefill(taps, np.array([0, 40], np.int32), kv=kv, slots=[7])  # slot out of range
+    assert e.value.status == OT.EINVAL
+    with pytest.raises(OT.OutletsError) as e:
+        pred.prefill(taps, np.array([0, 20, 40], np.int32), kv=kv, slots=[1, 1])  # duplicate slots
+    assert e.value.status == OT.EINVAL
+    pred.prefill(taps, np.array([0, 40], np.int32), kv=kv, slots=[0])
+    free = kv.free_pages
+    big = [to_device(t, "bf16") for t in _taps(shape, 300, off=7)]
+    with pytest.raises(OT.OutletsError) as e:                          # needs 5 pages, 4 left
+        pred.prefill(big, np.array([0, 300], np.int32), kv=kv, slots=[1])
+    assert e.value.status == OT.ECAPACITY
+    assert kv.free_pages == free and kv.slot_length(1) == 0 and kv.slot_length(0) == 40
+    with pytest.raises(OT.OutletsError) as e:
+        pred.step([t[:2] for t in taps], kv, [0, 0])
+    assert e.value.status == OT.EINVAL
+    assert kv.slot_length(0) == 40
+    pred.check()
+    kv.close()
+
+
+# ---------------------------------------------------------------- full-size configurations
+def _sampled_prefill(shape, lengths, max_tokens, sample, seed_off):
+    from paper_2609_01068_gb300 import outlets as OT
+    w = synth.make_weights(shape, 0)
+    pred = OT.Predictor(shape, w, max_tokens=max_tokens, max_batch=len(lengths), max_position=8192)
+    cu = synth.cu_seqlens(lengths)
+    taps = synth.make_taps(shape, int(cu[-1]), 0, seed_off)
+    z, ln = pred.prefill([to_device(t, "bf16") for t in taps], cu)
+    torch.cuda.synchronize()
+    pred.check()
+    hd = to_np(pred.intermediate(OT.T_HDRAFT))
+    ref = OR.sample_prefill_rows(w, shape, taps, cu, sample)
+    check_z_len(z[sample], ln[sample], ref["z"], ref["length"], "bf16", shape.name)
+    check_hidden(hd[sample], ref["h_draft"], "bf16", f"{shape.name} h_draft")
+    pred.close()
+
+
+def test_llama8b_prefill_full_size_sampled():
+    lengths = synth.lengths_8b_prefill(0)
+    order = np.argsort(lengths)
+    sample = [int(order[0]), int(order[1]), int(order[len(order) // 2]), int(order[-1])]
+    _sampled_prefill(synth.LLAMA8B, lengths, 32768, sample, 0)
+
+
+def test_llama70b_prefill_sampled():
+    lengths = synth.lengths_70b_prefill(0)
+    order = np.argsort(lengths)
+    sample = [int(order[0]), int(order[len(order) // 2])]
+    _sampled_prefill(synth.LLAMA70B, lengths, 65536, sample, 0)
+
+
+def test_llama8b_step_full_size_sampled():
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = synth.LLAMA8B
+    w = synth.make_weights(shape, 0)
+    lens = synth.lengths_8b_step_cache(0)
+    B = len(lens)
+    pred = OT.Predictor(shape, w, max_tokens=32768, max_batch=B, max_position=8192)
+    kv = OT.KVCache(pred, max_slots=B, max_tokens_total=int(lens.sum()) + 64 * B)
+    order = np.argsort(lens)
+    sample = [int(order[0]), int(order[1]), int(np.argmin(np.abs(lens - 700))), int(np.argmin(np.abs(lens - 1500)))]
+    gen = torch.Generator(device="cuda").manual_seed(0)
+    sample_taps = {b: synth.make_taps(shape, int(lens[b]), 0, 100 + b) for b in sample}
+    # fill the cache: prompts packed into prefill calls of <= 32768 rows
+    b = 0
+    while b < B:
+        e, tot = b, 0
+        while e < B and tot + lens[e] <= 32768:
+            tot += int(lens[e])
+            e += 1
+        parts = [[], [], []]
+        for r in range(b, e):
+            for i in range(3):
+                if r in sample_taps:
+                    parts[i].append(to_device(sample_taps[r][i], "bf16"))
+                else:
+                    parts[i].append(torch.randn(int(lens[r]), shape.d, device="cuda", generator=gen).to(torch.bfloat16))
+        taps = [torch.cat(p).contiguous() for p in parts]
+        pred.prefill(taps, synth.cu_seqlens(lens[b:e]), kv=kv, slots=np.arange(b, e, dtype=np.int32))
+        b = e
+    step_taps = synth.make_taps(shape, B, 0, 99)
+    z, ln = pred.step([to_device(t, "bf16") for t in step_taps], kv, np.arange(B, dtype=np.int32))
+    torch.cuda.synchronize()
+    pred.check()
+    attn = to_np(pred.intermediate(OT.T_ATTN))
+    for r in sample:
+        pre = OR.predict_prefill(w, shape, sample_taps[r], np.array([0, lens[r]]))
+        ref = OR.predict_step(w, shape, [t[r:r + 1] for t in step_taps], OR.caches_from_prefill(pre, [0, lens[r]]))
+        check_z_len(z[r:r + 1], ln[r:r + 1], ref["z"], ref["length"], "bf16", f"step request {r} (Lc={lens[r]})")
+        check_hidden(attn[r:r + 1], ref["attn"], "bf16", f"step attn request {r}")
+    kv.close()
+    pred.close()

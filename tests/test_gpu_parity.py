@@ -185,9 +185,11 @@ def test_argument_errors_change_nothing():
     assert e.value.status == OT.EINVAL
     pred.prefill(taps, np.array([0, 40], np.int32), kv=kv, slots=[0])
     free = kv.free_pages
-    big = [to_device(t, "bf16") for t in _taps(shape, 300, off=7)]
-    with pytest.raises(OT.OutletsError) as e:                          # needs 5 pages, 4 left
-        pred.prefill(big, np.array([0, 300], np.int32), kv=kv, slots=[1])
+    # the pool holds ceil(128 / 64) + 4 = 6 pages; one is taken, 400 rows need 7
+    assert free == 5
+    big = [to_device(t, "bf16") for t in _taps(shape, 400, off=7)]
+    with pytest.raises(OT.OutletsError) as e:
+        pred.prefill(big, np.array([0, 400], np.int32), kv=kv, slots=[1])
     assert e.value.status == OT.ECAPACITY
     assert kv.free_pages == free and kv.slot_length(1) == 0 and kv.slot_length(0) == 40
     with pytest.raises(OT.OutletsError) as e:

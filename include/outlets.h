@@ -231,6 +231,27 @@ const char* outlets_stage_name(int32_t stage);
 /* Number of kernels this context has launched for prediction calls so far. */
 uint64_t outlets_launch_count(const outlets_ctx* ctx);
 
+/* Length head without device allocation.  The paper has no counterpart: this
+ * exists for callers that cannot call cudaMalloc while they serve (a process
+ * that gives all spare device memory to its KV-cache pool at start-up and
+ * treats later allocations as failures, or a latency-critical caller that
+ * cannot accept cudaMalloc's implicit device synchronization).
+ *   h_draft  device [rows, d] (bf16 or f32 like the context), 16-byte aligned:
+ *            final-normed draft states (OUTLETS_T_HDRAFT of a prediction call).
+ *   z_out, len_out  device f32 [rows]: z_hat and max(0, expm1(z_hat));
+ *            len_out may be NULL.
+ * Same arithmetic as the head stage of the prediction calls.  The hidden
+ * activations live in a 16 MiB array inside the library image (held by every
+ * GPU that loads the library until the process exits) instead of allocated
+ * memory; rows x (widest hidden layer) x (2 if the head has more than one
+ * hidden layer) must fit in 4 Mi floats, else OUTLETS_ECAPACITY with a message
+ * in outlets_last_error.  The first call on a device looks up the array's
+ * device address; make that first call before any stream capture.  All calls
+ * on a device share the array: calls that overlap on the GPU race.  Allocates
+ * nothing (no cudaMalloc, cudaFree or allocating library routine). */
+outlets_status outlets_length_head_noalloc(outlets_ctx* ctx, const void* h_draft, int32_t rows, float* z_out,
+                                           float* len_out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1094,3 +1094,86 @@ outlets_status outlets_get_intermediate(outlets_ctx* c, int32_t which, void* dst
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Length head without device allocation.
+//
+// Some callers cannot call cudaMalloc while they serve: a serving process that
+// hands all spare device memory to its KV-cache pool at start-up and treats any
+// later allocation as a failure, or a caller on a latency-critical path where
+// cudaMalloc's implicit device-wide synchronization is not acceptable.  For
+// them, outlets_length_head_noalloc runs the length head (Linear+ReLU layers
+// and the output row) with its hidden activations in the file-scope array
+// below instead of in memory it allocates.  The array is part of the library
+// image: every GPU that loads the library holds its 16 MiB until the process
+// exits.  All calls on a device share it, so calls that overlap on the GPU
+// race; nothing in it has to start at zero (every value read was written
+// earlier in the same call).
+namespace {
+
+constexpr size_t kHeadScratchFloats = (size_t)4 << 20;  // 16 MiB
+static __device__ __align__(256) float g_head_scratch[kHeadScratchFloats];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_head_scratch_mu;
+float* g_head_scratch_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device (looked up once
+// per device; host code must not use the symbol itself as an address).
+cudaError_t head_scratch_ptr(int device, float** out) {
+  std::lock_guard<std::mutex> lock(g_head_scratch_mu);
+  if (!g_head_scratch_ptr[device]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_head_scratch);
+    if (e != cudaSuccess) return e;
+    g_head_scratch_ptr[device] = static_cast<float*>(p);
+  }
+  *out = g_head_scratch_ptr[device];
+  return cudaSuccess;
+}
+
+}  // namespace
+
+extern "C" outlets_status outlets_length_head_noalloc(outlets_ctx* c, const void* h_draft, int32_t rows,
+                                                      float* z_out, float* len_out, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  if (!h_draft || !z_out) return c->fail(OUTLETS_EINVAL, "h_draft and z_out must not be NULL");
+  if (rows < 0) return c->fail(OUTLETS_EINVAL, "rows must be >= 0");
+  if (rows == 0) return OUTLETS_OK;
+  if (c->cfg.device < 0 || c->cfg.device >= kMaxDevices) return c->fail(OUTLETS_EUNSUPPORTED, "device ordinal too large");
+  if (!is_device_ptr(h_draft) || !is_device_ptr(z_out) || (len_out && !is_device_ptr(len_out)))
+    return c->fail(OUTLETS_EINVAL, "h_draft, z_out and len_out must be device memory");
+  if (reinterpret_cast<uintptr_t>(h_draft) % 16) return c->fail(OUTLETS_EINVAL, "h_draft must be 16-byte aligned");
+  const int nl = (int)c->head_dims.size() - 1;
+  int wmax = 1;
+  for (int i = 1; i < nl; ++i) wmax = std::max(wmax, c->head_dims[i]);
+  const size_t need = (size_t)rows * (nl > 2 ? 2 * (size_t)wmax : (size_t)c->head_dims[1]);
+  if (need > kHeadScratchFloats)
+    return c->fail(OUTLETS_ECAPACITY, "rows x head width exceeds the 16 MiB scratch of outlets_length_head_noalloc (" +
+                                          std::to_string(need) + " > " + std::to_string(kHeadScratchFloats) +
+                                          " floats)");
+  OUT_CK(c, cudaSetDevice(c->cfg.device));
+  float* scratch = nullptr;
+  OUT_CK(c, head_scratch_ptr(c->cfg.device, &scratch));
+  cudaStream_t s = (cudaStream_t)stream;
+  const int d = c->d;
+  float* buf[2] = {scratch, scratch + (size_t)rows * wmax};
+  float* cur = buf[0];
+  const void* a1[3] = {h_draft, h_draft, h_draft};
+  const int w1 = c->head_dims[1];
+  if (c->bf16)
+    OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->head_w0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0, c->head_b[0], s));
+  else
+    OUT_TRY(gemm_f32(c, a1, d, rows, c->head_w0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0, c->head_b[0], s));
+  for (int i = 1; i < nl - 1; ++i) {
+    float* nxt = (cur == buf[0]) ? buf[1] : buf[0];
+    const void* ai[3] = {cur, cur, cur};
+    OUT_TRY(gemm_f32(c, ai, c->head_dims[i], rows, c->head_wf[i], c->head_dims[i + 1], c->head_dims[i],
+                     EPI_BIAS_RELU, nxt, c->head_dims[i + 1], nullptr, 0, c->head_b[i], s));
+    cur = nxt;
+  }
+  OUT_CK(c, head_tail_launch(cur, nullptr, c->head_wf[nl - 1], c->head_b[nl - 1], rows, c->head_dims[nl - 1], z_out,
+                             len_out, s));
+  return OUTLETS_OK;
+}

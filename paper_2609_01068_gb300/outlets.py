@@ -81,6 +81,7 @@ def load():
         "outlets_profile_read": (c_i32, [c_vp, P(ctypes.c_double), P(c_i32)]),
         "outlets_stage_name": (ctypes.c_char_p, [c_i32]),
         "outlets_launch_count": (ctypes.c_uint64, [c_vp]),
+        "outlets_length_head_noalloc": (c_i32, [c_vp, c_vp, c_i32, c_vp, c_vp, c_vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)

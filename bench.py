@@ -42,7 +42,11 @@ def parse():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--no-step-mode", action="store_true")
+    ap.add_argument("--mode", default="both", choices=["both", "prefill", "step"],
+                    help="static prediction (headline), dynamic prediction, or both")
+    ap.add_argument("--prompts", type=int, default=64, help="first N prompts of the workload (profiling cases)")
+    ap.add_argument("--step-requests", type=int, default=256, help="live requests of the dynamic-prediction run")
+    ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
 
@@ -195,7 +199,7 @@ def run_ours(args):
     peaks = load_peaks()
     shape = synth.LLAMA8B
     w = synth.make_weights(shape, 0)
-    lengths = synth.lengths_8b_prefill(0)
+    lengths = synth.lengths_8b_prefill(0)[:args.prompts]
     cu = synth.cu_seqlens(lengths)
     T, Bq = int(cu[-1]), len(lengths)
     taps = synth.make_taps(shape, T, 0, rank)
@@ -204,8 +208,10 @@ def run_ours(args):
         return torch.from_numpy(synth.bf16_bits(a).view(np.int16)).view(torch.bfloat16).cuda()
 
     taps_d = [dev(t) for t in taps]
-    step_B = 256
-    pred = outlets.Predictor(shape, w, max_tokens=32768, max_batch=step_B, max_position=8192, device=local)
+    step_B = args.step_requests
+    max_tokens = max(8192, (T + 1023) // 1024 * 1024)
+    pred = outlets.Predictor(shape, w, max_tokens=max_tokens, max_batch=max(step_B, Bq), max_position=8192,
+                             device=local)
     stream = torch.cuda.current_stream()
 
     def barrier():
@@ -220,6 +226,28 @@ def run_ours(args):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         return float(t.item())
 
+    out = {"metric": METRIC, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic"}
+    if args.mode in ("both", "prefill"):
+        out.update(run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, world, rank, local,
+                                    barrier, max_over_ranks, stream))
+    if args.mode in ("both", "step"):
+        sm = run_step_mode(args, pred, shape, peaks, step_B, world, barrier, max_over_ranks, stream, max_tokens)
+        if args.mode == "step":
+            out.update({k: sm[k] for k in ("value", "unit", "ms_per_step")})
+            out["config"] = {"workload": sm["workload"], "parallelism": f"replicas x{world}"}
+        out["step_mode"] = sm
+    if rank == 0:
+        print(json.dumps(out))
+    pred.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, world, rank, local, barrier,
+                     max_over_ranks, stream):
+    import torch
+    T, Bq = int(cu[-1]), len(lengths)
     # ---------------- device-timed static prediction
     z = torch.empty(Bq, dtype=torch.float32, device="cuda")
     ln = torch.empty(Bq, dtype=torch.float32, device="cuda")
@@ -259,30 +287,25 @@ def run_ours(args):
               for k, v in prof.items() if v[1]}
 
     # ---------------- end to end through the C ABI with host buffers
-    host_taps = [t.cpu().pin_memory() for t in taps_d]
-    zh = torch.empty(Bq, dtype=torch.float32).pin_memory()
-    lh = torch.empty(Bq, dtype=torch.float32).pin_memory()
-    for _ in range(max(2, args.warmup // 2)):
-        pred.prefill(host_taps, cu, z_out=zh, len_out=lh)
-        stream.synchronize()
-    barrier()
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        pred.prefill(host_taps, cu, z_out=zh, len_out=lh)
-        stream.synchronize()
-    e2e_s = max_over_ranks(time.perf_counter() - t0)
-    e2e = {"value": world * Bq * args.steps / e2e_s, "unit": "predictions/s",
-           "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps)),
-           "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4)}
+    e2e = None
+    if not args.no_e2e:
+        host_taps = [t.cpu().pin_memory() for t in taps_d]
+        zh = torch.empty(Bq, dtype=torch.float32).pin_memory()
+        lh = torch.empty(Bq, dtype=torch.float32).pin_memory()
+        for _ in range(max(2, args.warmup // 2)):
+            pred.prefill(host_taps, cu, z_out=zh, len_out=lh)
+            stream.synchronize()
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            pred.prefill(host_taps, cu, z_out=zh, len_out=lh)
+            stream.synchronize()
+        e2e_s = max_over_ranks(time.perf_counter() - t0)
+        e2e = {"value": world * Bq * args.steps / e2e_s, "unit": "predictions/s",
+               "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps)),
+               "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4)}
 
-    # ---------------- dynamic prediction (per-step path)
-    step_mode = None
-    if not args.no_step_mode:
-        step_mode = run_step_mode(args, pred, shape, peaks, step_B, world, barrier, max_over_ranks, stream)
-
-    out = {"metric": METRIC, "value": value, "unit": "predictions/s", "n_gpus": world, "steps": args.steps,
-           "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
-           "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+    out = {"value": value, "unit": "predictions/s", "ms_per_step": ms_step,
            "config": {"workload": WORKLOAD, "prompts_per_gpu": Bq, "tokens_per_gpu": T,
                       "l2": "inputs larger than L2 (taps 3x[T,4096] bf16 = %.0f MB, weights 545 MB)"
                             % (3 * T * 4096 * 2 / 1e6),
@@ -291,20 +314,16 @@ def run_ours(args):
            "tflops_per_s": flops * args.steps / (ms / 1e3) / 1e12,
            "tensor_peak_frac_step": flops * args.steps / (ms / 1e3) / 1e12 / peaks["bf16_sus"],
            "roofline": roofline, "stages": stages, "clocks": clocks, "e2e": e2e,
-           "gpu_launches": launches, "step_mode": step_mode}
+           "gpu_launches": launches}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n_pred, n_tok, secs = oracle_sample(shape, w, taps, cu, lengths, 1200)
         out["cpu_baseline"] = {"value": n_pred / secs, "unit": "predictions/s", "cores": cpu_threads(),
                                "kind": "oracle",
                                "sample": f"{n_pred} whole prompts ({n_tok} tokens) of the same workload, {secs:.1f} s"}
-    if rank == 0:
-        print(json.dumps(out))
-    pred.close()
-    if world > 1:
-        dist.destroy_process_group()
+    return out
 
 
-def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, stream):
+def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, stream, max_tokens):
     import torch
 
     from paper_2609_01068_gb300 import outlets, synth
@@ -315,7 +334,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     b = 0
     while b < B:   # fill the draft cache (untimed set-up)
         e, tot = b, 0
-        while e < B and tot + lens[e] <= 32768:
+        while e < B and tot + lens[e] <= max_tokens:
             tot += int(lens[e])
             e += 1
         taps = [torch.randn(tot, shape.d, device="cuda", generator=gen).to(torch.bfloat16) for _ in range(3)]
@@ -330,6 +349,9 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     pred.check()
     cache0 = sum(kv.slot_length(int(s)) for s in slots)
     pred.profile(True)
+    launches0 = pred.launch_count
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.start()
     barrier()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
@@ -338,7 +360,9 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     ev1.record(stream)
     ev1.synchronize()
     barrier()
+    clocks = sampler.stop()
     ms = max_over_ranks(ev0.elapsed_time(ev1))
+    launches = pred.launch_count - launches0
     prof = pred.profile_read()
     pred.profile(False)
     pred.check()
@@ -353,8 +377,8 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     at_gbs = kv_bytes / (at_ms / at_n / 1e3) / 1e9
     ms_step = ms / args.steps
     kv.close()
-    return {"workload": "dynamic prediction, 256 live requests x 1 new token, cache lengths lognormal "
-                        "median 512 clipped 1-4096 (sum %d)" % int(lens.sum()),
+    return {"workload": "dynamic prediction, %d live requests x 1 new token, cache lengths lognormal "
+                        "median 512 clipped 1-4096 (sum %d), Llama-3.1-8B-shaped draft layer" % (B, int(lens.sum())),
             "value": world * B * args.steps / (ms / 1e3), "unit": "predictions/s", "ms_per_step": ms_step,
             "hbm_frac_step": step_bytes / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"],
             "algorithmic_bytes_per_step": step_bytes,
@@ -362,7 +386,8 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
                          "achieved": at_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                          "frac": at_gbs / peaks["hbm_gbs"], "traffic": None,
                          "algorithmic_per_launch": f"{kv_bytes:.4g} B of K/V (cached + new)"},
-            "stages": {k: v[0] / max(args.steps, 1) for k, v in prof.items() if v[1]}}
+            "stages": {k: v[0] / max(args.steps, 1) for k, v in prof.items() if v[1]},
+            "clocks": clocks, "gpu_launches": launches}
 
 
 def main():

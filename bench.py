@@ -355,8 +355,10 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     barrier()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
+    h0 = time.perf_counter()
     for _ in range(args.steps):
         pred.step(st_taps, kv, slots, z_out=z, len_out=ln)
+    host_ms = (time.perf_counter() - h0) * 1e3 / args.steps
     ev1.record(stream)
     ev1.synchronize()
     barrier()
@@ -387,7 +389,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
                          "frac": at_gbs / peaks["hbm_gbs"], "traffic": None,
                          "algorithmic_per_launch": f"{kv_bytes:.4g} B of K/V (cached + new)"},
             "stages": {k: v[0] / max(args.steps, 1) for k, v in prof.items() if v[1]},
-            "clocks": clocks, "gpu_launches": launches}
+            "clocks": clocks, "gpu_launches": launches, "host_issue_ms_per_step": host_ms}
 
 
 def main():

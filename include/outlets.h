@@ -71,7 +71,7 @@ typedef struct outlets_config {
   int32_t d_model;        /* d: width of each tap, of f_ctx and of the draft state */
   int32_t n_heads;        /* H query heads */
   int32_t n_kv_heads;     /* KVH key/value heads; H % KVH == 0 */
-  int32_t head_dim;       /* hd (even; 64 or 128 on the bf16 path) */
+  int32_t head_dim;       /* hd (multiple of 16; 64 or 128 on the bf16 path) */
   int32_t ffn_dim;        /* F: SwiGLU inner width */
   int32_t n_head_hidden;  /* hidden Linear+ReLU layers of MLP_len (1 .. OUTLETS_MAX_HEAD_HIDDEN) */
   int32_t head_hidden[OUTLETS_MAX_HEAD_HIDDEN];  /* their widths; the last Linear maps to 1 */

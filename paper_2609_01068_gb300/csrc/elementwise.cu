@@ -43,29 +43,123 @@ __device__ __forceinline__ void store4<bf16>(bf16* p, float a, float b, float c,
   *reinterpret_cast<uint2*>(p) = v;
 }
 
-template <typename Act>
-__global__ void k_rmsnorm(const float* __restrict__ x, const int* __restrict__ row_index,
+// v = residual[src] + sum_s x[s][src] (split-K slices of the producing GEMM);
+// y[r] = v * g * rsqrt(mean(v^2) + eps); copy_out[r] = v (f32) when given.
+// REDUCE = false: v = x[src] (one slice, no residual).
+template <typename Act, bool REDUCE>
+__global__ void k_rmsnorm(const float* __restrict__ x, int n_split, long long split_stride,
+                          const float* __restrict__ residual, const int* __restrict__ row_index,
                           const float* __restrict__ g, Act* __restrict__ y, float* __restrict__ copy_out, int d,
                           float eps) {
   __shared__ float red[33];
+  extern __shared__ float4 rowbuf[];  // the reduced row (REDUCE only)
   const int r = blockIdx.x;
   const long long src = row_index ? row_index[r] : r;
-  const float* xr = x + src * d;
   float ss = 0.f;
   for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
-    const float4 v = *reinterpret_cast<const float4*>(xr + i);
+    float4 v = *reinterpret_cast<const float4*>(x + src * d + i);
+    if constexpr (REDUCE) {
+      float4 v2 = make_float4(0.f, 0.f, 0.f, 0.f);
+      int sp = 1;
+      for (; sp + 1 < n_split; sp += 2) {  // two independent partial sums
+        const float4 a = *reinterpret_cast<const float4*>(x + sp * split_stride + src * d + i);
+        const float4 b = *reinterpret_cast<const float4*>(x + (sp + 1) * split_stride + src * d + i);
+        v.x += a.x;
+        v.y += a.y;
+        v.z += a.z;
+        v.w += a.w;
+        v2.x += b.x;
+        v2.y += b.y;
+        v2.z += b.z;
+        v2.w += b.w;
+      }
+      if (sp < n_split) {
+        const float4 a = *reinterpret_cast<const float4*>(x + sp * split_stride + src * d + i);
+        v.x += a.x;
+        v.y += a.y;
+        v.z += a.z;
+        v.w += a.w;
+      }
+      if (residual) {
+        const float4 a = *reinterpret_cast<const float4*>(residual + src * d + i);
+        v2.x += a.x;
+        v2.y += a.y;
+        v2.z += a.z;
+        v2.w += a.w;
+      }
+      v.x += v2.x;
+      v.y += v2.y;
+      v.z += v2.z;
+      v.w += v2.w;
+      rowbuf[i >> 2] = v;
+    }
     ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
   }
   const float inv = rsqrtf(block_sum(ss, red) / (float)d + eps);
   Act* yr = y + (long long)r * d;
   for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
-    const float4 v = *reinterpret_cast<const float4*>(xr + i);
+    float4 v;
+    if constexpr (REDUCE) v = rowbuf[i >> 2];
+    else v = *reinterpret_cast<const float4*>(x + src * d + i);
     const float4 gg = *reinterpret_cast<const float4*>(g + i);
     store4<Act>(yr + i, v.x * inv * gg.x, v.y * inv * gg.y, v.z * inv * gg.z, v.w * inv * gg.w);
     if (copy_out) *reinterpret_cast<float4*>(copy_out + (long long)r * d + i) = v;
   }
 }
 
+// 8 consecutive elements of a row as f32, summed over n_split slices.
+template <typename In>
+__device__ __forceinline__ void load8(const In* p, long long idx, int n_split, long long stride, float* v);
+template <>
+__device__ __forceinline__ void load8<bf16>(const bf16* p, long long idx, int, long long, float* v) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p + idx);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float2 f = __bfloat1622float2(h[k]);
+    v[2 * k] = f.x;
+    v[2 * k + 1] = f.y;
+  }
+}
+template <>
+__device__ __forceinline__ void load8<float>(const float* p, long long idx, int n_split, long long stride,
+                                             float* v) {
+  float4 a = *reinterpret_cast<const float4*>(p + idx);
+  float4 b = *reinterpret_cast<const float4*>(p + idx + 4);
+  for (int sp = 1; sp < n_split; ++sp) {
+    const float4 c = *reinterpret_cast<const float4*>(p + sp * stride + idx);
+    const float4 e = *reinterpret_cast<const float4*>(p + sp * stride + idx + 4);
+    a.x += c.x;
+    a.y += c.y;
+    a.z += c.z;
+    a.w += c.w;
+    b.x += e.x;
+    b.y += e.y;
+    b.z += e.z;
+    b.w += e.w;
+  }
+  v[0] = a.x, v[1] = a.y, v[2] = a.z, v[3] = a.w, v[4] = b.x, v[5] = b.y, v[6] = b.z, v[7] = b.w;
+}
+
+template <typename Act>
+__device__ __forceinline__ void store8(Act* p, const float* v);
+template <>
+__device__ __forceinline__ void store8<bf16>(bf16* p, const float* v) {
+  uint4 u;
+  u.x = pack_bf16x2(v[0], v[1]);
+  u.y = pack_bf16x2(v[2], v[3]);
+  u.z = pack_bf16x2(v[4], v[5]);
+  u.w = pack_bf16x2(v[6], v[7]);
+  *reinterpret_cast<uint4*>(p) = u;
+}
+template <>
+__device__ __forceinline__ void store8<float>(float* p, const float* v) {
+  *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
+}
+
+// One CTA per row; a thread rotates 8 pairs (i..i+7 with i+hd/2..i+hd/2+7) of
+// one head and copies 8 values of V.  hd is a multiple of 16.
 template <typename In, typename Act>
 __global__ void k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
   const int row = blockIdx.x;
@@ -102,39 +196,51 @@ __global__ void k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
     const int page = a.page_list[a.page_off[seq] + pos / a.page_tokens];
     cache_base = ((long long)page * KVH) * a.page_tokens + pos % a.page_tokens;
   }
-  for (int idx = threadIdx.x; idx < (H + KVH) * half; idx += blockDim.x) {
-    const int head = idx / half;
-    const int i = idx - head * half;
-    const float x1 = to_f(src[head * hd + i]);
-    const float x2 = to_f(src[head * hd + i + half]);
-    const float c = cs[i], s = sn[i];
-    const float y1 = x1 * c - x2 * s;
-    const float y2 = x2 * c + x1 * s;
+  const int cpr = half / 8;  // 8-element chunks per half head
+  for (int idx = threadIdx.x; idx < (H + KVH) * cpr; idx += blockDim.x) {
+    const int head = idx / cpr;
+    const int i = (idx - head * cpr) * 8;
+    float x1[8], x2[8], y1[8], y2[8];
+    load8<In>(src, head * hd + i, a.n_split, a.split_stride, x1);
+    load8<In>(src, head * hd + i + half, a.n_split, a.split_stride, x2);
+    const float4 c0 = *reinterpret_cast<const float4*>(cs + i);
+    const float4 c1 = *reinterpret_cast<const float4*>(cs + i + 4);
+    const float4 s0 = *reinterpret_cast<const float4*>(sn + i);
+    const float4 s1 = *reinterpret_cast<const float4*>(sn + i + 4);
+    const float c[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+    const float sv[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      y1[k] = x1[k] * c[k] - x2[k] * sv[k];
+      y2[k] = x2[k] * c[k] + x1[k] * sv[k];
+    }
     if (head < H) {
       Act* qo = q_out + ((long long)row * H + head) * hd;
-      qo[i] = from_f<Act>(y1);
-      qo[i + half] = from_f<Act>(y2);
+      store8<Act>(qo + i, y1);
+      store8<Act>(qo + i + half, y2);
     } else {
       const int kh = head - H;
       if (k_out) {
         Act* ko = k_out + ((long long)kh * a.kv_ld_rows + row) * hd;
-        ko[i] = from_f<Act>(y1);
-        ko[i + half] = from_f<Act>(y2);
+        store8<Act>(ko + i, y1);
+        store8<Act>(ko + i + half, y2);
       }
       if (k_pool) {
         Act* kc = k_pool + (cache_base + (long long)kh * a.page_tokens) * hd;
-        kc[i] = from_f<Act>(y1);
-        kc[i + half] = from_f<Act>(y2);
+        store8<Act>(kc + i, y1);
+        store8<Act>(kc + i + half, y2);
       }
     }
   }
-  const In* vs = src + (long long)(H + KVH) * hd;
-  for (int idx = threadIdx.x; idx < KVH * hd; idx += blockDim.x) {
-    const int kh = idx / hd;
-    const int dd = idx - kh * hd;
-    const Act val = from_f<Act>(to_f(vs[idx]));
-    if (v_out) v_out[((long long)kh * a.kv_ld_rows + row) * hd + dd] = val;
-    if (v_pool) v_pool[(cache_base + (long long)kh * a.page_tokens) * hd + dd] = val;
+  const long long voff = (long long)(H + KVH) * hd;
+  for (int idx = threadIdx.x; idx < KVH * hd / 8; idx += blockDim.x) {
+    const int e = idx * 8;
+    const int kh = e / hd;
+    const int dd = e - kh * hd;
+    float v[8];
+    load8<In>(src, voff + e, a.n_split, a.split_stride, v);
+    if (v_out) store8<Act>(v_out + ((long long)kh * a.kv_ld_rows + row) * hd + dd, v);
+    if (v_pool) store8<Act>(v_pool + (cache_base + (long long)kh * a.page_tokens) * hd + dd, v);
   }
 }
 
@@ -145,27 +251,35 @@ __global__ void k_swiglu(const float* __restrict__ gu, Act* __restrict__ u, int 
        idx += (long long)gridDim.x * blockDim.x) {
     const long long r = idx / f_pad;
     const int j = (int)(idx - r * f_pad);
-    const float* row = gu + r * 2 * f_pad + (j >> 7) * 256 + (j & 127);
-    const float gt = row[0], up = row[128];
+    const float* row = gu + r * 2 * f_pad + (j >> 5) * 64 + (j & 31);
+    const float gt = row[0], up = row[32];
     u[idx] = from_f<Act>(gt / (1.f + __expf(-gt)) * up);
   }
 }
 
-__global__ void k_head_tail(const float* __restrict__ h, const float* __restrict__ b_prev,
-                            const float* __restrict__ w_last, const float* __restrict__ b_last, int rows, int width,
-                            float* __restrict__ z, float* __restrict__ len) {
-  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (r >= rows) return;
+// One CTA per row: h = sum of slices, a = relu(h + b_prev), z = w_last . a + b_last.
+__global__ void k_head_tail(const float* __restrict__ h, int n_split, long long split_stride,
+                            const float* __restrict__ b_prev, const float* __restrict__ w_last,
+                            const float* __restrict__ b_last, int rows, int width, float* __restrict__ z,
+                            float* __restrict__ len) {
+  __shared__ float red[33];
+  const int r = blockIdx.x;
   const float* hr = h + (long long)r * width;
   float acc = 0.f;
-  for (int j = lane; j < width; j += 32) {
-    float x = hr[j];
+  for (int j = threadIdx.x; j < width; j += blockDim.x) {
+    float x0 = hr[j], x1 = 0.f;
+    int sp = 1;
+    for (; sp + 1 < n_split; sp += 2) {
+      x0 += hr[sp * split_stride + j];
+      x1 += hr[(sp + 1) * split_stride + j];
+    }
+    if (sp < n_split) x0 += hr[sp * split_stride + j];
+    float x = x0 + x1;
     if (b_prev) x = fmaxf(x + b_prev[j], 0.f);
     acc += w_last[j] * x;
   }
-  acc = warp_sum(acc);
-  if (lane == 0) {
+  acc = block_sum(acc, red);
+  if (threadIdx.x == 0) {
     const float zz = acc + b_last[0];
     z[r] = zz;
     if (len) len[r] = fmaxf(0.f, expm1f(zz));
@@ -174,17 +288,25 @@ __global__ void k_head_tail(const float* __restrict__ h, const float* __restrict
 
 template <typename Act>
 __global__ void k_convert_rows(const float* __restrict__ src, Act* __restrict__ dst, int rows, int cols,
-                               long long dst_ld, int row_mode, int row_base) {
+                               long long dst_ld, int row_mode, int row_base, long long kb_np) {
   const long long n = (long long)rows * cols;
   for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n;
        idx += (long long)gridDim.x * blockDim.x) {
     const int r = (int)(idx / cols);
     const int c = (int)(idx - (long long)r * cols);
-    int dr;
-    if (row_mode == 0) dr = row_base + r;
-    else if (row_mode == 1) dr = (r >> 7) * 256 + (r & 127);        // gate rows of an interleaved [gate|up] block
-    else dr = (r >> 7) * 256 + 128 + (r & 127);                      // up rows
-    dst[(long long)dr * dst_ld + c] = from_f<Act>(src[idx]);
+    const int rg = row_base + r;
+    long long dr;
+    if (row_mode == 0) dr = rg;
+    else if (row_mode == 1) dr = (rg >> 5) * 64 + (rg & 31);        // gate rows of an interleaved [gate 32 | up 32] block
+    else dr = (rg >> 5) * 64 + 32 + (rg & 31);                      // up rows
+    long long o;
+    if (kb_np > 0) {
+      const int cc = c & 63;
+      o = ((long long)(c >> 6) * kb_np + dr) * 64 + ((((cc >> 3) ^ (int)(dr & 7)) << 3) | (cc & 7));
+    } else {
+      o = dr * dst_ld + c;
+    }
+    dst[o] = from_f<Act>(src[idx]);
   }
 }
 
@@ -256,16 +378,36 @@ inline int grid_for(long long n, int threads) {
 template <typename Act>
 cudaError_t rmsnorm_launch(const float* x, const float* g, Act* y, float* copy_out, int rows, int d, float eps,
                            cudaStream_t stream) {
-  if (rows == 0) return cudaSuccess;
-  k_rmsnorm<Act><<<rows, 256, 0, stream>>>(x, nullptr, g, y, copy_out, d, eps);
-  return cudaGetLastError();
+  return rmsnorm_reduce_launch<Act>(x, 1, 0, nullptr, nullptr, g, y, copy_out, rows, d, eps, stream);
 }
 
 template <typename Act>
 cudaError_t rmsnorm_gather_launch(const float* x, const int* row_index, const float* g, Act* y, int rows, int d,
                                   float eps, cudaStream_t stream) {
+  return rmsnorm_reduce_launch<Act>(x, 1, 0, nullptr, row_index, g, y, nullptr, rows, d, eps, stream);
+}
+
+template <typename Act>
+cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_stride, const float* residual,
+                                  const int* row_index, const float* g, Act* y, float* copy_out, int rows, int d,
+                                  float eps, cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
-  k_rmsnorm<Act><<<rows, 256, 0, stream>>>(x, row_index, g, y, nullptr, d, eps);
+  if (n_split > 1 || residual) {
+    const size_t smem = (size_t)d * sizeof(float);
+    if (smem > 48 * 1024) {
+      static bool attr = false;
+      if (!attr) {
+        cudaError_t e =
+            cudaFuncSetAttribute(k_rmsnorm<Act, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        if (e != cudaSuccess) return e;
+        attr = true;
+      }
+    }
+    k_rmsnorm<Act, true><<<rows, 256, smem, stream>>>(x, n_split, split_stride, residual, row_index, g, y, copy_out,
+                                                      d, eps);
+  } else {
+    k_rmsnorm<Act, false><<<rows, 256, 0, stream>>>(x, 1, 0, nullptr, row_index, g, y, copy_out, d, eps);
+  }
   return cudaGetLastError();
 }
 
@@ -283,19 +425,20 @@ cudaError_t swiglu_launch(const float* gu, Act* u, int rows, int f_pad, cudaStre
   return cudaGetLastError();
 }
 
-cudaError_t head_tail_launch(const float* h_pre, const float* b_prev, const float* w_last, const float* b_last,
-                             int rows, int width, float* z, float* len, cudaStream_t stream) {
+cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_stride, const float* b_prev,
+                             const float* w_last, const float* b_last, int rows, int width, float* z, float* len,
+                             cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
-  k_head_tail<<<(rows + 7) / 8, 256, 0, stream>>>(h_pre, b_prev, w_last, b_last, rows, width, z, len);
+  k_head_tail<<<rows, 128, 0, stream>>>(h_pre, n_split, split_stride, b_prev, w_last, b_last, rows, width, z, len);
   return cudaGetLastError();
 }
 
 template <typename Act>
 cudaError_t convert_rows_launch(const float* src, Act* dst, int rows, int cols, long long dst_ld, int row_mode,
-                                int row_base, cudaStream_t stream) {
+                                int row_base, long long kb_np, cudaStream_t stream) {
   if (rows == 0 || cols == 0) return cudaSuccess;
   k_convert_rows<Act><<<grid_for((long long)rows * cols, 256), 256, 0, stream>>>(src, dst, rows, cols, dst_ld,
-                                                                                row_mode, row_base);
+                                                                                row_mode, row_base, kb_np);
   return cudaGetLastError();
 }
 
@@ -308,20 +451,26 @@ cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int ep
 }
 
 #define OUTLETS_INST_ACT(Act)                                                                                   \
+  template cudaError_t rmsnorm_reduce_launch<Act>(const float*, int, long long, const float*, const int*,        \
+                                                  const float*, Act*, float*, int, int, float, cudaStream_t);   \
   template cudaError_t rmsnorm_launch<Act>(const float*, const float*, Act*, float*, int, int, float,          \
                                            cudaStream_t);                                                      \
   template cudaError_t rmsnorm_gather_launch<Act>(const float*, const int*, const float*, Act*, int, int, float, \
                                                   cudaStream_t);                                               \
   template cudaError_t swiglu_launch<Act>(const float*, Act*, int, int, cudaStream_t);                         \
-  template cudaError_t convert_rows_launch<Act>(const float*, Act*, int, int, long long, int, int, cudaStream_t); \
+  template cudaError_t convert_rows_launch<Act>(const float*, Act*, int, int, long long, int, int, long long,       \
+                                                cudaStream_t);                                                  \
   template cudaError_t rope_scatter_launch<float, Act>(const float*, const RopeArgs&, cudaStream_t);           \
   template cudaError_t rope_scatter_launch<Act, Act>(const Act*, const RopeArgs&, cudaStream_t);
 OUTLETS_INST_ACT(bf16)
+template cudaError_t rmsnorm_reduce_launch<float>(const float*, int, long long, const float*, const int*,
+                                                  const float*, float*, float*, int, int, float, cudaStream_t);
 template cudaError_t rmsnorm_launch<float>(const float*, const float*, float*, float*, int, int, float, cudaStream_t);
 template cudaError_t rmsnorm_gather_launch<float>(const float*, const int*, const float*, float*, int, int, float,
                                                   cudaStream_t);
 template cudaError_t swiglu_launch<float>(const float*, float*, int, int, cudaStream_t);
-template cudaError_t convert_rows_launch<float>(const float*, float*, int, int, long long, int, int, cudaStream_t);
+template cudaError_t convert_rows_launch<float>(const float*, float*, int, int, long long, int, int, long long,
+                                                cudaStream_t);
 template cudaError_t rope_scatter_launch<float, float>(const float*, const RopeArgs&, cudaStream_t);
 #undef OUTLETS_INST_ACT
 

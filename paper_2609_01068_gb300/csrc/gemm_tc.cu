@@ -21,24 +21,34 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;  // one 128-byte swizzle row of bf16
 
-template <int BN>
+// BN: tile width (N); MT: 128-row M sub-tiles per tile (1 or 2).  With MT = 2 a
+// CTA computes 256 rows against one staged B tile (two MMAs per K step into two
+// TMEM accumulators), so each weight tile is read once for up to 256 rows.
+template <int BN, int MT>
 struct TcCfg {
-  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
-  static constexpr uint32_t A_BYTES = BM * BK * 2;
+  static constexpr int ACC = (512 / (MT * BN)) >= 2 ? 2 : 1;  // TMEM accumulator stages
+  static_assert(BN % 64 == 0 && BN <= 256, "tile width");
+  static constexpr uint32_t A_BYTES = MT * BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr uint32_t TMEM_COLS = 2 * BN;
+  static constexpr int STAGES = (196608 / STAGE_BYTES) > 8 ? 8 : (196608 / STAGE_BYTES);
+  static constexpr uint32_t TMEM_USED = ACC * MT * BN;
+  static constexpr uint32_t TMEM_COLS = TMEM_USED <= 32 ? 32 : TMEM_USED <= 64 ? 64 : TMEM_USED <= 128 ? 128
+                                                               : TMEM_USED <= 256 ? 256 : 512;  // power of 2
   static constexpr size_t SMEM = 1024 + STAGES * STAGE_BYTES + 256;
+  static_assert(TMEM_USED <= 512, "TMEM columns");
 };
 
 struct Tile {
-  int m_blk, n_blk, kb0, kb1;
+  int m_blk, n_blk, kb0, kb1, split;
 };
 
-__device__ __forceinline__ Tile decode_tile(int t, int num_m, int num_n, int group_m, int kb_total, int kb_per) {
+__device__ __forceinline__ Tile decode_tile(int t, int num_m, int num_n, int group_m, int kb_total, int kb_per,
+                                            int splits, bool cluster_order) {
   const int per_split = num_m * num_n;
-  const int split = t / per_split;
-  const int r = t - split * per_split;
+  // cluster order: the splits of one output tile are consecutive CTAs (one cluster)
+  const int split = cluster_order ? t % splits : t / per_split;
+  const int r = cluster_order ? t / splits : t - split * per_split;
   const int width = group_m * num_n;
   const int group = r / width;
   const int first_m = group * group_m;
@@ -49,6 +59,7 @@ __device__ __forceinline__ Tile decode_tile(int t, int num_m, int num_n, int gro
   tl.n_blk = rr / gm;
   tl.kb0 = split * kb_per;
   tl.kb1 = min(kb_total, tl.kb0 + kb_per);
+  tl.split = split;
   return tl;
 }
 
@@ -85,12 +96,12 @@ __device__ __forceinline__ void store_row32<bf16>(bf16* dst, const float* v, int
   }
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, int MT>
 __global__ void __launch_bounds__(192, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_a1,
-              const __grid_constant__ CUtensorMap map_a2, const __grid_constant__ CUtensorMap map_b,
-              const GemmArgs p) {
-  using C = TcCfg<BN>;
+              const __grid_constant__ CUtensorMap map_a2, const GemmArgs p) {
+  using C = TcCfg<BN, MT>;
+  constexpr int TM = BM * MT;  // rows per tile
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
@@ -108,7 +119,7 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    for (int a = 0; a < 2; ++a) {
+    for (int a = 0; a < C::ACC; ++a) {
       mbar_init(&tfull[a], 1);
       mbar_init(&tempty[a], 128);
     }
@@ -119,7 +130,6 @@ __global__ void __launch_bounds__(192, 1)
     tma_prefetch_map(&map_a0);
     tma_prefetch_map(&map_a1);
     tma_prefetch_map(&map_a2);
-    tma_prefetch_map(&map_b);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -130,7 +140,7 @@ __global__ void __launch_bounds__(192, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int num_m = (p.M + BM - 1) / BM;
+  const int num_m = (p.M + TM - 1) / TM;
   const int num_n = (p.N + BN - 1) / BN;
   const int kb_total = (p.K + BK - 1) / BK;
   const int kb_per = (kb_total + p.splits - 1) / p.splits;
@@ -141,8 +151,14 @@ __global__ void __launch_bounds__(192, 1)
       int stage = 0;
       uint32_t phase = 0;
       for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
+        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per, p.splits, EPI == EPI_CLUSTER);
+        const bf16* btile = reinterpret_cast<const bf16*>(p.b) + (long long)tl.n_blk * BN * BK;
+        // weights streamed once: keep p.prefetch K blocks of B in flight toward L2
+        for (int kb = tl.kb0; kb < min(tl.kb1, tl.kb0 + p.prefetch); ++kb)
+          bulk_prefetch_l2(btile + (long long)kb * p.b_np * BK, C::B_BYTES);
         for (int kb = tl.kb0; kb < tl.kb1; ++kb) {
+          if (p.prefetch && kb + p.prefetch < tl.kb1)
+            bulk_prefetch_l2(btile + (long long)(kb + p.prefetch) * p.b_np * BK, C::B_BYTES);
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.err)) goto producer_done;
           uint8_t* sa = smem + stage * C::STAGE_BYTES;
           uint8_t* sb = sa + C::A_BYTES;
@@ -151,8 +167,11 @@ __global__ void __launch_bounds__(192, 1)
           const int piece = kg / p.k_per_map;
           const int kl = kg - piece * p.k_per_map;
           const CUtensorMap* am = piece == 0 ? &map_a0 : (piece == 1 ? &map_a1 : &map_a2);
-          tma_load_2d(sa, am, &full[stage], kl, tl.m_blk * BM);
-          tma_load_2d(sb, &map_b, &full[stage], kg, tl.n_blk * BN);
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt)
+            tma_load_2d(sa + mt * (BM * BK * 2), am, &full[stage], kl, tl.m_blk * TM + mt * BM);
+          bulk_load(sb, reinterpret_cast<const bf16*>(p.b) + ((long long)kb * p.b_np + tl.n_blk * BN) * BK,
+                    C::B_BYTES, &full[stage]);
           if (++stage == C::STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -169,21 +188,25 @@ __global__ void __launch_bounds__(192, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
+        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per, p.splits, EPI == EPI_CLUSTER);
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, p.err)) goto mma_done;
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * MT * BN);
         for (int kb = tl.kb0; kb < tl.kb1; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, p.err)) goto mma_done;
           tc_fence_after();
           const uint32_t a_addr = smem_u32(smem + stage * C::STAGE_BYTES);
           const uint32_t b_addr = a_addr + C::A_BYTES;
-          const uint64_t adesc = sw128_kmajor_desc(a_addr);
           const uint64_t bdesc = sw128_kmajor_desc(b_addr);
 #pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk) {
-            // advance 16 elements (32 bytes = 2 units of 16 bytes) along K
-            tc_mma_bf16(d_tmem, adesc + 2u * kk, bdesc + 2u * kk, idesc, (kb > tl.kb0 || kk > 0) ? 1u : 0u);
+          for (int mt = 0; mt < MT; ++mt) {
+            const uint64_t adesc = sw128_kmajor_desc(a_addr + mt * (BM * BK * 2));
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk) {
+              // advance 16 elements (32 bytes = 2 units of 16 bytes) along K
+              tc_mma_bf16(d_tmem + mt * BN, adesc + 2u * kk, bdesc + 2u * kk, idesc,
+                          (kb > tl.kb0 || kk > 0) ? 1u : 0u);
+            }
           }
           tc_commit(&empty[stage]);
           if (++stage == C::STAGES) {
@@ -192,36 +215,39 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
         tc_commit(&tfull[acc]);
-        if (++acc == 2) {
+        if (++acc == C::ACC) {
           acc = 0;
           acc_phase ^= 1u;
         }
       }
     mma_done:;
     }
-  } else {
+  } else if constexpr (EPI != EPI_CLUSTER) {
     // epilogue warps 2..5
     const int quarter = warp & 3;
     const int row_in_tile = quarter * 32 + lane;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-      const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
+      const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per, p.splits, EPI == EPI_CLUSTER);
       if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err)) break;
       tc_fence_after();
-      const int m = tl.m_blk * BM + row_in_tile;
+#pragma unroll 1
+      for (int mt = 0; mt < MT; ++mt) {
+      const int m = tl.m_blk * TM + mt * BM + row_in_tile;
       const bool row_ok = m < p.M;
-      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                             static_cast<uint32_t>((acc * MT + mt) * BN);
       if constexpr (EPI == EPI_SWIGLU) {
-        // tile columns [0, BN/2) are gate, [BN/2, BN) are up, for the same outputs
-        constexpr int HALF = BN / 2;
+        // B rows are interleaved in blocks of 32: tile columns [64j, 64j+32) are
+        // gate and [64j+32, 64j+64) up for the same 32 outputs
         const int n_out = p.N / 2;
-        for (int c = 0; c < HALF; c += 32) {
+        for (int c = 0; c < BN; c += 64) {
           uint32_t g[32], u[32];
           tmem_ld_32x32b_x32(tbase + c, g);
-          tmem_ld_32x32b_x32(tbase + HALF + c, u);
+          tmem_ld_32x32b_x32(tbase + c + 32, u);
           tmem_ld_wait();
-          const int n0 = tl.n_blk * HALF + c;
+          const int n0 = (tl.n_blk * BN + c) / 2;
           if (row_ok && n0 < n_out) {
             float v[32];
 #pragma unroll
@@ -275,12 +301,91 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
       }
+      }  // mt
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
-      if (++acc == 2) {
+      if (++acc == C::ACC) {
         acc = 0;
         acc_phase ^= 1u;
       }
+    }
+  }
+
+  if constexpr (EPI == EPI_CLUSTER) {
+    // One tile per CTA; the cluster's CTAs hold the K-split partial sums of the
+    // same output tile.  Per round of CW columns: every CTA stages its partial
+    // in its own shared memory (the pipeline ring is idle now), then each CTA
+    // adds up a contiguous column stripe across all CTAs of the cluster through
+    // DSMEM and writes it.  Every thread of every CTA passes every cluster
+    // barrier, also after an abort, so no CTA waits for one that left.
+    constexpr int CW = BN < 128 ? BN : 128;
+    constexpr int LD = CW + 4;  // padded row (floats): conflict-free row-wise staging
+    constexpr int G = CW / 4;   // float4 groups per row
+    __syncwarp();
+    const int S = p.splits;
+    const uint32_t rank = cluster_ctarank();
+    const Tile tl = decode_tile(blockIdx.x, num_m, num_n, p.group_m, kb_total, kb_per, p.splits, true);
+    bool have = false;
+    if (warp >= 2) {
+      have = mbar_wait(&tfull[0], 0, abort_flag, p.err);
+      tc_fence_after();
+    }
+    float* red = reinterpret_cast<float*>(smem);
+    const int per = (G + S - 1) / S;  // groups owned by each CTA
+    const int g0 = min(G, (int)rank * per);
+    const int g1 = min(G, g0 + per);
+    const int my_groups = g1 - g0;
+    const uint32_t red_addr = smem_u32(red);
+    for (int rd = 0; rd < BN / CW; ++rd) {
+      if (warp >= 2 && have) {
+        const int quarter = warp & 3;
+#pragma unroll 1
+        for (int mt = 0; mt < MT; ++mt) {
+          const int row = mt * BM + quarter * 32 + lane;
+          const uint32_t tb = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                              static_cast<uint32_t>(mt * BN + rd * CW);
+          for (int c = 0; c < CW; c += 32) {
+            uint32_t r[32];
+            tmem_ld_32x32b_x32(tb + c, r);
+            tmem_ld_wait();
+            float* dst = red + row * LD + c;
+#pragma unroll
+            for (int j = 0; j < 32; j += 4)
+              *reinterpret_cast<float4*>(dst + j) = make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]),
+                                                                __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3]));
+          }
+        }
+      }
+      cluster_sync_all();
+      if (!*abort_flag && my_groups > 0) {
+        const int items = TM * my_groups;
+        for (int it = threadIdx.x; it < items; it += blockDim.x) {
+          const int row = it / my_groups;
+          const int col = (g0 + it - row * my_groups) * 4;
+          const uint32_t off = red_addr + static_cast<uint32_t>((row * LD + col) * 4);
+          float4 acc = dsmem_ld_f4(dsmem_map(off, 0));
+          for (int q = 1; q < S; ++q) {
+            const float4 v = dsmem_ld_f4(dsmem_map(off, q));
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
+          }
+          const int m = tl.m_blk * TM + row;
+          const int n = tl.n_blk * BN + rd * CW + col;
+          if (m < p.M && n < p.N) {
+            if (p.residual) {
+              const float4 rv = *reinterpret_cast<const float4*>(p.residual + (long long)m * p.ldr + n);
+              acc.x += rv.x;
+              acc.y += rv.y;
+              acc.z += rv.z;
+              acc.w += rv.w;
+            }
+            *reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n) = acc;
+          }
+        }
+      }
+      cluster_sync_all();
     }
   }
 
@@ -293,43 +398,117 @@ __global__ void __launch_bounds__(192, 1)
   }
 }
 
-template <int BN, int EPI>
-cudaError_t launch_one(const CUtensorMap a_maps[3], const CUtensorMap& b_map, const GemmArgs& args, int num_sms,
+template <int BN, int EPI, int MT>
+cudaError_t launch_one(const CUtensorMap a_maps[3], const GemmArgs& args, int num_sms,
                        cudaStream_t stream) {
-  using C = TcCfg<BN>;
-  auto kern = k_gemm_tc<BN, EPI>;
+  using C = TcCfg<BN, MT>;
+  auto kern = k_gemm_tc<BN, EPI, MT>;
   static bool attr_set = false;  // per (BN, EPI) instantiation
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  const long long tiles = (long long)((args.M + BM - 1) / BM) * ((args.N + BN - 1) / BN) * args.splits;
+  const long long tiles = (long long)((args.M + BM * MT - 1) / (BM * MT)) * ((args.N + BN - 1) / BN) * args.splits;
   const int grid = (int)(tiles < num_sms ? tiles : num_sms);
   if (grid <= 0) return cudaSuccess;
-  kern<<<grid, 192, C::SMEM, stream>>>(a_maps[0], a_maps[1], a_maps[2], b_map, args);
+  kern<<<grid, 192, C::SMEM, stream>>>(a_maps[0], a_maps[1], a_maps[2], args);
   return cudaGetLastError();
+}
+
+template <int BN, int MT>
+cudaError_t launch_cluster(const CUtensorMap a_maps[3], const GemmArgs& args,
+                           cudaStream_t stream) {
+  using C = TcCfg<BN, MT>;
+  auto kern = k_gemm_tc<BN, EPI_CLUSTER, MT>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int tiles = ((args.M + BM * MT - 1) / (BM * MT)) * ((args.N + BN - 1) / BN);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(tiles * args.splits);
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = stream;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = args.splits;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a_maps[0], a_maps[1], a_maps[2], args);
+}
+
+template <int BN, int MT>
+int cluster_capacity(int splits) {
+  using C = TcCfg<BN, MT>;
+  auto kern = k_gemm_tc<BN, EPI_CLUSTER, MT>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(splits * 64);
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = splits;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
 }
 
 }  // namespace
 
-cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], const CUtensorMap& b_map, int bn, int epi,
-                           const GemmArgs& args, int num_sms, cudaStream_t stream) {
-#define OUTLETS_TC_CASE(BNV, EV) \
-  if (bn == BNV && epi == EV) return launch_one<BNV, EV>(a_maps, b_map, args, num_sms, stream);
-  OUTLETS_TC_CASE(256, EPI_F32)
-  OUTLETS_TC_CASE(256, EPI_ACT)
-  OUTLETS_TC_CASE(256, EPI_SWIGLU)
-  OUTLETS_TC_CASE(256, EPI_BIAS_RELU)
-  OUTLETS_TC_CASE(256, EPI_ATOMIC)
-  OUTLETS_TC_CASE(128, EPI_F32)
-  OUTLETS_TC_CASE(128, EPI_ACT)
-  OUTLETS_TC_CASE(128, EPI_BIAS_RELU)
-  OUTLETS_TC_CASE(128, EPI_ATOMIC)
-  OUTLETS_TC_CASE(64, EPI_F32)
-  OUTLETS_TC_CASE(64, EPI_ACT)
-  OUTLETS_TC_CASE(64, EPI_BIAS_RELU)
-  OUTLETS_TC_CASE(64, EPI_ATOMIC)
+cudaError_t gemm_tc_cluster_launch(const CUtensorMap a_maps[3], int bn, int mt, const GemmArgs& args,
+                                   cudaStream_t stream) {
+  if (args.splits < 1 || args.splits > 8) return cudaErrorInvalidValue;
+  if (bn == 256 && mt == 2) return launch_cluster<256, 2>(a_maps, args, stream);
+  if (bn == 256 && mt == 1) return launch_cluster<256, 1>(a_maps, args, stream);
+  if (bn == 128 && mt == 2) return launch_cluster<128, 2>(a_maps, args, stream);
+  if (bn == 128 && mt == 1) return launch_cluster<128, 1>(a_maps, args, stream);
+  return cudaErrorInvalidValue;
+}
+
+int gemm_tc_cluster_capacity(int bn, int mt, int splits) {
+  if (bn == 256 && mt == 2) return cluster_capacity<256, 2>(splits);
+  if (bn == 256 && mt == 1) return cluster_capacity<256, 1>(splits);
+  if (bn == 128 && mt == 2) return cluster_capacity<128, 2>(splits);
+  if (bn == 128 && mt == 1) return cluster_capacity<128, 1>(splits);
+  return 0;
+}
+
+cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args, int num_sms,
+                           cudaStream_t stream) {
+#define OUTLETS_TC_CASE(BNV, EV, MTV) \
+  if (bn == BNV && epi == EV && mt == MTV) return launch_one<BNV, EV, MTV>(a_maps, args, num_sms, stream);
+  // large M (prefill): one 128-row sub-tile per tile, two TMEM accumulators
+  OUTLETS_TC_CASE(256, EPI_F32, 1)
+  OUTLETS_TC_CASE(256, EPI_ACT, 1)
+  OUTLETS_TC_CASE(256, EPI_SWIGLU, 1)
+  OUTLETS_TC_CASE(128, EPI_F32, 1)
+  OUTLETS_TC_CASE(128, EPI_ACT, 1)
+  OUTLETS_TC_CASE(64, EPI_F32, 1)
+  OUTLETS_TC_CASE(64, EPI_ACT, 1)
+  OUTLETS_TC_CASE(64, EPI_BIAS_RELU, 1)
+  // small M (dynamic prediction): fused SwiGLU, one wave of tiles
+  OUTLETS_TC_CASE(256, EPI_SWIGLU, 2)
+  OUTLETS_TC_CASE(192, EPI_SWIGLU, 2)
+  OUTLETS_TC_CASE(192, EPI_SWIGLU, 1)
+  OUTLETS_TC_CASE(128, EPI_SWIGLU, 2)
+  OUTLETS_TC_CASE(128, EPI_SWIGLU, 1)
 #undef OUTLETS_TC_CASE
   return cudaErrorInvalidValue;
 }

@@ -22,16 +22,27 @@ enum : int {
 enum Epi : int {
   EPI_F32 = 0,        // out f32 = acc (+ residual f32)
   EPI_ACT = 1,        // out act (bf16 on the tensor-core path, f32 on the CUDA-core path) = acc
-  EPI_SWIGLU = 2,     // B rows interleaved in blocks of 128 [gate | up]; out act = silu(g) * u
+  EPI_SWIGLU = 2,     // B rows interleaved in blocks of 32 [gate | up]; out act = silu(g) * u
   EPI_BIAS_RELU = 3,  // out f32 = max(acc + bias, 0)
   EPI_ATOMIC = 4,     // out f32 += acc (split-K partial sums)
+  EPI_CLUSTER = 6,    // split-K inside a thread-block cluster, reduced through DSMEM: out f32 = sum (+ residual)
 };
 
+// B operands (weights) live in a k-block-major, pre-swizzled layout owned by the
+// library: element (n, k) of a [N, K] weight is stored at
+//   ((k / 64) * b_np + n) * 64 + (((k % 64) / 8) ^ (n % 8)) * 8 + k % 8
+// with b_np >= every tile's last row (zero rows beyond N).  A tile of BN rows of
+// one 64-wide K block is then one contiguous run of BN * 128 bytes, already in
+// the 128-byte-swizzled order the tensor-core descriptors expect, loaded by one
+// bulk copy.
 struct GemmArgs {
   int M, N, K;
+  const void* b;          // weights, layout above
+  long long b_np;         // padded rows per K block
   int k_per_map;          // K extent of each A piece (multiple of 64 when pieces > 1)
   int splits;             // split-K factor (> 1 only with EPI_ATOMIC); every split non-empty
   int group_m;            // tile raster: M blocks per group
+  int prefetch;           // K blocks of B to prefetch into L2 ahead of the smem ring (0 = off)
   void* out;
   long long ldo;          // elements
   const float* residual;  // EPI_F32 only, may be null
@@ -41,9 +52,17 @@ struct GemmArgs {
 };
 
 // tcgen05 path (bf16 operands).  a_maps: 3 tensor maps over the A pieces (box
-// 64 x 128), b_map: tensor map over B (box 64 x bn).  grid = min(tiles, num_sms).
-cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], const CUtensorMap& b_map, int bn, int epi,
-                           const GemmArgs& args, int num_sms, cudaStream_t stream);
+// 64 x 128).  mt: 128-row sub-tiles per tile (1 or 2).  grid = min(tiles, num_sms).
+cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args, int num_sms,
+                           cudaStream_t stream);
+
+// Split-K GEMM whose args.splits CTAs per output tile form one cluster and add
+// their accumulators through distributed shared memory (EPI_CLUSTER): every
+// output element is written once, in a fixed order.  args.splits <= 8.
+cudaError_t gemm_tc_cluster_launch(const CUtensorMap a_maps[3], int bn, int mt, const GemmArgs& args,
+                                   cudaStream_t stream);
+// Most clusters of `splits` CTAs of that kernel that can be resident at once (0 if unknown).
+int gemm_tc_cluster_capacity(int bn, int mt, int splits);
 
 // CUDA-core path of the f32 configuration.  a[0..2]: A pieces with row stride k_per_map.
 cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int epi, const GemmArgs& args,
@@ -58,6 +77,13 @@ cudaError_t rmsnorm_launch(const float* x, const float* g, Act* y, float* copy_o
 // y[i] = norm(x[row_index[i]]).
 template <typename Act>
 cudaError_t rmsnorm_gather_launch(const float* x, const int* row_index, const float* g, Act* y, int rows, int d,
+                                  float eps, cudaStream_t stream);
+
+// v[i] = residual[src] + sum_s x[s * split_stride + src], src = row_index ? row_index[i] : i;
+// y[i] = norm(v[i]) * g; copy_out[i] = v[i] when copy_out is given.
+template <typename Act>
+cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_stride, const float* residual,
+                                  const int* row_index, const float* g, Act* y, float* copy_out, int rows, int d,
                                   float eps, cudaStream_t stream);
 
 struct RopeArgs {
@@ -78,25 +104,30 @@ struct RopeArgs {
   const int* page_list;  // pages of each sequence/request, concatenated
   const int* page_off;   // [B+1] (prefill: per sequence; step: per row)
   int page_tokens;
+  int n_split;           // qkv holds n_split slices (split-K partial sums) to add up
+  long long split_stride;
   int* err;
 };
 template <typename In, typename Act>
 cudaError_t rope_scatter_launch(const In* qkv, const RopeArgs& a, cudaStream_t stream);
 
-// u[r, j] = silu(gu[r, gate(j)]) * gu[r, up(j)], gu interleaved in blocks of 128.
+// u[r, j] = silu(gu[r, gate(j)]) * gu[r, up(j)], gu interleaved in blocks of 32.
 template <typename Act>
 cudaError_t swiglu_launch(const float* gu, Act* u, int rows, int f_pad, cudaStream_t stream);
 
-// z[r] = w_last . a(h[r]) + b_last, a(x) = relu(x + b_prev) (identity if b_prev is null);
-// len[r] = max(0, expm1(z[r])).
-cudaError_t head_tail_launch(const float* h_pre, const float* b_prev, const float* w_last, const float* b_last,
-                             int rows, int width, float* z, float* len, cudaStream_t stream);
+// h[r] = sum_s h_pre[s * split_stride + r]; z[r] = w_last . a(h[r]) + b_last with
+// a(x) = relu(x + b_prev) (identity if b_prev is null); len[r] = max(0, expm1(z[r])).
+cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_stride, const float* b_prev,
+                             const float* w_last, const float* b_last, int rows, int width, float* z, float* len,
+                             cudaStream_t stream);
 
-// dst[map(r)][c] = src[r][c] (f32 -> Act); row_mode 0: row_base + r, 1: gate rows, 2: up rows
-// of the [gate | up] interleave (blocks of 128).
+// dst row map(row_base + r) <- src row r (f32 -> Act); map: row_mode 0 identity,
+// 1 gate rows, 2 up rows of the [gate 32 | up 32] interleave.  kb_np == 0:
+// row-major with row stride dst_ld; kb_np > 0: the k-block-major swizzled
+// weight layout of GemmArgs with b_np = kb_np.
 template <typename Act>
 cudaError_t convert_rows_launch(const float* src, Act* dst, int rows, int cols, long long dst_ld, int row_mode,
-                                int row_base, cudaStream_t stream);
+                                int row_base, long long kb_np, cudaStream_t stream);
 
 // ---------------------------------------------------------------- attention
 struct AttnTile {

@@ -19,6 +19,7 @@
 #include <cstring>
 #include <mutex>
 #include <string>
+#include <unordered_map>
 #include <vector>
 
 #include "kernels.h"
@@ -64,6 +65,25 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, ui
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Memo of encoded tensor maps: weights and workspace buffers are re-used by
+// every call with the same shapes, so their maps are encoded once.
+struct MapKey {
+  const void* base;
+  uint64_t cols, rows, ld;
+  uint32_t box_rows;
+  bool operator==(const MapKey& o) const {
+    return base == o.base && cols == o.cols && rows == o.rows && ld == o.ld && box_rows == o.box_rows;
+  }
+};
+struct MapKeyHash {
+  size_t operator()(const MapKey& k) const {
+    size_t h = std::hash<const void*>()(k.base);
+    h ^= std::hash<uint64_t>()(k.cols * 1000003ull + k.rows * 7919ull + k.ld * 131ull + k.box_rows) + 0x9e3779b9 +
+         (h << 6) + (h >> 2);
+    return h;
+  }
+};
+
 bool is_device_ptr(const void* p) {
   cudaPointerAttributes at;
   if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
@@ -90,6 +110,8 @@ struct outlets_ctx {
 
   void *w_proj = nullptr, *w_qkv = nullptr, *w_o = nullptr, *w_gu = nullptr, *w_down = nullptr,
        *head_w0 = nullptr;
+  // padded rows per K block of each weight in the k-block-major layout (bf16 path; 0 = row-major)
+  long long np_proj = 0, np_qkv = 0, np_o = 0, np_gu = 0, np_down = 0, np_h0 = 0;
   float *g_in = nullptr, *g_post = nullptr, *g_final = nullptr;
   std::vector<float*> head_wf, head_b;
   float *rope_cos = nullptr, *rope_sin = nullptr;
@@ -100,6 +122,8 @@ struct outlets_ctx {
        *attn = nullptr, *u = nullptr, *hn = nullptr;
   void* taps_stage[3] = {nullptr, nullptr, nullptr};
   int* err_dev = nullptr;
+  float* part = nullptr;  // f32 QKV rows of the small-M path
+  size_t part_floats = 0;
   int* meta_dev = nullptr;
   size_t meta_cap = 0;  // ints
 
@@ -115,6 +139,8 @@ struct outlets_ctx {
 
   int last_rows = 0, last_out_rows = 0;
   bool oom = false;
+  std::unordered_map<MapKey, CUtensorMap, MapKeyHash> map_cache;  // library-owned buffers only
+  std::unordered_map<int, int> cluster_cap;                       // resident clusters per GEMM shape
 
   // stage timing and launch accounting
   struct ProfRec {
@@ -196,25 +222,27 @@ struct outlets_kv {
 
 namespace {
 
+// True for buffers the context allocated itself (their tensor maps may be memoized).
+bool owned_by(const outlets_ctx* c, const void* p) {
+  for (void* q : c->allocs)
+    if (q == p) return true;
+  for (int i = 0; i < 3; ++i)
+    if (c->taps_stage[i] == p) return true;
+  return false;
+}
+
 // Uploads a host f32 matrix [rows, cols] through a device staging buffer and
-// converts it (f32 -> act) into dst with the given row mapping.
+// converts it (f32 -> act) into dst with the given row mapping and layout
+// (kb_np > 0: k-block-major swizzled weight layout, else row-major, stride dst_ld).
 outlets_status upload_rows(outlets_ctx* c, const float* src, int rows, int cols, void* dst, long long dst_ld,
-                           int row_mode, int row_base, float* stage, size_t stage_floats) {
+                           int row_mode, int row_base, long long kb_np, float* stage, size_t stage_floats) {
   const int chunk = (int)std::max<size_t>(1, stage_floats / (size_t)cols);
   for (int r0 = 0; r0 < rows; r0 += chunk) {
     const int n = std::min(chunk, rows - r0);
     OUT_CK(c, cudaMemcpy(stage, src + (size_t)r0 * cols, (size_t)n * cols * 4, cudaMemcpyHostToDevice));
-    // rows r0.. map like global rows: shift the mapping by r0
-    cudaError_t e;
-    if (row_mode == 0) {
-      e = c->bf16 ? convert_rows_launch<bf16>(stage, (bf16*)dst, n, cols, dst_ld, 0, row_base + r0, 0)
-                  : convert_rows_launch<float>(stage, (float*)dst, n, cols, dst_ld, 0, row_base + r0, 0);
-    } else {
-      // chunk boundaries are multiples of 128 rows (see caller) so the interleave maps locally
-      const long long off = (long long)(r0 >> 7) * 256 * dst_ld;
-      e = c->bf16 ? convert_rows_launch<bf16>(stage, (bf16*)dst + off, n, cols, dst_ld, row_mode, 0, 0)
-                  : convert_rows_launch<float>(stage, (float*)dst + off, n, cols, dst_ld, row_mode, 0, 0);
-    }
+    const cudaError_t e =
+        c->bf16 ? convert_rows_launch<bf16>(stage, (bf16*)dst, n, cols, dst_ld, row_mode, row_base + r0, kb_np, 0)
+                : convert_rows_launch<float>(stage, (float*)dst, n, cols, dst_ld, row_mode, row_base + r0, kb_np, 0);
     OUT_CK(c, e);
     OUT_CK(c, cudaDeviceSynchronize());
   }
@@ -230,7 +258,7 @@ outlets_status validate_config(const outlets_config* cfg, std::string& why) {
   if (cfg->d_model <= 0 || cfg->d_model % 64) return bad("d_model must be a positive multiple of 64");
   if (cfg->n_heads <= 0 || cfg->n_kv_heads <= 0 || cfg->n_heads % cfg->n_kv_heads)
     return bad("n_heads must be a positive multiple of n_kv_heads");
-  if (cfg->head_dim <= 0 || cfg->head_dim % 2) return bad("head_dim must be positive and even");
+  if (cfg->head_dim <= 0 || cfg->head_dim % 16) return bad("head_dim must be a positive multiple of 16");
   if ((cfg->n_heads * cfg->head_dim) % 64) return bad("n_heads * head_dim must be a multiple of 64");
   if (cfg->ffn_dim <= 0) return bad("ffn_dim must be positive");
   if (cfg->n_head_hidden < 1 || cfg->n_head_hidden > OUTLETS_MAX_HEAD_HIDDEN)
@@ -299,32 +327,62 @@ struct MetaBuilder {
   size_t put(const std::vector<int>& x) { return put(x.data(), x.size()); }
 };
 
-// bf16 GEMM through tcgen05.  A pieces: row-major [M, k_piece] with row stride lda.
-outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
-                       const void* b, int N, int K, int epi, void* out, long long ldo, const float* residual,
-                       long long ldr, const float* bias, cudaStream_t s) {
-  if (M == 0) return OUTLETS_OK;
-  int bn = 256;
-  if (epi != EPI_SWIGLU) {
-    auto tiles = [&](int bnv) { return cdiv(M, 128) * cdiv(N, bnv); };
-    if (tiles(256) >= c->num_sms) bn = 256;
-    else if (tiles(128) >= c->num_sms) bn = 128;
-    else bn = 64;
+// Tensor map of a library-owned buffer (weights, workspace): encoded once.
+bool cached_map(outlets_ctx* c, CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld,
+                uint32_t box_rows) {
+  const MapKey k{base, cols, rows, ld, box_rows};
+  auto it = c->map_cache.find(k);
+  if (it != c->map_cache.end()) {
+    *m = it->second;
+    return true;
   }
-  CUtensorMap am[3], bm;
+  if (!make_map(m, base, cols, rows, ld, box_rows)) return false;
+  if (c->map_cache.size() > 4096) c->map_cache.clear();
+  c->map_cache.emplace(k, *m);
+  return true;
+}
+
+bool owned_by(const outlets_ctx* c, const void* p);
+
+#define OUT_TRY(expr)                      \
+  do {                                     \
+    outlets_status st_ = (expr);           \
+    if (st_ != OUTLETS_OK) return st_;     \
+  } while (0)
+
+// Tensor maps of the (up to three) A pieces of a GEMM.
+outlets_status a_maps(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
+                      CUtensorMap* am) {
   for (int i = 0; i < 3; ++i) {
     const void* base = a[i < n_pieces ? i : 0];
-    if (!make_map(&am[i], base, (uint64_t)k_piece, (uint64_t)M, (uint64_t)lda, 128))
-      return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for a GEMM A operand");
+    if (i > 0 && n_pieces == 1) {
+      am[i] = am[0];
+      continue;
+    }
+    const bool ok = owned_by(c, base) ? cached_map(c, &am[i], base, (uint64_t)k_piece, (uint64_t)M, (uint64_t)lda, 128)
+                                      : make_map(&am[i], base, (uint64_t)k_piece, (uint64_t)M, (uint64_t)lda, 128);
+    if (!ok) return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for a GEMM A operand");
   }
-  if (!make_map(&bm, b, (uint64_t)K, (uint64_t)N, (uint64_t)K, (uint32_t)bn))
-    return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for a GEMM B operand");
+  return OUTLETS_OK;
+}
+
+// bf16 GEMM through tcgen05 with an explicit tile plan.  A pieces: row-major
+// [M, k_piece] with row stride lda.
+outlets_status gemm_tc_ex(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
+                          const void* b, long long b_np, int N, int K, int epi, int bn, int mt, int splits, void* out,
+                          long long ldo, const float* residual, long long ldr, const float* bias, cudaStream_t s) {
+  if (M == 0) return OUTLETS_OK;
+  CUtensorMap am[3];
+  OUT_TRY(a_maps(c, a, n_pieces, k_piece, lda, M, am));
   GemmArgs g{};
   g.M = M;
   g.N = N;
   g.K = K;
+  g.b = b;
+  g.b_np = b_np;
   g.k_per_map = k_piece;
-  g.splits = 1;
+  g.splits = splits;
+  g.prefetch = M <= 256 ? 8 : 0;  // small M streams every weight tile once
   g.group_m = 16;
   g.out = out;
   g.ldo = ldo;
@@ -332,9 +390,67 @@ outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k
   g.ldr = ldr;
   g.bias = bias;
   g.err = c->err_dev;
-  OUT_CK(c, gemm_tc_launch(am, bm, bn, epi, g, c->num_sms, s));
+  OUT_CK(c, gemm_tc_launch(am, bn, epi, mt, g, c->num_sms, s));
   return OUTLETS_OK;
 }
+
+// Large-M GEMM (prefill): 128-row tiles, tile width chosen to fill the SMs.
+outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
+                       const void* b, long long b_np, int N, int K, int epi, void* out, long long ldo,
+                       const float* residual, long long ldr, const float* bias, cudaStream_t s) {
+  int bn = 256;
+  if (epi != EPI_SWIGLU) {
+    auto tiles = [&](int bnv) { return cdiv(M, 128) * cdiv(N, bnv); };
+    if (tiles(256) >= c->num_sms) bn = 256;
+    else if (tiles(128) >= c->num_sms) bn = 128;
+    else bn = 64;
+  }
+  return gemm_tc_ex(c, a, n_pieces, k_piece, lda, M, b, b_np, N, K, epi, bn, 1, 1, out, ldo, residual, ldr, bias, s);
+}
+
+// Small-M GEMM with the K splits of each output tile reduced inside a
+// thread-block cluster (DSMEM): out f32 [M, N] = A B^T (+ residual), written once.
+outlets_status gemm_cluster(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
+                            const void* b, long long b_np, int N, int K, float* out, long long ldo,
+                            const float* residual, long long ldr, cudaStream_t s) {
+  if (M == 0) return OUTLETS_OK;
+  const int mt = M <= 128 ? 1 : 2;
+  const int bn = cdiv(N, 256) >= 8 ? 256 : 128;
+  const long long n_tiles = cdiv(N, bn);
+  const long long kb = cdiv(K, 64);
+  int sp = (int)std::max<long long>(1, std::min<long long>(std::min<long long>(8, c->num_sms / n_tiles), kb));
+  // keep every cluster resident in one wave when the hardware allows it
+  while (sp > 1) {
+    const int key = bn * 100 + mt * 10 + sp;
+    auto it = c->cluster_cap.find(key);
+    const int cap = it != c->cluster_cap.end() ? it->second : (c->cluster_cap[key] = gemm_tc_cluster_capacity(bn, mt, sp));
+    if (cap >= n_tiles) break;
+    --sp;
+  }
+  const long long kb_per = cdiv(kb, sp);
+  sp = (int)cdiv(kb, kb_per);
+  CUtensorMap am[3];
+  OUT_TRY(a_maps(c, a, n_pieces, k_piece, lda, M, am));
+  GemmArgs g{};
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.k_per_map = k_piece;
+  g.b = b;
+  g.b_np = b_np;
+  g.splits = sp;
+  g.group_m = 1;
+  g.prefetch = 8;
+  g.out = out;
+  g.ldo = ldo;
+  g.residual = residual;
+  g.ldr = ldr;
+  g.err = c->err_dev;
+  OUT_CK(c, gemm_tc_cluster_launch(am, bn, mt, g, s));
+  return OUTLETS_OK;
+}
+
+inline bool small_path(const outlets_ctx* c, int M) { return c->bf16 && M <= 256; }
 
 outlets_status gemm_f32(outlets_ctx* c, const void* const* a, int k_piece, int M, const void* b, int N, int K,
                         int epi, void* out, long long ldo, const float* residual, long long ldr, const float* bias,
@@ -357,39 +473,52 @@ outlets_status gemm_f32(outlets_ctx* c, const void* const* a, int k_piece, int M
   return OUTLETS_OK;
 }
 
-#define OUT_TRY(expr)                      \
-  do {                                     \
-    outlets_status st_ = (expr);           \
-    if (st_ != OUTLETS_OK) return st_;     \
-  } while (0)
 
 // Everything after attention: O projection + residual, post-attention norm,
 // SwiGLU MLP + residual, final norm of the predicted rows, length head.
 outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_row_idx_dev, float* z_dev,
                         float* len_dev, cudaStream_t s) {
   const int d = c->d;
-  // O projection + residual: a = f + attn W_o^T
+  const float eps = c->cfg.rms_eps;
+  const bool small = small_path(c, rows);
+  // O projection + residual: a = f + attn W_o^T; post-attention RMSNorm
   c->stage_begin(OUTLETS_S_O);
   {
     const void* a1[3] = {c->attn, c->attn, c->attn};
-    if (c->bf16)
-      OUT_TRY(gemm_tc(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d,
+    if (small)
+      OUT_TRY(gemm_cluster(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, c->a, d, c->f, d, s));
+    else if (c->bf16)
+      OUT_TRY(gemm_tc(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d,
                       nullptr, s));
     else
       OUT_TRY(gemm_f32(c, a1, c->attn_w, rows, c->w_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d, nullptr, s));
   }
   c->stage_end(1);
-  // post-attention RMSNorm
   c->stage_begin(OUTLETS_S_NORM_POST);
-  if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->a, c->g_post, (bf16*)c->ahat, nullptr, rows, d, c->cfg.rms_eps, s));
-  else OUT_CK(c, rmsnorm_launch<float>(c->a, c->g_post, (float*)c->ahat, nullptr, rows, d, c->cfg.rms_eps, s));
+  if (c->bf16)
+    OUT_CK(c, rmsnorm_launch<bf16>(c->a, c->g_post, (bf16*)c->ahat, nullptr, rows, d, eps, s));
+  else
+    OUT_CK(c, rmsnorm_launch<float>(c->a, c->g_post, (float*)c->ahat, nullptr, rows, d, eps, s));
   c->stage_end(1);
   // gate/up + SwiGLU
   c->stage_begin(OUTLETS_S_GATEUP);
   {
     const void* a1[3] = {c->ahat, c->ahat, c->ahat};
-    if (c->bf16) {
-      OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_gu, 2 * c->Fp, d, EPI_SWIGLU, c->u, c->Fp, nullptr, 0, nullptr, s));
+    if (small) {
+      // one wave of tiles: the width (multiple of 64) that minimizes waves x width
+      int best_bn = 256;
+      long long best = -1;
+      for (int bnv : {256, 192, 128}) {
+        const long long cost = cdiv(cdiv(2 * c->Fp, bnv), c->num_sms) * bnv;
+        if (best < 0 || cost < best) {
+          best = cost;
+          best_bn = bnv;
+        }
+      }
+      OUT_TRY(gemm_tc_ex(c, a1, 1, d, d, rows, c->w_gu, c->np_gu, 2 * c->Fp, d, EPI_SWIGLU, best_bn,
+                         rows <= 128 ? 1 : 2, 1, c->u, c->Fp, nullptr, 0, nullptr, s));
+    } else if (c->bf16) {
+      OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_gu, c->np_gu, 2 * c->Fp, d, EPI_SWIGLU, c->u, c->Fp, nullptr, 0, nullptr, s));
     } else {
       OUT_TRY(gemm_f32(c, a1, d, rows, c->w_gu, 2 * c->Fp, d, EPI_F32, c->gu32, 2 * c->Fp, nullptr, 0, nullptr, s));
       OUT_CK(c, swiglu_launch<float>(c->gu32, (float*)c->u, rows, c->Fp, s));
@@ -401,8 +530,10 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   c->stage_begin(OUTLETS_S_DOWN);
   {
     const void* a1[3] = {c->u, c->u, c->u};
-    if (c->bf16)
-      OUT_TRY(gemm_tc(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, d, c->Fp, EPI_F32, c->y, d, c->a, d, nullptr, s));
+    if (small)
+      OUT_TRY(gemm_cluster(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, c->np_down, d, c->Fp, c->y, d, c->a, d, s));
+    else if (c->bf16)
+      OUT_TRY(gemm_tc(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, c->np_down, d, c->Fp, EPI_F32, c->y, d, c->a, d, nullptr, s));
     else
       OUT_TRY(gemm_f32(c, a1, c->Fp, rows, c->w_down, d, c->Fp, EPI_F32, c->y, d, c->a, d, nullptr, s));
   }
@@ -410,25 +541,27 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   // final RMSNorm of the predicted rows -> h^draft
   c->stage_begin(OUTLETS_S_FINAL_NORM);
   if (c->bf16)
-    OUT_CK(c, rmsnorm_gather_launch<bf16>(c->y, out_row_idx_dev, c->g_final, (bf16*)c->hn, out_rows, d,
-                                          c->cfg.rms_eps, s));
+    OUT_CK(c, rmsnorm_gather_launch<bf16>(c->y, out_row_idx_dev, c->g_final, (bf16*)c->hn, out_rows, d, eps, s));
   else
-    OUT_CK(c, rmsnorm_gather_launch<float>(c->y, out_row_idx_dev, c->g_final, (float*)c->hn, out_rows, d,
-                                           c->cfg.rms_eps, s));
+    OUT_CK(c, rmsnorm_gather_launch<float>(c->y, out_row_idx_dev, c->g_final, (float*)c->hn, out_rows, d, eps, s));
   c->stage_end(1);
   // length head: Linear+ReLU layers, then the output row
   c->stage_begin(OUTLETS_S_HEAD);
   const int nl = (int)c->head_dims.size() - 1;
-  float* cur = c->h1a;
-  {
-    const void* a1[3] = {c->hn, c->hn, c->hn};
-    const int w1 = c->head_dims[1];
-    if (c->bf16)
-      OUT_TRY(gemm_tc(c, a1, 1, d, d, out_rows, c->head_w0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0,
-                      c->head_b[0], s));
-    else
-      OUT_TRY(gemm_f32(c, a1, d, out_rows, c->head_w0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0, c->head_b[0], s));
+  const int w1 = c->head_dims[1];
+  const void* ah[3] = {c->hn, c->hn, c->hn};
+  if (small_path(c, out_rows) && nl == 2) {
+    OUT_TRY(gemm_cluster(c, ah, 1, d, d, out_rows, c->head_w0, c->np_h0, w1, d, c->h1a, w1, nullptr, 0, s));
+    OUT_CK(c, head_tail_launch(c->h1a, 1, 0, c->head_b[0], c->head_wf[1], c->head_b[1], out_rows, w1, z_dev, len_dev,
+                               s));
+    c->stage_end(2);
+    return OUTLETS_OK;
   }
+  float* cur = c->h1a;
+  if (c->bf16)
+    OUT_TRY(gemm_tc(c, ah, 1, d, d, out_rows, c->head_w0, c->np_h0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0, c->head_b[0], s));
+  else
+    OUT_TRY(gemm_f32(c, ah, d, out_rows, c->head_w0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0, c->head_b[0], s));
   for (int i = 1; i < nl - 1; ++i) {
     float* nxt = (cur == c->h1a) ? c->h1b : c->h1a;
     const void* a1[3] = {cur, cur, cur};
@@ -436,9 +569,61 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
                      EPI_BIAS_RELU, nxt, c->head_dims[i + 1], nullptr, 0, c->head_b[i], s));
     cur = nxt;
   }
-  OUT_CK(c, head_tail_launch(cur, nullptr, c->head_wf[nl - 1], c->head_b[nl - 1], out_rows, c->head_dims[nl - 1],
-                             z_dev, len_dev, s));
+  OUT_CK(c, head_tail_launch(cur, 1, 0, nullptr, c->head_wf[nl - 1], c->head_b[nl - 1], out_rows,
+                             c->head_dims[nl - 1], z_dev, len_dev, s));
   c->stage_end(nl);
+  return OUTLETS_OK;
+}
+
+// FC (Eq. 1) -> input RMSNorm -> QKV projection.  Fills the input side of the
+// RoPE arguments (fused qkv rows, or split slices on the small-M path).
+struct QkvSrc {
+  const void* p;
+  bool f32;
+  int n_split;
+  long long stride;
+};
+
+outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvSrc* q, cudaStream_t s) {
+  const int d = c->d;
+  const float eps = c->cfg.rms_eps;
+  const bool small = small_path(c, rows);
+  c->stage_begin(OUTLETS_S_FC);
+  if (small) OUT_TRY(gemm_cluster(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, c->f, d, nullptr, 0, s));
+  else if (c->bf16) OUT_TRY(gemm_tc(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
+  else OUT_TRY(gemm_f32(c, tp, d, rows, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
+  c->stage_end(1);
+  c->stage_begin(OUTLETS_S_NORM_IN);
+  if (c->bf16)
+    OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xhat, nullptr, rows, d, eps, s));
+  else
+    OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
+  c->stage_end(1);
+  c->stage_begin(OUTLETS_S_QKV);
+  const void* a1[3] = {c->xhat, c->xhat, c->xhat};
+  if (small) {
+    OUT_TRY(gemm_cluster(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, c->part, c->qkv_n, nullptr, 0, s));
+    *q = {c->part, true, 1, 0};
+  } else if (c->bf16) {
+    OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, EPI_ACT, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
+    *q = {c->qkv, false, 1, 0};
+  } else {
+    OUT_TRY(gemm_f32(c, a1, d, rows, c->w_qkv, c->qkv_n, d, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
+    *q = {c->qkv, true, 1, 0};
+  }
+  c->stage_end(1);
+  return OUTLETS_OK;
+}
+
+outlets_status launch_rope(outlets_ctx* c, const QkvSrc& q, RopeArgs& ra, cudaStream_t s) {
+  ra.n_split = q.n_split;
+  ra.split_stride = q.stride;
+  if (c->bf16) {
+    if (q.f32) OUT_CK(c, rope_scatter_launch<float, bf16>((const float*)q.p, ra, s));
+    else OUT_CK(c, rope_scatter_launch<bf16, bf16>((const bf16*)q.p, ra, s));
+  } else {
+    OUT_CK(c, rope_scatter_launch<float, float>((const float*)q.p, ra, s));
+  }
   return OUTLETS_OK;
 }
 
@@ -529,19 +714,28 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   };
   const int d = c->d;
   const size_t es = c->esz;
-  // ---- weights
-  c->w_proj = c->alloc((size_t)d * 3 * d * es);
-  c->w_qkv = c->alloc((size_t)c->qkv_n * d * es);
-  c->w_o = c->alloc((size_t)d * c->attn_w * es);
-  c->w_gu = c->alloc((size_t)2 * c->Fp * d * es);
-  c->w_down = c->alloc((size_t)d * c->Fp * es);
+  // ---- weights (bf16: k-block-major swizzled, rows padded to a multiple of 768 =
+  // lcm of the tile widths 64..256, so every tile's bulk copy stays in bounds)
+  auto np_of = [&](int n) -> long long { return c->bf16 ? cdiv(n, 768) * 768 : 0; };
+  c->np_proj = np_of(d);
+  c->np_qkv = np_of(c->qkv_n);
+  c->np_o = np_of(d);
+  c->np_gu = np_of(2 * c->Fp);
+  c->np_down = np_of(d);
+  c->np_h0 = np_of(c->head_dims[1]);
+  auto rows_of = [&](long long np, int n) -> size_t { return (size_t)(np ? np : n); };
+  c->w_proj = c->alloc(rows_of(c->np_proj, d) * 3 * d * es);
+  c->w_qkv = c->alloc(rows_of(c->np_qkv, c->qkv_n) * d * es);
+  c->w_o = c->alloc(rows_of(c->np_o, d) * c->attn_w * es);
+  c->w_gu = c->alloc(rows_of(c->np_gu, 2 * c->Fp) * d * es);
+  c->w_down = c->alloc(rows_of(c->np_down, d) * c->Fp * es);
   c->g_in = (float*)c->alloc((size_t)d * 4);
   c->g_post = (float*)c->alloc((size_t)d * 4);
   c->g_final = (float*)c->alloc((size_t)d * 4);
   const int nl = (int)c->head_dims.size() - 1;
   c->head_wf.assign(nl, nullptr);
   c->head_b.assign(nl, nullptr);
-  c->head_w0 = c->alloc((size_t)c->head_dims[1] * d * es);
+  c->head_w0 = c->alloc(rows_of(c->np_h0, c->head_dims[1]) * d * es);
   for (int i = 1; i < nl; ++i) c->head_wf[i] = (float*)c->alloc((size_t)c->head_dims[i + 1] * c->head_dims[i] * 4);
   for (int i = 0; i < nl; ++i) c->head_b[i] = (float*)c->alloc((size_t)c->head_dims[i + 1] * 4);
   c->rope_cos = (float*)c->alloc((size_t)cfg->max_position * (c->hd / 2) * 4);
@@ -568,6 +762,10 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->z = (float*)c->alloc(R * 4);
   c->len = (float*)c->alloc(R * 4);
   c->err_dev = (int*)c->alloc(16);
+  if (c->bf16) {  // f32 QKV rows of the small-M path
+    c->part_floats = std::min<size_t>(R, 256) * (size_t)c->qkv_n;
+    c->part = (float*)c->alloc(c->part_floats * 4);
+  }
   if (c->oom) return cleanup_fail(OUTLETS_ENOMEM);
   for (auto& p : c->ring)
     if (cudaEventCreateWithFlags(&p.ev, cudaEventDisableTiming) != cudaSuccess) return cleanup_fail(OUTLETS_ECUDA);
@@ -583,19 +781,19 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   // keep interleaved uploads chunked on 128-row boundaries
   const size_t il_floats = std::max<size_t>((stage_floats / d) / 128 * 128, 128) * d;
   outlets_status st = OUTLETS_OK;
-  auto up = [&](const float* src, int rows, int cols, void* dst, long long ld, int mode, int base) {
+  auto up = [&](const float* src, int rows, int cols, void* dst, long long ld, int mode, int base, long long np) {
     if (st == OUTLETS_OK)
-      st = upload_rows(c, src, rows, cols, dst, ld, mode, base, stage, mode == 0 ? stage_floats : il_floats);
+      st = upload_rows(c, src, rows, cols, dst, ld, mode, base, np, stage, mode == 0 ? stage_floats : il_floats);
   };
-  up(w->w_proj, d, 3 * d, c->w_proj, 3 * d, 0, 0);
-  up(w->w_q, c->H * c->hd, d, c->w_qkv, d, 0, 0);
-  up(w->w_k, c->KVH * c->hd, d, c->w_qkv, d, 0, c->H * c->hd);
-  up(w->w_v, c->KVH * c->hd, d, c->w_qkv, d, 0, (c->H + c->KVH) * c->hd);
-  up(w->w_o, d, c->attn_w, c->w_o, c->attn_w, 0, 0);
-  up(w->w_gate, c->F, d, c->w_gu, d, 1, 0);
-  up(w->w_up, c->F, d, c->w_gu, d, 2, 0);
-  up(w->w_down, d, c->F, c->w_down, c->Fp, 0, 0);
-  up(w->head_w[0], c->head_dims[1], d, c->head_w0, d, 0, 0);
+  up(w->w_proj, d, 3 * d, c->w_proj, 3 * d, 0, 0, c->np_proj);
+  up(w->w_q, c->H * c->hd, d, c->w_qkv, d, 0, 0, c->np_qkv);
+  up(w->w_k, c->KVH * c->hd, d, c->w_qkv, d, 0, c->H * c->hd, c->np_qkv);
+  up(w->w_v, c->KVH * c->hd, d, c->w_qkv, d, 0, (c->H + c->KVH) * c->hd, c->np_qkv);
+  up(w->w_o, d, c->attn_w, c->w_o, c->attn_w, 0, 0, c->np_o);
+  up(w->w_gate, c->F, d, c->w_gu, d, 1, 0, c->np_gu);
+  up(w->w_up, c->F, d, c->w_gu, d, 2, 0, c->np_gu);
+  up(w->w_down, d, c->F, c->w_down, c->Fp, 0, 0, c->np_down);
+  up(w->head_w[0], c->head_dims[1], d, c->head_w0, d, 0, 0, c->np_h0);
   cudaFree(stage);
   if (st != OUTLETS_OK) return cleanup_fail(st);
   auto h2d = [&](void* dst, const void* src, size_t bytes) {
@@ -863,24 +1061,9 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
   const int* cu_dev = m + off_cu;
 
   const int d = c->d;
-  // ---- FC (Eq. 1): f = [tap0 | tap1 | tap2] W_proj^T
-  c->stage_begin(OUTLETS_S_FC);
-  if (c->bf16) OUT_TRY(gemm_tc(c, tp, 3, d, d, T, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
-  else OUT_TRY(gemm_f32(c, tp, d, T, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
-  c->stage_end(1);
-  // ---- input RMSNorm
-  c->stage_begin(OUTLETS_S_NORM_IN);
-  if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xhat, nullptr, T, d, c->cfg.rms_eps, s));
-  else OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, T, d, c->cfg.rms_eps, s));
-  c->stage_end(1);
-  // ---- QKV
-  c->stage_begin(OUTLETS_S_QKV);
-  {
-    const void* a1[3] = {c->xhat, c->xhat, c->xhat};
-    if (c->bf16) OUT_TRY(gemm_tc(c, a1, 1, d, d, T, c->w_qkv, c->qkv_n, d, EPI_ACT, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
-    else OUT_TRY(gemm_f32(c, a1, d, T, c->w_qkv, c->qkv_n, d, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
-  }
-  c->stage_end(1);
+  // ---- FC (Eq. 1) -> input RMSNorm -> QKV
+  QkvSrc qsrc;
+  OUT_TRY(run_front(c, tp, T, &qsrc, s));
   // ---- RoPE, q, head-major k/v, cache
   c->stage_begin(OUTLETS_S_ROPE);
   {
@@ -906,8 +1089,7 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
       ra.page_tokens = kPageTokens;
     }
     ra.err = c->err_dev;
-    if (c->bf16) OUT_CK(c, rope_scatter_launch<bf16, bf16>((const bf16*)c->qkv, ra, s));
-    else OUT_CK(c, rope_scatter_launch<float, float>((const float*)c->qkv, ra, s));
+    OUT_TRY(launch_rope(c, qsrc, ra, s));
   }
   c->stage_end(1);
   // ---- attention
@@ -915,8 +1097,8 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
   if (c->bf16) {
     CUtensorMap qm, km, vm;
     const uint64_t kv_rows = (uint64_t)c->KVH * c->cfg.max_tokens;
-    if (!make_map(&qm, c->q, c->attn_w, T, c->attn_w, 64) || !make_map(&km, c->kh, c->hd, kv_rows, c->hd, 64) ||
-        !make_map(&vm, c->vh, c->hd, kv_rows, c->hd, 64))
+    if (!cached_map(c, &qm, c->q, c->attn_w, T, c->attn_w, 64) || !cached_map(c, &km, c->kh, c->hd, kv_rows, c->hd, 64) ||
+        !cached_map(c, &vm, c->vh, c->hd, kv_rows, c->hd, 64))
       return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for attention");
     OUT_CK(c, attn_prefill_bf16_launch(qm, km, vm, reinterpret_cast<const AttnTile*>(m + off_tiles), n_tiles,
                                        c->cfg.max_tokens, c->H, c->KVH, c->hd, c->attn, c->err_dev, s));
@@ -989,21 +1171,8 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
   const int* m = c->meta_dev;
   const int d = c->d;
 
-  c->stage_begin(OUTLETS_S_FC);
-  if (c->bf16) OUT_TRY(gemm_tc(c, tp, 3, d, d, B, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
-  else OUT_TRY(gemm_f32(c, tp, d, B, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
-  c->stage_end(1);
-  c->stage_begin(OUTLETS_S_NORM_IN);
-  if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xhat, nullptr, B, d, c->cfg.rms_eps, s));
-  else OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, B, d, c->cfg.rms_eps, s));
-  c->stage_end(1);
-  c->stage_begin(OUTLETS_S_QKV);
-  {
-    const void* a1[3] = {c->xhat, c->xhat, c->xhat};
-    if (c->bf16) OUT_TRY(gemm_tc(c, a1, 1, d, d, B, c->w_qkv, c->qkv_n, d, EPI_ACT, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
-    else OUT_TRY(gemm_f32(c, a1, d, B, c->w_qkv, c->qkv_n, d, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
-  }
-  c->stage_end(1);
+  QkvSrc qsrc;
+  OUT_TRY(run_front(c, tp, B, &qsrc, s));
   c->stage_begin(OUTLETS_S_ROPE);
   {
     RopeArgs ra{};
@@ -1023,8 +1192,7 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
     ra.page_off = m + off_po;
     ra.page_tokens = kPageTokens;
     ra.err = c->err_dev;
-    if (c->bf16) OUT_CK(c, rope_scatter_launch<bf16, bf16>((const bf16*)c->qkv, ra, s));
-    else OUT_CK(c, rope_scatter_launch<float, float>((const float*)c->qkv, ra, s));
+    OUT_TRY(launch_rope(c, qsrc, ra, s));
   }
   c->stage_end(1);
   c->stage_begin(OUTLETS_S_ATTN);
@@ -1053,7 +1221,7 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
     if (c->bf16) {
       CUtensorMap km, vm;
       const uint64_t rows = (uint64_t)kv->num_pages * c->KVH * kPageTokens;
-      if (!make_map(&km, kv->k_pool, c->hd, rows, c->hd, 64) || !make_map(&vm, kv->v_pool, c->hd, rows, c->hd, 64))
+      if (!cached_map(c, &km, kv->k_pool, c->hd, rows, c->hd, 64) || !cached_map(c, &vm, kv->v_pool, c->hd, rows, c->hd, 64))
         return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for the KV pools");
       OUT_CK(c, attn_decode_bf16_launch(km, vm, da, s));
       c->stage_end(2);
@@ -1163,7 +1331,7 @@ extern "C" outlets_status outlets_length_head_noalloc(outlets_ctx* c, const void
   const void* a1[3] = {h_draft, h_draft, h_draft};
   const int w1 = c->head_dims[1];
   if (c->bf16)
-    OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->head_w0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0, c->head_b[0], s));
+    OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->head_w0, c->np_h0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0, c->head_b[0], s));
   else
     OUT_TRY(gemm_f32(c, a1, d, rows, c->head_w0, w1, d, EPI_BIAS_RELU, cur, w1, nullptr, 0, c->head_b[0], s));
   for (int i = 1; i < nl - 1; ++i) {
@@ -1173,7 +1341,7 @@ extern "C" outlets_status outlets_length_head_noalloc(outlets_ctx* c, const void
                      EPI_BIAS_RELU, nxt, c->head_dims[i + 1], nullptr, 0, c->head_b[i], s));
     cur = nxt;
   }
-  OUT_CK(c, head_tail_launch(cur, nullptr, c->head_wf[nl - 1], c->head_b[nl - 1], rows, c->head_dims[nl - 1], z_out,
-                             len_out, s));
+  OUT_CK(c, head_tail_launch(cur, 1, 0, nullptr, c->head_wf[nl - 1], c->head_b[nl - 1], rows, c->head_dims[nl - 1],
+                             z_out, len_out, s));
   return OUTLETS_OK;
 }

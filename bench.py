@@ -254,7 +254,7 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     for _ in range(args.warmup):
         pred.prefill(taps_d, cu, z_out=z, len_out=ln)
     pred.check()
-    pred.profile(True)
+    pred.profile(True, ["gateup_swiglu_gemm"])  # the dominant kernel, timed live on its stream
     launches0 = pred.launch_count
     sampler = ClockSampler(local)
     sampler.start()
@@ -269,13 +269,19 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     clocks = sampler.stop()
     ms = max_over_ranks(ev0.elapsed_time(ev1))
     launches = pred.launch_count - launches0
-    prof = pred.profile_read()
+    prof_live = pred.profile_read()
     pred.profile(False)
     pred.check()
+    # per-stage breakdown in a separate (untimed) pass: stage events serialize the kernels
+    pred.profile(True)
+    for _ in range(3):
+        pred.prefill(taps_d, cu, z_out=z, len_out=ln)
+    prof = pred.profile_read()
+    pred.profile(False)
     ms_step = ms / args.steps
     value = world * Bq * args.steps / (ms / 1e3)
     flops = prefill_flops(shape, lengths, Bq)
-    gu_ms, gu_n = prof["gateup_swiglu_gemm"]
+    gu_ms, gu_n = prof_live["gateup_swiglu_gemm"]
     gu_flops = 2.0 * T * (2 * shape.ffn) * shape.d
     gu_tflops = gu_flops / (gu_ms / gu_n / 1e3) / 1e12
     roofline = {"bound": "tensor", "kernel": "gateup_swiglu_gemm (k_gemm_tc<256, SWIGLU>)",
@@ -283,7 +289,7 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
                 "frac": gu_tflops / peaks["bf16_sus"], "peak_kind": f"bf16 sustained {peaks['src']}",
                 "traffic": None,
                 "algorithmic_per_launch": f"{gu_flops:.4g} FLOP = 2*T*(2F)*d, T={T}"}
-    stages = {k: {"ms_per_step": v[0] / max(args.steps, 1), "share": v[0] / max(sum(x[0] for x in prof.values()), 1e-9)}
+    stages = {k: {"ms_per_step": v[0] / max(v[1], 1), "share": v[0] / max(sum(x[0] for x in prof.values()), 1e-9)}
               for k, v in prof.items() if v[1]}
 
     # ---------------- end to end through the C ABI with host buffers
@@ -329,7 +335,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     from paper_2609_01068_gb300 import outlets, synth
     lens = synth.lengths_8b_step_cache(0, B)
     n_steps = args.steps + args.warmup
-    kv = outlets.KVCache(pred, max_slots=B, max_tokens_total=int(lens.sum()) + (n_steps + 64) * B)
+    kv = outlets.KVCache(pred, max_slots=B, max_tokens_total=int(lens.sum()) + (n_steps + 8 + 64) * B)
     gen = torch.Generator(device="cuda").manual_seed(1)
     b = 0
     while b < B:   # fill the draft cache (untimed set-up)
@@ -348,7 +354,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
         pred.step(st_taps, kv, slots, z_out=z, len_out=ln)
     pred.check()
     cache0 = sum(kv.slot_length(int(s)) for s in slots)
-    pred.profile(True)
+    pred.profile(True, ["attention"])  # the dominant kernel, timed live on its stream
     launches0 = pred.launch_count
     sampler = ClockSampler(torch.cuda.current_device())
     sampler.start()
@@ -365,9 +371,15 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     clocks = sampler.stop()
     ms = max_over_ranks(ev0.elapsed_time(ev1))
     launches = pred.launch_count - launches0
-    prof = pred.profile_read()
+    prof_live = pred.profile_read()
     pred.profile(False)
     pred.check()
+    pred.profile(True)  # per-stage breakdown, separate pass (stage events serialize kernels)
+    n_prof = 3
+    for _ in range(n_prof):
+        pred.step(st_taps, kv, slots, z_out=z, len_out=ln)
+    prof = pred.profile_read()
+    pred.profile(False)
     d, KVH, hd, F = shape.d, shape.n_kv_heads, shape.head_dim, shape.ffn
     # keys read per step: every cached position plus the new one, K and V, bf16
     keys_avg = cache0 + B * (args.steps + 1) / 2.0
@@ -375,7 +387,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     widths = (d,) + tuple(shape.head_widths) + (1,)
     w_bytes = 2 * (3 * d * d + d * shape.qkv_out + shape.n_heads * hd * d + 3 * d * F + widths[0] * widths[1])
     step_bytes = kv_bytes + w_bytes + 3 * B * d * 2
-    at_ms, at_n = prof["attention"]
+    at_ms, at_n = prof_live["attention"]
     at_gbs = kv_bytes / (at_ms / at_n / 1e3) / 1e9
     ms_step = ms / args.steps
     kv.close()
@@ -388,7 +400,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
                          "achieved": at_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                          "frac": at_gbs / peaks["hbm_gbs"], "traffic": None,
                          "algorithmic_per_launch": f"{kv_bytes:.4g} B of K/V (cached + new)"},
-            "stages": {k: v[0] / max(args.steps, 1) for k, v in prof.items() if v[1]},
+            "stages": {k: v[0] / max(v[1], 1) for k, v in prof.items() if v[1]},
             "clocks": clocks, "gpu_launches": launches, "host_issue_ms_per_step": host_ms}
 
 

@@ -200,8 +200,10 @@ outlets_status outlets_get_intermediate(outlets_ctx* ctx, int32_t which, void* d
                                         outlets_tensor_info* info, void* stream);
 
 /* Per-stage device timing.  While enabled, every prediction call records a
- * CUDA event pair around each stage on the call's stream (a stage is one
- * kernel, or the two kernels of split-KV decode attention). */
+ * CUDA event pair around each selected stage on the call's stream (a stage is
+ * one kernel, or the two kernels of split-KV decode attention).  An event pair
+ * serializes its stage with its neighbours (no launch overlap across it), so
+ * time only the stages you need inside a measured region. */
 typedef enum outlets_stage {
   OUTLETS_S_FC = 0,          /* Eq. 1 tap-fusion GEMM */
   OUTLETS_S_NORM_IN = 1,     /* input RMSNorm */
@@ -217,8 +219,9 @@ typedef enum outlets_stage {
   OUTLETS_N_STAGES = 11
 } outlets_stage;
 
-/* Turns stage timing on (1) or off (0) for later calls; clears recorded times. */
-outlets_status outlets_profile_enable(outlets_ctx* ctx, int32_t enable);
+/* Times the stages whose bit (1 << outlets_stage) is set in stage_mask for
+ * later calls (-1: all, 0: off); clears recorded times. */
+outlets_status outlets_profile_enable(outlets_ctx* ctx, int32_t stage_mask);
 
 /* Waits for the recorded events, then writes for each stage the summed
  * duration in milliseconds (ms[OUTLETS_N_STAGES]) and how many times it ran

@@ -36,6 +36,8 @@ template <int HD>
 __global__ void __launch_bounds__(128)
     k_attn_decode_bf16(const __grid_constant__ CUtensorMap k_map, const __grid_constant__ CUtensorMap v_map,
                        const DecodeArgs a) {
+  pdl_trigger();
+  pdl_wait();
   using C = DecCfg<HD>;
   constexpr int NB = HD / 64;
   extern __shared__ uint8_t smem_raw[];
@@ -265,6 +267,8 @@ __global__ void __launch_bounds__(128)
 // Merge split partials: out = sum_s w_s o_s / sum_s w_s, w_s = l_s * 2^(m_s - max m).
 template <typename Act>
 __global__ void k_decode_combine(const DecodeArgs a, int hd) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const int head = blockIdx.y;
   const int w0 = a.work_off[b], w1 = a.work_off[b + 1];
@@ -287,6 +291,8 @@ __global__ void k_decode_combine(const DecodeArgs a, int hd) {
 // f32 path: warp per (request, head); keys walked through the page list.
 template <typename Act>
 __global__ void k_attn_decode_simt(const DecodeArgs a) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int MAXD = 8;
   const int b = blockIdx.x;
   const int h = blockIdx.y * 4 + (threadIdx.x >> 5);
@@ -348,10 +354,10 @@ cudaError_t launch_decode_tc(const CUtensorMap& k_map, const CUtensorMap& v_map,
     attr = true;
   }
   dim3 grid(a.n_work, a.KVH);
-  k_attn_decode_bf16<HD><<<grid, 128, C::SMEM, stream>>>(k_map, v_map, a);
+  OUTLETS_TRY_LAUNCH(launch_k(k_attn_decode_bf16<HD>, dim3(grid), dim3(128), C::SMEM, stream, k_map, v_map, a));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_decode_combine<bf16><<<dim3(a.B, a.H), 128, 0, stream>>>(a, HD);
+  OUTLETS_TRY_LAUNCH(launch_k(k_decode_combine<bf16>, dim3(dim3(a.B, a.H)), dim3(128), 0, stream, a, HD));
   return cudaGetLastError();
 }
 
@@ -370,7 +376,7 @@ template <typename Act>
 cudaError_t attn_decode_simt_launch(const DecodeArgs& a, cudaStream_t stream) {
   if (a.B == 0) return cudaSuccess;
   if (a.hd > 256) return cudaErrorInvalidValue;
-  k_attn_decode_simt<Act><<<dim3(a.B, (a.H + 3) / 4), 128, 0, stream>>>(a);
+  OUTLETS_TRY_LAUNCH(launch_k(k_attn_decode_simt<Act>, dim3(dim3(a.B, (a.H + 3) / 4)), dim3(128), 0, stream, a));
   return cudaGetLastError();
 }
 template cudaError_t attn_decode_simt_launch<float>(const DecodeArgs&, cudaStream_t);

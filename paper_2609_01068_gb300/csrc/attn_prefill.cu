@@ -30,6 +30,8 @@ __global__ void __launch_bounds__(128)
     k_attn_prefill_bf16(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap k_map,
                         const __grid_constant__ CUtensorMap v_map, const AttnTile* __restrict__ tiles, int T,
                         int H, int KVH, bf16* __restrict__ out, int* err) {
+  pdl_trigger();
+  pdl_wait();
   using C = PrefillCfg<HD>;
   constexpr int NB = HD / 64;
   extern __shared__ uint8_t smem_raw[];
@@ -232,6 +234,8 @@ template <typename Act>
 __global__ void k_attn_prefill_simt(const Act* __restrict__ q, const Act* __restrict__ k,
                                     const Act* __restrict__ v, const int* __restrict__ cu, int B, int kv_ld, int H,
                                     int KVH, int hd, Act* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int MAXD = 8;  // hd <= 256
   const int row = blockIdx.x;
   const int h = blockIdx.y * 4 + (threadIdx.x >> 5);
@@ -296,8 +300,8 @@ cudaError_t attn_prefill_bf16_launch(const CUtensorMap& q_map, const CUtensorMap
       attr = true;
     }
     dim3 grid(H, n_tiles);
-    k_attn_prefill_bf16<128><<<grid, 128, C::SMEM, stream>>>(q_map, k_map, v_map, tiles, T, H, KVH,
-                                                             reinterpret_cast<bf16*>(out), err);
+    OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_bf16<128>, dim3(grid), dim3(128), C::SMEM, stream, q_map, k_map, v_map, tiles, T, H, KVH,
+                                                             reinterpret_cast<bf16*>(out), err));
     return cudaGetLastError();
   }
   if (hd == 64) {
@@ -310,8 +314,8 @@ cudaError_t attn_prefill_bf16_launch(const CUtensorMap& q_map, const CUtensorMap
       attr = true;
     }
     dim3 grid(H, n_tiles);
-    k_attn_prefill_bf16<64><<<grid, 128, C::SMEM, stream>>>(q_map, k_map, v_map, tiles, T, H, KVH,
-                                                            reinterpret_cast<bf16*>(out), err);
+    OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_bf16<64>, dim3(grid), dim3(128), C::SMEM, stream, q_map, k_map, v_map, tiles, T, H, KVH,
+                                                            reinterpret_cast<bf16*>(out), err));
     return cudaGetLastError();
   }
   return cudaErrorInvalidValue;
@@ -323,7 +327,7 @@ cudaError_t attn_prefill_simt_launch(const Act* q, const Act* k, const Act* v, c
   if (n_rows == 0) return cudaSuccess;
   if (hd > 256) return cudaErrorInvalidValue;
   dim3 grid(n_rows, (H + 3) / 4);
-  k_attn_prefill_simt<Act><<<grid, 128, 0, stream>>>(q, k, v, cu, B, kv_ld, H, KVH, hd, out);
+  OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_simt<Act>, dim3(grid), dim3(128), 0, stream, q, k, v, cu, B, kv_ld, H, KVH, hd, out));
   return cudaGetLastError();
 }
 

@@ -51,6 +51,8 @@ __global__ void k_rmsnorm(const float* __restrict__ x, int n_split, long long sp
                           const float* __restrict__ residual, const int* __restrict__ row_index,
                           const float* __restrict__ g, Act* __restrict__ y, float* __restrict__ copy_out, int d,
                           float eps) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[33];
   extern __shared__ float4 rowbuf[];  // the reduced row (REDUCE only)
   const int r = blockIdx.x;
@@ -162,6 +164,8 @@ __device__ __forceinline__ void store8<float>(float* p, const float* v) {
 // one head and copies 8 values of V.  hd is a multiple of 16.
 template <typename In, typename Act>
 __global__ void k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
+  pdl_trigger();
+  pdl_wait();
   const int row = blockIdx.x;
   int pos, seq;
   if (a.cu) {
@@ -246,6 +250,8 @@ __global__ void k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
 
 template <typename Act>
 __global__ void k_swiglu(const float* __restrict__ gu, Act* __restrict__ u, int rows, int f_pad) {
+  pdl_trigger();
+  pdl_wait();
   const long long n = (long long)rows * f_pad;
   for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n;
        idx += (long long)gridDim.x * blockDim.x) {
@@ -262,6 +268,8 @@ __global__ void k_head_tail(const float* __restrict__ h, int n_split, long long 
                             const float* __restrict__ b_prev, const float* __restrict__ w_last,
                             const float* __restrict__ b_last, int rows, int width, float* __restrict__ z,
                             float* __restrict__ len) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[33];
   const int r = blockIdx.x;
   const float* hr = h + (long long)r * width;
@@ -316,6 +324,8 @@ constexpr int ST = 64, SK = 16;
 __global__ void __launch_bounds__(256) k_gemm_simt(const float* __restrict__ a0, const float* __restrict__ a1,
                                                    const float* __restrict__ a2, const float* __restrict__ bm,
                                                    int epi, const GemmArgs p) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float As[SK][ST + 1];
   __shared__ float Bs[SK][ST + 1];
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -403,10 +413,10 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
         attr = true;
       }
     }
-    k_rmsnorm<Act, true><<<rows, 256, smem, stream>>>(x, n_split, split_stride, residual, row_index, g, y, copy_out,
-                                                      d, eps);
+    OUTLETS_TRY_LAUNCH(launch_k(k_rmsnorm<Act, true>, dim3(rows), dim3(256), smem, stream, x, n_split, split_stride, residual, row_index, g, y, copy_out,
+                                                      d, eps));
   } else {
-    k_rmsnorm<Act, false><<<rows, 256, 0, stream>>>(x, 1, 0, nullptr, row_index, g, y, copy_out, d, eps);
+    OUTLETS_TRY_LAUNCH(launch_k(k_rmsnorm<Act, false>, dim3(rows), dim3(256), 0, stream, x, 1, 0, nullptr, row_index, g, y, copy_out, d, eps));
   }
   return cudaGetLastError();
 }
@@ -414,14 +424,14 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
 template <typename In, typename Act>
 cudaError_t rope_scatter_launch(const In* qkv, const RopeArgs& a, cudaStream_t stream) {
   if (a.T == 0) return cudaSuccess;
-  k_rope_scatter<In, Act><<<a.T, 128, 0, stream>>>(qkv, a);
+  OUTLETS_TRY_LAUNCH(launch_k(k_rope_scatter<In, Act>, dim3(a.T), dim3(128), 0, stream, qkv, a));
   return cudaGetLastError();
 }
 
 template <typename Act>
 cudaError_t swiglu_launch(const float* gu, Act* u, int rows, int f_pad, cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
-  k_swiglu<Act><<<grid_for((long long)rows * f_pad, 256), 256, 0, stream>>>(gu, u, rows, f_pad);
+  OUTLETS_TRY_LAUNCH(launch_k(k_swiglu<Act>, dim3(grid_for((long long)rows * f_pad, 256)), dim3(256), 0, stream, gu, u, rows, f_pad));
   return cudaGetLastError();
 }
 
@@ -429,7 +439,7 @@ cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_st
                              const float* w_last, const float* b_last, int rows, int width, float* z, float* len,
                              cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
-  k_head_tail<<<rows, 128, 0, stream>>>(h_pre, n_split, split_stride, b_prev, w_last, b_last, rows, width, z, len);
+  OUTLETS_TRY_LAUNCH(launch_k(k_head_tail, dim3(rows), dim3(128), 0, stream, h_pre, n_split, split_stride, b_prev, w_last, b_last, rows, width, z, len));
   return cudaGetLastError();
 }
 
@@ -437,8 +447,8 @@ template <typename Act>
 cudaError_t convert_rows_launch(const float* src, Act* dst, int rows, int cols, long long dst_ld, int row_mode,
                                 int row_base, long long kb_np, cudaStream_t stream) {
   if (rows == 0 || cols == 0) return cudaSuccess;
-  k_convert_rows<Act><<<grid_for((long long)rows * cols, 256), 256, 0, stream>>>(src, dst, rows, cols, dst_ld,
-                                                                                row_mode, row_base, kb_np);
+  OUTLETS_TRY_LAUNCH(launch_k(k_convert_rows<Act>, dim3(grid_for((long long)rows * cols, 256)), dim3(256), 0, stream, src, dst, rows, cols, dst_ld,
+                                                                                row_mode, row_base, kb_np));
   return cudaGetLastError();
 }
 
@@ -446,7 +456,7 @@ cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int ep
                                  cudaStream_t stream) {
   if (args.M == 0 || args.N == 0) return cudaSuccess;
   dim3 grid((args.N + ST - 1) / ST, (args.M + ST - 1) / ST);
-  k_gemm_simt<<<grid, 256, 0, stream>>>(a[0], a[1], a[2], b, epi, args);
+  OUTLETS_TRY_LAUNCH(launch_k(k_gemm_simt, dim3(grid), dim3(256), 0, stream, a[0], a[1], a[2], b, epi, args));
   return cudaGetLastError();
 }
 

@@ -12,6 +12,8 @@
 // Used for Eq. 1 (three-tap fusion: A is split along K over the three taps),
 // the QKV / O / gate-up / down projections of the draft decoder layer, and
 // the first Linear of the length head (Sec. 4.2).
+#include <stdlib.h>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -139,6 +141,20 @@ __global__ void __launch_bounds__(192, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_trigger();
+  if (warp == 0 && lane == 0 && p.prefetch) {
+    // weights never change: start pulling this CTA's first weight tiles toward L2
+    // while the previous kernel finishes
+    const int nm = (p.M + TM - 1) / TM, nn = (p.N + BN - 1) / BN, kbt = (p.K + BK - 1) / BK;
+    if ((int)blockIdx.x < nm * nn * p.splits) {
+    const Tile t0 = decode_tile(blockIdx.x, nm, nn, p.group_m, kbt, (kbt + p.splits - 1) / p.splits, p.splits,
+                                EPI == EPI_CLUSTER);
+    const bf16* bt = reinterpret_cast<const bf16*>(p.b) + (long long)t0.n_blk * BN * BK;
+    for (int kb = t0.kb0; kb < min(t0.kb1, t0.kb0 + p.prefetch); ++kb)
+      bulk_prefetch_l2(bt + (long long)kb * p.b_np * BK, C::B_BYTES);
+    }
+  }
+  pdl_wait();  // activations and outputs are touched only after the previous kernel is done
 
   const int num_m = (p.M + TM - 1) / TM;
   const int num_n = (p.N + BN - 1) / BN;
@@ -412,7 +428,7 @@ cudaError_t launch_one(const CUtensorMap a_maps[3], const GemmArgs& args, int nu
   const long long tiles = (long long)((args.M + BM * MT - 1) / (BM * MT)) * ((args.N + BN - 1) / BN) * args.splits;
   const int grid = (int)(tiles < num_sms ? tiles : num_sms);
   if (grid <= 0) return cudaSuccess;
-  kern<<<grid, 192, C::SMEM, stream>>>(a_maps[0], a_maps[1], a_maps[2], args);
+  OUTLETS_TRY_LAUNCH(launch_k(kern, dim3(grid), dim3(192), C::SMEM, stream, a_maps[0], a_maps[1], a_maps[2], args));
   return cudaGetLastError();
 }
 
@@ -433,13 +449,15 @@ cudaError_t launch_cluster(const CUtensorMap a_maps[3], const GemmArgs& args,
   cfg.blockDim = dim3(192);
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = stream;
-  cudaLaunchAttribute at[1];
+  cudaLaunchAttribute at[2];
   at[0].id = cudaLaunchAttributeClusterDimension;
   at[0].val.clusterDim.x = args.splits;
   at[0].val.clusterDim.y = 1;
   at[0].val.clusterDim.z = 1;
+  at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = at;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl_enabled() ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, kern, a_maps[0], a_maps[1], a_maps[2], args);
 }
 
@@ -471,6 +489,14 @@ int cluster_capacity(int splits) {
 }
 
 }  // namespace
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = getenv("OUTLETS_PDL");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
 
 cudaError_t gemm_tc_cluster_launch(const CUtensorMap a_maps[3], int bn, int mt, const GemmArgs& args,
                                    cudaStream_t stream) {

@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace outlets {
 
 typedef __nv_bfloat16 bf16;
@@ -16,6 +18,35 @@ enum : int {
   ERR_TIMEOUT = 1,    // a bounded wait ran out (an mbarrier phase never completed)
   ERR_BAD_INDEX = 2,  // a kernel met an index it refused to use
 };
+
+// Every prediction kernel is launched with programmatic stream serialization:
+// it signals its dependents at once and runs its prologue (barrier init, TMEM
+// allocation, L2 prefetch of weights) before waiting (griddepcontrol.wait) for
+// the previous kernel's memory, so launch latency and prologues overlap the
+// previous kernel's tail.  OUTLETS_PDL=0 in the environment turns this off.
+bool pdl_enabled();
+
+#define OUTLETS_TRY_LAUNCH(...)                \
+  do {                                         \
+    const cudaError_t e_launch_ = (__VA_ARGS__); \
+    if (e_launch_ != cudaSuccess) return e_launch_; \
+  } while (0)
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                     Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
 
 // GEMM: C[M, N] = A[M, K] * B[N, K]^T, A optionally split along K across up to
 // three separately addressed row-major matrices (the three taps of Eq. 1).

@@ -147,7 +147,8 @@ struct outlets_ctx {
     int stage;
     cudaEvent_t a, b;
   };
-  bool prof = false;
+  unsigned prof = 0;  // bit mask of timed stages
+  int cur_stage = -1;
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_used = 0;
   std::vector<ProfRec> recs;
@@ -166,16 +167,19 @@ struct outlets_ctx {
     return ev_pool[ev_used++];
   }
   void stage_begin(int stage) {
-    if (!prof) return;
+    cur_stage = -1;
+    if (!((prof >> stage) & 1u)) return;
     ProfRec r{stage, next_event(), next_event()};
     if (!r.a || !r.b) return;
     cudaEventRecord(r.a, cur_stream);
     recs.push_back(r);
+    cur_stage = stage;
   }
   void stage_end(int n_kernels) {
     launches += (unsigned long long)n_kernels;
-    if (!prof || recs.empty()) return;
+    if (cur_stage < 0 || recs.empty()) return;
     cudaEventRecord(recs.back().b, cur_stream);
+    cur_stage = -1;
   }
 
   outlets_status fail(outlets_status st, const std::string& msg) {
@@ -848,7 +852,7 @@ outlets_status outlets_profile_enable(outlets_ctx* c, int32_t enable) {
   if (!c) return OUTLETS_EINVAL;
   OUT_CK(c, cudaSetDevice(c->cfg.device));
   OUT_CK(c, cudaDeviceSynchronize());
-  c->prof = enable != 0;
+  c->prof = static_cast<unsigned>(enable) & ((1u << OUTLETS_N_STAGES) - 1u);
   c->recs.clear();
   c->ev_used = 0;
   return OUTLETS_OK;

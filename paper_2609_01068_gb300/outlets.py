@@ -212,8 +212,17 @@ class Predictor:
         if st != OK:
             self._raise(st)
 
-    def profile(self, enable: bool):
-        st = self.lib.outlets_profile_enable(self.h, 1 if enable else 0)
+    def profile(self, enable, stages=None):
+        """Time the named stages (all if None) of later calls; enable=False turns timing off."""
+        mask = 0
+        if enable:
+            if stages is None:
+                mask = -1
+            else:
+                names = [self.lib.outlets_stage_name(i).decode() for i in range(N_STAGES)]
+                for n in stages:
+                    mask |= 1 << names.index(n)
+        st = self.lib.outlets_profile_enable(self.h, mask)
         if st != OK:
             self._raise(st)
 

@@ -1,6 +1,8 @@
-// tcgen05 GEMM for sm_103a: C[M, N] = A[M, K] * B[N, K]^T, bf16 in, f32 accumulate.
+// tcgen05 GEMMs for sm_103a: C[M, N] = A[M, K] * B[N, K]^T, bf16 in, f32 accumulate.
+// A (activations) is loaded by TMA tensor copies (128-byte swizzle); B (weights)
+// lives in a k-block-major, pre-swizzled layout and is loaded by bulk copies.
 //
-// Persistent, one CTA per SM, 6 warps:
+// k_gemm_tc (large M, prefill): persistent, one CTA per SM, 6 warps:
 //   warp 0      TMA producer (one thread): A and B K-blocks into a smem ring
 //   warp 1      MMA issuer (one thread): tcgen05.mma 128 x BN x 16 into TMEM;
 //               also owns the TMEM allocation
@@ -8,6 +10,10 @@
 //               store to global.  Warp w reads TMEM lanes 32*(w%4) .. +31.
 // Two TMEM accumulators (2 * BN columns) let the epilogue of tile i overlap
 // the main loop of tile i+1.  Every mbarrier wait is bounded.
+//
+// k_gemm_small (M <= 256, dynamic prediction and the head): one output tile and
+// one K split per CTA, every weight tile streamed once; K splits of a tile form
+// thread-block clusters reduced through distributed shared memory.
 //
 // Used for Eq. 1 (three-tap fusion: A is split along K over the three taps),
 // the QKV / O / gate-up / down projections of the draft decoder layer, and
@@ -33,7 +39,8 @@ struct TcCfg {
   static constexpr uint32_t A_BYTES = MT * BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = (196608 / STAGE_BYTES) > 8 ? 8 : (196608 / STAGE_BYTES);
+  // every byte of the 227 KB a CTA may use goes to the ring (1 KB alignment + barriers aside)
+  static constexpr int STAGES = ((232448 - 1024 - 256) / STAGE_BYTES) > 8 ? 8 : ((232448 - 1024 - 256) / STAGE_BYTES);
   static constexpr uint32_t TMEM_USED = ACC * MT * BN;
   static constexpr uint32_t TMEM_COLS = TMEM_USED <= 32 ? 32 : TMEM_USED <= 64 ? 64 : TMEM_USED <= 128 ? 128
                                                                : TMEM_USED <= 256 ? 256 : 512;  // power of 2
@@ -45,12 +52,10 @@ struct Tile {
   int m_blk, n_blk, kb0, kb1, split;
 };
 
-__device__ __forceinline__ Tile decode_tile(int t, int num_m, int num_n, int group_m, int kb_total, int kb_per,
-                                            int splits, bool cluster_order) {
+__device__ __forceinline__ Tile decode_tile(int t, int num_m, int num_n, int group_m, int kb_total, int kb_per) {
   const int per_split = num_m * num_n;
-  // cluster order: the splits of one output tile are consecutive CTAs (one cluster)
-  const int split = cluster_order ? t % splits : t / per_split;
-  const int r = cluster_order ? t / splits : t - split * per_split;
+  const int split = t / per_split;
+  const int r = t - split * per_split;
   const int width = group_m * num_n;
   const int group = r / width;
   const int first_m = group * group_m;
@@ -147,8 +152,7 @@ __global__ void __launch_bounds__(192, 1)
     // while the previous kernel finishes
     const int nm = (p.M + TM - 1) / TM, nn = (p.N + BN - 1) / BN, kbt = (p.K + BK - 1) / BK;
     if ((int)blockIdx.x < nm * nn * p.splits) {
-    const Tile t0 = decode_tile(blockIdx.x, nm, nn, p.group_m, kbt, (kbt + p.splits - 1) / p.splits, p.splits,
-                                EPI == EPI_CLUSTER);
+    const Tile t0 = decode_tile(blockIdx.x, nm, nn, p.group_m, kbt, (kbt + p.splits - 1) / p.splits);
     const bf16* bt = reinterpret_cast<const bf16*>(p.b) + (long long)t0.n_blk * BN * BK;
     for (int kb = t0.kb0; kb < min(t0.kb1, t0.kb0 + p.prefetch); ++kb)
       bulk_prefetch_l2(bt + (long long)kb * p.b_np * BK, C::B_BYTES);
@@ -167,7 +171,7 @@ __global__ void __launch_bounds__(192, 1)
       int stage = 0;
       uint32_t phase = 0;
       for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per, p.splits, EPI == EPI_CLUSTER);
+        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
         const bf16* btile = reinterpret_cast<const bf16*>(p.b) + (long long)tl.n_blk * BN * BK;
         // weights streamed once: keep p.prefetch K blocks of B in flight toward L2
         for (int kb = tl.kb0; kb < min(tl.kb1, tl.kb0 + p.prefetch); ++kb)
@@ -204,7 +208,7 @@ __global__ void __launch_bounds__(192, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per, p.splits, EPI == EPI_CLUSTER);
+        const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, p.err)) goto mma_done;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * MT * BN);
@@ -238,14 +242,14 @@ __global__ void __launch_bounds__(192, 1)
       }
     mma_done:;
     }
-  } else if constexpr (EPI != EPI_CLUSTER) {
+  } else {
     // epilogue warps 2..5
     const int quarter = warp & 3;
     const int row_in_tile = quarter * 32 + lane;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-      const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per, p.splits, EPI == EPI_CLUSTER);
+      const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
       if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err)) break;
       tc_fence_after();
 #pragma unroll 1
@@ -327,84 +331,6 @@ __global__ void __launch_bounds__(192, 1)
     }
   }
 
-  if constexpr (EPI == EPI_CLUSTER) {
-    // One tile per CTA; the cluster's CTAs hold the K-split partial sums of the
-    // same output tile.  Per round of CW columns: every CTA stages its partial
-    // in its own shared memory (the pipeline ring is idle now), then each CTA
-    // adds up a contiguous column stripe across all CTAs of the cluster through
-    // DSMEM and writes it.  Every thread of every CTA passes every cluster
-    // barrier, also after an abort, so no CTA waits for one that left.
-    constexpr int CW = BN < 128 ? BN : 128;
-    constexpr int LD = CW + 4;  // padded row (floats): conflict-free row-wise staging
-    constexpr int G = CW / 4;   // float4 groups per row
-    __syncwarp();
-    const int S = p.splits;
-    const uint32_t rank = cluster_ctarank();
-    const Tile tl = decode_tile(blockIdx.x, num_m, num_n, p.group_m, kb_total, kb_per, p.splits, true);
-    bool have = false;
-    if (warp >= 2) {
-      have = mbar_wait(&tfull[0], 0, abort_flag, p.err);
-      tc_fence_after();
-    }
-    float* red = reinterpret_cast<float*>(smem);
-    const int per = (G + S - 1) / S;  // groups owned by each CTA
-    const int g0 = min(G, (int)rank * per);
-    const int g1 = min(G, g0 + per);
-    const int my_groups = g1 - g0;
-    const uint32_t red_addr = smem_u32(red);
-    for (int rd = 0; rd < BN / CW; ++rd) {
-      if (warp >= 2 && have) {
-        const int quarter = warp & 3;
-#pragma unroll 1
-        for (int mt = 0; mt < MT; ++mt) {
-          const int row = mt * BM + quarter * 32 + lane;
-          const uint32_t tb = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
-                              static_cast<uint32_t>(mt * BN + rd * CW);
-          for (int c = 0; c < CW; c += 32) {
-            uint32_t r[32];
-            tmem_ld_32x32b_x32(tb + c, r);
-            tmem_ld_wait();
-            float* dst = red + row * LD + c;
-#pragma unroll
-            for (int j = 0; j < 32; j += 4)
-              *reinterpret_cast<float4*>(dst + j) = make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]),
-                                                                __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3]));
-          }
-        }
-      }
-      cluster_sync_all();
-      if (!*abort_flag && my_groups > 0) {
-        const int items = TM * my_groups;
-        for (int it = threadIdx.x; it < items; it += blockDim.x) {
-          const int row = it / my_groups;
-          const int col = (g0 + it - row * my_groups) * 4;
-          const uint32_t off = red_addr + static_cast<uint32_t>((row * LD + col) * 4);
-          float4 acc = dsmem_ld_f4(dsmem_map(off, 0));
-          for (int q = 1; q < S; ++q) {
-            const float4 v = dsmem_ld_f4(dsmem_map(off, q));
-            acc.x += v.x;
-            acc.y += v.y;
-            acc.z += v.z;
-            acc.w += v.w;
-          }
-          const int m = tl.m_blk * TM + row;
-          const int n = tl.n_blk * BN + rd * CW + col;
-          if (m < p.M && n < p.N) {
-            if (p.residual) {
-              const float4 rv = *reinterpret_cast<const float4*>(p.residual + (long long)m * p.ldr + n);
-              acc.x += rv.x;
-              acc.y += rv.y;
-              acc.z += rv.z;
-              acc.w += rv.w;
-            }
-            *reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n) = acc;
-          }
-        }
-      }
-      cluster_sync_all();
-    }
-  }
-
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -432,11 +358,269 @@ cudaError_t launch_one(const CUtensorMap a_maps[3], const GemmArgs& args, int nu
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// Small-M kernel.  A CTA computes one (up to 256) x BN output tile over one
+// K split (balanced, never empty).  Activations and weights have their own
+// ring barriers (AS and WS slots; the producer may run the weight ring
+// WS - AS blocks ahead); with AS == WS this is one ring holding both tiles of
+// a K block, which is what the latency of both operands needs.
 template <int BN, int MT>
-cudaError_t launch_cluster(const CUtensorMap a_maps[3], const GemmArgs& args,
-                           cudaStream_t stream) {
-  using C = TcCfg<BN, MT>;
-  auto kern = k_gemm_tc<BN, EPI_CLUSTER, MT>;
+struct SmCfg {
+  static constexpr uint32_t A_BYTES = MT * BM * BK * 2;
+  static constexpr uint32_t B_BYTES = BN * BK * 2;
+  // one ring slot per K block for activations and weights alike: latency hides
+  // behind total bytes in flight, so the ring takes every byte of the 227 KB
+  static constexpr int FIT = (int)((232448u - 1024u - 256u) / (A_BYTES + B_BYTES));
+  static constexpr int AS = FIT > 8 ? 8 : FIT;
+  static constexpr int WS = AS;
+  static constexpr uint32_t RING_BYTES = AS * A_BYTES + WS * B_BYTES;
+  static constexpr uint32_t TMEM_USED = MT * BN;
+  static constexpr uint32_t TMEM_COLS = TMEM_USED <= 64 ? 64 : TMEM_USED <= 128 ? 128 : TMEM_USED <= 256 ? 256 : 512;
+  static constexpr size_t SMEM = 1024 + RING_BYTES + 256;
+  static_assert(AS >= 2, "ring");
+  static_assert(TMEM_USED <= 512, "TMEM columns");
+};
+
+template <int BN, int EPI, int MT>
+__global__ void __launch_bounds__(192, 1)
+    k_gemm_small(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_a1,
+                 const __grid_constant__ CUtensorMap map_a2, const GemmArgs p) {
+  using C = SmCfg<BN, MT>;
+  constexpr int TM = BM * MT;
+  constexpr int AS = C::AS, WS = C::WS;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sW = smem + AS * C::A_BYTES;
+  uint64_t* fullA = reinterpret_cast<uint64_t*>(smem + C::RING_BYTES);
+  uint64_t* emptyA = fullA + AS;
+  uint64_t* fullW = emptyA + AS;
+  uint64_t* emptyW = fullW + WS;
+  uint64_t* tfull = emptyW + WS;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tfull + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < AS; ++i) {
+      mbar_init(&fullA[i], 1);
+      mbar_init(&emptyA[i], 1);
+    }
+    for (int i = 0; i < WS; ++i) {
+      mbar_init(&fullW[i], 1);
+      mbar_init(&emptyW[i], 1);
+    }
+    mbar_init(&tfull[0], 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&map_a0);
+    tma_prefetch_map(&map_a1);
+    tma_prefetch_map(&map_a2);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();
+
+  const int S = p.splits;
+  const int tile = blockIdx.x / S;
+  const int split = blockIdx.x - tile * S;
+  const int num_n = (p.N + BN - 1) / BN;
+  const int m_blk = tile / num_n;
+  const int n_blk = tile - m_blk * num_n;
+  const int kb_total = (p.K + BK - 1) / BK;
+  // balanced split: every split gets floor or ceil of kb_total / S blocks (S <= kb_total)
+  const int kb0 = (int)(((long long)split * kb_total) / S);
+  const int kb1 = (int)(((long long)(split + 1) * kb_total) / S);
+  const bf16* wt = reinterpret_cast<const bf16*>(p.b) + (long long)n_blk * BN * BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      constexpr int lag = WS - AS;  // >= 0
+      int ws = 0, as = 0;
+      uint32_t wph = 0, aph = 0;
+      for (int i = kb0; i < kb1 + lag; ++i) {
+        if (i < kb1) {
+          if (!mbar_wait(&emptyW[ws], wph ^ 1u, abort_flag, p.err)) break;
+          mbar_arrive_expect_tx(&fullW[ws], C::B_BYTES);
+          bulk_load(sW + ws * C::B_BYTES, wt + (long long)i * p.b_np * BK, C::B_BYTES, &fullW[ws]);
+          if (++ws == WS) {
+            ws = 0;
+            wph ^= 1u;
+          }
+        }
+        const int j = i - lag;
+        if (j >= kb0 && j < kb1) {
+          if (!mbar_wait(&emptyA[as], aph ^ 1u, abort_flag, p.err)) break;
+          mbar_arrive_expect_tx(&fullA[as], C::A_BYTES);
+          const int kg = j * BK;
+          const int piece = kg / p.k_per_map;
+          const int kl = kg - piece * p.k_per_map;
+          const CUtensorMap* am = piece == 0 ? &map_a0 : (piece == 1 ? &map_a1 : &map_a2);
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt)
+            tma_load_2d(sA + as * C::A_BYTES + mt * (BM * BK * 2), am, &fullA[as], kl, m_blk * TM + mt * BM);
+          if (++as == AS) {
+            as = 0;
+            aph ^= 1u;
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      int ws = 0, as = 0;
+      uint32_t wph = 0, aph = 0;
+      for (int kb = kb0; kb < kb1; ++kb) {
+        if (!mbar_wait(&fullA[as], aph, abort_flag, p.err)) break;
+        if (!mbar_wait(&fullW[ws], wph, abort_flag, p.err)) break;
+        tc_fence_after();
+        const uint32_t a_addr = smem_u32(sA + as * C::A_BYTES);
+        const uint64_t bdesc = sw128_kmajor_desc(smem_u32(sW + ws * C::B_BYTES));
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+          const uint64_t adesc = sw128_kmajor_desc(a_addr + mt * (BM * BK * 2));
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            tc_mma_bf16(tmem_base + mt * BN, adesc + 2u * kk, bdesc + 2u * kk, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+        }
+        tc_commit(&emptyA[as]);
+        tc_commit(&emptyW[ws]);
+        if (++ws == WS) {
+          ws = 0;
+          wph ^= 1u;
+        }
+        if (++as == AS) {
+          as = 0;
+          aph ^= 1u;
+        }
+      }
+      tc_commit(&tfull[0]);
+    }
+  }
+  __syncwarp();
+
+  bool have = false;
+  if (warp >= 2) {
+    have = mbar_wait(&tfull[0], 0, abort_flag, p.err);
+    tc_fence_after();
+  }
+  const int quarter = warp & 3;
+  if constexpr (EPI == EPI_SWIGLU) {
+    if (warp >= 2 && have) {
+      const int n_out = p.N / 2;
+#pragma unroll 1
+      for (int mt = 0; mt < MT; ++mt) {
+        const int m = m_blk * TM + mt * BM + quarter * 32 + lane;
+        const uint32_t tb = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(mt * BN);
+        for (int c = 0; c < BN; c += 64) {
+          uint32_t g[32], u[32];
+          tmem_ld_32x32b_x32(tb + c, g);
+          tmem_ld_32x32b_x32(tb + c + 32, u);
+          tmem_ld_wait();
+          const int n0 = (n_blk * BN + c) / 2;
+          if (m < p.M && n0 < n_out) {
+            float v[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = silu_f(__uint_as_float(g[j])) * __uint_as_float(u[j]);
+            store_row32(reinterpret_cast<bf16*>(p.out) + (long long)m * p.ldo + n0, v, min(32, n_out - n0));
+          }
+        }
+      }
+    }
+  } else {
+    // Cluster reduction: the p.cluster CTAs of a cluster hold partial sums of
+    // the same tile over different K splits.  Per round of CW columns each CTA
+    // stages its partial in its (now idle) rings, then adds one contiguous
+    // column stripe across the cluster through DSMEM and writes it to the
+    // slice of its cluster group.  All threads pass every cluster barrier.
+    constexpr int CW = BN < 128 ? BN : 128;
+    constexpr int LD = CW + 4;
+    constexpr int G = CW / 4;
+    const int Sc = p.cluster;
+    const uint32_t rank = Sc > 1 ? cluster_ctarank() : 0u;
+    const int group = split / Sc;
+    float* red = reinterpret_cast<float*>(smem);
+    const uint32_t red_addr = smem_u32(red);
+    const int per = (G + Sc - 1) / Sc;
+    const int g0 = min(G, (int)rank * per);
+    const int g1 = min(G, g0 + per);
+    const int my_groups = g1 - g0;
+    float* out = reinterpret_cast<float*>(p.out) + (long long)group * p.group_stride;
+    for (int rd = 0; rd < BN / CW; ++rd) {
+      if (warp >= 2 && have) {
+#pragma unroll 1
+        for (int mt = 0; mt < MT; ++mt) {
+          const int row = mt * BM + quarter * 32 + lane;
+          const uint32_t tb = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                              static_cast<uint32_t>(mt * BN + rd * CW);
+          for (int c = 0; c < CW; c += 32) {
+            uint32_t r[32];
+            tmem_ld_32x32b_x32(tb + c, r);
+            tmem_ld_wait();
+            float* dst = red + row * LD + c;
+#pragma unroll
+            for (int j = 0; j < 32; j += 4)
+              *reinterpret_cast<float4*>(dst + j) = make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]),
+                                                                __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3]));
+          }
+        }
+      }
+      if (Sc > 1) cluster_sync_all();
+      else __syncthreads();
+      if (!*abort_flag && my_groups > 0) {
+        const int items = TM * my_groups;
+        for (int it = threadIdx.x; it < items; it += blockDim.x) {
+          const int row = it / my_groups;
+          const int col = (g0 + it - row * my_groups) * 4;
+          const int m = m_blk * TM + row;
+          const int n = n_blk * BN + rd * CW + col;
+          if (m >= p.M || n >= p.N) continue;
+          const uint32_t off = red_addr + static_cast<uint32_t>((row * LD + col) * 4);
+          float4 acc;
+          if (Sc > 1) {
+            acc = dsmem_ld_f4(dsmem_map(off, 0));
+            for (int q = 1; q < Sc; ++q) {
+              const float4 v = dsmem_ld_f4(dsmem_map(off, q));
+              acc.x += v.x;
+              acc.y += v.y;
+              acc.z += v.z;
+              acc.w += v.w;
+            }
+          } else {
+            acc = *reinterpret_cast<const float4*>(red + row * LD + col);
+          }
+          *reinterpret_cast<float4*>(out + (long long)m * p.ldo + n) = acc;
+        }
+      }
+      if (Sc > 1) cluster_sync_all();
+      else __syncthreads();
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+template <int BN, int EPI, int MT>
+cudaError_t launch_small(const CUtensorMap a_maps[3], const GemmArgs& args, cudaStream_t stream) {
+  using C = SmCfg<BN, MT>;
+  auto kern = k_gemm_small<BN, EPI, MT>;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
@@ -450,42 +634,22 @@ cudaError_t launch_cluster(const CUtensorMap a_maps[3], const GemmArgs& args,
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = stream;
   cudaLaunchAttribute at[2];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = args.splits;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  at[1].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = pdl_enabled() ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, kern, a_maps[0], a_maps[1], a_maps[2], args);
-}
-
-template <int BN, int MT>
-int cluster_capacity(int splits) {
-  using C = TcCfg<BN, MT>;
-  auto kern = k_gemm_tc<BN, EPI_CLUSTER, MT>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
-  }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(splits * 64);
-  cfg.blockDim = dim3(192);
-  cfg.dynamicSmemBytes = C::SMEM;
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = splits;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
+  if (EPI == EPI_CLUSTER && args.cluster > 1) {
+    at[n].id = cudaLaunchAttributeClusterDimension;
+    at[n].val.clusterDim.x = args.cluster;
+    at[n].val.clusterDim.y = 1;
+    at[n].val.clusterDim.z = 1;
+    ++n;
   }
-  return n;
+  if (pdl_enabled()) {
+    at[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  cfg.attrs = at;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kern, a_maps[0], a_maps[1], a_maps[2], args);
 }
 
 }  // namespace
@@ -498,21 +662,58 @@ bool pdl_enabled() {
   return on;
 }
 
-cudaError_t gemm_tc_cluster_launch(const CUtensorMap a_maps[3], int bn, int mt, const GemmArgs& args,
-                                   cudaStream_t stream) {
-  if (args.splits < 1 || args.splits > 8) return cudaErrorInvalidValue;
-  if (bn == 256 && mt == 2) return launch_cluster<256, 2>(a_maps, args, stream);
-  if (bn == 256 && mt == 1) return launch_cluster<256, 1>(a_maps, args, stream);
-  if (bn == 128 && mt == 2) return launch_cluster<128, 2>(a_maps, args, stream);
-  if (bn == 128 && mt == 1) return launch_cluster<128, 1>(a_maps, args, stream);
+cudaError_t gemm_small_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args,
+                              cudaStream_t stream) {
+  if (args.splits < 1 || args.cluster < 1 || args.splits % args.cluster || args.cluster > 8)
+    return cudaErrorInvalidValue;
+#define OUTLETS_SM_CASE(BNV, EV, MTV) \
+  if (bn == BNV && epi == EV && mt == MTV) return launch_small<BNV, EV, MTV>(a_maps, args, stream);
+  OUTLETS_SM_CASE(256, EPI_CLUSTER, 2)
+  OUTLETS_SM_CASE(256, EPI_CLUSTER, 1)
+  OUTLETS_SM_CASE(128, EPI_CLUSTER, 2)
+  OUTLETS_SM_CASE(128, EPI_CLUSTER, 1)
+  OUTLETS_SM_CASE(256, EPI_SWIGLU, 2)
+  OUTLETS_SM_CASE(256, EPI_SWIGLU, 1)
+  OUTLETS_SM_CASE(192, EPI_SWIGLU, 2)  // 4 slots of 56 KB
+  OUTLETS_SM_CASE(192, EPI_SWIGLU, 1)
+  OUTLETS_SM_CASE(128, EPI_SWIGLU, 2)
+  OUTLETS_SM_CASE(128, EPI_SWIGLU, 1)
+#undef OUTLETS_SM_CASE
   return cudaErrorInvalidValue;
 }
 
-int gemm_tc_cluster_capacity(int bn, int mt, int splits) {
-  if (bn == 256 && mt == 2) return cluster_capacity<256, 2>(splits);
-  if (bn == 256 && mt == 1) return cluster_capacity<256, 1>(splits);
-  if (bn == 128 && mt == 2) return cluster_capacity<128, 2>(splits);
-  if (bn == 128 && mt == 1) return cluster_capacity<128, 1>(splits);
+template <int BN, int MT>
+int small_capacity(int cluster) {
+  using C = SmCfg<BN, MT>;
+  auto kern = k_gemm_small<BN, EPI_CLUSTER, MT>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(cluster * 64);
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = cluster;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+int gemm_small_cluster_capacity(int bn, int mt, int cluster) {
+  if (bn == 256 && mt == 2) return small_capacity<256, 2>(cluster);
+  if (bn == 256 && mt == 1) return small_capacity<256, 1>(cluster);
+  if (bn == 128 && mt == 2) return small_capacity<128, 2>(cluster);
+  if (bn == 128 && mt == 1) return small_capacity<128, 1>(cluster);
   return 0;
 }
 

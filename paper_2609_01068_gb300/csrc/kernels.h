@@ -56,7 +56,7 @@ enum Epi : int {
   EPI_SWIGLU = 2,     // B rows interleaved in blocks of 32 [gate | up]; out act = silu(g) * u
   EPI_BIAS_RELU = 3,  // out f32 = max(acc + bias, 0)
   EPI_ATOMIC = 4,     // out f32 += acc (split-K partial sums)
-  EPI_CLUSTER = 6,    // split-K inside a thread-block cluster, reduced through DSMEM: out f32 = sum (+ residual)
+  EPI_CLUSTER = 6,    // small M: split-K reduced inside thread-block clusters (DSMEM), one f32 slice per group
 };
 
 // B operands (weights) live in a k-block-major, pre-swizzled layout owned by the
@@ -74,6 +74,8 @@ struct GemmArgs {
   int splits;             // split-K factor (> 1 only with EPI_ATOMIC); every split non-empty
   int group_m;            // tile raster: M blocks per group
   int prefetch;           // K blocks of B to prefetch into L2 ahead of the smem ring (0 = off)
+  int cluster;            // small-M split-K: CTAs per cluster (splits reduced together through DSMEM)
+  long long group_stride; // small-M split-K: elements between the output slices of cluster groups
   void* out;
   long long ldo;          // elements
   const float* residual;  // EPI_F32 only, may be null
@@ -87,13 +89,16 @@ struct GemmArgs {
 cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args, int num_sms,
                            cudaStream_t stream);
 
-// Split-K GEMM whose args.splits CTAs per output tile form one cluster and add
-// their accumulators through distributed shared memory (EPI_CLUSTER): every
-// output element is written once, in a fixed order.  args.splits <= 8.
-cudaError_t gemm_tc_cluster_launch(const CUtensorMap a_maps[3], int bn, int mt, const GemmArgs& args,
-                                   cudaStream_t stream);
-// Most clusters of `splits` CTAs of that kernel that can be resident at once (0 if unknown).
-int gemm_tc_cluster_capacity(int bn, int mt, int splits);
+// Small-M GEMM (M <= 128 * mt): one output tile per CTA, activation and weight
+// tiles in separate shared-memory rings (weights run further ahead).
+//   epi == EPI_SWIGLU: args.splits == 1, fused SwiGLU epilogue (bf16 out).
+//   epi == EPI_CLUSTER: args.splits K splits per tile, in clusters of
+//     args.cluster CTAs; each cluster adds its splits through DSMEM and writes
+//     f32 slice (split / cluster) at out + slice * group_stride.
+cudaError_t gemm_small_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args,
+                              cudaStream_t stream);
+// Most clusters of `cluster` CTAs of the small-M split-K kernel resident at once (0 if unknown).
+int gemm_small_cluster_capacity(int bn, int mt, int cluster);
 
 // CUDA-core path of the f32 configuration.  a[0..2]: A pieces with row stride k_per_map.
 cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int epi, const GemmArgs& args,

@@ -15,6 +15,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -95,6 +96,16 @@ bool is_device_ptr(const void* p) {
 
 inline long long cdiv(long long a, long long b) { return (a + b - 1) / b; }
 
+// K blocks of weights each small-M GEMM CTA keeps in flight toward L2 ahead of
+// its shared-memory ring (OUTLETS_PREFETCH overrides; default 8).
+int prefetch_blocks() {
+  static const int n = [] {
+    const char* v = getenv("OUTLETS_PREFETCH");
+    return v ? atoi(v) : 8;
+  }();
+  return n;
+}
+
 }  // namespace
 
 struct outlets_ctx {
@@ -122,7 +133,7 @@ struct outlets_ctx {
        *attn = nullptr, *u = nullptr, *hn = nullptr;
   void* taps_stage[3] = {nullptr, nullptr, nullptr};
   int* err_dev = nullptr;
-  float* part = nullptr;  // f32 QKV rows of the small-M path
+  float* part = nullptr;  // f32 split-K slices of the small-M path
   size_t part_floats = 0;
   int* meta_dev = nullptr;
   size_t meta_cap = 0;  // ints
@@ -386,7 +397,7 @@ outlets_status gemm_tc_ex(outlets_ctx* c, const void* const* a, int n_pieces, in
   g.b_np = b_np;
   g.k_per_map = k_piece;
   g.splits = splits;
-  g.prefetch = M <= 256 ? 8 : 0;  // small M streams every weight tile once
+  g.prefetch = M <= 256 ? prefetch_blocks() : 0;  // small M streams every weight tile once
   g.group_m = 16;
   g.out = out;
   g.ldo = ldo;
@@ -412,45 +423,58 @@ outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k
   return gemm_tc_ex(c, a, n_pieces, k_piece, lda, M, b, b_np, N, K, epi, bn, 1, 1, out, ldo, residual, ldr, bias, s);
 }
 
-// Small-M GEMM with the K splits of each output tile reduced inside a
-// thread-block cluster (DSMEM): out f32 [M, N] = A B^T (+ residual), written once.
+// Small-M GEMM (M <= 256): every weight tile is streamed once; K is split so
+// that about one wave of CTAs streams the weights.  The splits of a tile form
+// clusters of sc CTAs that add their partials through DSMEM; the g cluster
+// groups of a tile write g f32 slices part[g][M][N] that the consuming kernel
+// adds up.  Returns the slice count in *slices.
 outlets_status gemm_cluster(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
-                            const void* b, long long b_np, int N, int K, float* out, long long ldo,
-                            const float* residual, long long ldr, cudaStream_t s) {
+                            const void* b, long long b_np, int N, int K, float* part, int* slices, cudaStream_t s) {
   if (M == 0) return OUTLETS_OK;
   const int mt = M <= 128 ? 1 : 2;
   const int bn = cdiv(N, 256) >= 8 ? 256 : 128;
   const long long n_tiles = cdiv(N, bn);
   const long long kb = cdiv(K, 64);
-  int sp = (int)std::max<long long>(1, std::min<long long>(std::min<long long>(8, c->num_sms / n_tiles), kb));
-  // keep every cluster resident in one wave when the hardware allows it
-  while (sp > 1) {
-    const int key = bn * 100 + mt * 10 + sp;
-    auto it = c->cluster_cap.find(key);
-    const int cap = it != c->cluster_cap.end() ? it->second : (c->cluster_cap[key] = gemm_tc_cluster_capacity(bn, mt, sp));
-    if (cap >= n_tiles) break;
-    --sp;
+  int best_sc = 1, best_g = 1;
+  long long best_ctas = -1;
+  for (int sc : {4, 3, 2, 1}) {
+    long long g = std::min<long long>(8, c->num_sms / (n_tiles * sc));
+    while (g > 1 && sc * g > kb) --g;
+    if (g < 1 || sc > kb) continue;
+    if (sc > 1) {
+      const int key = 100000 + bn * 100 + mt * 10 + sc;
+      auto it = c->cluster_cap.find(key);
+      const int cap =
+          it != c->cluster_cap.end() ? it->second : (c->cluster_cap[key] = gemm_small_cluster_capacity(bn, mt, sc));
+      while (g > 1 && n_tiles * g > cap) --g;
+      if (n_tiles * g > cap) continue;
+    }
+    const long long ctas = n_tiles * sc * g;
+    if (ctas > best_ctas) {
+      best_ctas = ctas;
+      best_sc = sc;
+      best_g = (int)g;
+    }
   }
-  const long long kb_per = cdiv(kb, sp);
-  sp = (int)cdiv(kb, kb_per);
+  if ((size_t)best_g * M * N > c->part_floats) return c->fail(OUTLETS_ECAPACITY, "split-K workspace too small");
   CUtensorMap am[3];
   OUT_TRY(a_maps(c, a, n_pieces, k_piece, lda, M, am));
   GemmArgs g{};
   g.M = M;
   g.N = N;
   g.K = K;
-  g.k_per_map = k_piece;
   g.b = b;
   g.b_np = b_np;
-  g.splits = sp;
+  g.k_per_map = k_piece;
+  g.splits = best_sc * best_g;
+  g.cluster = best_sc;
+  g.group_stride = (long long)M * N;
   g.group_m = 1;
-  g.prefetch = 8;
-  g.out = out;
-  g.ldo = ldo;
-  g.residual = residual;
-  g.ldr = ldr;
+  g.out = part;
+  g.ldo = N;
   g.err = c->err_dev;
-  OUT_CK(c, gemm_tc_cluster_launch(am, bn, mt, g, s));
+  OUT_CK(c, gemm_small_launch(am, bn, EPI_CLUSTER, mt, g, s));
+  *slices = best_g;
   return OUTLETS_OK;
 }
 
@@ -485,12 +509,13 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   const int d = c->d;
   const float eps = c->cfg.rms_eps;
   const bool small = small_path(c, rows);
+  int sl = 1;
   // O projection + residual: a = f + attn W_o^T; post-attention RMSNorm
   c->stage_begin(OUTLETS_S_O);
   {
     const void* a1[3] = {c->attn, c->attn, c->attn};
     if (small)
-      OUT_TRY(gemm_cluster(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, c->a, d, c->f, d, s));
+      OUT_TRY(gemm_cluster(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, c->part, &sl, s));
     else if (c->bf16)
       OUT_TRY(gemm_tc(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d,
                       nullptr, s));
@@ -499,7 +524,10 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   }
   c->stage_end(1);
   c->stage_begin(OUTLETS_S_NORM_POST);
-  if (c->bf16)
+  if (small)
+    OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, c->f, nullptr, c->g_post, (bf16*)c->ahat,
+                                          c->a, rows, d, eps, s));
+  else if (c->bf16)
     OUT_CK(c, rmsnorm_launch<bf16>(c->a, c->g_post, (bf16*)c->ahat, nullptr, rows, d, eps, s));
   else
     OUT_CK(c, rmsnorm_launch<float>(c->a, c->g_post, (float*)c->ahat, nullptr, rows, d, eps, s));
@@ -519,8 +547,22 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
           best_bn = bnv;
         }
       }
-      OUT_TRY(gemm_tc_ex(c, a1, 1, d, d, rows, c->w_gu, c->np_gu, 2 * c->Fp, d, EPI_SWIGLU, best_bn,
-                         rows <= 128 ? 1 : 2, 1, c->u, c->Fp, nullptr, 0, nullptr, s));
+      CUtensorMap am[3];
+      OUT_TRY(a_maps(c, a1, 1, d, d, rows, am));
+      GemmArgs g{};
+      g.M = rows;
+      g.N = 2 * c->Fp;
+      g.K = d;
+      g.b = c->w_gu;
+      g.b_np = c->np_gu;
+      g.k_per_map = d;
+      g.splits = 1;
+      g.cluster = 1;
+      g.group_m = 1;
+      g.out = c->u;
+      g.ldo = c->Fp;
+      g.err = c->err_dev;
+      OUT_CK(c, gemm_small_launch(am, best_bn, EPI_SWIGLU, rows <= 128 ? 1 : 2, g, s));
     } else if (c->bf16) {
       OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_gu, c->np_gu, 2 * c->Fp, d, EPI_SWIGLU, c->u, c->Fp, nullptr, 0, nullptr, s));
     } else {
@@ -535,7 +577,7 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   {
     const void* a1[3] = {c->u, c->u, c->u};
     if (small)
-      OUT_TRY(gemm_cluster(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, c->np_down, d, c->Fp, c->y, d, c->a, d, s));
+      OUT_TRY(gemm_cluster(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, c->np_down, d, c->Fp, c->part, &sl, s));
     else if (c->bf16)
       OUT_TRY(gemm_tc(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, c->np_down, d, c->Fp, EPI_F32, c->y, d, c->a, d, nullptr, s));
     else
@@ -544,20 +586,34 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   c->stage_end(1);
   // final RMSNorm of the predicted rows -> h^draft
   c->stage_begin(OUTLETS_S_FINAL_NORM);
-  if (c->bf16)
-    OUT_CK(c, rmsnorm_gather_launch<bf16>(c->y, out_row_idx_dev, c->g_final, (bf16*)c->hn, out_rows, d, eps, s));
-  else
-    OUT_CK(c, rmsnorm_gather_launch<float>(c->y, out_row_idx_dev, c->g_final, (float*)c->hn, out_rows, d, eps, s));
-  c->stage_end(1);
+  int n_final = 1;
+  if (small && !out_row_idx_dev) {
+    // every row is predicted: add the slices and the residual, normalize, in one pass
+    OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, c->a, nullptr, c->g_final, (bf16*)c->hn,
+                                          c->y, rows, d, eps, s));
+  } else {
+    if (small) {
+      // y for every row (the normed copy goes to a dead buffer), then the predicted rows
+      OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, c->a, nullptr, c->g_final,
+                                            (bf16*)c->ahat, c->y, rows, d, eps, s));
+      n_final = 2;
+    }
+    if (c->bf16)
+      OUT_CK(c, rmsnorm_gather_launch<bf16>(c->y, out_row_idx_dev, c->g_final, (bf16*)c->hn, out_rows, d, eps, s));
+    else
+      OUT_CK(c, rmsnorm_gather_launch<float>(c->y, out_row_idx_dev, c->g_final, (float*)c->hn, out_rows, d, eps, s));
+  }
+  c->stage_end(n_final);
   // length head: Linear+ReLU layers, then the output row
   c->stage_begin(OUTLETS_S_HEAD);
   const int nl = (int)c->head_dims.size() - 1;
   const int w1 = c->head_dims[1];
   const void* ah[3] = {c->hn, c->hn, c->hn};
   if (small_path(c, out_rows) && nl == 2) {
-    OUT_TRY(gemm_cluster(c, ah, 1, d, d, out_rows, c->head_w0, c->np_h0, w1, d, c->h1a, w1, nullptr, 0, s));
-    OUT_CK(c, head_tail_launch(c->h1a, 1, 0, c->head_b[0], c->head_wf[1], c->head_b[1], out_rows, w1, z_dev, len_dev,
-                               s));
+    int hs = 1;
+    OUT_TRY(gemm_cluster(c, ah, 1, d, d, out_rows, c->head_w0, c->np_h0, w1, d, c->part, &hs, s));
+    OUT_CK(c, head_tail_launch(c->part, hs, (long long)out_rows * w1, c->head_b[0], c->head_wf[1], c->head_b[1],
+                               out_rows, w1, z_dev, len_dev, s));
     c->stage_end(2);
     return OUTLETS_OK;
   }
@@ -593,12 +649,16 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
   const float eps = c->cfg.rms_eps;
   const bool small = small_path(c, rows);
   c->stage_begin(OUTLETS_S_FC);
-  if (small) OUT_TRY(gemm_cluster(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, c->f, d, nullptr, 0, s));
+  int sl = 1;
+  if (small) OUT_TRY(gemm_cluster(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, c->part, &sl, s));
   else if (c->bf16) OUT_TRY(gemm_tc(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
   else OUT_TRY(gemm_f32(c, tp, d, rows, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
   c->stage_end(1);
   c->stage_begin(OUTLETS_S_NORM_IN);
-  if (c->bf16)
+  if (small)
+    OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, nullptr, nullptr, c->g_in, (bf16*)c->xhat,
+                                          c->f, rows, d, eps, s));
+  else if (c->bf16)
     OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xhat, nullptr, rows, d, eps, s));
   else
     OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
@@ -606,8 +666,8 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
   c->stage_begin(OUTLETS_S_QKV);
   const void* a1[3] = {c->xhat, c->xhat, c->xhat};
   if (small) {
-    OUT_TRY(gemm_cluster(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, c->part, c->qkv_n, nullptr, 0, s));
-    *q = {c->part, true, 1, 0};
+    OUT_TRY(gemm_cluster(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, c->part, &sl, s));
+    *q = {c->part, true, sl, (long long)rows * c->qkv_n};
   } else if (c->bf16) {
     OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, EPI_ACT, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
     *q = {c->qkv, false, 1, 0};
@@ -766,8 +826,9 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->z = (float*)c->alloc(R * 4);
   c->len = (float*)c->alloc(R * 4);
   c->err_dev = (int*)c->alloc(16);
-  if (c->bf16) {  // f32 QKV rows of the small-M path
-    c->part_floats = std::min<size_t>(R, 256) * (size_t)c->qkv_n;
+  if (c->bf16) {  // f32 split-K slices of the small-M path (up to 8 per GEMM)
+    const size_t widest = (size_t)std::max(std::max(d, c->qkv_n), c->head_dims[1]);
+    c->part_floats = (size_t)8 * std::min<size_t>(R, 256) * widest;
     c->part = (float*)c->alloc(c->part_floats * 4);
   }
   if (c->oom) return cleanup_fail(OUTLETS_ENOMEM);

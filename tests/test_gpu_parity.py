@@ -272,3 +272,48 @@ def test_llama8b_step_full_size_sampled():
         check_hidden(attn[r:r + 1], ref["attn"], "bf16", f"step attn request {r}")
     kv.close()
     pred.close()
+
+
+def test_sweep_batch_full_size_sampled():
+    """The serving sweep's largest prefill batch (<= 131072 tokens of the heavy-tailed
+    mixture, arrival order) and one step over its requests, sampled against the oracle."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = synth.LLAMA8B
+    w = synth.make_weights(shape, 0)
+    lengths = synth.lengths_sweep(0)
+    batch, tot = [], 0
+    for i, L in enumerate(lengths):
+        if tot + L > 131072:
+            break
+        batch.append(i)
+        tot += int(L)
+    lens = lengths[batch]
+    B = len(batch)
+    pred = OT.Predictor(shape, w, max_tokens=131072, max_batch=512, max_position=16384)
+    kv = OT.KVCache(pred, max_slots=B, max_tokens_total=tot + 128 * B)
+    order = np.argsort(lens)
+    sample = [int(order[0]), int(order[1]), int(np.argmin(np.abs(lens - 600)))]
+    sample_taps = {b: synth.make_taps(shape, int(lens[b]), 0, 500 + b) for b in sample}
+    gen = torch.Generator(device="cuda").manual_seed(3)
+    parts = [[], [], []]
+    for r in range(B):
+        for i in range(3):
+            if r in sample_taps:
+                parts[i].append(to_device(sample_taps[r][i], "bf16"))
+            else:
+                parts[i].append(torch.randn(int(lens[r]), shape.d, device="cuda", generator=gen).to(torch.bfloat16))
+    taps = [torch.cat(p).contiguous() for p in parts]
+    z, ln = pred.prefill(taps, synth.cu_seqlens(lens), kv=kv, slots=np.arange(B, dtype=np.int32))
+    torch.cuda.synchronize()
+    pred.check()
+    step_taps = synth.make_taps(shape, B, 0, 501)
+    zs, ls = pred.step([to_device(t, "bf16") for t in step_taps], kv, np.arange(B, dtype=np.int32))
+    torch.cuda.synchronize()
+    pred.check()
+    for r in sample:
+        pre = OR.predict_prefill(w, shape, sample_taps[r], np.array([0, lens[r]]))
+        check_z_len(z[r:r + 1], ln[r:r + 1], pre["z"], pre["length"], "bf16", f"sweep prefill request {r}")
+        st = OR.predict_step(w, shape, [t[r:r + 1] for t in step_taps], OR.caches_from_prefill(pre, [0, lens[r]]))
+        check_z_len(zs[r:r + 1], ls[r:r + 1], st["z"], st["length"], "bf16", f"sweep step request {r}")
+    kv.close()
+    pred.close()

@@ -51,6 +51,35 @@ def parse():
     return ap.parse_args()
 
 
+TRAFFIC_SOURCES = {  # files whose content decides the kernel's DRAM traffic (incl. the tile raster)
+    "gateup_swiglu_gemm": ["gemm_tc.cu", "common.cuh", "kernels.h", "outlets.cu"],
+    "decode_attention": ["attn_decode.cu", "mma_sync.cuh", "common.cuh", "kernels.h", "outlets.cu"],
+}
+
+
+def sources_sha(kernel):
+    import hashlib
+    h = hashlib.sha256()
+    for f in TRAFFIC_SOURCES[kernel]:
+        with open(os.path.join(ROOT, "paper_2609_01068_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def measured_traffic(kernel, workload):
+    """DRAM bytes per launch from the committed ncu capture, or None if the kernel's
+    sources changed since (profiles/traffic.json records their hash)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as fh:
+        j = json.load(fh)
+    e = j.get(kernel)
+    if not e or e.get("workload") != workload or e.get("sources_sha256") != sources_sha(kernel):
+        return None
+    return e["dram_bytes_per_launch"]
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -298,7 +327,7 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     roofline = {"bound": "tensor", "kernel": "gateup_swiglu_gemm (k_gemm_tc<256, SWIGLU>)",
                 "achieved": gu_tflops, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
                 "frac": gu_tflops / peaks["bf16_sus"], "peak_kind": f"bf16 sustained {peaks['src']}",
-                "traffic": None,
+                "traffic": measured_traffic("gateup_swiglu_gemm", f"8b-static-{Bq}p-T{T}"),
                 "algorithmic_per_launch": f"{gu_flops:.4g} FLOP = 2*T*(2F)*d, T={T}"}
     stages = {k: {"ms_per_step": v[0] / max(v[1], 1), "share": v[0] / max(sum(x[0] for x in prof.values()), 1e-9)}
               for k, v in prof.items() if v[1]}
@@ -409,7 +438,8 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
             "algorithmic_bytes_per_step": step_bytes,
             "roofline": {"bound": "hbm", "kernel": "decode attention (k_attn_decode_bf16 + combine)",
                          "achieved": at_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                         "frac": at_gbs / peaks["hbm_gbs"], "traffic": None,
+                         "frac": at_gbs / peaks["hbm_gbs"],
+                         "traffic": measured_traffic("decode_attention", f"8b-step-{B}r-L{int(lens.sum())}"),
                          "algorithmic_per_launch": f"{kv_bytes:.4g} B of K/V (cached + new)"},
             "stages": {k: v[0] / max(v[1], 1) for k, v in prof.items() if v[1]},
             "clocks": clocks, "gpu_launches": launches, "host_issue_ms_per_step": host_ms}

@@ -39,12 +39,16 @@ struct TcCfg {
   static constexpr uint32_t A_BYTES = MT * BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  // every byte of the 227 KB a CTA may use goes to the ring (1 KB alignment + barriers aside)
-  static constexpr int STAGES = ((232448 - 1024 - 256) / STAGE_BYTES) > 8 ? 8 : ((232448 - 1024 - 256) / STAGE_BYTES);
+  // epilogue staging: one 32 x 32 f32 chunk per epilogue warp, rows padded to 36 words
+  static constexpr uint32_t EPI_BYTES = 4 * 32 * 36 * 4;
+  // the rest of the 227 KB a CTA may use goes to the ring (1 KB alignment + barriers aside)
+  static constexpr int STAGES = ((232448 - 1024 - 256 - EPI_BYTES) / STAGE_BYTES) > 8
+                                    ? 8
+                                    : ((232448 - 1024 - 256 - EPI_BYTES) / STAGE_BYTES);
   static constexpr uint32_t TMEM_USED = ACC * MT * BN;
   static constexpr uint32_t TMEM_COLS = TMEM_USED <= 32 ? 32 : TMEM_USED <= 64 ? 64 : TMEM_USED <= 128 ? 128
                                                                : TMEM_USED <= 256 ? 256 : 512;  // power of 2
-  static constexpr size_t SMEM = 1024 + STAGES * STAGE_BYTES + 256;
+  static constexpr size_t SMEM = 1024 + STAGES * STAGE_BYTES + 256 + EPI_BYTES;
   static_assert(TMEM_USED <= 512, "TMEM columns");
 };
 
@@ -117,6 +121,7 @@ __global__ void __launch_bounds__(192, 1)
   uint64_t* tempty = tfull + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* epi_stage = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES + 256);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -281,43 +286,61 @@ __global__ void __launch_bounds__(192, 1)
           tmem_ld_32x32b_x32(tbase + c, r);
           tmem_ld_wait();
           const int n0 = tl.n_blk * BN + c;
-          if (row_ok && n0 < p.N) {
+          if constexpr (EPI == EPI_F32 || EPI == EPI_ACT) {
+            // stage the 32 x 32 chunk (thread = row) in shared memory, then write it
+            // out line by line: 8 lanes x 16 bytes cover one row's 32 columns, 4 rows
+            // per instruction.  Row stride 36 words: both directions conflict-free.
+            float* stg = epi_stage + (warp - 2) * (32 * 36);
+#pragma unroll
+            for (int j = 0; j < 32; j += 4)
+              *reinterpret_cast<float4*>(stg + lane * 36 + j) = make_float4(
+                  __uint_as_float(r[j]), __uint_as_float(r[j + 1]), __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3]));
+            __syncwarp();
+            const int row0 = tl.m_blk * TM + mt * BM + quarter * 32;
+            const int cq = (lane & 7) * 4;  // this lane's 4 columns of the chunk
+            const int n = n0 + cq;
+            if (n < p.N) {                  // N % 4 == 0: a lane's 4 columns are all in or all out
+              if constexpr (EPI == EPI_F32) {
+                float4 res[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {  // all residual loads first, then the stores
+                  const int mm = row0 + k * 4 + (lane >> 3);
+                  res[k] = (p.residual && mm < p.M)
+                               ? __ldg(reinterpret_cast<const float4*>(p.residual + (long long)mm * p.ldr + n))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                  const int rr = k * 4 + (lane >> 3);
+                  if (row0 + rr < p.M) {
+                    const float4 v = *reinterpret_cast<const float4*>(stg + rr * 36 + cq);
+                    *reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (long long)(row0 + rr) * p.ldo + n) =
+                        make_float4(v.x + res[k].x, v.y + res[k].y, v.z + res[k].z, v.w + res[k].w);
+                  }
+                }
+              } else {
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                  const int rr = k * 4 + (lane >> 3);
+                  if (row0 + rr < p.M) {
+                    const float4 v = *reinterpret_cast<const float4*>(stg + rr * 36 + cq);
+                    uint2 packed;
+                    packed.x = pack_bf16x2(v.x, v.y);
+                    packed.y = pack_bf16x2(v.z, v.w);
+                    *reinterpret_cast<uint2*>(reinterpret_cast<bf16*>(p.out) + (long long)(row0 + rr) * p.ldo + n) =
+                        packed;
+                  }
+                }
+              }
+            }
+            __syncwarp();
+          } else if (row_ok && n0 < p.N) {  // EPI_BIAS_RELU
             const int valid = min(32, p.N - n0);
             float v[32];
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-            if constexpr (EPI == EPI_F32) {
-              if (p.residual) {
-                const float* res = p.residual + (long long)m * p.ldr + n0;
-                if (valid >= 32) {
-#pragma unroll
-                  for (int j = 0; j < 32; j += 4) {
-                    const float4 q = *reinterpret_cast<const float4*>(res + j);
-                    v[j] += q.x;
-                    v[j + 1] += q.y;
-                    v[j + 2] += q.z;
-                    v[j + 3] += q.w;
-                  }
-                } else {
-                  for (int j = 0; j < valid; ++j) v[j] += res[j];
-                }
-              }
-              store_row32(reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n0, v, valid);
-            } else if constexpr (EPI == EPI_ACT) {
-              store_row32(reinterpret_cast<bf16*>(p.out) + (long long)m * p.ldo + n0, v, valid);
-            } else if constexpr (EPI == EPI_BIAS_RELU) {
-              for (int j = 0; j < valid; ++j) v[j] = fmaxf(v[j] + p.bias[n0 + j], 0.0f);
-              store_row32(reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n0, v, valid);
-            } else {  // EPI_ATOMIC
-              float* dst = reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n0;
-              if (valid >= 32) {
-#pragma unroll
-                for (int j = 0; j < 32; j += 4)
-                  atomicAdd(reinterpret_cast<float4*>(dst + j), make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]));
-              } else {
-                for (int j = 0; j < valid; ++j) atomicAdd(dst + j, v[j]);
-              }
-            }
+            for (int j = 0; j < valid; ++j) v[j] = fmaxf(v[j] + p.bias[n0 + j], 0.0f);
+            store_row32(reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n0, v, valid);
           }
         }
       }

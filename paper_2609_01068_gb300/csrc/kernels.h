@@ -55,7 +55,6 @@ enum Epi : int {
   EPI_ACT = 1,        // out act (bf16 on the tensor-core path, f32 on the CUDA-core path) = acc
   EPI_SWIGLU = 2,     // B rows interleaved in blocks of 32 [gate | up]; out act = silu(g) * u
   EPI_BIAS_RELU = 3,  // out f32 = max(acc + bias, 0)
-  EPI_ATOMIC = 4,     // out f32 += acc (split-K partial sums)
   EPI_CLUSTER = 6,    // small M: split-K reduced inside thread-block clusters (DSMEM), one f32 slice per group
 };
 
@@ -71,7 +70,7 @@ struct GemmArgs {
   const void* b;          // weights, layout above
   long long b_np;         // padded rows per K block
   int k_per_map;          // K extent of each A piece (multiple of 64 when pieces > 1)
-  int splits;             // split-K factor (> 1 only with EPI_ATOMIC); every split non-empty
+  int splits;             // split-K factor (small-M kernel); 1 for the persistent kernel
   int group_m;            // tile raster: M blocks per group
   int prefetch;           // K blocks of B to prefetch into L2 ahead of the smem ring (0 = off)
   int cluster;            // small-M split-K: CTAs per cluster (splits reduced together through DSMEM)

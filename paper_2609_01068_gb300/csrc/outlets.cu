@@ -398,7 +398,9 @@ outlets_status gemm_tc_ex(outlets_ctx* c, const void* const* a, int n_pieces, in
   g.k_per_map = k_piece;
   g.splits = splits;
   g.prefetch = M <= 256 ? prefetch_blocks() : 0;  // small M streams every weight tile once
-  g.group_m = 16;
+  // tile raster: groups of M blocks whose activation panel (128 x K bf16 each)
+  // fills about 48 MB of L2, so each weight tile is fetched once per group
+  g.group_m = (int)std::max<long long>(8, std::min<long long>(cdiv(M, 128), (48ll << 20) / (128ll * K * 2)));
   g.out = out;
   g.ldo = ldo;
   g.residual = residual;
@@ -1125,7 +1127,6 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
   const int* m = c->meta_dev;
   const int* cu_dev = m + off_cu;
 
-  const int d = c->d;
   // ---- FC (Eq. 1) -> input RMSNorm -> QKV
   QkvSrc qsrc;
   OUT_TRY(run_front(c, tp, T, &qsrc, s));
@@ -1234,7 +1235,6 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
   const size_t off_wo = mb.put(work_off);
   OUT_TRY(upload_meta(c, mb.v, s));
   const int* m = c->meta_dev;
-  const int d = c->d;
 
   QkvSrc qsrc;
   OUT_TRY(run_front(c, tp, B, &qsrc, s));

@@ -452,7 +452,6 @@ __global__ void __launch_bounds__(192, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   pdl_trigger();
-  pdl_wait();
 
   const int S = p.splits;
   const int tile = blockIdx.x / S;
@@ -465,14 +464,24 @@ __global__ void __launch_bounds__(192, 1)
   const int kb0 = (int)(((long long)split * kb_total) / S);
   const int kb1 = (int)(((long long)(split + 1) * kb_total) / S);
   const bf16* wt = reinterpret_cast<const bf16*>(p.b) + (long long)n_blk * BN * BK;
+  // Weights do not depend on the previous kernel: fill the first weight slots
+  // while it is still running, before waiting for its outputs (activations).
+  const int pre = min(WS, kb1 - kb0);
+  if (warp == 0 && lane == 0) {
+    for (int i = 0; i < pre; ++i) {
+      mbar_arrive_expect_tx(&fullW[i], C::B_BYTES);
+      bulk_load(sW + i * C::B_BYTES, wt + (long long)(kb0 + i) * p.b_np * BK, C::B_BYTES, &fullW[i]);
+    }
+  }
+  pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
       constexpr int lag = WS - AS;  // >= 0
-      int ws = 0, as = 0;
-      uint32_t wph = 0, aph = 0;
+      int ws = pre % WS, as = 0;
+      uint32_t wph = pre == WS ? 1u : 0u, aph = 0;
       for (int i = kb0; i < kb1 + lag; ++i) {
-        if (i < kb1) {
+        if (i < kb1 && i >= kb0 + pre) {
           if (!mbar_wait(&emptyW[ws], wph ^ 1u, abort_flag, p.err)) break;
           mbar_arrive_expect_tx(&fullW[ws], C::B_BYTES);
           bulk_load(sW + ws * C::B_BYTES, wt + (long long)i * p.b_np * BK, C::B_BYTES, &fullW[ws]);

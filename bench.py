@@ -182,6 +182,34 @@ def oracle_sample(shape, w, taps, cu, lengths, budget_tokens):
     return len(picks), tot, dt
 
 
+class ReplicaGroup:
+    """N independent replicas, one per GPU (requests never interact, so nothing
+    is exchanged on the data path): a barrier around the timed region and a
+    max over ranks of its duration.  Whole-job throughput = N * units / max time."""
+
+    def __init__(self, world, rank, device, sync=None):
+        self.world, self.rank, self.device, self.sync = world, rank, device, sync
+
+    def barrier(self):
+        import torch.distributed as dist
+        if self.sync:
+            self.sync()
+        if self.world > 1:
+            dist.barrier()
+
+    def max(self, x):
+        if self.world == 1:
+            return float(x)
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([float(x)], dtype=torch.float64, device=self.device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def throughput(self, units_per_rank, seconds):
+        return self.world * units_per_rank / self.max(seconds)
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -243,17 +271,8 @@ def run_ours(args):
                              device=local)
     stream = torch.cuda.current_stream()
 
-    def barrier():
-        torch.cuda.synchronize()
-        if world > 1:
-            dist.barrier()
-
-    def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+    group = ReplicaGroup(world, rank, "cuda", sync=torch.cuda.synchronize)
+    barrier, max_over_ranks = group.barrier, group.max
 
     out = {"metric": METRIC, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic"}

@@ -231,6 +231,14 @@ outlets_status outlets_profile_read(outlets_ctx* ctx, double* ms, int32_t* count
 /* Static name of a stage ("fc_gemm", ...), or "" for an invalid id. */
 const char* outlets_stage_name(int32_t stage);
 
+/* Failure-path self-test (the paper has no counterpart).  Enqueues one kernel
+ * whose bounded wait on an mbarrier can never complete -- the wait every
+ * prediction pipeline uses -- so it gives up after timeout_ns (1 us .. 1 s)
+ * and raises the context's device error word, as a stalled pipeline would.
+ * The next outlets_check then returns OUTLETS_ETIMEOUT (and clears the word);
+ * the context stays usable.  Faults nothing, hangs nothing. */
+outlets_status outlets_selftest_bounded_wait(outlets_ctx* ctx, uint64_t timeout_ns, void* stream);
+
 /* Number of kernels this context has launched for prediction calls so far. */
 uint64_t outlets_launch_count(const outlets_ctx* ctx);
 

@@ -64,14 +64,15 @@ OUTLETS_DEV bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // Waits for the phase with the given parity to complete.  Gives up (returns
 // false) when the CTA-wide abort flag is raised or after kWaitTimeoutNs, in
 // which case it raises the abort flag and the global error word.
-OUTLETS_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err) {
+OUTLETS_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
+                           unsigned long long timeout_ns = kWaitTimeoutNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = global_timer_ns();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((i & 31u) == 0) {
       if (*abort_flag) return false;
-      if (global_timer_ns() - t0 > kWaitTimeoutNs) {
+      if (global_timer_ns() - t0 > timeout_ns) {
         *abort_flag = 1;
         if (err) atomicOr(err, ERR_TIMEOUT);
         return false;

@@ -377,6 +377,21 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const float* __restrict__ a0,
   }
 }
 
+// A wait that nothing completes: the bounded-wait path every pipeline uses
+// (mbar_wait) gives up after timeout_ns and raises ERR_TIMEOUT.
+__global__ void k_wait_selftest(int* err, unsigned long long timeout_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_wait(&bar, 0, &abort_flag, err, timeout_ns);
+  __syncthreads();
+}
+
 inline int grid_for(long long n, int threads) {
   long long g = (n + threads - 1) / threads;
   if (g > 152LL * 32) g = 152LL * 32;
@@ -449,6 +464,11 @@ cudaError_t convert_rows_launch(const float* src, Act* dst, int rows, int cols, 
   if (rows == 0 || cols == 0) return cudaSuccess;
   OUTLETS_TRY_LAUNCH(launch_k(k_convert_rows<Act>, dim3(grid_for((long long)rows * cols, 256)), dim3(256), 0, stream, src, dst, rows, cols, dst_ld,
                                                                                 row_mode, row_base, kb_np));
+  return cudaGetLastError();
+}
+
+cudaError_t wait_selftest_launch(int* err, unsigned long long timeout_ns, cudaStream_t stream) {
+  k_wait_selftest<<<1, 32, 0, stream>>>(err, timeout_ns);
   return cudaGetLastError();
 }
 

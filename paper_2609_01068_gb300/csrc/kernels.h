@@ -164,6 +164,9 @@ template <typename Act>
 cudaError_t convert_rows_launch(const float* src, Act* dst, int rows, int cols, long long dst_ld, int row_mode,
                                 int row_base, long long kb_np, cudaStream_t stream);
 
+// One CTA whose bounded mbarrier wait can never complete: raises ERR_TIMEOUT in err.
+cudaError_t wait_selftest_launch(int* err, unsigned long long timeout_ns, cudaStream_t stream);
+
 // ---------------------------------------------------------------- attention
 struct AttnTile {
   int q_start;    // first query row (packed index)

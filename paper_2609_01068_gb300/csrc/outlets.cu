@@ -911,6 +911,16 @@ void outlets_destroy(outlets_ctx* c) {
   delete c;
 }
 
+outlets_status outlets_selftest_bounded_wait(outlets_ctx* c, uint64_t timeout_ns, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  if (timeout_ns < 1000 || timeout_ns > 1000000000ull)
+    return c->fail(OUTLETS_EINVAL, "timeout_ns must be in [1 us, 1 s]");
+  OUT_CK(c, cudaSetDevice(c->cfg.device));
+  OUT_CK(c, wait_selftest_launch(c->err_dev, timeout_ns, (cudaStream_t)stream));
+  return OUTLETS_OK;
+}
+
 outlets_status outlets_profile_enable(outlets_ctx* c, int32_t enable) {
   if (!c) return OUTLETS_EINVAL;
   OUT_CK(c, cudaSetDevice(c->cfg.device));

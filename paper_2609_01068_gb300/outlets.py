@@ -82,6 +82,7 @@ def load():
         "outlets_stage_name": (ctypes.c_char_p, [c_i32]),
         "outlets_launch_count": (ctypes.c_uint64, [c_vp]),
         "outlets_length_head_noalloc": (c_i32, [c_vp, c_vp, c_i32, c_vp, c_vp, c_vp]),
+        "outlets_selftest_bounded_wait": (c_i32, [c_vp, ctypes.c_uint64, c_vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -206,6 +207,12 @@ class Predictor:
         if st != OK:
             self._raise(st)
         return z_out, len_out
+
+    def selftest_bounded_wait(self, timeout_ns=1_000_000, stream=None):
+        """Enqueue a kernel whose bounded wait runs out (see outlets_check)."""
+        st = self.lib.outlets_selftest_bounded_wait(self.h, timeout_ns, _stream_handle(stream))
+        if st != OK:
+            self._raise(st)
 
     def check(self, stream=None):
         st = self.lib.outlets_check(self.h, _stream_handle(stream))

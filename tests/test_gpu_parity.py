@@ -317,3 +317,23 @@ def test_sweep_batch_full_size_sampled():
         check_z_len(zs[r:r + 1], ls[r:r + 1], st["z"], st["length"], "bf16", f"sweep step request {r}")
     kv.close()
     pred.close()
+
+
+def test_bounded_wait_timeout_is_reported_and_context_survives():
+    """A kernel whose wait never completes gives up after its limit, the host
+    reads OUTLETS_ETIMEOUT, and the next prediction is still correct."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = MID128
+    pred, w = predictor("mid128")
+    pred.check()
+    pred.selftest_bounded_wait(timeout_ns=2_000_000)
+    with pytest.raises(OT.OutletsError) as e:
+        pred.check()
+    assert e.value.status == OT.ETIMEOUT
+    pred.check()  # the error word was cleared
+    cu = synth.cu_seqlens([9, 70])
+    taps = _taps(shape, int(cu[-1]), off=8)
+    z, ln = pred.prefill([to_device(t, "bf16") for t in taps], cu)
+    ref = OR.predict_prefill(w, shape, taps, cu)
+    check_z_len(z, ln, ref["z"], ref["length"], "bf16", "after timeout")
+    pred.check()

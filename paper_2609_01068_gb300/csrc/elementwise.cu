@@ -10,6 +10,8 @@
 //   SwiGLU            silu(gate) * up (the decoder layer's MLP block)
 //   head tail         z_hat = w . relu(h + b) + b_out, length = max(0, expm1(z_hat))
 //                     (Sec. 4.2: log-space target z = log(1 + length))
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -29,6 +31,55 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return red[32];
 }
 
+// Split-K slices: s[0] + s[1] + ... + s[n-1] at p, p + stride, ..., added in
+// slice order (the same order on every call); the loads of up to nine slices
+// are in flight together.
+__device__ __forceinline__ void add4(float4& a, const float4& b) {
+  a.x += b.x;
+  a.y += b.y;
+  a.z += b.z;
+  a.w += b.w;
+}
+__device__ __forceinline__ float4 ld_sum4(const float* p, int n, long long stride) {
+  float4 acc = *reinterpret_cast<const float4*>(p);
+  for (int s0 = 1; s0 < n; s0 += 8) {
+    float4 v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (s0 + k < n) v[k] = *reinterpret_cast<const float4*>(p + (s0 + k) * stride);
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (s0 + k < n) add4(acc, v[k]);
+  }
+  return acc;
+}
+// Two float4 runs (8 floats at p and 8 at q) summed over the slices; up to five
+// slices of both in flight together.
+__device__ __forceinline__ void ld_sum16(const float* p, const float* q, int n, long long stride, float4 (&o)[4]) {
+  o[0] = *reinterpret_cast<const float4*>(p);
+  o[1] = *reinterpret_cast<const float4*>(p + 4);
+  o[2] = *reinterpret_cast<const float4*>(q);
+  o[3] = *reinterpret_cast<const float4*>(q + 4);
+  for (int s0 = 1; s0 < n; s0 += 4) {
+    float4 v[4][4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (s0 + k < n) {
+        const long long off = (s0 + k) * stride;
+        v[k][0] = *reinterpret_cast<const float4*>(p + off);
+        v[k][1] = *reinterpret_cast<const float4*>(p + off + 4);
+        v[k][2] = *reinterpret_cast<const float4*>(q + off);
+        v[k][3] = *reinterpret_cast<const float4*>(q + off + 4);
+      }
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (s0 + k < n) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) add4(o[j], v[k][j]);
+      }
+  }
+}
+
 template <typename Act>
 __device__ __forceinline__ void store4(Act* p, float a, float b, float c, float d);
 template <>
@@ -43,11 +94,11 @@ __device__ __forceinline__ void store4<bf16>(bf16* p, float a, float b, float c,
   *reinterpret_cast<uint2*>(p) = v;
 }
 
-// v = residual[src] + sum_s x[s][src] (split-K slices of the producing GEMM);
+// v = (sum_s x[s][src]) + residual[src] (split-K slices of the producing GEMM, in slice order);
 // y[r] = v * g * rsqrt(mean(v^2) + eps); copy_out[r] = v (f32) when given.
 // REDUCE = false: v = x[src] (one slice, no residual).
 template <typename Act, bool REDUCE>
-__global__ void k_rmsnorm(const float* __restrict__ x, int n_split, long long split_stride,
+__global__ void __launch_bounds__(1024) k_rmsnorm(const float* __restrict__ x, int n_split, long long split_stride,
                           const float* __restrict__ residual, const int* __restrict__ row_index,
                           const float* __restrict__ g, Act* __restrict__ y, float* __restrict__ copy_out, int d,
                           float eps) {
@@ -59,41 +110,13 @@ __global__ void k_rmsnorm(const float* __restrict__ x, int n_split, long long sp
   const long long src = row_index ? row_index[r] : r;
   float ss = 0.f;
   for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
-    float4 v = *reinterpret_cast<const float4*>(x + src * d + i);
+    float4 v;
     if constexpr (REDUCE) {
-      float4 v2 = make_float4(0.f, 0.f, 0.f, 0.f);
-      int sp = 1;
-      for (; sp + 1 < n_split; sp += 2) {  // two independent partial sums
-        const float4 a = *reinterpret_cast<const float4*>(x + sp * split_stride + src * d + i);
-        const float4 b = *reinterpret_cast<const float4*>(x + (sp + 1) * split_stride + src * d + i);
-        v.x += a.x;
-        v.y += a.y;
-        v.z += a.z;
-        v.w += a.w;
-        v2.x += b.x;
-        v2.y += b.y;
-        v2.z += b.z;
-        v2.w += b.w;
-      }
-      if (sp < n_split) {
-        const float4 a = *reinterpret_cast<const float4*>(x + sp * split_stride + src * d + i);
-        v.x += a.x;
-        v.y += a.y;
-        v.z += a.z;
-        v.w += a.w;
-      }
-      if (residual) {
-        const float4 a = *reinterpret_cast<const float4*>(residual + src * d + i);
-        v2.x += a.x;
-        v2.y += a.y;
-        v2.z += a.z;
-        v2.w += a.w;
-      }
-      v.x += v2.x;
-      v.y += v2.y;
-      v.z += v2.z;
-      v.w += v2.w;
+      v = ld_sum4(x + src * d + i, n_split, split_stride);
+      if (residual) add4(v, *reinterpret_cast<const float4*>(residual + src * d + i));
       rowbuf[i >> 2] = v;
+    } else {
+      v = *reinterpret_cast<const float4*>(x + src * d + i);
     }
     ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
   }
@@ -126,21 +149,26 @@ __device__ __forceinline__ void load8<bf16>(const bf16* p, long long idx, int, l
 template <>
 __device__ __forceinline__ void load8<float>(const float* p, long long idx, int n_split, long long stride,
                                              float* v) {
-  float4 a = *reinterpret_cast<const float4*>(p + idx);
-  float4 b = *reinterpret_cast<const float4*>(p + idx + 4);
-  for (int sp = 1; sp < n_split; ++sp) {
-    const float4 c = *reinterpret_cast<const float4*>(p + sp * stride + idx);
-    const float4 e = *reinterpret_cast<const float4*>(p + sp * stride + idx + 4);
-    a.x += c.x;
-    a.y += c.y;
-    a.z += c.z;
-    a.w += c.w;
-    b.x += e.x;
-    b.y += e.y;
-    b.z += e.z;
-    b.w += e.w;
-  }
+  const float4 a = ld_sum4(p + idx, n_split, stride);
+  const float4 b = ld_sum4(p + idx + 4, n_split, stride);
   v[0] = a.x, v[1] = a.y, v[2] = a.z, v[3] = a.w, v[4] = b.x, v[5] = b.y, v[6] = b.z, v[7] = b.w;
+}
+// Both halves of a rotation pair (8 elements at idx and at idx + half).
+template <typename In>
+__device__ __forceinline__ void load8x2(const In* p, long long idx, long long half, int n_split, long long stride,
+                                        float* v1, float* v2) {
+  load8<In>(p, idx, n_split, stride, v1);
+  load8<In>(p, idx + half, n_split, stride, v2);
+}
+template <>
+__device__ __forceinline__ void load8x2<float>(const float* p, long long idx, long long half, int n_split,
+                                               long long stride, float* v1, float* v2) {
+  float4 o[4];
+  ld_sum16(p + idx, p + idx + half, n_split, stride, o);
+  v1[0] = o[0].x, v1[1] = o[0].y, v1[2] = o[0].z, v1[3] = o[0].w;
+  v1[4] = o[1].x, v1[5] = o[1].y, v1[6] = o[1].z, v1[7] = o[1].w;
+  v2[0] = o[2].x, v2[1] = o[2].y, v2[2] = o[2].z, v2[3] = o[2].w;
+  v2[4] = o[3].x, v2[5] = o[3].y, v2[6] = o[3].z, v2[7] = o[3].w;
 }
 
 template <typename Act>
@@ -163,7 +191,7 @@ __device__ __forceinline__ void store8<float>(float* p, const float* v) {
 // One CTA per row; a thread rotates 8 pairs (i..i+7 with i+hd/2..i+hd/2+7) of
 // one head and copies 8 values of V.  hd is a multiple of 16.
 template <typename In, typename Act>
-__global__ void k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
+__global__ void __launch_bounds__(512) k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
   pdl_trigger();
   pdl_wait();
   const int row = blockIdx.x;
@@ -205,8 +233,7 @@ __global__ void k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
     const int head = idx / cpr;
     const int i = (idx - head * cpr) * 8;
     float x1[8], x2[8], y1[8], y2[8];
-    load8<In>(src, head * hd + i, a.n_split, a.split_stride, x1);
-    load8<In>(src, head * hd + i + half, a.n_split, a.split_stride, x2);
+    load8x2<In>(src, head * hd + i, half, a.n_split, a.split_stride, x1, x2);
     const float4 c0 = *reinterpret_cast<const float4*>(cs + i);
     const float4 c1 = *reinterpret_cast<const float4*>(cs + i + 4);
     const float4 s0 = *reinterpret_cast<const float4*>(sn + i);
@@ -264,7 +291,7 @@ __global__ void k_swiglu(const float* __restrict__ gu, Act* __restrict__ u, int 
 }
 
 // One CTA per row: h = sum of slices, a = relu(h + b_prev), z = w_last . a + b_last.
-__global__ void k_head_tail(const float* __restrict__ h, int n_split, long long split_stride,
+__global__ void __launch_bounds__(512) k_head_tail(const float* __restrict__ h, int n_split, long long split_stride,
                             const float* __restrict__ b_prev, const float* __restrict__ w_last,
                             const float* __restrict__ b_last, int rows, int width, float* __restrict__ z,
                             float* __restrict__ len) {
@@ -274,17 +301,23 @@ __global__ void k_head_tail(const float* __restrict__ h, int n_split, long long 
   const int r = blockIdx.x;
   const float* hr = h + (long long)r * width;
   float acc = 0.f;
-  for (int j = threadIdx.x; j < width; j += blockDim.x) {
-    float x0 = hr[j], x1 = 0.f;
-    int sp = 1;
-    for (; sp + 1 < n_split; sp += 2) {
-      x0 += hr[sp * split_stride + j];
-      x1 += hr[(sp + 1) * split_stride + j];
+  if ((width & 3) == 0) {
+    for (int j = threadIdx.x * 4; j < width; j += blockDim.x * 4) {
+      float4 x = ld_sum4(hr + j, n_split, split_stride);
+      if (b_prev) {
+        const float4 b = *reinterpret_cast<const float4*>(b_prev + j);
+        x = make_float4(fmaxf(x.x + b.x, 0.f), fmaxf(x.y + b.y, 0.f), fmaxf(x.z + b.z, 0.f), fmaxf(x.w + b.w, 0.f));
+      }
+      const float4 wl = *reinterpret_cast<const float4*>(w_last + j);
+      acc += wl.x * x.x + wl.y * x.y + wl.z * x.z + wl.w * x.w;
     }
-    if (sp < n_split) x0 += hr[sp * split_stride + j];
-    float x = x0 + x1;
-    if (b_prev) x = fmaxf(x + b_prev[j], 0.f);
-    acc += w_last[j] * x;
+  } else {
+    for (int j = threadIdx.x; j < width; j += blockDim.x) {
+      float x = hr[j];
+      for (int sp = 1; sp < n_split; ++sp) x += hr[sp * split_stride + j];
+      if (b_prev) x = fmaxf(x + b_prev[j], 0.f);
+      acc += w_last[j] * x;
+    }
   }
   acc = block_sum(acc, red);
   if (threadIdx.x == 0) {
@@ -428,7 +461,9 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
         attr = true;
       }
     }
-    OUTLETS_TRY_LAUNCH(launch_k(k_rmsnorm<Act, true>, dim3(rows), dim3(256), smem, stream, x, n_split, split_stride, residual, row_index, g, y, copy_out,
+    // one float4 of the row per thread where d allows: every slice load of a row in flight at once
+    const int threads = std::min(1024, std::max(64, ((d / 4 + 31) / 32) * 32));
+    OUTLETS_TRY_LAUNCH(launch_k(k_rmsnorm<Act, true>, dim3(rows), dim3(threads), smem, stream, x, n_split, split_stride, residual, row_index, g, y, copy_out,
                                                       d, eps));
   } else {
     OUTLETS_TRY_LAUNCH(launch_k(k_rmsnorm<Act, false>, dim3(rows), dim3(256), 0, stream, x, 1, 0, nullptr, row_index, g, y, copy_out, d, eps));
@@ -439,7 +474,9 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
 template <typename In, typename Act>
 cudaError_t rope_scatter_launch(const In* qkv, const RopeArgs& a, cudaStream_t stream) {
   if (a.T == 0) return cudaSuccess;
-  OUTLETS_TRY_LAUNCH(launch_k(k_rope_scatter<In, Act>, dim3(a.T), dim3(128), 0, stream, qkv, a));
+  const int items = (a.H + a.KVH) * (a.hd / 16);  // rotation chunks per row: about one per thread
+  const int threads = std::min(512, std::max(64, ((items + 31) / 32) * 32));
+  OUTLETS_TRY_LAUNCH(launch_k(k_rope_scatter<In, Act>, dim3(a.T), dim3(threads), 0, stream, qkv, a));
   return cudaGetLastError();
 }
 
@@ -454,7 +491,8 @@ cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_st
                              const float* w_last, const float* b_last, int rows, int width, float* z, float* len,
                              cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
-  OUTLETS_TRY_LAUNCH(launch_k(k_head_tail, dim3(rows), dim3(128), 0, stream, h_pre, n_split, split_stride, b_prev, w_last, b_last, rows, width, z, len));
+  const int threads = std::min(512, std::max(64, ((width / 4 + 31) / 32) * 32));
+  OUTLETS_TRY_LAUNCH(launch_k(k_head_tail, dim3(rows), dim3(threads), 0, stream, h_pre, n_split, split_stride, b_prev, w_last, b_last, rows, width, z, len));
   return cudaGetLastError();
 }
 

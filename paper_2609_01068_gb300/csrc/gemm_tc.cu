@@ -12,8 +12,8 @@
 // the main loop of tile i+1.  Every mbarrier wait is bounded.
 //
 // k_gemm_small (M <= 256, dynamic prediction and the head): one output tile and
-// one K split per CTA, every weight tile streamed once; K splits of a tile form
-// thread-block clusters reduced through distributed shared memory.
+// one K split per CTA, every weight tile streamed once; each K split writes an
+// f32 slice that the consuming kernel adds up.
 //
 // Used for Eq. 1 (three-tap fusion: A is split along K over the three taps),
 // the QKV / O / gate-up / down projections of the draft decoder layer, and
@@ -86,7 +86,9 @@ __device__ __forceinline__ void store_row32<float>(float* dst, const float* v, i
     for (int j = 0; j < 32; j += 4)
       *reinterpret_cast<float4*>(dst + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
   } else {
-    for (int j = 0; j < valid; ++j) dst[j] = v[j];
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < valid) dst[j] = v[j];
   }
 }
 
@@ -103,7 +105,9 @@ __device__ __forceinline__ void store_row32<bf16>(bf16* dst, const float* v, int
       *reinterpret_cast<uint4*>(dst + j) = p;
     }
   } else {
-    for (int j = 0; j < valid; ++j) dst[j] = __float2bfloat16_rn(v[j]);
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < valid) dst[j] = __float2bfloat16_rn(v[j]);
   }
 }
 
@@ -338,8 +342,7 @@ __global__ void __launch_bounds__(192, 1)
             const int valid = min(32, p.N - n0);
             float v[32];
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-            for (int j = 0; j < valid; ++j) v[j] = fmaxf(v[j] + p.bias[n0 + j], 0.0f);
+            for (int j = 0; j < 32; ++j) v[j] = j < valid ? fmaxf(__uint_as_float(r[j]) + p.bias[n0 + j], 0.0f) : 0.0f;
             store_row32(reinterpret_cast<float*>(p.out) + (long long)m * p.ldo + n0, v, valid);
           }
         }
@@ -571,36 +574,33 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else {
-    // Cluster reduction: the p.cluster CTAs of a cluster hold partial sums of
-    // the same tile over different K splits.  Per round of CW columns each CTA
-    // stages its partial in its (now idle) rings, then adds one contiguous
-    // column stripe across the cluster through DSMEM and writes it to the
-    // slice of its cluster group.  All threads pass every cluster barrier.
+    // Split-K partial: the f32 tile of this K split goes to slice `split`
+    // (out + split * group_stride); the consuming kernel adds the slices in
+    // slice order, so the sum does not depend on scheduling.  The tile is
+    // staged in the idle ring CW columns at a time (warps 2..5 read TMEM, one
+    // row per thread) and written by all six warps with row-contiguous float4
+    // stores (a warp store covers one 512-byte row segment).
     constexpr int CW = BN < 128 ? BN : 128;
-    constexpr int LD = CW + 4;
-    constexpr int G = CW / 4;
-    const int Sc = p.cluster;
-    const uint32_t rank = Sc > 1 ? cluster_ctarank() : 0u;
-    const int group = split / Sc;
-    float* red = reinterpret_cast<float*>(smem);
-    const uint32_t red_addr = smem_u32(red);
-    const int per = (G + Sc - 1) / Sc;
-    const int g0 = min(G, (int)rank * per);
-    const int g1 = min(G, g0 + per);
-    const int my_groups = g1 - g0;
-    float* out = reinterpret_cast<float*>(p.out) + (long long)group * p.group_stride;
+    constexpr int LD = CW + 4;  // 16-byte row skew: conflict-free thread-per-row staging
+    constexpr int Q = CW / 4;   // float4 per staged row
+    constexpr int ITEMS = TM * Q;
+    static_assert((size_t)TM * LD * 4 <= C::RING_BYTES, "stage fits in the ring");
+    float* stage = reinterpret_cast<float*>(smem);
+    float* out = reinterpret_cast<float*>(p.out) + (long long)split * p.group_stride;
     for (int rd = 0; rd < BN / CW; ++rd) {
+      if (rd > 0) __syncthreads();  // the previous round's reads of the stage are done
       if (warp >= 2 && have) {
 #pragma unroll 1
         for (int mt = 0; mt < MT; ++mt) {
           const int row = mt * BM + quarter * 32 + lane;
           const uint32_t tb = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                               static_cast<uint32_t>(mt * BN + rd * CW);
+#pragma unroll 1
           for (int c = 0; c < CW; c += 32) {
             uint32_t r[32];
             tmem_ld_32x32b_x32(tb + c, r);
             tmem_ld_wait();
-            float* dst = red + row * LD + c;
+            float* dst = stage + row * LD + c;
 #pragma unroll
             for (int j = 0; j < 32; j += 4)
               *reinterpret_cast<float4*>(dst + j) = make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]),
@@ -608,35 +608,20 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
       }
-      if (Sc > 1) cluster_sync_all();
-      else __syncthreads();
-      if (!*abort_flag && my_groups > 0) {
-        const int items = TM * my_groups;
-        for (int it = threadIdx.x; it < items; it += blockDim.x) {
-          const int row = it / my_groups;
-          const int col = (g0 + it - row * my_groups) * 4;
+      __syncthreads();
+      if (!*abort_flag) {
+        const int n0 = n_blk * BN + rd * CW;
+#pragma unroll 4
+        for (int it = threadIdx.x; it < ITEMS; it += 192) {
+          const int row = it / Q;
+          const int col = (it - row * Q) * 4;
           const int m = m_blk * TM + row;
-          const int n = n_blk * BN + rd * CW + col;
-          if (m >= p.M || n >= p.N) continue;
-          const uint32_t off = red_addr + static_cast<uint32_t>((row * LD + col) * 4);
-          float4 acc;
-          if (Sc > 1) {
-            acc = dsmem_ld_f4(dsmem_map(off, 0));
-            for (int q = 1; q < Sc; ++q) {
-              const float4 v = dsmem_ld_f4(dsmem_map(off, q));
-              acc.x += v.x;
-              acc.y += v.y;
-              acc.z += v.z;
-              acc.w += v.w;
-            }
-          } else {
-            acc = *reinterpret_cast<const float4*>(red + row * LD + col);
-          }
-          *reinterpret_cast<float4*>(out + (long long)m * p.ldo + n) = acc;
+          const int n = n0 + col;
+          if (m < p.M && n < p.N)
+            *reinterpret_cast<float4*>(out + (long long)m * p.ldo + n) =
+                *reinterpret_cast<const float4*>(stage + row * LD + col);
         }
       }
-      if (Sc > 1) cluster_sync_all();
-      else __syncthreads();
     }
   }
 
@@ -665,15 +650,8 @@ cudaError_t launch_small(const CUtensorMap a_maps[3], const GemmArgs& args, cuda
   cfg.blockDim = dim3(192);
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = stream;
-  cudaLaunchAttribute at[2];
+  cudaLaunchAttribute at[1];
   int n = 0;
-  if (EPI == EPI_CLUSTER && args.cluster > 1) {
-    at[n].id = cudaLaunchAttributeClusterDimension;
-    at[n].val.clusterDim.x = args.cluster;
-    at[n].val.clusterDim.y = 1;
-    at[n].val.clusterDim.z = 1;
-    ++n;
-  }
   if (pdl_enabled()) {
     at[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     at[n].val.programmaticStreamSerializationAllowed = 1;
@@ -696,14 +674,13 @@ bool pdl_enabled() {
 
 cudaError_t gemm_small_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args,
                               cudaStream_t stream) {
-  if (args.splits < 1 || args.cluster < 1 || args.splits % args.cluster || args.cluster > 8)
-    return cudaErrorInvalidValue;
+  if (args.splits < 1 || (epi == EPI_SLICES && args.N % 4)) return cudaErrorInvalidValue;
 #define OUTLETS_SM_CASE(BNV, EV, MTV) \
   if (bn == BNV && epi == EV && mt == MTV) return launch_small<BNV, EV, MTV>(a_maps, args, stream);
-  OUTLETS_SM_CASE(256, EPI_CLUSTER, 2)
-  OUTLETS_SM_CASE(256, EPI_CLUSTER, 1)
-  OUTLETS_SM_CASE(128, EPI_CLUSTER, 2)
-  OUTLETS_SM_CASE(128, EPI_CLUSTER, 1)
+  OUTLETS_SM_CASE(256, EPI_SLICES, 2)
+  OUTLETS_SM_CASE(256, EPI_SLICES, 1)
+  OUTLETS_SM_CASE(128, EPI_SLICES, 2)
+  OUTLETS_SM_CASE(128, EPI_SLICES, 1)
   OUTLETS_SM_CASE(256, EPI_SWIGLU, 2)
   OUTLETS_SM_CASE(256, EPI_SWIGLU, 1)
   OUTLETS_SM_CASE(192, EPI_SWIGLU, 2)  // 4 slots of 56 KB
@@ -712,41 +689,6 @@ cudaError_t gemm_small_launch(const CUtensorMap a_maps[3], int bn, int epi, int 
   OUTLETS_SM_CASE(128, EPI_SWIGLU, 1)
 #undef OUTLETS_SM_CASE
   return cudaErrorInvalidValue;
-}
-
-template <int BN, int MT>
-int small_capacity(int cluster) {
-  using C = SmCfg<BN, MT>;
-  auto kern = k_gemm_small<BN, EPI_CLUSTER, MT>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
-  }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(cluster * 64);
-  cfg.blockDim = dim3(192);
-  cfg.dynamicSmemBytes = C::SMEM;
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = cluster;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
-  int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
-  }
-  return n;
-}
-
-int gemm_small_cluster_capacity(int bn, int mt, int cluster) {
-  if (bn == 256 && mt == 2) return small_capacity<256, 2>(cluster);
-  if (bn == 256 && mt == 1) return small_capacity<256, 1>(cluster);
-  if (bn == 128 && mt == 2) return small_capacity<128, 2>(cluster);
-  if (bn == 128 && mt == 1) return small_capacity<128, 1>(cluster);
-  return 0;
 }
 
 cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args, int num_sms,

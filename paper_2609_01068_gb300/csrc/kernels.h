@@ -55,7 +55,7 @@ enum Epi : int {
   EPI_ACT = 1,        // out act (bf16 on the tensor-core path, f32 on the CUDA-core path) = acc
   EPI_SWIGLU = 2,     // B rows interleaved in blocks of 32 [gate | up]; out act = silu(g) * u
   EPI_BIAS_RELU = 3,  // out f32 = max(acc + bias, 0)
-  EPI_CLUSTER = 6,    // small M: split-K reduced inside thread-block clusters (DSMEM), one f32 slice per group
+  EPI_SLICES = 6,     // small M: split-K, K split s writes its f32 partial to slice s (summed by the consumer)
 };
 
 // B operands (weights) live in a k-block-major, pre-swizzled layout owned by the
@@ -73,8 +73,7 @@ struct GemmArgs {
   int splits;             // split-K factor (small-M kernel); 1 for the persistent kernel
   int group_m;            // tile raster: M blocks per group
   int prefetch;           // K blocks of B to prefetch into L2 ahead of the smem ring (0 = off)
-  int cluster;            // small-M split-K: CTAs per cluster (splits reduced together through DSMEM)
-  long long group_stride; // small-M split-K: elements between the output slices of cluster groups
+  long long group_stride; // small-M split-K: elements between the f32 slices of consecutive K splits
   void* out;
   long long ldo;          // elements
   const float* residual;  // EPI_F32 only, may be null
@@ -88,16 +87,12 @@ struct GemmArgs {
 cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args, int num_sms,
                            cudaStream_t stream);
 
-// Small-M GEMM (M <= 128 * mt): one output tile per CTA, activation and weight
-// tiles in separate shared-memory rings (weights run further ahead).
+// Small-M GEMM (M <= 128 * mt): one output tile and one K split per CTA.
 //   epi == EPI_SWIGLU: args.splits == 1, fused SwiGLU epilogue (bf16 out).
-//   epi == EPI_CLUSTER: args.splits K splits per tile, in clusters of
-//     args.cluster CTAs; each cluster adds its splits through DSMEM and writes
-//     f32 slice (split / cluster) at out + slice * group_stride.
+//   epi == EPI_SLICES: args.splits balanced K splits per tile; split s writes
+//     its f32 partial [M, N] to out + s * group_stride (N % 4 == 0).
 cudaError_t gemm_small_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args,
                               cudaStream_t stream);
-// Most clusters of `cluster` CTAs of the small-M split-K kernel resident at once (0 if unknown).
-int gemm_small_cluster_capacity(int bn, int mt, int cluster);
 
 // CUDA-core path of the f32 configuration.  a[0..2]: A pieces with row stride k_per_map.
 cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int epi, const GemmArgs& args,

@@ -151,7 +151,6 @@ struct outlets_ctx {
   int last_rows = 0, last_out_rows = 0;
   bool oom = false;
   std::unordered_map<MapKey, CUtensorMap, MapKeyHash> map_cache;  // library-owned buffers only
-  std::unordered_map<int, int> cluster_cap;                       // resident clusters per GEMM shape
 
   // stage timing and launch accounting
   struct ProfRec {
@@ -425,40 +424,37 @@ outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k
   return gemm_tc_ex(c, a, n_pieces, k_piece, lda, M, b, b_np, N, K, epi, bn, 1, 1, out, ldo, residual, ldr, bias, s);
 }
 
-// Small-M GEMM (M <= 256): every weight tile is streamed once; K is split so
-// that about one wave of CTAs streams the weights.  The splits of a tile form
-// clusters of sc CTAs that add their partials through DSMEM; the g cluster
-// groups of a tile write g f32 slices part[g][M][N] that the consuming kernel
-// adds up.  Returns the slice count in *slices.
-outlets_status gemm_cluster(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
-                            const void* b, long long b_np, int N, int K, float* part, int* slices, cudaStream_t s) {
+// Small-M GEMM (M <= 256): every weight tile is streamed once.  K is split so
+// that enough CTAs stream the weights, but every split adds an f32 slice
+// part[s][M][N] that is written and read back through L2 by the consuming
+// kernel.  Tile width and split count minimise an estimate of both costs:
+// operand streaming per CTA (A and B tiles, ~85 GB/s per CTA) plus the slice
+// traffic (~6 TB/s), rates measured on GB300.  Returns the slice count in
+// *slices.
+outlets_status gemm_split(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
+                          const void* b, long long b_np, int N, int K, float* part, int* slices, cudaStream_t s) {
   if (M == 0) return OUTLETS_OK;
   const int mt = M <= 128 ? 1 : 2;
-  const int bn = cdiv(N, 256) >= 8 ? 256 : 128;
-  const long long n_tiles = cdiv(N, bn);
+  const long long tm = 128LL * mt;
   const long long kb = cdiv(K, 64);
-  int best_sc = 1, best_g = 1;
-  long long best_ctas = -1;
-  for (int sc : {4, 3, 2, 1}) {
-    long long g = std::min<long long>(8, c->num_sms / (n_tiles * sc));
-    while (g > 1 && sc * g > kb) --g;
-    if (g < 1 || sc > kb) continue;
-    if (sc > 1) {
-      const int key = 100000 + bn * 100 + mt * 10 + sc;
-      auto it = c->cluster_cap.find(key);
-      const int cap =
-          it != c->cluster_cap.end() ? it->second : (c->cluster_cap[key] = gemm_small_cluster_capacity(bn, mt, sc));
-      while (g > 1 && n_tiles * g > cap) --g;
-      if (n_tiles * g > cap) continue;
-    }
-    const long long ctas = n_tiles * sc * g;
-    if (ctas > best_ctas) {
-      best_ctas = ctas;
-      best_sc = sc;
-      best_g = (int)g;
+  const long long max_s = std::min<long long>(kb, (long long)(c->part_floats / ((size_t)M * N)));
+  if (max_s < 1 || N % 4) return c->fail(OUTLETS_ECAPACITY, "split-K workspace too small");
+  int best_bn = 256, best_s = 1;
+  double best_t = -1.0;
+  for (int bn : {256, 128}) {
+    const long long tiles = cdiv(N, bn) * cdiv(M, tm);
+    for (long long sp = 1; sp <= max_s && (sp == 1 || tiles * sp <= c->num_sms); ++sp) {
+      const double waves = (double)cdiv(tiles * sp, c->num_sms);
+      const double per_cta = (double)(bn + tm) * 64.0 * 2.0 * (double)cdiv(kb, sp);
+      const double t = waves * per_cta / 85e3 + 2.0 * sp * M * N * 4.0 / 6e6;
+      if (best_t < 0 || t < best_t) {
+        best_t = t;
+        best_bn = bn;
+        best_s = (int)sp;
+      }
     }
   }
-  if ((size_t)best_g * M * N > c->part_floats) return c->fail(OUTLETS_ECAPACITY, "split-K workspace too small");
+  const int bn = best_bn;
   CUtensorMap am[3];
   OUT_TRY(a_maps(c, a, n_pieces, k_piece, lda, M, am));
   GemmArgs g{};
@@ -468,15 +464,14 @@ outlets_status gemm_cluster(outlets_ctx* c, const void* const* a, int n_pieces, 
   g.b = b;
   g.b_np = b_np;
   g.k_per_map = k_piece;
-  g.splits = best_sc * best_g;
-  g.cluster = best_sc;
+  g.splits = best_s;
   g.group_stride = (long long)M * N;
   g.group_m = 1;
   g.out = part;
   g.ldo = N;
   g.err = c->err_dev;
-  OUT_CK(c, gemm_small_launch(am, bn, EPI_CLUSTER, mt, g, s));
-  *slices = best_g;
+  OUT_CK(c, gemm_small_launch(am, bn, EPI_SLICES, mt, g, s));
+  *slices = best_s;
   return OUTLETS_OK;
 }
 
@@ -517,7 +512,7 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   {
     const void* a1[3] = {c->attn, c->attn, c->attn};
     if (small)
-      OUT_TRY(gemm_cluster(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, c->part, &sl, s));
+      OUT_TRY(gemm_split(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, c->part, &sl, s));
     else if (c->bf16)
       OUT_TRY(gemm_tc(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d,
                       nullptr, s));
@@ -559,7 +554,6 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
       g.b_np = c->np_gu;
       g.k_per_map = d;
       g.splits = 1;
-      g.cluster = 1;
       g.group_m = 1;
       g.out = c->u;
       g.ldo = c->Fp;
@@ -579,7 +573,7 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   {
     const void* a1[3] = {c->u, c->u, c->u};
     if (small)
-      OUT_TRY(gemm_cluster(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, c->np_down, d, c->Fp, c->part, &sl, s));
+      OUT_TRY(gemm_split(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, c->np_down, d, c->Fp, c->part, &sl, s));
     else if (c->bf16)
       OUT_TRY(gemm_tc(c, a1, 1, c->Fp, c->Fp, rows, c->w_down, c->np_down, d, c->Fp, EPI_F32, c->y, d, c->a, d, nullptr, s));
     else
@@ -613,7 +607,7 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   const void* ah[3] = {c->hn, c->hn, c->hn};
   if (small_path(c, out_rows) && nl == 2) {
     int hs = 1;
-    OUT_TRY(gemm_cluster(c, ah, 1, d, d, out_rows, c->head_w0, c->np_h0, w1, d, c->part, &hs, s));
+    OUT_TRY(gemm_split(c, ah, 1, d, d, out_rows, c->head_w0, c->np_h0, w1, d, c->part, &hs, s));
     OUT_CK(c, head_tail_launch(c->part, hs, (long long)out_rows * w1, c->head_b[0], c->head_wf[1], c->head_b[1],
                                out_rows, w1, z_dev, len_dev, s));
     c->stage_end(2);
@@ -652,7 +646,7 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
   const bool small = small_path(c, rows);
   c->stage_begin(OUTLETS_S_FC);
   int sl = 1;
-  if (small) OUT_TRY(gemm_cluster(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, c->part, &sl, s));
+  if (small) OUT_TRY(gemm_split(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, c->part, &sl, s));
   else if (c->bf16) OUT_TRY(gemm_tc(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
   else OUT_TRY(gemm_f32(c, tp, d, rows, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
   c->stage_end(1);
@@ -668,7 +662,7 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
   c->stage_begin(OUTLETS_S_QKV);
   const void* a1[3] = {c->xhat, c->xhat, c->xhat};
   if (small) {
-    OUT_TRY(gemm_cluster(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, c->part, &sl, s));
+    OUT_TRY(gemm_split(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, c->part, &sl, s));
     *q = {c->part, true, sl, (long long)rows * c->qkv_n};
   } else if (c->bf16) {
     OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, EPI_ACT, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
@@ -828,9 +822,9 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->z = (float*)c->alloc(R * 4);
   c->len = (float*)c->alloc(R * 4);
   c->err_dev = (int*)c->alloc(16);
-  if (c->bf16) {  // f32 split-K slices of the small-M path (up to 8 per GEMM)
+  if (c->bf16) {  // f32 split-K slices of the small-M path (up to 12 of the widest GEMM)
     const size_t widest = (size_t)std::max(std::max(d, c->qkv_n), c->head_dims[1]);
-    c->part_floats = (size_t)8 * std::min<size_t>(R, 256) * widest;
+    c->part_floats = (size_t)12 * std::min<size_t>(R, 256) * widest;
     c->part = (float*)c->alloc(c->part_floats * 4);
   }
   if (c->oom) return cleanup_fail(OUTLETS_ENOMEM);

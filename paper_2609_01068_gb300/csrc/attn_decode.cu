@@ -11,8 +11,9 @@
 // (64 keys x hd) of K and V are staged by TMA (128-byte swizzle, 3 stages);
 // each of the 4 warps takes 16 keys of a page, keeps its own online softmax,
 // and the warps are merged through shared memory.  Requests with one split
-// write the output directly; others write (o, m, l) partials merged by a
-// second kernel.
+// write the output directly; others write (o, m, l) partials, and the last
+// split CTA of each (request, kv head) to finish merges them (a fenced
+// completion counter; no CTA waits for another).
 //
 // f32 path: one warp per (request, head), lanes own head dims.
 #include "common.cuh"
@@ -32,6 +33,55 @@ struct DecCfg {
   static constexpr size_t SMEM = 1024 + Q_BYTES + kStages * 2 * PAGE_BYTES + 128;
 };
 
+// Merge the split partials of request b, heads h0 .. h0 + nh - 1:
+// out = sum_s w_s o_s / sum_s w_s with w_s = l_s * 2^(m_s - max m), splits
+// added in order.  The (m, l) pairs and the weights are staged in `scratch`
+// (2 * nh * ns + nh floats); each output then issues the loads of up to eight
+// splits together.  Partials written by other CTAs are read through L2.
+template <int HD>
+__device__ __forceinline__ void merge_splits(const DecodeArgs& a, int b, int h0, int nh, float* scratch) {
+  const int w0 = a.work_off[b];
+  const int ns = a.work_off[b + 1] - w0;
+  float* ml = scratch;           // [nh][ns][2]
+  float* wt = scratch + 2 * nh * ns;  // [nh][ns] weights, then [nh] their sums
+  float* lsum = wt + nh * ns;
+  for (int i = threadIdx.x; i < nh * ns * 2; i += blockDim.x) {
+    const int r = i / (2 * ns), rem = i - r * 2 * ns;
+    ml[i] = __ldcg(&a.part_ml[((long long)(w0 + (rem >> 1)) * a.H + h0 + r) * 2 + (rem & 1)]);
+  }
+  __syncthreads();
+  for (int r = threadIdx.x; r < nh; r += blockDim.x) {
+    float M = -INFINITY;
+    for (int w = 0; w < ns; ++w) M = fmaxf(M, ml[(r * ns + w) * 2]);
+    const float Mu = (M == -INFINITY) ? 0.f : M;
+    float Ls = 0.f;
+    for (int w = 0; w < ns; ++w) {
+      const float f = exp2f(ml[(r * ns + w) * 2] - Mu) * ml[(r * ns + w) * 2 + 1];
+      wt[r * ns + w] = f;
+      Ls += f;
+    }
+    lsum[r] = Ls;
+  }
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < nh * HD; idx += blockDim.x) {
+    const int r = idx / HD;
+    const int d = idx - r * HD;
+    const float* po = a.part_o + ((long long)w0 * a.H + h0 + r) * HD + d;
+    const long long wstride = (long long)a.H * HD;
+    float Os = 0.f;
+    for (int w = 0; w < ns; w += 8) {
+      float o[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (w + k < ns) o[k] = __ldcg(po + (w + k) * wstride);
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (w + k < ns) Os += wt[r * ns + w + k] * o[k];
+    }
+    reinterpret_cast<bf16*>(a.out)[((long long)b * a.H + h0 + r) * HD + d] = __float2bfloat16_rn(Os / lsum[r]);
+  }
+}
+
 template <int HD>
 __global__ void __launch_bounds__(128)
     k_attn_decode_bf16(const __grid_constant__ CUtensorMap k_map, const __grid_constant__ CUtensorMap v_map,
@@ -48,7 +98,8 @@ __global__ void __launch_bounds__(128)
   uint64_t* empty = full + kStages;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(empty + kStages);
 
-  const int2 wk = reinterpret_cast<const int2*>(a.work)[blockIdx.x];
+  const int item = a.order ? a.order[blockIdx.x] : (int)blockIdx.x;  // work item of this CTA
+  const int2 wk = reinterpret_cast<const int2*>(a.work)[item];
   const int b = wk.x;
   const int split = wk.y;
   const int g = blockIdx.y;
@@ -254,7 +305,7 @@ __global__ void __launch_bounds__(128)
     if (n_split == 1) {
       reinterpret_cast<bf16*>(a.out)[((long long)b * a.H + head) * HD + d] = __float2bfloat16_rn(Os / Ls);
     } else {
-      const long long pi = (long long)blockIdx.x * a.H + head;  // partial index: (work item, head)
+      const long long pi = (long long)item * a.H + head;  // partial index: (work item, head)
       a.part_o[pi * HD + d] = Os / Ls;
       if (d == 0) {
         a.part_ml[pi * 2 + 0] = M;
@@ -262,30 +313,23 @@ __global__ void __launch_bounds__(128)
       }
     }
   }
-}
-
-// Merge split partials: out = sum_s w_s o_s / sum_s w_s, w_s = l_s * 2^(m_s - max m).
-template <typename Act>
-__global__ void k_decode_combine(const DecodeArgs a, int hd) {
-  pdl_trigger();
-  pdl_wait();
-  const int b = blockIdx.x;
-  const int head = blockIdx.y;
-  const int w0 = a.work_off[b], w1 = a.work_off[b + 1];
-  if (w1 - w0 <= 1) return;
-  float M = -INFINITY;
-  for (int w = w0; w < w1; ++w) M = fmaxf(M, a.part_ml[((long long)w * a.H + head) * 2]);
-  const float Mu = (M == -INFINITY) ? 0.f : M;
-  for (int d = threadIdx.x; d < hd; d += blockDim.x) {
-    float Ls = 0.f, Os = 0.f;
-    for (int w = w0; w < w1; ++w) {
-      const long long pi = (long long)w * a.H + head;
-      const float f = exp2f(a.part_ml[pi * 2] - Mu) * a.part_ml[pi * 2 + 1];
-      Ls += f;
-      Os += f * a.part_o[pi * hd + d];
-    }
-    reinterpret_cast<Act*>(a.out)[((long long)b * a.H + head) * hd + d] = from_f<Act>(Os / Ls);
+  if (n_split == 1) return;
+  // The last split CTA of (request, KV group) to finish merges all splits:
+  // each CTA publishes its partial (fence, then count); the one that brings
+  // the count to n_split reads every partial and resets the counter for the
+  // next call.  No CTA waits for another.
+  __shared__ int is_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int prev = atomicAdd(&a.combine_count[b * a.KVH + g], 1);
+    is_last = prev == n_split - 1;
   }
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  merge_splits<HD>(a, b, g * G, G, reinterpret_cast<float*>(sKV));  // the K/V stages are idle now
+  if (threadIdx.x == 0) a.combine_count[b * a.KVH + g] = 0;
 }
 
 // f32 path: warp per (request, head); keys walked through the page list.
@@ -353,11 +397,10 @@ cudaError_t launch_decode_tc(const CUtensorMap& k_map, const CUtensorMap& v_map,
     if (e != cudaSuccess) return e;
     attr = true;
   }
+  // the split merge stages (3 * splits + 1) floats per query head in the K/V stages
+  if ((3LL * a.max_splits + 1) * (a.H / a.KVH) * 4 > (long long)kStages * 2 * C::PAGE_BYTES) return cudaErrorInvalidValue;
   dim3 grid(a.n_work, a.KVH);
   OUTLETS_TRY_LAUNCH(launch_k(k_attn_decode_bf16<HD>, dim3(grid), dim3(128), C::SMEM, stream, k_map, v_map, a));
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  OUTLETS_TRY_LAUNCH(launch_k(k_decode_combine<bf16>, dim3(dim3(a.B, a.H)), dim3(128), 0, stream, a, HD));
   return cudaGetLastError();
 }
 

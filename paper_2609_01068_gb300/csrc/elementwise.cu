@@ -32,7 +32,7 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 }
 
 // Split-K slices: s[0] + s[1] + ... + s[n-1] at p, p + stride, ..., added in
-// slice order (the same order on every call); the loads of up to nine slices
+// slice order (the same order on every call); the loads of up to U + 1 slices
 // are in flight together.
 __device__ __forceinline__ void add4(float4& a, const float4& b) {
   a.x += b.x;
@@ -40,30 +40,31 @@ __device__ __forceinline__ void add4(float4& a, const float4& b) {
   a.z += b.z;
   a.w += b.w;
 }
+template <int U = 8>
 __device__ __forceinline__ float4 ld_sum4(const float* p, int n, long long stride) {
   float4 acc = *reinterpret_cast<const float4*>(p);
-  for (int s0 = 1; s0 < n; s0 += 8) {
-    float4 v[8];
+  for (int s0 = 1; s0 < n; s0 += U) {
+    float4 v[U];
 #pragma unroll
-    for (int k = 0; k < 8; ++k)
+    for (int k = 0; k < U; ++k)
       if (s0 + k < n) v[k] = *reinterpret_cast<const float4*>(p + (s0 + k) * stride);
 #pragma unroll
-    for (int k = 0; k < 8; ++k)
+    for (int k = 0; k < U; ++k)
       if (s0 + k < n) add4(acc, v[k]);
   }
   return acc;
 }
-// Two float4 runs (8 floats at p and 8 at q) summed over the slices; up to five
-// slices of both in flight together.
+// Two float4 runs (8 floats at p and 8 at q) summed over the slices; up to
+// three slices of both in flight together.
 __device__ __forceinline__ void ld_sum16(const float* p, const float* q, int n, long long stride, float4 (&o)[4]) {
   o[0] = *reinterpret_cast<const float4*>(p);
   o[1] = *reinterpret_cast<const float4*>(p + 4);
   o[2] = *reinterpret_cast<const float4*>(q);
   o[3] = *reinterpret_cast<const float4*>(q + 4);
-  for (int s0 = 1; s0 < n; s0 += 4) {
-    float4 v[4][4];
+  for (int s0 = 1; s0 < n; s0 += 2) {
+    float4 v[2][4];
 #pragma unroll
-    for (int k = 0; k < 4; ++k)
+    for (int k = 0; k < 2; ++k)
       if (s0 + k < n) {
         const long long off = (s0 + k) * stride;
         v[k][0] = *reinterpret_cast<const float4*>(p + off);
@@ -72,7 +73,7 @@ __device__ __forceinline__ void ld_sum16(const float* p, const float* q, int n, 
         v[k][3] = *reinterpret_cast<const float4*>(q + off + 4);
       }
 #pragma unroll
-    for (int k = 0; k < 4; ++k)
+    for (int k = 0; k < 2; ++k)
       if (s0 + k < n) {
 #pragma unroll
         for (int j = 0; j < 4; ++j) add4(o[j], v[k][j]);
@@ -98,7 +99,7 @@ __device__ __forceinline__ void store4<bf16>(bf16* p, float a, float b, float c,
 // y[r] = v * g * rsqrt(mean(v^2) + eps); copy_out[r] = v (f32) when given.
 // REDUCE = false: v = x[src] (one slice, no residual).
 template <typename Act, bool REDUCE>
-__global__ void __launch_bounds__(1024) k_rmsnorm(const float* __restrict__ x, int n_split, long long split_stride,
+__global__ void __launch_bounds__(512, 2) k_rmsnorm(const float* __restrict__ x, int n_split, long long split_stride,
                           const float* __restrict__ residual, const int* __restrict__ row_index,
                           const float* __restrict__ g, Act* __restrict__ y, float* __restrict__ copy_out, int d,
                           float eps) {
@@ -149,8 +150,8 @@ __device__ __forceinline__ void load8<bf16>(const bf16* p, long long idx, int, l
 template <>
 __device__ __forceinline__ void load8<float>(const float* p, long long idx, int n_split, long long stride,
                                              float* v) {
-  const float4 a = ld_sum4(p + idx, n_split, stride);
-  const float4 b = ld_sum4(p + idx + 4, n_split, stride);
+  const float4 a = ld_sum4<4>(p + idx, n_split, stride);
+  const float4 b = ld_sum4<4>(p + idx + 4, n_split, stride);
   v[0] = a.x, v[1] = a.y, v[2] = a.z, v[3] = a.w, v[4] = b.x, v[5] = b.y, v[6] = b.z, v[7] = b.w;
 }
 // Both halves of a rotation pair (8 elements at idx and at idx + half).
@@ -191,7 +192,7 @@ __device__ __forceinline__ void store8<float>(float* p, const float* v) {
 // One CTA per row; a thread rotates 8 pairs (i..i+7 with i+hd/2..i+hd/2+7) of
 // one head and copies 8 values of V.  hd is a multiple of 16.
 template <typename In, typename Act>
-__global__ void __launch_bounds__(512) k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
+__global__ void __launch_bounds__(320, 2) k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
   pdl_trigger();
   pdl_wait();
   const int row = blockIdx.x;
@@ -461,8 +462,8 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
         attr = true;
       }
     }
-    // one float4 of the row per thread where d allows: every slice load of a row in flight at once
-    const int threads = std::min(1024, std::max(64, ((d / 4 + 31) / 32) * 32));
+    // two CTAs (rows) per SM fit beside each other: a one-wave grid for up to 2 x SMs rows
+    const int threads = std::min(512, std::max(64, ((d / 4 + 31) / 32) * 32));
     OUTLETS_TRY_LAUNCH(launch_k(k_rmsnorm<Act, true>, dim3(rows), dim3(threads), smem, stream, x, n_split, split_stride, residual, row_index, g, y, copy_out,
                                                       d, eps));
   } else {
@@ -474,8 +475,9 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
 template <typename In, typename Act>
 cudaError_t rope_scatter_launch(const In* qkv, const RopeArgs& a, cudaStream_t stream) {
   if (a.T == 0) return cudaSuccess;
-  const int items = (a.H + a.KVH) * (a.hd / 16);  // rotation chunks per row: about one per thread
-  const int threads = std::min(512, std::max(64, ((items + 31) / 32) * 32));
+  // rotation chunks per row, about one per thread; two CTAs (rows) fit per SM
+  const int items = (a.H + a.KVH) * (a.hd / 16);
+  const int threads = std::min(320, std::max(64, ((items + 31) / 32) * 32));
   OUTLETS_TRY_LAUNCH(launch_k(k_rope_scatter<In, Act>, dim3(a.T), dim3(threads), 0, stream, qkv, a));
   return cudaGetLastError();
 }

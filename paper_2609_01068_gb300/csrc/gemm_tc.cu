@@ -74,7 +74,8 @@ __device__ __forceinline__ Tile decode_tile(int t, int num_m, int num_n, int gro
   return tl;
 }
 
-__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + __expf(-x)); }
+// silu(x) = x * sigmoid(x); the fast division is exact to ~2 ulp (the result is rounded to bf16)
+__device__ __forceinline__ float silu_f(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
 
 template <typename T>
 __device__ __forceinline__ void store_row32(T* dst, const float* v, int valid);

@@ -192,10 +192,13 @@ struct DecodeArgs {
   const int* seq_len;     // [B] keys per request (cached + the new token)
   const int* work;        // [n_work] pairs (request, split), grouped by request
   const int* work_off;    // [B+1] first work item of each request
+  const int* order;       // [n_work] launch order of the work items (longest first), or null
   int n_work;
   int split_len;          // keys per split (multiple of page_tokens)
+  int max_splits;         // most splits of one request
   float* part_o;          // [n_work, H, hd] normalized partial outputs
   float* part_ml;         // [n_work, H, 2] (max in log2 units, sum)
+  int* combine_count;     // [B, KVH] split completion counters, zero between calls
   void* out;              // [B, H, hd]
   int* err;
 };

@@ -31,7 +31,8 @@ using namespace outlets;
 namespace {
 
 constexpr int kPageTokens = 64;
-constexpr int kSplitLen = 512;
+constexpr int kSplitLen = 512;        // shortest split-KV work item (keys)
+constexpr int kDecodeCtasPerSm = 2;   // resident decode-attention CTAs per SM
 constexpr int kRing = 4;
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -133,6 +134,7 @@ struct outlets_ctx {
        *attn = nullptr, *u = nullptr, *hn = nullptr;
   void* taps_stage[3] = {nullptr, nullptr, nullptr};
   int* err_dev = nullptr;
+  int* dec_count = nullptr;  // [max_batch, KVH] split-KV completion counters of decode attention
   float* part = nullptr;  // f32 split-K slices of the small-M path
   size_t part_floats = 0;
   int* meta_dev = nullptr;
@@ -822,6 +824,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->z = (float*)c->alloc(R * 4);
   c->len = (float*)c->alloc(R * 4);
   c->err_dev = (int*)c->alloc(16);
+  c->dec_count = (int*)c->alloc((size_t)cfg->max_batch * c->KVH * sizeof(int));
   if (c->bf16) {  // f32 split-K slices of the small-M path (up to 12 of the widest GEMM)
     const size_t widest = (size_t)std::max(std::max(d, c->qkv_n), c->head_dims[1]);
     c->part_floats = (size_t)12 * std::min<size_t>(R, 256) * widest;
@@ -1028,6 +1031,8 @@ outlets_status outlets_check(outlets_ctx* c, void* stream) {
   OUT_CK(c, cudaMemcpy(&e, c->err_dev, sizeof(int), cudaMemcpyDeviceToHost));
   if (e) {
     OUT_CK(c, cudaMemset(c->err_dev, 0, sizeof(int)));
+    // a CTA that gave up may have left a split counter mid-count
+    OUT_CK(c, cudaMemset(c->dec_count, 0, (size_t)c->cfg.max_batch * c->KVH * sizeof(int)));
     if (e & ERR_TIMEOUT) return c->fail(OUTLETS_ETIMEOUT, "a kernel's bounded wait ran out");
     return c->fail(OUTLETS_EDEVICE, "a kernel refused an out-of-range index");
   }
@@ -1211,6 +1216,14 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
 
   // ---- commit the append and build metadata
   std::vector<int> pos(B), seq_len(B), po(B + 1, 0), pl, work, work_off(B + 1, 0);
+  // Keys per split-KV work item: about a third of one resident CTA's share of
+  // all keys (never below 512), so most requests need no split (and no merge)
+  // while the longest items still fit several times into the whole pass.
+  long long total_keys = 0;
+  for (int b = 0; b < B; ++b) total_keys += kv->len[slots[b]] + 1;
+  const long long share = cdiv(total_keys * c->KVH, 3LL * kDecodeCtasPerSm * c->num_sms);
+  const int split_len = (int)std::max<long long>(kSplitLen, cdiv(share, kPageTokens) * kPageTokens);
+  int max_splits = 1;
   for (int b = 0; b < B; ++b) {
     const int sl = slots[b];
     if (kv->len[sl] % kPageTokens == 0) {
@@ -1222,7 +1235,8 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
     seq_len[b] = kv->len[sl];
     pl.insert(pl.end(), kv->pages[sl].begin(), kv->pages[sl].end());
     po[b + 1] = (int)pl.size();
-    const int ns = (int)cdiv(seq_len[b], kSplitLen);
+    const int ns = (int)cdiv(seq_len[b], split_len);
+    max_splits = std::max(max_splits, ns);
     for (int sp = 0; sp < ns; ++sp) {
       work.push_back(b);
       work.push_back(sp);
@@ -1230,6 +1244,13 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
     work_off[b + 1] = (int)(work.size() / 2);
   }
   const int n_work = work_off[B];
+  // launch order: longest work items first (the short ones fill the tail)
+  std::vector<int> order(n_work), item_keys(n_work);
+  for (int w = 0; w < n_work; ++w) {
+    order[w] = w;
+    item_keys[w] = std::min(split_len, seq_len[work[2 * w]] - work[2 * w + 1] * split_len);
+  }
+  std::stable_sort(order.begin(), order.end(), [&](int x, int y) { return item_keys[x] > item_keys[y]; });
   MetaBuilder mb;
   const size_t off_pos = mb.put(pos);
   const size_t off_sl = mb.put(seq_len);
@@ -1237,6 +1258,7 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
   const size_t off_pl = mb.put(pl);
   const size_t off_w = mb.put(work);
   const size_t off_wo = mb.put(work_off);
+  const size_t off_ord = mb.put(order);
   OUT_TRY(upload_meta(c, mb.v, s));
   const int* m = c->meta_dev;
 
@@ -1281,9 +1303,12 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
     da.work = m + off_w;
     da.work_off = m + off_wo;
     da.n_work = n_work;
-    da.split_len = kSplitLen;
+    da.split_len = split_len;
+    da.order = m + off_ord;
+    da.max_splits = max_splits;
     da.part_o = kv->part_o;
     da.part_ml = kv->part_ml;
+    da.combine_count = c->dec_count;
     da.out = c->attn;
     da.err = c->err_dev;
     if ((size_t)n_work > kv->part_items) return c->fail(OUTLETS_ECAPACITY, "split-KV partial buffer too small");
@@ -1293,7 +1318,7 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
       if (!cached_map(c, &km, kv->k_pool, c->hd, rows, c->hd, 64) || !cached_map(c, &vm, kv->v_pool, c->hd, rows, c->hd, 64))
         return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for the KV pools");
       OUT_CK(c, attn_decode_bf16_launch(km, vm, da, s));
-      c->stage_end(2);
+      c->stage_end(1);
     } else {
       OUT_CK(c, attn_decode_simt_launch<float>(da, s));
       c->stage_end(1);

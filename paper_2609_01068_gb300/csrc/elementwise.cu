@@ -11,6 +11,7 @@
 //   head tail         z_hat = w . relu(h + b) + b_out, length = max(0, expm1(z_hat))
 //                     (Sec. 4.2: log-space target z = log(1 + length))
 #include <algorithm>
+#include <type_traits>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -191,8 +192,17 @@ __device__ __forceinline__ void store8<float>(float* p, const float* v) {
 
 // One CTA per row; a thread rotates 8 pairs (i..i+7 with i+hd/2..i+hd/2+7) of
 // one head and copies 8 values of V.  hd is a multiple of 16.
+// Block shape of the RoPE/scatter kernel.  f32 input (split-K slices, small
+// batches): one rotation chunk per thread, two CTAs (rows) per SM.  bf16 input
+// (prefill, one CTA per token over ~T rows): small CTAs, many per SM.
+template <typename In>
+struct RopeBlock {
+  static constexpr int kThreads = std::is_same<In, float>::value ? 320 : 128;
+  static constexpr int kMinBlocks = std::is_same<In, float>::value ? 2 : 12;
+};
+
 template <typename In, typename Act>
-__global__ void __launch_bounds__(320, 2) k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
+__global__ void __launch_bounds__(RopeBlock<In>::kThreads, RopeBlock<In>::kMinBlocks) k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
   pdl_trigger();
   pdl_wait();
   const int row = blockIdx.x;
@@ -475,9 +485,8 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
 template <typename In, typename Act>
 cudaError_t rope_scatter_launch(const In* qkv, const RopeArgs& a, cudaStream_t stream) {
   if (a.T == 0) return cudaSuccess;
-  // rotation chunks per row, about one per thread; two CTAs (rows) fit per SM
-  const int items = (a.H + a.KVH) * (a.hd / 16);
-  const int threads = std::min(320, std::max(64, ((items + 31) / 32) * 32));
+  const int items = (a.H + a.KVH) * (a.hd / 16);  // rotation chunks per row
+  const int threads = std::min(RopeBlock<In>::kThreads, std::max(64, ((items + 31) / 32) * 32));
   OUTLETS_TRY_LAUNCH(launch_k(k_rope_scatter<In, Act>, dim3(a.T), dim3(threads), 0, stream, qkv, a));
   return cudaGetLastError();
 }

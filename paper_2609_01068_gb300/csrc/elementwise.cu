@@ -205,7 +205,7 @@ template <typename In, typename Act>
 __global__ void __launch_bounds__(RopeBlock<In>::kThreads, RopeBlock<In>::kMinBlocks) k_rope_scatter(const In* __restrict__ qkv, const RopeArgs a) {
   pdl_trigger();
   pdl_wait();
-  const int row = blockIdx.x;
+  const int row = a.row0 + (int)blockIdx.x;
   int pos, seq;
   if (a.cu) {
     int lo = 0, hi = a.B;

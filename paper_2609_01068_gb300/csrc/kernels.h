@@ -117,7 +117,8 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
                                   float eps, cudaStream_t stream);
 
 struct RopeArgs {
-  int T;                 // rows of this call
+  int T;                 // rows of this launch (rows row0 .. row0 + T - 1 of the call)
+  int row0;              // first row (a prefill call may run its rows in chunks)
   int H, KVH, hd;
   const int* cu;         // prefill: sequence offsets [B+1] (position = row - cu[b]); else null
   int B;

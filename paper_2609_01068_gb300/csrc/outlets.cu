@@ -31,6 +31,8 @@ using namespace outlets;
 namespace {
 
 constexpr int kPageTokens = 64;
+constexpr int kMaxTapChunks = 4;      // row chunks of host taps copied while earlier chunks compute
+constexpr int kMinTapChunkRows = 2048;
 constexpr int kSplitLen = 512;        // shortest split-KV work item (keys)
 constexpr int kDecodeCtasPerSm = 2;   // resident decode-attention CTAs per SM
 constexpr int kRing = 4;
@@ -148,6 +150,10 @@ struct outlets_ctx {
   } ring[kRing];
   int ring_i = 0;
   cudaEvent_t done_ev = nullptr;
+  // copies of host taps in row chunks, overlapped with the prefill front
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t copy_start = nullptr;
+  cudaEvent_t chunk_ev[kMaxTapChunks] = {};
   bool have_prev = false;
 
   int last_rows = 0, last_out_rows = 0;
@@ -642,14 +648,19 @@ struct QkvSrc {
   long long stride;
 };
 
-outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvSrc* q, cudaStream_t s) {
+// FC (Eq. 1) -> input RMSNorm -> QKV for rows row0 .. row0 + rows - 1 (tp
+// points at row row0 of each tap; row0 > 0 only on the large-M path).
+outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvSrc* q, cudaStream_t s,
+                         int row0 = 0) {
   const int d = c->d;
   const float eps = c->cfg.rms_eps;
   const bool small = small_path(c, rows);
   c->stage_begin(OUTLETS_S_FC);
   int sl = 1;
   if (small) OUT_TRY(gemm_split(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, c->part, &sl, s));
-  else if (c->bf16) OUT_TRY(gemm_tc(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
+  else if (c->bf16)
+    OUT_TRY(gemm_tc(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, EPI_F32, c->f + (size_t)row0 * d, d, nullptr,
+                    0, nullptr, s));
   else OUT_TRY(gemm_f32(c, tp, d, rows, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
   c->stage_end(1);
   c->stage_begin(OUTLETS_S_NORM_IN);
@@ -657,17 +668,20 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
     OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, nullptr, nullptr, c->g_in, (bf16*)c->xhat,
                                           c->f, rows, d, eps, s));
   else if (c->bf16)
-    OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xhat, nullptr, rows, d, eps, s));
+    OUT_CK(c, rmsnorm_launch<bf16>(c->f + (size_t)row0 * d, c->g_in, (bf16*)c->xhat + (size_t)row0 * d, nullptr, rows,
+                                   d, eps, s));
   else
     OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
   c->stage_end(1);
   c->stage_begin(OUTLETS_S_QKV);
-  const void* a1[3] = {c->xhat, c->xhat, c->xhat};
+  const void* xr = (const char*)c->xhat + (size_t)row0 * d * c->esz;
+  const void* a1[3] = {xr, xr, xr};
   if (small) {
     OUT_TRY(gemm_split(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, c->part, &sl, s));
     *q = {c->part, true, sl, (long long)rows * c->qkv_n};
   } else if (c->bf16) {
-    OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, EPI_ACT, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
+    OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, EPI_ACT,
+                    (char*)c->qkv + (size_t)row0 * c->qkv_n * c->esz, c->qkv_n, nullptr, 0, nullptr, s));
     *q = {c->qkv, false, 1, 0};
   } else {
     OUT_TRY(gemm_f32(c, a1, d, rows, c->w_qkv, c->qkv_n, d, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
@@ -705,6 +719,40 @@ outlets_status prepare_taps(outlets_ctx* c, const void* const taps[3], int rows,
       OUT_CK(c, cudaMemcpyAsync(c->taps_stage[i], taps[i], (size_t)rows * c->d * c->esz, cudaMemcpyHostToDevice, s));
       out[i] = c->taps_stage[i];
     }
+  }
+  return OUTLETS_OK;
+}
+
+// Host taps of a large call: copied in n row chunks on the context's copy
+// stream (after the work already queued on s, which may still read the
+// staging buffers); chunk i's completion is recorded in chunk_ev[i] so the
+// front of the pipeline can start on rows that have landed while later rows
+// are still in transit.  tp receives the staging buffers.
+outlets_status stage_taps_chunked(outlets_ctx* c, const void* const taps[3], int rows, int n, int chunk_rows,
+                                  const void* tp[3], cudaStream_t s) {
+  if (!c->copy_stream) {
+    OUT_CK(c, cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking));
+    OUT_CK(c, cudaEventCreateWithFlags(&c->copy_start, cudaEventDisableTiming));
+    for (auto& e : c->chunk_ev) OUT_CK(c, cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+  }
+  const size_t row_bytes = (size_t)c->d * c->esz;
+  for (int i = 0; i < 3; ++i) {
+    if (!taps[i]) return c->fail(OUTLETS_EINVAL, "taps[i] is NULL");
+    if (!c->taps_stage[i]) {
+      c->taps_stage[i] = c->alloc((size_t)c->max_rows * row_bytes);
+      if (!c->taps_stage[i]) return c->fail(OUTLETS_ENOMEM, "tap staging allocation failed");
+    }
+    tp[i] = c->taps_stage[i];
+  }
+  OUT_CK(c, cudaEventRecord(c->copy_start, s));
+  OUT_CK(c, cudaStreamWaitEvent(c->copy_stream, c->copy_start, 0));
+  for (int k = 0; k < n; ++k) {
+    const int r0 = k * chunk_rows, r1 = std::min(rows, r0 + chunk_rows);
+    for (int i = 0; i < 3; ++i)
+      OUT_CK(c, cudaMemcpyAsync((char*)c->taps_stage[i] + (size_t)r0 * row_bytes,
+                                (const char*)taps[i] + (size_t)r0 * row_bytes, (size_t)(r1 - r0) * row_bytes,
+                                cudaMemcpyHostToDevice, c->copy_stream));
+    OUT_CK(c, cudaEventRecord(c->chunk_ev[k], c->copy_stream));
   }
   return OUTLETS_OK;
 }
@@ -905,6 +953,10 @@ void outlets_destroy(outlets_ctx* c) {
   }
   if (c->done_ev) cudaEventDestroy(c->done_ev);
   for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
+  if (c->copy_start) cudaEventDestroy(c->copy_start);
+  for (cudaEvent_t e : c->chunk_ev)
+    if (e) cudaEventDestroy(e);
+  if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
   delete c;
 }
 
@@ -1081,8 +1133,18 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
   const int out_rows = all_tokens ? T : B;
 
   OUT_TRY(begin_call(c, s));
+  // Large calls with host taps overlap the copy with the front of the pipeline
+  // (FC, input norm, QKV, RoPE are row-wise): rows run in chunks of whole
+  // 128-row tiles as their taps land.
+  int n_chunks = 1, chunk_rows = T;
+  if (c->bf16 && !small_path(c, T) && !is_device_ptr(taps[0]) && !is_device_ptr(taps[1]) && !is_device_ptr(taps[2])) {
+    n_chunks = std::max(1, std::min(kMaxTapChunks, T / kMinTapChunkRows));
+    chunk_rows = (int)(cdiv(cdiv(T, n_chunks), 128) * 128);
+    n_chunks = (int)cdiv(T, chunk_rows);
+  }
   const void* tp[3];
-  OUT_TRY(prepare_taps(c, taps, T, tp, s));
+  if (n_chunks > 1) OUT_TRY(stage_taps_chunked(c, taps, T, n_chunks, chunk_rows, tp, s));
+  else OUT_TRY(prepare_taps(c, taps, T, tp, s));
 
   // ---- host metadata
   MetaBuilder mb;
@@ -1136,11 +1198,8 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
   const int* m = c->meta_dev;
   const int* cu_dev = m + off_cu;
 
-  // ---- FC (Eq. 1) -> input RMSNorm -> QKV
-  QkvSrc qsrc;
-  OUT_TRY(run_front(c, tp, T, &qsrc, s));
-  // ---- RoPE, q, head-major k/v, cache
-  c->stage_begin(OUTLETS_S_ROPE);
+  // ---- per row chunk: FC (Eq. 1) -> input RMSNorm -> QKV -> RoPE (q,
+  // head-major k/v, cache)
   {
     RopeArgs ra{};
     ra.T = T;
@@ -1164,9 +1223,20 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
       ra.page_tokens = kPageTokens;
     }
     ra.err = c->err_dev;
-    OUT_TRY(launch_rope(c, qsrc, ra, s));
+    for (int k = 0; k < n_chunks; ++k) {
+      const int r0 = k * chunk_rows, rows = std::min(T, r0 + chunk_rows) - r0;
+      if (n_chunks > 1) OUT_CK(c, cudaStreamWaitEvent(s, c->chunk_ev[k], 0));
+      const size_t off = (size_t)r0 * c->d * c->esz;
+      const void* tpc[3] = {(const char*)tp[0] + off, (const char*)tp[1] + off, (const char*)tp[2] + off};
+      QkvSrc qsrc;
+      OUT_TRY(run_front(c, tpc, rows, &qsrc, s, r0));
+      c->stage_begin(OUTLETS_S_ROPE);
+      ra.row0 = r0;
+      ra.T = rows;
+      OUT_TRY(launch_rope(c, qsrc, ra, s));
+      c->stage_end(1);
+    }
   }
-  c->stage_end(1);
   // ---- attention
   c->stage_begin(OUTLETS_S_ATTN);
   if (c->bf16) {

@@ -168,6 +168,34 @@ def test_host_buffers_match_device_buffers():
     np.testing.assert_array_equal(l_h.numpy(), l_d.cpu().numpy())
 
 
+def test_chunked_host_taps_match_device_taps():
+    """Host taps of a large call are copied in row chunks that the front of the
+    pipeline consumes as they land (a chunk boundary falls inside a sequence):
+    the predictions, every cached key and the draft states must be identical to
+    the same call on device taps."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = MID128
+    pred, w = predictor("mid128", max_tokens=8192)
+    lengths = [1500, 2100, 1400, 37]
+    cu = synth.cu_seqlens(lengths)
+    T = int(cu[-1])
+    taps = _taps(shape, T, off=13)
+    dev = [to_device(t, "bf16") for t in taps]
+    z_d, l_d = pred.prefill(dev, cu, all_tokens=True)
+    h_d = to_np(pred.intermediate(OT.T_HDRAFT)).copy()
+    host = [t.cpu().pin_memory() for t in dev]
+    z_h = torch.empty(T, dtype=torch.float32).pin_memory()
+    l_h = torch.empty(T, dtype=torch.float32).pin_memory()
+    pred.prefill(host, cu, all_tokens=True, z_out=z_h, len_out=l_h)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(z_h.numpy(), z_d.cpu().numpy())
+    np.testing.assert_array_equal(l_h.numpy(), l_d.cpu().numpy())
+    np.testing.assert_array_equal(to_np(pred.intermediate(OT.T_HDRAFT)), h_d)
+    ref = OR.predict_prefill(w, shape, taps, cu)
+    last = torch.as_tensor(np.asarray(cu[1:]) - 1, dtype=torch.long)
+    check_z_len(z_h[last], l_h[last], ref["z"], ref["length"], "bf16", "chunked host taps")
+
+
 def test_argument_errors_change_nothing():
     from paper_2609_01068_gb300 import outlets as OT
     shape = MID128

@@ -285,6 +285,54 @@ __global__ void __launch_bounds__(192, 1)
             store_row32(reinterpret_cast<bf16*>(p.out) + (long long)m * p.ldo + n0, v, min(32, n_out - n0));
           }
         }
+      } else if (EPI == EPI_F32 && p.residual) {
+        // f32 out + residual: the chunk loop is unrolled so the residual loads
+        // of the next LA chunks are in flight while a chunk is written (a short
+        // K loop, as in the O projection, leaves no time to wait for each).
+        constexpr int NC = BN / 32;
+        constexpr int LA = NC < 3 ? NC : 3;
+        const int row0 = tl.m_blk * TM + mt * BM + quarter * 32;
+        const int cq = (lane & 7) * 4;
+        float* stg = epi_stage + (warp - 2) * (32 * 36);
+        float4 res[LA][8];
+        auto load_res = [&](int ci, float4 (&rr)[8]) {
+          const int n = tl.n_blk * BN + ci * 32 + cq;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const int mm = row0 + k * 4 + (lane >> 3);
+            rr[k] = (mm < p.M && n < p.N)
+                        ? __ldg(reinterpret_cast<const float4*>(p.residual + (long long)mm * p.ldr + n))
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+        };
+#pragma unroll
+        for (int i = 0; i < LA; ++i) load_res(i, res[i]);
+#pragma unroll
+        for (int ci = 0; ci < NC; ++ci) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tbase + ci * 32, r);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 32; j += 4)
+            *reinterpret_cast<float4*>(stg + lane * 36 + j) = make_float4(
+                __uint_as_float(r[j]), __uint_as_float(r[j + 1]), __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3]));
+          __syncwarp();
+          const int n = tl.n_blk * BN + ci * 32 + cq;
+          if (n < p.N) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const int rr = k * 4 + (lane >> 3);
+              if (row0 + rr < p.M) {
+                const float4 v = *reinterpret_cast<const float4*>(stg + rr * 36 + cq);
+                const float4 q = res[ci % LA][k];
+                *reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (long long)(row0 + rr) * p.ldo + n) =
+                    make_float4(v.x + q.x, v.y + q.y, v.z + q.z, v.w + q.w);
+              }
+            }
+          }
+          if (ci + LA < NC) load_res(ci + LA, res[ci % LA]);
+          __syncwarp();
+        }
       } else {
         for (int c = 0; c < BN; c += 32) {
           uint32_t r[32];

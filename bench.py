@@ -34,6 +34,18 @@ sys.path.insert(0, ROOT)
 METRIC = "length predictions/s and draft tokens/s on 1 GB300; % bf16 tensor peak / % HBM BW"
 WORKLOAD = ("static length prediction, Llama-3.1-8B-shaped EAGLE-3 draft layer + length head, "
             "64 ragged prompts (lognormal median 256, clipped 16-2048), packed varlen")
+WORKLOAD_70B = ("static length prediction, Llama-3.3-70B-shaped EAGLE-3 draft layer + length head, "
+                "32 ragged prompts (lognormal median 1024, clipped 64-4096), packed varlen")
+
+
+def model_setup(args):
+    """Shape, prompt lengths, workload text and traffic key prefix of --model."""
+    from paper_2609_01068_gb300 import synth
+    if args.model == "70b":
+        lengths = synth.lengths_70b_prefill(0)
+        return synth.LLAMA70B, lengths[:args.prompts] if args.prompts else lengths, WORKLOAD_70B, "70b"
+    lengths = synth.lengths_8b_prefill(0)
+    return synth.LLAMA8B, lengths[:args.prompts] if args.prompts else lengths, WORKLOAD, "8b"
 
 
 def parse():
@@ -44,7 +56,10 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--mode", default="both", choices=["both", "prefill", "step", "sweep"],
                     help="static prediction (headline), dynamic prediction, both, or the serving sweep")
-    ap.add_argument("--prompts", type=int, default=64, help="first N prompts of the workload (profiling cases)")
+    ap.add_argument("--prompts", type=int, default=None,
+                    help="first N prompts of the workload (profiling cases; default: all)")
+    ap.add_argument("--model", default="8b", choices=["8b", "70b"],
+                    help="draft-layer shape; 70b (Llama-3.3-70B-shaped, 32 prompts) runs the static mode only")
     ap.add_argument("--step-requests", type=int, default=256, help="live requests of the dynamic-prediction run")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -145,6 +160,12 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm), "power_w_max": max(power) if power else None}
 
 
+def weight_bytes(shape):
+    """bf16 bytes of the draft layer's matrices and the head's first layer."""
+    d, H, KVH, hd, F = shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
+    return 2 * (3 * d * d + d * (H + 2 * KVH) * hd + H * hd * d + 3 * d * F + d * shape.head_widths[0])
+
+
 def prefill_flops(shape, lengths, n_out):
     """Algorithmic FLOPs of one static-prediction pass (dense GEMMs + causal attention + head)."""
     d, H, KVH, hd, F = shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
@@ -215,9 +236,8 @@ def run_reference(args):
     if rank != 0:
         return
     from paper_2609_01068_gb300 import synth
-    shape = synth.LLAMA8B
+    shape, lengths, workload, _ = model_setup(args)
     w = synth.make_weights(shape, 0)
-    lengths = synth.lengths_8b_prefill(0)
     cu = synth.cu_seqlens(lengths)
     taps = synth.make_taps(shape, int(cu[-1]), 0)
     budget = 400
@@ -232,7 +252,7 @@ def run_reference(args):
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * secs / args.steps,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "draft_tokens_per_s": n_tok / secs,
-           "config": {"workload": WORKLOAD, "sample": f"~{budget} prompt tokens per step (whole prompts)"},
+           "config": {"workload": workload, "sample": f"~{budget} prompt tokens per step (whole prompts)"},
            "cpu_baseline": {"value": value, "unit": "predictions/s", "cores": cpu_threads(), "kind": "oracle",
                             "sample": f"{n_pred} prompts / {n_tok} tokens over {args.steps} steps"},
            "e2e": {"value": value, "unit": "predictions/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -254,9 +274,11 @@ def run_ours(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     B.build()
     peaks = load_peaks()
-    shape = synth.LLAMA8B
+    if args.model == "70b" and args.mode != "prefill":
+        raise SystemExit("--model 70b runs the static (prefill) mode only")
+    shape, lengths, workload, tkey = model_setup(args)
+    args.workload, args.traffic_key = workload, tkey
     w = synth.make_weights(shape, 0)
-    lengths = synth.lengths_8b_prefill(0)[:args.prompts]
     cu = synth.cu_seqlens(lengths)
     T, Bq = int(cu[-1]), len(lengths)
     taps = synth.make_taps(shape, T, 0, rank)
@@ -346,7 +368,7 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     roofline = {"bound": "tensor", "kernel": "gateup_swiglu_gemm (k_gemm_tc<256, SWIGLU>)",
                 "achieved": gu_tflops, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
                 "frac": gu_tflops / peaks["bf16_sus"], "peak_kind": f"bf16 sustained {peaks['src']}",
-                "traffic": measured_traffic("gateup_swiglu_gemm", f"8b-static-{Bq}p-T{T}"),
+                "traffic": measured_traffic("gateup_swiglu_gemm", f"{args.traffic_key}-static-{Bq}p-T{T}"),
                 "algorithmic_per_launch": f"{gu_flops:.4g} FLOP = 2*T*(2F)*d, T={T}"}
     stages = {k: {"ms_per_step": v[0] / max(v[1], 1), "share": v[0] / max(sum(x[0] for x in prof.values()), 1e-9)}
               for k, v in prof.items() if v[1]}
@@ -371,9 +393,9 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
                "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4)}
 
     out = {"value": value, "unit": "predictions/s", "ms_per_step": ms_step,
-           "config": {"workload": WORKLOAD, "prompts_per_gpu": Bq, "tokens_per_gpu": T,
-                      "l2": "inputs larger than L2 (taps 3x[T,4096] bf16 = %.0f MB, weights 545 MB)"
-                            % (3 * T * 4096 * 2 / 1e6),
+           "config": {"workload": args.workload, "prompts_per_gpu": Bq, "tokens_per_gpu": T,
+                      "l2": "inputs larger than L2 (taps 3x[T,%d] bf16 = %.0f MB, weights %.0f MB)"
+                            % (shape.d, 3 * T * shape.d * 2 / 1e6, weight_bytes(shape) / 1e6),
                       "parallelism": f"replicas x{world}"},
            "draft_tokens_per_s": world * T * args.steps / (ms / 1e3),
            "tflops_per_s": flops * args.steps / (ms / 1e3) / 1e12,

@@ -8,7 +8,8 @@
 // bf16 path: split-KV.  One CTA = (request, split of <= split_len keys, kv
 // head).  The G = H / KVH query heads of the kv head form the rows of one
 // 16-row mma.sync tile, so every K/V byte is read from HBM once.  Page blocks
-// (64 keys x hd) of K and V are staged by TMA (128-byte swizzle, 3 stages);
+// (64 keys x hd) of K and V are staged by TMA (128-byte swizzle, 2 stages,
+// three CTAs per SM so one CTA's start-up is covered by two streaming ones);
 // each of the 4 warps takes 16 keys of a page, keeps its own online softmax,
 // and the warps are merged through shared memory.  Requests with one split
 // write the output directly; others write (o, m, l) partials, and the last
@@ -24,7 +25,7 @@ namespace outlets {
 namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr int kStages = 3;
+constexpr int kStages = 2;
 
 template <int HD>
 struct DecCfg {
@@ -83,7 +84,7 @@ __device__ __forceinline__ void merge_splits(const DecodeArgs& a, int b, int h0,
 }
 
 template <int HD>
-__global__ void __launch_bounds__(128)
+__global__ void __launch_bounds__(128, 3)
     k_attn_decode_bf16(const __grid_constant__ CUtensorMap k_map, const __grid_constant__ CUtensorMap v_map,
                        const DecodeArgs a) {
   pdl_trigger();

@@ -34,7 +34,7 @@ constexpr int kPageTokens = 64;
 constexpr int kMaxTapChunks = 4;      // row chunks of host taps copied while earlier chunks compute
 constexpr int kMinTapChunkRows = 2048;
 constexpr int kSplitLen = 512;        // shortest split-KV work item (keys)
-constexpr int kDecodeCtasPerSm = 2;   // resident decode-attention CTAs per SM
+constexpr int kDecodeCtasPerSm = 3;   // resident decode-attention CTAs per SM
 constexpr int kRing = 4;
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,

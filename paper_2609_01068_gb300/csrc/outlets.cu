@@ -139,16 +139,23 @@ struct outlets_ctx {
   int* dec_count = nullptr;  // [max_batch, KVH] split-KV completion counters of decode attention
   float* part = nullptr;  // f32 split-K slices of the small-M path
   size_t part_floats = 0;
-  int* meta_dev = nullptr;
-  size_t meta_cap = 0;  // ints
+  int* meta_dev = nullptr;  // device metadata of the current call (a ring slot's buffer)
 
+  // Ring of metadata slots: pinned host staging + device buffer.  A slot is
+  // reused only after the call that last used it has finished on the GPU
+  // (`done`), so the upload of one call overlaps the kernels of the previous.
   struct Pin {
     int* h = nullptr;
     size_t cap = 0;
-    cudaEvent_t ev = nullptr;
+    int* dev = nullptr;
+    size_t dev_cap = 0;
+    cudaEvent_t ev = nullptr;    // upload complete (copy stream)
+    cudaEvent_t done = nullptr;  // the call that used the slot is complete (its stream)
     bool used = false;
   } ring[kRing];
   int ring_i = 0;
+  int cur_slot = -1;
+  bool meta_waited = false;
   cudaEvent_t done_ev = nullptr;
   // copies of host taps in row chunks, overlapped with the prefill front
   cudaStream_t copy_stream = nullptr;
@@ -300,43 +307,84 @@ outlets_status validate_config(const outlets_config* cfg, std::string& why) {
   return OUTLETS_OK;
 }
 
-// Pinned staging of one call's index metadata, then one H2D copy.
+#define OUT_TRY(expr)                      \
+  do {                                     \
+    outlets_status st_ = (expr);           \
+    if (st_ != OUTLETS_OK) return st_;     \
+  } while (0)
+
+outlets_status ensure_copy_stream(outlets_ctx* c) {
+  if (c->copy_stream) return OUTLETS_OK;
+  OUT_CK(c, cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking));
+  OUT_CK(c, cudaEventCreateWithFlags(&c->copy_start, cudaEventDisableTiming));
+  for (auto& e : c->chunk_ev) OUT_CK(c, cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+  return OUTLETS_OK;
+}
+
+// One call's index metadata: pinned staging, one H2D copy on the copy stream
+// into the slot's device buffer.  Sets c->meta_dev; kernels that read it are
+// enqueued after wait_meta (the FC, norm and QKV kernels before them keep
+// their programmatic launch chain).  The slot is released when the call's
+// stream passes the slot's `done` event (recorded by CallSlot on every exit).
 outlets_status upload_meta(outlets_ctx* c, const std::vector<int>& meta, cudaStream_t s) {
   if (meta.empty()) return OUTLETS_OK;
-  if (meta.size() > c->meta_cap) {
-    if (c->meta_dev) {
-      OUT_CK(c, cudaStreamSynchronize(s));
-      cudaFree(c->meta_dev);
-      c->meta_dev = nullptr;
-    }
-    size_t cap = std::max<size_t>(meta.size() * 2, 1 << 16);
-    if (cudaMalloc(&c->meta_dev, cap * sizeof(int)) != cudaSuccess) {
-      cudaGetLastError();
-      c->meta_cap = 0;
-      return c->fail(OUTLETS_ENOMEM, "metadata buffer allocation failed");
-    }
-    c->meta_cap = cap;
-  }
-  outlets_ctx::Pin& p = c->ring[c->ring_i];
+  OUT_TRY(ensure_copy_stream(c));
+  const int slot = c->ring_i;
+  outlets_ctx::Pin& p = c->ring[slot];
   c->ring_i = (c->ring_i + 1) % kRing;
-  if (p.used) OUT_CK(c, cudaEventSynchronize(p.ev));
+  if (p.used) OUT_CK(c, cudaEventSynchronize(p.done));
+  const size_t cap = std::max<size_t>(meta.size() * 2, 1 << 16);
   if (meta.size() > p.cap) {
     if (p.h) cudaFreeHost(p.h);
     p.h = nullptr;
-    size_t cap = std::max<size_t>(meta.size() * 2, 1 << 16);
+    p.cap = 0;
     if (cudaMallocHost(&p.h, cap * sizeof(int)) != cudaSuccess) {
       cudaGetLastError();
-      p.cap = 0;
       return c->fail(OUTLETS_ENOMEM, "pinned metadata buffer allocation failed");
     }
     p.cap = cap;
   }
+  if (meta.size() > p.dev_cap) {
+    if (p.dev) cudaFree(p.dev);
+    p.dev = nullptr;
+    p.dev_cap = 0;
+    if (cudaMalloc(&p.dev, cap * sizeof(int)) != cudaSuccess) {
+      cudaGetLastError();
+      return c->fail(OUTLETS_ENOMEM, "metadata buffer allocation failed");
+    }
+    p.dev_cap = cap;
+  }
   std::memcpy(p.h, meta.data(), meta.size() * sizeof(int));
-  OUT_CK(c, cudaMemcpyAsync(c->meta_dev, p.h, meta.size() * sizeof(int), cudaMemcpyHostToDevice, s));
-  OUT_CK(c, cudaEventRecord(p.ev, s));
+  OUT_CK(c, cudaMemcpyAsync(p.dev, p.h, meta.size() * sizeof(int), cudaMemcpyHostToDevice, c->copy_stream));
+  OUT_CK(c, cudaEventRecord(p.ev, c->copy_stream));
   p.used = true;
+  c->cur_slot = slot;
+  c->meta_waited = false;
+  c->meta_dev = p.dev;
   return OUTLETS_OK;
 }
+
+// Makes stream s wait for the current call's metadata upload (once).
+outlets_status wait_meta(outlets_ctx* c, cudaStream_t s) {
+  if (c->cur_slot < 0 || c->meta_waited) return OUTLETS_OK;
+  OUT_CK(c, cudaStreamWaitEvent(s, c->ring[c->cur_slot].ev, 0));
+  c->meta_waited = true;
+  return OUTLETS_OK;
+}
+
+// Releases the call's metadata slot on every exit from a prediction call:
+// records the slot's `done` event after everything the call enqueued.
+struct CallSlot {
+  outlets_ctx* c;
+  cudaStream_t s;
+  ~CallSlot() {
+    if (c->cur_slot >= 0) {
+      if (!c->meta_waited) cudaStreamWaitEvent(s, c->ring[c->cur_slot].ev, 0);  // done implies uploaded
+      cudaEventRecord(c->ring[c->cur_slot].done, s);
+      c->cur_slot = -1;
+    }
+  }
+};
 
 struct MetaBuilder {
   std::vector<int> v;
@@ -365,12 +413,6 @@ bool cached_map(outlets_ctx* c, CUtensorMap* m, const void* base, uint64_t cols,
 }
 
 bool owned_by(const outlets_ctx* c, const void* p);
-
-#define OUT_TRY(expr)                      \
-  do {                                     \
-    outlets_status st_ = (expr);           \
-    if (st_ != OUTLETS_OK) return st_;     \
-  } while (0)
 
 // Tensor maps of the (up to three) A pieces of a GEMM.
 outlets_status a_maps(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
@@ -730,11 +772,7 @@ outlets_status prepare_taps(outlets_ctx* c, const void* const taps[3], int rows,
 // are still in transit.  tp receives the staging buffers.
 outlets_status stage_taps_chunked(outlets_ctx* c, const void* const taps[3], int rows, int n, int chunk_rows,
                                   const void* tp[3], cudaStream_t s) {
-  if (!c->copy_stream) {
-    OUT_CK(c, cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking));
-    OUT_CK(c, cudaEventCreateWithFlags(&c->copy_start, cudaEventDisableTiming));
-    for (auto& e : c->chunk_ev) OUT_CK(c, cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
-  }
+  OUT_TRY(ensure_copy_stream(c));
   const size_t row_bytes = (size_t)c->d * c->esz;
   for (int i = 0; i < 3; ++i) {
     if (!taps[i]) return c->fail(OUTLETS_EINVAL, "taps[i] is NULL");
@@ -880,7 +918,9 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   }
   if (c->oom) return cleanup_fail(OUTLETS_ENOMEM);
   for (auto& p : c->ring)
-    if (cudaEventCreateWithFlags(&p.ev, cudaEventDisableTiming) != cudaSuccess) return cleanup_fail(OUTLETS_ECUDA);
+    if (cudaEventCreateWithFlags(&p.ev, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&p.done, cudaEventDisableTiming) != cudaSuccess)
+      return cleanup_fail(OUTLETS_ECUDA);
   if (cudaEventCreateWithFlags(&c->done_ev, cudaEventDisableTiming) != cudaSuccess) return cleanup_fail(OUTLETS_ECUDA);
 
   // ---- upload
@@ -946,10 +986,11 @@ void outlets_destroy(outlets_ctx* c) {
   cudaDeviceSynchronize();
   for (void* p : c->allocs)
     if (p) cudaFree(p);
-  if (c->meta_dev) cudaFree(c->meta_dev);
   for (auto& p : c->ring) {
     if (p.h) cudaFreeHost(p.h);
+    if (p.dev) cudaFree(p.dev);
     if (p.ev) cudaEventDestroy(p.ev);
+    if (p.done) cudaEventDestroy(p.done);
   }
   if (c->done_ev) cudaEventDestroy(c->done_ev);
   for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
@@ -1133,6 +1174,7 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
   const int out_rows = all_tokens ? T : B;
 
   OUT_TRY(begin_call(c, s));
+  CallSlot slot_guard{c, s};
   // Large calls with host taps overlap the copy with the front of the pipeline
   // (FC, input norm, QKV, RoPE are row-wise): rows run in chunks of whole
   // 128-row tiles as their taps land.
@@ -1142,9 +1184,6 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
     chunk_rows = (int)(cdiv(cdiv(T, n_chunks), 128) * 128);
     n_chunks = (int)cdiv(T, chunk_rows);
   }
-  const void* tp[3];
-  if (n_chunks > 1) OUT_TRY(stage_taps_chunked(c, taps, T, n_chunks, chunk_rows, tp, s));
-  else OUT_TRY(prepare_taps(c, taps, T, tp, s));
 
   // ---- host metadata
   MetaBuilder mb;
@@ -1195,6 +1234,11 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
     off_po = mb.put(po);
   }
   OUT_TRY(upload_meta(c, mb.v, s));
+  // taps after the metadata: both go through the copy stream, and the call's
+  // stream waits for the metadata before its first kernel
+  const void* tp[3];
+  if (n_chunks > 1) OUT_TRY(stage_taps_chunked(c, taps, T, n_chunks, chunk_rows, tp, s));
+  else OUT_TRY(prepare_taps(c, taps, T, tp, s));
   const int* m = c->meta_dev;
   const int* cu_dev = m + off_cu;
 
@@ -1230,6 +1274,7 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
       const void* tpc[3] = {(const char*)tp[0] + off, (const char*)tp[1] + off, (const char*)tp[2] + off};
       QkvSrc qsrc;
       OUT_TRY(run_front(c, tpc, rows, &qsrc, s, r0));
+      OUT_TRY(wait_meta(c, s));
       c->stage_begin(OUTLETS_S_ROPE);
       ra.row0 = r0;
       ra.T = rows;
@@ -1281,6 +1326,7 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
   if (need > (int)kv->free_list.size()) return c->fail(OUTLETS_ECAPACITY, "not enough free KV pages");
 
   OUT_TRY(begin_call(c, s));
+  CallSlot slot_guard{c, s};
   const void* tp[3];
   OUT_TRY(prepare_taps(c, taps, B, tp, s));
 
@@ -1334,6 +1380,7 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
 
   QkvSrc qsrc;
   OUT_TRY(run_front(c, tp, B, &qsrc, s));
+  OUT_TRY(wait_meta(c, s));  // RoPE is the first kernel that reads the metadata
   c->stage_begin(OUTLETS_S_ROPE);
   {
     RopeArgs ra{};

@@ -304,7 +304,7 @@ def run_ours(args):
     if args.mode in ("both", "step"):
         sm = run_step_mode(args, pred, shape, peaks, step_B, world, barrier, max_over_ranks, stream, max_tokens)
         if args.mode == "step":
-            out.update({k: sm[k] for k in ("value", "unit", "ms_per_step")})
+            out.update({k: sm[k] for k in ("value", "unit", "ms_per_step", "e2e", "gpu_launches", "clocks")})
             out["config"] = {"workload": sm["workload"], "parallelism": f"replicas x{world}"}
         out["step_mode"] = sm
     if args.mode == "sweep":
@@ -415,7 +415,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
 
     from paper_2609_01068_gb300 import outlets, synth
     lens = synth.lengths_8b_step_cache(0, B)
-    n_steps = args.steps + args.warmup
+    n_steps = 2 * args.steps + args.warmup  # timed steps, then as many again for the e2e pass
     kv = outlets.KVCache(pred, max_slots=B, max_tokens_total=int(lens.sum()) + (n_steps + 8 + 64) * B)
     gen = torch.Generator(device="cuda").manual_seed(1)
     b = 0
@@ -461,6 +461,24 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
         pred.step(st_taps, kv, slots, z_out=z, len_out=ln)
     prof = pred.profile_read()
     pred.profile(False)
+    # end to end through the C ABI: host taps in, host predictions out, every step
+    e2e = None
+    if not args.no_e2e:
+        host_taps = [t.cpu().pin_memory() for t in st_taps]
+        zh = torch.empty(B, dtype=torch.float32).pin_memory()
+        lh = torch.empty(B, dtype=torch.float32).pin_memory()
+        for _ in range(2):
+            pred.step(host_taps, kv, slots, z_out=zh, len_out=lh)
+            stream.synchronize()
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            pred.step(host_taps, kv, slots, z_out=zh, len_out=lh)
+            stream.synchronize()
+        e2e_s = max_over_ranks(time.perf_counter() - t0)
+        e2e = {"value": world * B * args.steps / e2e_s, "unit": "predictions/s",
+               "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps)),
+               "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4)}
     d, KVH, hd, F = shape.d, shape.n_kv_heads, shape.head_dim, shape.ffn
     # keys read per step: every cached position plus the new one, K and V, bf16
     keys_avg = cache0 + B * (args.steps + 1) / 2.0
@@ -483,7 +501,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
                          "traffic": measured_traffic("decode_attention", f"8b-step-{B}r-L{int(lens.sum())}"),
                          "algorithmic_per_launch": f"{kv_bytes:.4g} B of K/V (cached + new)"},
             "stages": {k: v[0] / max(v[1], 1) for k, v in prof.items() if v[1]},
-            "clocks": clocks, "gpu_launches": launches, "host_issue_ms_per_step": host_ms}
+            "clocks": clocks, "gpu_launches": launches, "host_issue_ms_per_step": host_ms, "e2e": e2e}
 
 
 def pack_batches(lengths, cap):

@@ -22,8 +22,13 @@ primitive used as a step.  The steps follow the paper in order:
 
 Readings where the paper is silent (the same list is kept in the design notes):
   * attention is standard causal GQA softmax(q k^T / sqrt(hd)) v; q-head h
-    uses kv-head floor(h * KVH / H); the gated variant (Sec. 4.1 cites Gated
-    Attention) is out of the default path;
+    uses kv-head floor(h * KVH / H);
+  * gated attention (Sec. 4.1 instantiates the layer's attention with the
+    cited Gated Attention, no formula given): read as that work's elementwise,
+    head-specific sigmoid gate computed from the normalized layer input,
+    o <- o * sigmoid(x_hat W_ag^T) with W_ag [H*hd, d], applied to the
+    attention output before W_o.  Used when the weights carry "w_attn_gate";
+    the default path has no gate;
   * RMSNorm y = x * g / sqrt(mean(x^2) + eps);
   * RoPE rotates pairs (i, i + hd/2) by angle pos * theta^(-2i/hd);
     positions restart at 0 for each packed sequence; a decode step's token
@@ -145,6 +150,17 @@ def attend_single(q_row, k_all, v_all):
     return out
 
 
+# ------------------------------------------------------------------ gated attention (Sec. 4.1)
+def sigmoid(x):
+    x = _f64(x)
+    return 1.0 / (1.0 + np.exp(-x))
+
+
+def attention_gate(x, w_attn_gate):
+    """Elementwise gate of gated attention: sigmoid(x_hat W_ag^T), [rows, H*hd]."""
+    return sigmoid(_f64(x) @ _f64(w_attn_gate).T)
+
+
 # ------------------------------------------------------------------ MLP
 def silu(x):
     x = _f64(x)
@@ -205,6 +221,8 @@ def predict_prefill(w, shape, taps, cu, all_tokens=False):
     q = apply_rope(q, pos, theta)
     k = apply_rope(k, pos, theta)
     o = causal_gqa_attention(q, k, v, cu).reshape(T, H * hd)
+    if w.get("w_attn_gate") is not None:
+        o = o * attention_gate(x, w["w_attn_gate"])
     a = f + o @ _f64(w["w_o"]).T
     ah = rms_norm(a, w["g_post"], eps)
     y = a + swiglu_mlp(ah, w["w_gate"], w["w_up"], w["w_down"])
@@ -248,6 +266,8 @@ def predict_step(w, shape, taps_rows, caches):
         o[b] = attend_single(q[b], kc, vc)
         new_caches.append((kc, vc))
     o = o.reshape(B, H * hd)
+    if w.get("w_attn_gate") is not None:
+        o = o * attention_gate(x, w["w_attn_gate"])
     a = f + o @ _f64(w["w_o"]).T
     y = a + swiglu_mlp(rms_norm(a, w["g_post"], eps), w["w_gate"], w["w_up"], w["w_down"])
     hd_state = rms_norm(y, w["g_final"], eps)

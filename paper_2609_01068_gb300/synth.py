@@ -136,10 +136,12 @@ def weight_names(shape: ModelShape):
 
 
 def make_weights(shape: ModelShape, seed: int = 0, std: float = 0.02,
-                 out_bias: float = math.log(257.0)) -> dict:
+                 out_bias: float = math.log(257.0), gated: bool = False) -> dict:
     """All draft weights, nn.Linear [out, in] row-major, float32 arrays.
 
     On the bf16 path the matrices and head parameters are bf16-representable.
+    gated=True adds the attention gate "w_attn_gate" [H*hd, d] (gated
+    attention), drawn after every other weight so the rest are unchanged.
     """
     rng = _streams(seed)[2]
     d, H, KVH, hd, F = shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
@@ -167,6 +169,8 @@ def make_weights(shape: ModelShape, seed: int = 0, std: float = 0.02,
             w[f"head_b{i}"] = rnd(rng.standard_normal(widths[i + 1], dtype=np.float32) * np.float32(std))
         else:
             w[f"head_b{i}"] = rnd(np.full(1, out_bias, np.float32))
+    if gated:
+        w["w_attn_gate"] = lin(H * hd, d)
     return w
 
 

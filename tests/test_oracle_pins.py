@@ -342,3 +342,80 @@ def test_generator_is_seeded_and_shaped():
     assert len(s) == 1024 and s.max() <= 8192
     cu = synth.cu_seqlens([3, 4])
     assert cu.tolist() == [0, 3, 7] and cu.dtype == np.int32
+
+
+# ---------------------------------------------------------------- gated attention (Sec. 4.1)
+def _gated_weights(shape=SMALL, seed=0):
+    return synth.make_weights(shape, seed, gated=True)
+
+
+def test_sigmoid_against_library_expit():
+    scipy_special = pytest.importorskip("scipy.special")
+    x = np.linspace(-40, 40, 161)
+    np.testing.assert_allclose(O.sigmoid(x), scipy_special.expit(x), rtol=1e-13, atol=1e-300)
+
+
+def test_zero_gate_weights_halve_the_attention_output():
+    """W_ag = 0 gives sigmoid(0) = 1/2 on every element: the gated layer equals
+    the ungated layer with W_o scaled by 1/2 (linearity of the output projection)."""
+    w = dict(_gated_weights())
+    w["w_attn_gate"] = np.zeros_like(w["w_attn_gate"])
+    gated, _, _ = _prefill(w, SMALL, [5, 3])
+    w2 = {k: v for k, v in w.items() if k != "w_attn_gate"}
+    w2["w_o"] = w["w_o"] * 0.5
+    plain, _, _ = _prefill(w2, SMALL, [5, 3])
+    np.testing.assert_allclose(gated["y"], plain["y"], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(gated["z"], plain["z"], rtol=1e-12, atol=1e-12)
+
+
+def test_gate_brute_force_elementwise():
+    """attn[r, c] = o[r, c] / (1 + exp(-sum_j x_hat[r, j] W_ag[c, j])), element by element."""
+    w = _gated_weights()
+    w2 = {k: v for k, v in w.items() if k != "w_attn_gate"}
+    gated, _, _ = _prefill(w, SMALL, [4, 3])
+    plain, _, _ = _prefill(w2, SMALL, [4, 3])
+    x, o, W = gated["x"], plain["attn"], w["w_attn_gate"].astype(np.float64)
+    ref = np.empty_like(o)
+    for r in range(o.shape[0]):
+        for c in range(o.shape[1]):
+            acc = 0.0
+            for j in range(x.shape[1]):
+                acc += float(x[r, j]) * float(W[c, j])
+            ref[r, c] = o[r, c] / (1.0 + math.exp(-acc))
+    np.testing.assert_allclose(gated["attn"], ref, rtol=1e-12, atol=1e-14)
+
+
+def test_gate_is_elementwise_per_output_column():
+    """Changing one row of W_ag changes only that column of the gated output."""
+    w = dict(_gated_weights())
+    base, _, _ = _prefill(w, SMALL, [6])
+    col = 5
+    w["w_attn_gate"] = w["w_attn_gate"].copy()
+    w["w_attn_gate"][col] += 0.5
+    moved, _, _ = _prefill(w, SMALL, [6])
+    diff = np.abs(moved["attn"] - base["attn"]).max(axis=0)
+    assert diff[col] > 0
+    assert np.all(np.delete(diff, col) == 0)
+
+
+def test_gated_prefill_equals_prefix_then_steps():
+    w = _gated_weights()
+    lengths = [5, 3]
+    full, taps, cu = _prefill(w, SMALL, lengths, all_tokens=True)
+    kpre = [2, 1]
+    pre_taps = [np.concatenate([t[cu[b]:cu[b] + kpre[b]] for b in range(2)]) for t in taps]
+    pre_cu = synth.cu_seqlens(kpre)
+    caches = O.caches_from_prefill(O.predict_prefill(w, SMALL, pre_taps, pre_cu), pre_cu)
+    for step in range(2):
+        rows = [cu[b] + kpre[b] + step for b in range(2)]
+        st = O.predict_step(w, SMALL, [t[rows] for t in taps], caches)
+        np.testing.assert_allclose(st["z"], full["z"][rows], rtol=1e-11, atol=1e-11)
+        caches = st["caches"]
+
+
+def test_default_weights_have_no_gate():
+    w = synth.make_weights(SMALL, 0)
+    wg = synth.make_weights(SMALL, 0, gated=True)
+    assert "w_attn_gate" not in w
+    for k in w:
+        np.testing.assert_array_equal(w[k], wg[k])

@@ -92,6 +92,11 @@ typedef struct outlets_config {
  *   w_gate [F, d], w_up [F, d], w_down [d, F]
  *   head_w[i] [w_{i+1}, w_i], head_b[i] [w_{i+1}] for i = 0 .. n_head_hidden,
  *   widths w_0 = d, w_1.. = head_hidden, last = 1.
+ *   w_attn_gate [H*hd, d] or NULL: gated attention (Sec. 4.1 uses the cited
+ *     Gated Attention for the draft layer).  When given, the attention output
+ *     o [rows, H*hd] is multiplied elementwise by sigmoid(x_hat w_attn_gate^T)
+ *     (x_hat: the RMS-normalized layer input that also feeds QKV) before W_o;
+ *     NULL gives standard attention.
  * The library copies everything during outlets_create; the caller may free
  * its arrays afterwards. */
 typedef struct outlets_weights {
@@ -108,6 +113,7 @@ typedef struct outlets_weights {
   const float* w_down;
   const float* head_w[OUTLETS_MAX_HEAD_HIDDEN + 1];
   const float* head_b[OUTLETS_MAX_HEAD_HIDDEN + 1];
+  const float* w_attn_gate;
 } outlets_weights;
 
 typedef struct outlets_ctx outlets_ctx;

@@ -79,7 +79,9 @@ __device__ __forceinline__ void merge_splits(const DecodeArgs& a, int b, int h0,
       for (int k = 0; k < 8; ++k)
         if (w + k < ns) Os += wt[r * ns + w + k] * o[k];
     }
-    reinterpret_cast<bf16*>(a.out)[((long long)b * a.H + h0 + r) * HD + d] = __float2bfloat16_rn(Os / lsum[r]);
+    const long long oi = ((long long)b * a.H + h0 + r) * HD + d;
+    const float gv = a.gate ? __bfloat162float(reinterpret_cast<const bf16*>(a.gate)[oi]) : 1.f;  // gated attention
+    reinterpret_cast<bf16*>(a.out)[oi] = __float2bfloat16_rn(Os / lsum[r] * gv);
   }
 }
 
@@ -304,7 +306,9 @@ __global__ void __launch_bounds__(128, 3)
     }
     const int head = g * G + r;
     if (n_split == 1) {
-      reinterpret_cast<bf16*>(a.out)[((long long)b * a.H + head) * HD + d] = __float2bfloat16_rn(Os / Ls);
+      const long long oi = ((long long)b * a.H + head) * HD + d;
+      const float gv = a.gate ? __bfloat162float(reinterpret_cast<const bf16*>(a.gate)[oi]) : 1.f;
+      reinterpret_cast<bf16*>(a.out)[oi] = __float2bfloat16_rn(Os / Ls * gv);
     } else {
       const long long pi = (long long)item * a.H + head;  // partial index: (work item, head)
       a.part_o[pi * HD + d] = Os / Ls;
@@ -380,10 +384,11 @@ __global__ void k_attn_decode_simt(const DecodeArgs a) {
     m = mn;
   }
   Act* op = reinterpret_cast<Act*>(a.out) + ((long long)b * a.H + h) * hd;
+  const Act* gp = a.gate ? reinterpret_cast<const Act*>(a.gate) + ((long long)b * a.H + h) * hd : nullptr;
 #pragma unroll
   for (int i = 0; i < MAXD; ++i) {
     const int d = lane + 32 * i;
-    if (d < hd) op[d] = from_f<Act>(ov[i] / l);
+    if (d < hd) op[d] = from_f<Act>(ov[i] / l * (gp ? to_f(gp[d]) : 1.f));
   }
 }
 

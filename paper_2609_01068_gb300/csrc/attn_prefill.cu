@@ -29,7 +29,7 @@ template <int HD>
 __global__ void __launch_bounds__(128)
     k_attn_prefill_bf16(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap k_map,
                         const __grid_constant__ CUtensorMap v_map, const AttnTile* __restrict__ tiles, int T,
-                        int H, int KVH, bf16* __restrict__ out, int* err) {
+                        int H, int KVH, bf16* __restrict__ out, const bf16* __restrict__ gate, int* err) {
   pdl_trigger();
   pdl_wait();
   using C = PrefillCfg<HD>;
@@ -213,10 +213,16 @@ __global__ void __launch_bounds__(128)
 #pragma unroll
   for (int j = 0; j < HD / 8; ++j) {
     const int d = h * HD + 8 * j + 2 * (lane & 3);
-    if (row0 < q_end)
-      *reinterpret_cast<uint32_t*>(out + row0 * ld + d) = pack_bf16x2(o[j][0] * inv0, o[j][1] * inv0);
-    if (row1 < q_end)
-      *reinterpret_cast<uint32_t*>(out + row1 * ld + d) = pack_bf16x2(o[j][2] * inv1, o[j][3] * inv1);
+    if (row0 < q_end) {
+      float2 gv = make_float2(1.f, 1.f);  // gated attention: elementwise output gate
+      if (gate) gv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(gate + row0 * ld + d));
+      *reinterpret_cast<uint32_t*>(out + row0 * ld + d) = pack_bf16x2(o[j][0] * inv0 * gv.x, o[j][1] * inv0 * gv.y);
+    }
+    if (row1 < q_end) {
+      float2 gv = make_float2(1.f, 1.f);
+      if (gate) gv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(gate + row1 * ld + d));
+      *reinterpret_cast<uint32_t*>(out + row1 * ld + d) = pack_bf16x2(o[j][2] * inv1 * gv.x, o[j][3] * inv1 * gv.y);
+    }
   }
 }
 
@@ -233,7 +239,7 @@ __device__ __forceinline__ void load_dims(const Act* p, int hd, int lane, float*
 template <typename Act>
 __global__ void k_attn_prefill_simt(const Act* __restrict__ q, const Act* __restrict__ k,
                                     const Act* __restrict__ v, const int* __restrict__ cu, int B, int kv_ld, int H,
-                                    int KVH, int hd, Act* __restrict__ out) {
+                                    int KVH, int hd, Act* __restrict__ out, const Act* __restrict__ gate) {
   pdl_trigger();
   pdl_wait();
   constexpr int MAXD = 8;  // hd <= 256
@@ -277,10 +283,11 @@ __global__ void k_attn_prefill_simt(const Act* __restrict__ q, const Act* __rest
     m = mn;
   }
   Act* op = out + ((long long)row * H + h) * hd;
+  const Act* gp = gate ? gate + ((long long)row * H + h) * hd : nullptr;
 #pragma unroll
   for (int i = 0; i < MAXD; ++i) {
     const int d = lane + 32 * i;
-    if (d < hd) op[d] = from_f<Act>(ov[i] / l);
+    if (d < hd) op[d] = from_f<Act>(ov[i] / l * (gp ? to_f(gp[d]) : 1.f));
   }
 }
 
@@ -288,7 +295,7 @@ __global__ void k_attn_prefill_simt(const Act* __restrict__ q, const Act* __rest
 
 cudaError_t attn_prefill_bf16_launch(const CUtensorMap& q_map, const CUtensorMap& k_map, const CUtensorMap& v_map,
                                      const AttnTile* tiles, int n_tiles, int T, int H, int KVH, int hd, void* out,
-                                     int* err, cudaStream_t stream) {
+                                     const void* gate, int* err, cudaStream_t stream) {
   if (n_tiles == 0) return cudaSuccess;
   if (hd == 128) {
     using C = PrefillCfg<128>;
@@ -301,7 +308,7 @@ cudaError_t attn_prefill_bf16_launch(const CUtensorMap& q_map, const CUtensorMap
     }
     dim3 grid(H, n_tiles);
     OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_bf16<128>, dim3(grid), dim3(128), C::SMEM, stream, q_map, k_map, v_map, tiles, T, H, KVH,
-                                                             reinterpret_cast<bf16*>(out), err));
+                                                             reinterpret_cast<bf16*>(out), reinterpret_cast<const bf16*>(gate), err));
     return cudaGetLastError();
   }
   if (hd == 64) {
@@ -315,7 +322,7 @@ cudaError_t attn_prefill_bf16_launch(const CUtensorMap& q_map, const CUtensorMap
     }
     dim3 grid(H, n_tiles);
     OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_bf16<64>, dim3(grid), dim3(128), C::SMEM, stream, q_map, k_map, v_map, tiles, T, H, KVH,
-                                                            reinterpret_cast<bf16*>(out), err));
+                                                            reinterpret_cast<bf16*>(out), reinterpret_cast<const bf16*>(gate), err));
     return cudaGetLastError();
   }
   return cudaErrorInvalidValue;
@@ -323,17 +330,18 @@ cudaError_t attn_prefill_bf16_launch(const CUtensorMap& q_map, const CUtensorMap
 
 template <typename Act>
 cudaError_t attn_prefill_simt_launch(const Act* q, const Act* k, const Act* v, const int* cu, int B, int n_rows,
-                                     int kv_ld, int H, int KVH, int hd, Act* out, cudaStream_t stream) {
+                                     int kv_ld, int H, int KVH, int hd, Act* out, const Act* gate,
+                                     cudaStream_t stream) {
   if (n_rows == 0) return cudaSuccess;
   if (hd > 256) return cudaErrorInvalidValue;
   dim3 grid(n_rows, (H + 3) / 4);
-  OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_simt<Act>, dim3(grid), dim3(128), 0, stream, q, k, v, cu, B, kv_ld, H, KVH, hd, out));
+  OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_simt<Act>, dim3(grid), dim3(128), 0, stream, q, k, v, cu, B, kv_ld, H, KVH, hd, out, gate));
   return cudaGetLastError();
 }
 
 template cudaError_t attn_prefill_simt_launch<float>(const float*, const float*, const float*, const int*, int,
-                                                     int, int, int, int, int, float*, cudaStream_t);
+                                                     int, int, int, int, int, float*, const float*, cudaStream_t);
 template cudaError_t attn_prefill_simt_launch<bf16>(const bf16*, const bf16*, const bf16*, const int*, int, int,
-                                                    int, int, int, int, bf16*, cudaStream_t);
+                                                    int, int, int, int, bf16*, const bf16*, cudaStream_t);
 
 }  // namespace outlets

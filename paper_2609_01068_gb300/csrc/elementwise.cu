@@ -225,7 +225,7 @@ __global__ void __launch_bounds__(RopeBlock<In>::kThreads, RopeBlock<In>::kMinBl
     pos = 0;
   }
   const int hd = a.hd, half = hd / 2, H = a.H, KVH = a.KVH;
-  const long long W = (long long)(H + 2 * KVH) * hd;
+  const long long W = a.qkv_ld;
   const In* src = qkv + (long long)row * W;
   const float* cs = a.cos_tab + (long long)pos * half;
   const float* sn = a.sin_tab + (long long)pos * half;
@@ -283,6 +283,19 @@ __global__ void __launch_bounds__(RopeBlock<In>::kThreads, RopeBlock<In>::kMinBl
     load8<In>(src, voff + e, a.n_split, a.split_stride, v);
     if (v_out) store8<Act>(v_out + ((long long)kh * a.kv_ld_rows + row) * hd + dd, v);
     if (v_pool) store8<Act>(v_pool + (cache_base + (long long)kh * a.page_tokens) * hd + dd, v);
+  }
+  if (a.gate_out) {
+    // gated attention (Sec. 4.1): the gate columns follow q, k, v in the qkv
+    // row; the attention kernels multiply their output by sigmoid(gate)
+    const long long goff = (long long)(H + 2 * KVH) * hd;
+    Act* go = reinterpret_cast<Act*>(a.gate_out) + (long long)row * H * hd;
+    for (int idx = threadIdx.x; idx < H * hd / 8; idx += blockDim.x) {
+      float g[8];
+      load8<In>(src, goff + idx * 8, a.n_split, a.split_stride, g);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) g[k] = 1.f / (1.f + __expf(-g[k]));
+      store8<Act>(go + idx * 8, g);
+    }
   }
 }
 

@@ -137,6 +137,8 @@ struct RopeArgs {
   int page_tokens;
   int n_split;           // qkv holds n_split slices (split-K partial sums) to add up
   long long split_stride;
+  int qkv_ld;            // elements per qkv row: (H + 2 KVH) hd, + H hd gate columns when gated
+  void* gate_out;        // gated attention: [T, H*hd] sigmoid of the gate columns, else null
   int* err;
 };
 template <typename In, typename Act>
@@ -171,16 +173,18 @@ struct AttnTile {
   int seq_len;    // rows of the sequence
 };
 
-// k/v head-major [KVH, kv_ld, hd]; q/out [n_rows, H, hd].
+// k/v head-major [KVH, kv_ld, hd]; q/out [n_rows, H, hd]; gate (or null) [n_rows, H*hd]
+// multiplies the output elementwise (gated attention).
 template <typename Act>
 cudaError_t attn_prefill_simt_launch(const Act* q, const Act* k, const Act* v, const int* cu, int B, int n_rows,
-                                     int kv_ld, int H, int KVH, int hd, Act* out, cudaStream_t stream);
+                                     int kv_ld, int H, int KVH, int hd, Act* out, const Act* gate,
+                                     cudaStream_t stream);
 
 // bf16 flash attention; q_map over [rows, H*hd] (box 64 x 64), k/v maps over
 // head-major [KVH * kv_ld, hd] (box 64 x 64); kv_ld passed as T.
 cudaError_t attn_prefill_bf16_launch(const CUtensorMap& q_map, const CUtensorMap& k_map, const CUtensorMap& v_map,
                                      const AttnTile* tiles, int n_tiles, int T, int H, int KVH, int hd, void* out,
-                                     int* err, cudaStream_t stream);
+                                     const void* gate, int* err, cudaStream_t stream);
 
 struct DecodeArgs {
   int B, H, KVH, hd;
@@ -201,6 +205,7 @@ struct DecodeArgs {
   float* part_ml;         // [n_work, H, 2] (max in log2 units, sum)
   int* combine_count;     // [B, KVH] split completion counters, zero between calls
   void* out;              // [B, H, hd]
+  const void* gate;       // [B, H*hd] elementwise output gate (gated attention) or null
   int* err;
 };
 cudaError_t attn_decode_bf16_launch(const CUtensorMap& k_map, const CUtensorMap& v_map, const DecodeArgs& a,

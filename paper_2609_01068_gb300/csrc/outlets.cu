@@ -118,6 +118,8 @@ struct outlets_ctx {
   bool bf16 = true;
   size_t esz = 2;
   int d = 0, H = 0, KVH = 0, hd = 0, F = 0, Fp = 0, qkv_n = 0, attn_w = 0, max_rows = 0;
+  bool gated = false;        // gated attention: QKV carries H*hd gate columns after q, k, v
+  void* gate_act = nullptr;  // [max_rows, H*hd] sigmoid(gate), act dtype
   std::vector<int> head_dims;  // d, hidden..., 1
   std::vector<void*> allocs;
   size_t dev_bytes = 0;
@@ -848,8 +850,9 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->hd = cfg->head_dim;
   c->F = cfg->ffn_dim;
   c->Fp = (int)cdiv(c->F, 128) * 128;
-  c->qkv_n = (c->H + 2 * c->KVH) * c->hd;
   c->attn_w = c->H * c->hd;
+  c->gated = w->w_attn_gate != nullptr;
+  c->qkv_n = (c->H + 2 * c->KVH) * c->hd + (c->gated ? c->attn_w : 0);
   c->max_rows = std::max(cfg->max_tokens, cfg->max_batch);
   c->head_dims.push_back(c->d);
   for (int i = 0; i < cfg->n_head_hidden; ++i) c->head_dims.push_back(cfg->head_hidden[i]);
@@ -898,6 +901,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->hn = c->alloc(R * d * es);
   c->qkv = c->alloc(R * c->qkv_n * es);
   c->q = c->alloc(R * c->attn_w * es);
+  if (c->gated) c->gate_act = c->alloc(R * c->attn_w * es);
   c->attn = c->alloc(R * c->attn_w * es);
   c->kh = c->alloc((size_t)c->KVH * cfg->max_tokens * c->hd * es);
   c->vh = c->alloc((size_t)c->KVH * cfg->max_tokens * c->hd * es);
@@ -941,6 +945,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   up(w->w_q, c->H * c->hd, d, c->w_qkv, d, 0, 0, c->np_qkv);
   up(w->w_k, c->KVH * c->hd, d, c->w_qkv, d, 0, c->H * c->hd, c->np_qkv);
   up(w->w_v, c->KVH * c->hd, d, c->w_qkv, d, 0, (c->H + c->KVH) * c->hd, c->np_qkv);
+  if (c->gated) up(w->w_attn_gate, c->attn_w, d, c->w_qkv, d, 0, (c->H + 2 * c->KVH) * c->hd, c->np_qkv);
   up(w->w_o, d, c->attn_w, c->w_o, c->attn_w, 0, 0, c->np_o);
   up(w->w_gate, c->F, d, c->w_gu, d, 1, 0, c->np_gu);
   up(w->w_up, c->F, d, c->w_gu, d, 2, 0, c->np_gu);
@@ -1266,6 +1271,8 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
       ra.page_off = m + off_po;
       ra.page_tokens = kPageTokens;
     }
+    ra.qkv_ld = c->qkv_n;
+    ra.gate_out = c->gated ? c->gate_act : nullptr;
     ra.err = c->err_dev;
     for (int k = 0; k < n_chunks; ++k) {
       const int r0 = k * chunk_rows, rows = std::min(T, r0 + chunk_rows) - r0;
@@ -1291,10 +1298,11 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
         !cached_map(c, &vm, c->vh, c->hd, kv_rows, c->hd, 64))
       return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for attention");
     OUT_CK(c, attn_prefill_bf16_launch(qm, km, vm, reinterpret_cast<const AttnTile*>(m + off_tiles), n_tiles,
-                                       c->cfg.max_tokens, c->H, c->KVH, c->hd, c->attn, c->err_dev, s));
+                                       c->cfg.max_tokens, c->H, c->KVH, c->hd, c->attn, c->gate_act, c->err_dev, s));
   } else {
     OUT_CK(c, attn_prefill_simt_launch<float>((const float*)c->q, (const float*)c->kh, (const float*)c->vh, cu_dev,
-                                              B, T, c->cfg.max_tokens, c->H, c->KVH, c->hd, (float*)c->attn, s));
+                                              B, T, c->cfg.max_tokens, c->H, c->KVH, c->hd, (float*)c->attn,
+                                              (const float*)c->gate_act, s));
   }
   c->stage_end(1);
   OUT_TRY(run_tail(c, T, out_rows, all_tokens ? nullptr : m + off_last, c->z, c->len, s));
@@ -1399,6 +1407,8 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
     ra.page_list = m + off_pl;
     ra.page_off = m + off_po;
     ra.page_tokens = kPageTokens;
+    ra.qkv_ld = c->qkv_n;
+    ra.gate_out = c->gated ? c->gate_act : nullptr;
     ra.err = c->err_dev;
     OUT_TRY(launch_rope(c, qsrc, ra, s));
   }
@@ -1427,6 +1437,7 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
     da.part_ml = kv->part_ml;
     da.combine_count = c->dec_count;
     da.out = c->attn;
+    da.gate = c->gate_act;  // null unless gated
     da.err = c->err_dev;
     if ((size_t)n_work > kv->part_items) return c->fail(OUTLETS_ECAPACITY, "split-KV partial buffer too small");
     if (c->bf16) {

@@ -37,7 +37,8 @@ _WNAMES = ["w_proj", "w_q", "w_k", "w_v", "w_o", "g_in", "g_post", "g_final", "w
 
 class Weights(ctypes.Structure):
     _fields_ = [(n, c_vp) for n in _WNAMES] + [("head_w", c_vp * (MAX_HEAD_HIDDEN + 1)),
-                                               ("head_b", c_vp * (MAX_HEAD_HIDDEN + 1))]
+                                               ("head_b", c_vp * (MAX_HEAD_HIDDEN + 1)),
+                                               ("w_attn_gate", c_vp)]
 
 
 class TensorInfo(ctypes.Structure):
@@ -144,6 +145,10 @@ class Predictor:
             keep[f"hw{i}"], keep[f"hb{i}"] = wa, ba
             w.head_w[i] = wa.ctypes.data
             w.head_b[i] = ba.ctypes.data
+        if weights.get("w_attn_gate") is not None:  # gated attention
+            ga = np.ascontiguousarray(weights["w_attn_gate"], dtype=np.float32)
+            keep["w_attn_gate"] = ga
+            w.w_attn_gate = ga.ctypes.data
         h = c_vp()
         st = self.lib.outlets_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h))
         if st != OK:

@@ -41,11 +41,13 @@ WORKLOAD_70B = ("static length prediction, Llama-3.3-70B-shaped EAGLE-3 draft la
 def model_setup(args):
     """Shape, prompt lengths, workload text and traffic key prefix of --model."""
     from paper_2609_01068_gb300 import synth
+    gate = ", gated attention" if getattr(args, "gated", False) else ""
+    gkey = "-gated" if getattr(args, "gated", False) else ""
     if args.model == "70b":
         lengths = synth.lengths_70b_prefill(0)
-        return synth.LLAMA70B, lengths[:args.prompts] if args.prompts else lengths, WORKLOAD_70B, "70b"
+        return synth.LLAMA70B, lengths[:args.prompts] if args.prompts else lengths, WORKLOAD_70B + gate, "70b" + gkey
     lengths = synth.lengths_8b_prefill(0)
-    return synth.LLAMA8B, lengths[:args.prompts] if args.prompts else lengths, WORKLOAD, "8b"
+    return synth.LLAMA8B, lengths[:args.prompts] if args.prompts else lengths, WORKLOAD + gate, "8b" + gkey
 
 
 def parse():
@@ -58,6 +60,8 @@ def parse():
                     help="static prediction (headline), dynamic prediction, both, or the serving sweep")
     ap.add_argument("--prompts", type=int, default=None,
                     help="first N prompts of the workload (profiling cases; default: all)")
+    ap.add_argument("--gated", action="store_true",
+                    help="gated attention (Sec. 4.1): sigmoid gate on the attention output, gate weights [H*hd, d]")
     ap.add_argument("--model", default="8b", choices=["8b", "70b"],
                     help="draft-layer shape; 70b (Llama-3.3-70B-shaped, 32 prompts) runs the static mode only")
     ap.add_argument("--step-requests", type=int, default=256, help="live requests of the dynamic-prediction run")
@@ -166,11 +170,11 @@ def weight_bytes(shape):
     return 2 * (3 * d * d + d * (H + 2 * KVH) * hd + H * hd * d + 3 * d * F + d * shape.head_widths[0])
 
 
-def prefill_flops(shape, lengths, n_out):
+def prefill_flops(shape, lengths, n_out, gated=False):
     """Algorithmic FLOPs of one static-prediction pass (dense GEMMs + causal attention + head)."""
     d, H, KVH, hd, F = shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
     T = int(np.sum(lengths))
-    per_tok = 2 * (3 * d * d + d * (H + 2 * KVH) * hd + H * hd * d + 3 * d * F)
+    per_tok = 2 * (3 * d * d + d * (H + 2 * KVH + (H if gated else 0)) * hd + H * hd * d + 3 * d * F)
     attn = 4 * H * hd * float(np.sum(lengths * (lengths + 1) / 2))
     widths = (d,) + tuple(shape.head_widths) + (1,)
     head = 2 * sum(widths[i] * widths[i + 1] for i in range(len(widths) - 1)) * n_out
@@ -237,7 +241,7 @@ def run_reference(args):
         return
     from paper_2609_01068_gb300 import synth
     shape, lengths, workload, _ = model_setup(args)
-    w = synth.make_weights(shape, 0)
+    w = synth.make_weights(shape, 0, gated=args.gated)
     cu = synth.cu_seqlens(lengths)
     taps = synth.make_taps(shape, int(cu[-1]), 0)
     budget = 400
@@ -278,7 +282,7 @@ def run_ours(args):
         raise SystemExit("--model 70b runs the static (prefill) mode only")
     shape, lengths, workload, tkey = model_setup(args)
     args.workload, args.traffic_key = workload, tkey
-    w = synth.make_weights(shape, 0)
+    w = synth.make_weights(shape, 0, gated=args.gated)
     cu = synth.cu_seqlens(lengths)
     T, Bq = int(cu[-1]), len(lengths)
     taps = synth.make_taps(shape, T, 0, rank)
@@ -361,7 +365,7 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     pred.profile(False)
     ms_step = ms / args.steps
     value = world * Bq * args.steps / (ms / 1e3)
-    flops = prefill_flops(shape, lengths, Bq)
+    flops = prefill_flops(shape, lengths, Bq, args.gated)
     gu_ms, gu_n = prof_live["gateup_swiglu_gemm"]
     gu_flops = 2.0 * T * (2 * shape.ffn) * shape.d
     gu_tflops = gu_flops / (gu_ms / gu_n / 1e3) / 1e12
@@ -485,20 +489,24 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     kv_bytes = keys_avg * KVH * hd * 2 * 2
     widths = (d,) + tuple(shape.head_widths) + (1,)
     w_bytes = 2 * (3 * d * d + d * shape.qkv_out + shape.n_heads * hd * d + 3 * d * F + widths[0] * widths[1])
+    if args.gated:
+        w_bytes += 2 * shape.n_heads * hd * d  # gate rows of the QKV weight
     step_bytes = kv_bytes + w_bytes + 3 * B * d * 2
     at_ms, at_n = prof_live["attention"]
     at_gbs = kv_bytes / (at_ms / at_n / 1e3) / 1e9
     ms_step = ms / args.steps
     kv.close()
     return {"workload": "dynamic prediction, %d live requests x 1 new token, cache lengths lognormal "
-                        "median 512 clipped 1-4096 (sum %d), Llama-3.1-8B-shaped draft layer" % (B, int(lens.sum())),
+                        "median 512 clipped 1-4096 (sum %d), Llama-3.1-8B-shaped draft layer%s"
+                        % (B, int(lens.sum()), ", gated attention" if args.gated else ""),
             "value": world * B * args.steps / (ms / 1e3), "unit": "predictions/s", "ms_per_step": ms_step,
             "hbm_frac_step": step_bytes / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"],
             "algorithmic_bytes_per_step": step_bytes,
             "roofline": {"bound": "hbm", "kernel": "decode attention (k_attn_decode_bf16 + combine)",
                          "achieved": at_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                          "frac": at_gbs / peaks["hbm_gbs"],
-                         "traffic": measured_traffic("decode_attention", f"8b-step-{B}r-L{int(lens.sum())}"),
+                         "traffic": measured_traffic("decode_attention", f"8b-step-{B}r-L{int(lens.sum())}"
+                                                     + ("-gated" if args.gated else "")),
                          "algorithmic_per_launch": f"{kv_bytes:.4g} B of K/V (cached + new)"},
             "stages": {k: v[0] / max(v[1], 1) for k, v in prof.items() if v[1]},
             "clocks": clocks, "gpu_launches": launches, "host_issue_ms_per_step": host_ms, "e2e": e2e}

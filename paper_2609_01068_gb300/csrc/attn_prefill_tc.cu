@@ -1,0 +1,443 @@
+// Causal GQA self-attention of the static-prediction pass (the draft decoder's
+// self-attention, Sec. 4.1) on the tcgen05 tensor cores:
+// o = softmax(q k^T / sqrt(hd) + causal mask) v per packed sequence, q-head h
+// reading kv-head floor(h * KVH / H), optionally gated (o * gate).
+//
+// Persistent kernel, one CTA per SM, 6 warps.  A work item is one 128-row
+// query tile of one sequence x one query head; items are taken longest first
+// (most key tiles) with a grid stride.
+//   warp 0      TMA producer: Q tile (two buffers), then K and V^T tiles of 128
+//               keys (two stages), continuously across items
+//   warp 1      TMEM owner and single-thread MMA issuer:
+//                 S_j = Q K_j^T     M=128 N=128 K=hd, into one of two TMEM S buffers
+//                 O  += P_j V_j     M=128 N=hd K=128, into the TMEM O accumulator
+//               S_{j+1} is issued before waiting for P_j, so the next scores
+//               are computed while the softmax of the current tile runs
+//   warps 2..5  softmax, one query row per thread (TMEM lane): row max of the
+//               masked, scaled scores, P = exp2(s - m) written as bf16 into a
+//               128-byte-swizzled shared tile (the A operand of the PV MMA),
+//               O and l rescaled in place only when a row max grows by more
+//               than 2^8 over the one in use (the result is exact either way);
+//               at the end of an item O / l (x gate) is stored as bf16
+// V is read through a transposed copy V^T [KVH*hd, columns] (keys contiguous)
+// so both MMAs take K-major operands; each sequence starts at a column that is
+// a multiple of 8 (TMA coordinates in 16-byte units).  Every wait is bounded.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace outlets {
+namespace {
+
+constexpr int kBQ = 128;                         // query rows per work item
+constexpr int kBK = 128;                         // keys per K/V tile
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kRescaleLog2 = 8.f;              // tolerated growth of a row max before O is rescaled
+
+// 2^x with the hardware approximation (ex2.approx.ftz: -inf -> 0); the result
+// is rounded to bf16 or divided out by the row sum, far coarser than its error.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+template <int HD>
+struct TcAttnCfg {
+  static constexpr int NB = HD / 64;                   // 64-wide blocks of a head
+  static constexpr uint32_t Q_BYTES = kBQ * HD * 2;    // [NB][128 rows][64]
+  static constexpr uint32_t K_BYTES = kBK * HD * 2;    // [NB][128 keys][64]
+  static constexpr uint32_t V_BYTES = HD * kBK * 2;    // V^T: [2][hd rows][64 keys]
+  static constexpr uint32_t P_BYTES = kBQ * kBK * 2;   // [2][128 rows][64 keys]
+  static constexpr size_t SMEM = 1024 + 2 * Q_BYTES + 2 * K_BYTES + 2 * V_BYTES + P_BYTES + 256;
+  static constexpr uint32_t O_COL = 2 * kBK;           // TMEM: S0 [0,128), S1 [128,256), O [256, 256+hd)
+  static_assert(SMEM <= 232448, "shared memory");
+};
+
+template <int HD>
+__global__ void __launch_bounds__(192, 1)
+    k_attn_prefill_tc(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap k_map,
+                      const __grid_constant__ CUtensorMap vt_map, const TcAttnItem* __restrict__ items,
+                      int n_items, int kv_ld, int H, int KVH, bf16* __restrict__ out, const bf16* __restrict__ gate,
+                      int* err) {
+  using C = TcAttnCfg<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;                    // two buffers
+  uint8_t* sK = sQ + 2 * C::Q_BYTES;     // two stages
+  uint8_t* sV = sK + 2 * C::K_BYTES;     // two stages
+  uint8_t* sP = sV + 2 * C::V_BYTES;
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(sP + C::P_BYTES);
+  uint64_t* q_empty = q_full + 2;
+  uint64_t* kv_full = q_empty + 2;
+  uint64_t* kv_empty = kv_full + 2;
+  uint64_t* s_full = kv_empty + 2;
+  uint64_t* p_full = s_full + 2;
+  uint64_t* pv_done = p_full + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pv_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&q_full[i], 1);
+      mbar_init(&q_empty[i], 1);
+      mbar_init(&kv_full[i], 1);
+      mbar_init(&kv_empty[i], 1);
+      mbar_init(&s_full[i], 1);
+    }
+    mbar_init(p_full, 4 * 32);
+    mbar_init(pv_done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&q_map);
+    tma_prefetch_map(&k_map);
+    tma_prefetch_map(&vt_map);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();  // q, k and V^T are written by the kernels before this one
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int g = 0;  // K/V tiles loaded by this CTA
+      int k = 0;  // items of this CTA
+      for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
+        const TcAttnItem w = items[it];
+        const int kvh = (w.head * KVH) / H;
+        const int qb = k & 1;
+        if (k >= 2 && !mbar_wait(&q_empty[qb], ((k - 2) >> 1) & 1, abort_flag, err)) break;
+        mbar_arrive_expect_tx(&q_full[qb], C::Q_BYTES);
+#pragma unroll
+        for (int b = 0; b < C::NB; ++b)
+          tma_load_2d(sQ + qb * C::Q_BYTES + b * (kBQ * 128), &q_map, &q_full[qb], w.head * HD + 64 * b, w.q_start);
+        bool ok = true;
+        for (int j = 0; j < w.n_kv; ++j, ++g) {
+          const int st = g & 1;
+          if (g >= 2 && !mbar_wait(&kv_empty[st], ((g - 2) >> 1) & 1, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&kv_full[st], C::K_BYTES + C::V_BYTES);
+#pragma unroll
+          for (int b = 0; b < C::NB; ++b)
+            tma_load_2d(sK + st * C::K_BYTES + b * (kBK * 128), &k_map, &kv_full[st], 64 * b,
+                        kvh * kv_ld + w.seq_start + kBK * j);
+#pragma unroll
+          for (int b = 0; b < 2; ++b)
+            tma_load_2d(sV + st * C::V_BYTES + b * (HD * 128), &vt_map, &kv_full[st], w.v_start + kBK * j + 64 * b,
+                        kvh * HD);
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t id_s = idesc_bf16_f32(kBQ, kBK);
+      constexpr uint32_t id_o = idesc_bf16_f32(kBQ, HD);
+      // issue cursor of S (runs one tile ahead of the PV cursor)
+      int s_it = blockIdx.x, s_k = 0, s_j = 0, s_g = 0;
+      int s_nkv = s_it < n_items ? items[s_it].n_kv : 0;
+      auto issue_s = [&]() -> bool {
+        if (s_it >= n_items) return true;
+        const int qb = s_k & 1;
+        if (s_j == 0 && !mbar_wait(&q_full[qb], (s_k >> 1) & 1, abort_flag, err)) return false;
+        const int st = s_g & 1;
+        if (!mbar_wait(&kv_full[st], (s_g >> 1) & 1, abort_flag, err)) return false;
+        tc_fence_after();
+        const uint32_t qa = smem_u32(sQ + qb * C::Q_BYTES);
+        const uint32_t ka = smem_u32(sK + st * C::K_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * (128 * 128);
+          tc_mma_bf16(tmem_base + st * kBK, sw128_kmajor_desc(qa + off) + 2u * (kk & 3),
+                      sw128_kmajor_desc(ka + off) + 2u * (kk & 3), id_s, kk > 0 ? 1u : 0u);
+        }
+        tc_commit(&s_full[st]);
+        if (s_j == s_nkv - 1) tc_commit(&q_empty[qb]);  // last S of the item: its Q buffer is free
+        ++s_g;
+        if (++s_j == s_nkv) {
+          s_j = 0;
+          ++s_k;
+          s_it += gridDim.x;
+          s_nkv = s_it < n_items ? items[s_it].n_kv : 0;
+        }
+        return true;
+      };
+      bool ok = issue_s();
+      int p_g = 0;
+      for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
+        const int nkv = items[it].n_kv;
+        for (int j = 0; j < nkv; ++j, ++p_g) {
+          if (!issue_s()) {
+            ok = false;
+            break;
+          }
+          if (!mbar_wait(p_full, p_g & 1, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const int st = p_g & 1;
+          const uint32_t pa = smem_u32(sP);
+          const uint32_t va = smem_u32(sV + st * C::V_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk)
+            tc_mma_bf16(tmem_base + C::O_COL, sw128_kmajor_desc(pa + (kk >> 2) * (kBQ * 128)) + 2u * (kk & 3),
+                        sw128_kmajor_desc(va + (kk >> 2) * (HD * 128)) + 2u * (kk & 3), id_o,
+                        (j > 0 || kk > 0) ? 1u : 0u);
+          tc_commit(pv_done);
+          tc_commit(&kv_empty[st]);  // S_j and PV_j have read this stage's K and V
+        }
+      }
+    }
+  } else {
+    // softmax warps: thread = query row = TMEM lane
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    const float sl2 = rsqrtf((float)HD) * kLog2e;
+    uint8_t* prow = sP + r * 128;
+    int g = 0;
+    bool ok = true;
+    for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
+      const TcAttnItem w = items[it];
+      const int qp = (w.q_start - w.seq_start) + r;  // position of this row in its sequence
+      float m_used = -INFINITY, l = 0.f;
+      for (int j = 0; j < w.n_kv; ++j, ++g) {
+        const int sb = g & 1;
+        if (!mbar_wait(&s_full[sb], (g >> 1) & 1, abort_flag, err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t s_addr = tmem_base + lane_off + static_cast<uint32_t>(sb * kBK);
+        const bool diag = j == w.n_kv - 1;
+        const int key0 = kBK * j;
+        // the row's 128 scores into registers: four loads, one wait
+        uint32_t v[kBK];
+#pragma unroll
+        for (int c = 0; c < kBK / 32; ++c) tmem_ld_32x32b_x32(s_addr + 32 * c, v + 32 * c);
+        tmem_ld_wait();
+        float mx = -INFINITY;
+#pragma unroll
+        for (int e = 0; e < kBK; ++e) {
+          float x = __uint_as_float(v[e]) * sl2;
+          if (diag && key0 + e > qp) x = -INFINITY;  // causal mask (diagonal tile only)
+          v[e] = __float_as_uint(x);
+          mx = fmaxf(mx, x);
+        }
+        float alpha = 1.f;
+        bool resc = false;
+        if (mx > m_used + kRescaleLog2) {
+          alpha = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - mx);
+          l *= alpha;
+          m_used = mx;
+          resc = j > 0;
+        }
+        // O and the P tile are free once the previous PV of this item is done
+        if (j > 0 && !mbar_wait(pv_done, (g - 1) & 1, abort_flag, err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, resc)) {
+          // rare: 32 columns at a time (the score row is still live in registers)
+          const float a = resc ? alpha : 1.f;
+#pragma unroll 1
+          for (int c = 0; c < HD / 32; ++c) {
+            uint32_t o[32];
+            const uint32_t o_addr = tmem_base + lane_off + C::O_COL + 32 * c;
+            tmem_ld_32x32b_x32(o_addr, o);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * a);
+            tmem_st_32x32b_x32(o_addr, o);
+          }
+          tmem_st_wait();
+        }
+        // P = exp2(s - m) as bf16 into the swizzled A tile, and the row sum of
+        // the bf16 values the PV product uses (O / l stays a convex combination)
+        float ps = 0.f;
+#pragma unroll
+        for (int c = 0; c < kBK / 32; ++c) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 32; e += 2) {
+            const float p0 = ex2_approx(__uint_as_float(v[32 * c + e]) - m_used);
+            const float p1 = ex2_approx(__uint_as_float(v[32 * c + e + 1]) - m_used);
+            pk[e >> 1] = pack_bf16x2(p0, p1);
+            const float2 pr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&pk[e >> 1]));
+            ps += pr.x + pr.y;
+          }
+          // keys 32c .. 32c+31: block c/2, 16-byte chunks 4(c%2) .. 4(c%2)+3 of the row
+          uint8_t* blk = prow + (c >> 1) * (kBQ * 128);
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const int chunk = ((c & 1) * 4 + t) ^ (r & 7);
+            *reinterpret_cast<uint4*>(blk + chunk * 16) = make_uint4(pk[4 * t], pk[4 * t + 1], pk[4 * t + 2], pk[4 * t + 3]);
+          }
+        }
+        l += ps;
+        fence_proxy_async_smem();  // the P tile is read by the tensor cores (async proxy)
+        tc_fence_before();
+        mbar_arrive(p_full);
+      }
+      if (!ok) break;
+      // end of the item: O / l (x gate) as bf16
+      if (!mbar_wait(pv_done, (g - 1) & 1, abort_flag, err)) break;
+      tc_fence_after();
+      const float inv = 1.f / l;
+      const bool row_ok = r < w.q_len;
+      bf16* orow = out + (long long)(w.q_start + r) * H * HD + w.head * HD;
+      const bf16* grow = gate ? gate + (long long)(w.q_start + r) * H * HD + w.head * HD : nullptr;
+      uint32_t ov[HD];
+#pragma unroll
+      for (int c = 0; c < HD / 32; ++c) tmem_ld_32x32b_x32(tmem_base + lane_off + C::O_COL + 32 * c, ov + 32 * c);
+      tmem_ld_wait();
+#pragma unroll
+      for (int c = 0; c < HD / 32; ++c) {
+        const uint32_t* v = ov + 32 * c;
+        if (row_ok) {
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            float f[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) f[e] = __uint_as_float(v[8 * t + e]) * inv;
+            if (grow) {
+              const uint4 gq = *reinterpret_cast<const uint4*>(grow + 32 * c + 8 * t);
+              const __nv_bfloat162* gh = reinterpret_cast<const __nv_bfloat162*>(&gq);
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float2 gf = __bfloat1622float2(gh[e]);
+                f[2 * e] *= gf.x;
+                f[2 * e + 1] *= gf.y;
+              }
+            }
+            *reinterpret_cast<uint4*>(orow + 32 * c + 8 * t) =
+                make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]), pack_bf16x2(f[4], f[5]),
+                           pack_bf16x2(f[6], f[7]));
+          }
+        }
+      }
+      tc_fence_before();
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem_base, 512);
+  }
+}
+
+// V^T [KVH * hd, vt_ld] from head-major V [KVH, kv_ld, hd]: token t of sequence
+// b goes to column v_start[b] + (t - cu[b]).  One CTA = 64 tokens of one kv head,
+// staged in shared memory so that both the reads and the writes are coalesced.
+template <int HD>
+__global__ void __launch_bounds__(256) k_v_transpose(const bf16* __restrict__ vh, const int* __restrict__ cu,
+                                                     const int* __restrict__ v_start, int B, int T, int kv_ld,
+                                                     bf16* __restrict__ vt, long long vt_ld) {
+  pdl_trigger();
+  pdl_wait();
+  constexpr int LDW = HD / 2 + 1;  // words per staged token (odd: conflict-free column reads)
+  __shared__ uint32_t tile[64 * LDW];
+  __shared__ int col[64];
+  const int t0 = blockIdx.x * 64;
+  const int g = blockIdx.y;
+  if (threadIdx.x < 64) {
+    const int t = t0 + threadIdx.x;
+    int c = -1;
+    if (t < T) {
+      int lo = 0, hi = B;
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (cu[mid] <= t) lo = mid;
+        else hi = mid;
+      }
+      c = v_start[lo] + (t - cu[lo]);
+    }
+    col[threadIdx.x] = c;
+  }
+  for (int idx = threadIdx.x; idx < 64 * (HD / 8); idx += blockDim.x) {
+    const int tok = idx / (HD / 8);
+    const int c8 = idx - tok * (HD / 8);
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (t0 + tok < T) v = *reinterpret_cast<const uint4*>(vh + ((long long)g * kv_ld + t0 + tok) * HD + c8 * 8);
+    uint32_t* dst = tile + tok * LDW + c8 * 4;
+    dst[0] = v.x;
+    dst[1] = v.y;
+    dst[2] = v.z;
+    dst[3] = v.w;
+  }
+  __syncthreads();
+  const uint16_t* t16 = reinterpret_cast<const uint16_t*>(tile);
+  for (int idx = threadIdx.x; idx < HD * 64; idx += blockDim.x) {
+    const int d = idx >> 6;
+    const int tok = idx & 63;
+    const int c = col[tok];
+    if (c >= 0) {
+      const uint16_t bits = t16[tok * (2 * LDW) + d];
+      reinterpret_cast<uint16_t*>(vt)[((long long)g * HD + d) * vt_ld + c] = bits;
+    }
+  }
+}
+
+template <int HD>
+cudaError_t launch_tc(const CUtensorMap& q_map, const CUtensorMap& k_map, const CUtensorMap& vt_map,
+                      const TcAttnItem* items, int n_items, int kv_ld, int H, int KVH, void* out, const void* gate,
+                      int* err, int num_sms, cudaStream_t stream) {
+  using C = TcAttnCfg<HD>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_attn_prefill_tc<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const int grid = n_items < num_sms ? n_items : num_sms;
+  OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_tc<HD>, dim3(grid), dim3(192), C::SMEM, stream, q_map, k_map, vt_map,
+                              items, n_items, kv_ld, H, KVH, reinterpret_cast<bf16*>(out),
+                              reinterpret_cast<const bf16*>(gate), err));
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t v_transpose_launch(const void* vh, const int* cu, const int* v_start, int B, int T, int kv_ld, int KVH,
+                               int hd, void* vt, long long vt_ld, cudaStream_t stream) {
+  if (T == 0) return cudaSuccess;
+  const dim3 grid((T + 63) / 64, KVH);
+  if (hd == 128) {
+    OUTLETS_TRY_LAUNCH(launch_k(k_v_transpose<128>, grid, dim3(256), 0, stream, reinterpret_cast<const bf16*>(vh), cu,
+                                v_start, B, T, kv_ld, reinterpret_cast<bf16*>(vt), vt_ld));
+  } else if (hd == 64) {
+    OUTLETS_TRY_LAUNCH(launch_k(k_v_transpose<64>, grid, dim3(256), 0, stream, reinterpret_cast<const bf16*>(vh), cu,
+                                v_start, B, T, kv_ld, reinterpret_cast<bf16*>(vt), vt_ld));
+  } else {
+    return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t attn_prefill_tc_launch(const CUtensorMap& q_map, const CUtensorMap& k_map, const CUtensorMap& vt_map,
+                                   const TcAttnItem* items, int n_items, int kv_ld, int H, int KVH, int hd, void* out,
+                                   const void* gate, int* err, int num_sms, cudaStream_t stream) {
+  if (n_items == 0) return cudaSuccess;
+  if (hd == 128) return launch_tc<128>(q_map, k_map, vt_map, items, n_items, kv_ld, H, KVH, out, gate, err, num_sms, stream);
+  if (hd == 64) return launch_tc<64>(q_map, k_map, vt_map, items, n_items, kv_ld, H, KVH, out, gate, err, num_sms, stream);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace outlets

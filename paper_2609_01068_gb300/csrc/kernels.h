@@ -166,13 +166,6 @@ cudaError_t convert_rows_launch(const float* src, Act* dst, int rows, int cols, 
 cudaError_t wait_selftest_launch(int* err, unsigned long long timeout_ns, cudaStream_t stream);
 
 // ---------------------------------------------------------------- attention
-struct AttnTile {
-  int q_start;    // first query row (packed index)
-  int q_len;      // rows in this tile (<= 64)
-  int seq_start;  // first row of the sequence
-  int seq_len;    // rows of the sequence
-};
-
 // k/v head-major [KVH, kv_ld, hd]; q/out [n_rows, H, hd]; gate (or null) [n_rows, H*hd]
 // multiplies the output elementwise (gated attention).
 template <typename Act>
@@ -180,11 +173,24 @@ cudaError_t attn_prefill_simt_launch(const Act* q, const Act* k, const Act* v, c
                                      int kv_ld, int H, int KVH, int hd, Act* out, const Act* gate,
                                      cudaStream_t stream);
 
-// bf16 flash attention; q_map over [rows, H*hd] (box 64 x 64), k/v maps over
-// head-major [KVH * kv_ld, hd] (box 64 x 64); kv_ld passed as T.
-cudaError_t attn_prefill_bf16_launch(const CUtensorMap& q_map, const CUtensorMap& k_map, const CUtensorMap& v_map,
-                                     const AttnTile* tiles, int n_tiles, int T, int H, int KVH, int hd, void* out,
-                                     const void* gate, int* err, cudaStream_t stream);
+// tcgen05 flash attention of the static pass.  A work item: one 128-row query
+// tile (rows q_start .. q_start + q_len - 1 of the pack, q_len <= 128) of the
+// sequence [seq_start, seq_start + seq_len) for one query head; n_kv = number
+// of 128-key tiles it attends to (the last one is the diagonal tile);
+// v_start = the sequence's first column in V^T (a multiple of 8).
+struct TcAttnItem {
+  int q_start, q_len, seq_start, seq_len, v_start, head, n_kv, pad;
+};
+// q_map over q [rows, H*hd] (box 64 x 128), k_map over head-major K
+// [KVH * kv_ld, hd] (box 64 x 128), vt_map over V^T [KVH * hd, vt_ld] (box
+// 64 x hd).  Persistent: min(n_items, num_sms) CTAs.  hd in {64, 128}.
+cudaError_t attn_prefill_tc_launch(const CUtensorMap& q_map, const CUtensorMap& k_map, const CUtensorMap& vt_map,
+                                   const TcAttnItem* items, int n_items, int kv_ld, int H, int KVH, int hd, void* out,
+                                   const void* gate, int* err, int num_sms, cudaStream_t stream);
+// V^T [KVH * hd, vt_ld] from head-major V [KVH, kv_ld, hd]; token t of sequence b
+// (cu[b] <= t < cu[b+1]) goes to column v_start[b] + t - cu[b].
+cudaError_t v_transpose_launch(const void* vh, const int* cu, const int* v_start, int B, int T, int kv_ld, int KVH,
+                               int hd, void* vt, long long vt_ld, cudaStream_t stream);
 
 struct DecodeArgs {
   int B, H, KVH, hd;

@@ -119,6 +119,8 @@ struct outlets_ctx {
   size_t esz = 2;
   int d = 0, H = 0, KVH = 0, hd = 0, F = 0, Fp = 0, qkv_n = 0, attn_w = 0, max_rows = 0;
   bool gated = false;        // gated attention: QKV carries H*hd gate columns after q, k, v
+  void* vt = nullptr;        // V^T [KVH * hd, vt_ld] for the tcgen05 prefill attention (bf16)
+  long long vt_ld = 0;
   void* gate_act = nullptr;  // [max_rows, H*hd] sigmoid(gate), act dtype
   std::vector<int> head_dims;  // d, hidden..., 1
   std::vector<void*> allocs;
@@ -905,6 +907,10 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->attn = c->alloc(R * c->attn_w * es);
   c->kh = c->alloc((size_t)c->KVH * cfg->max_tokens * c->hd * es);
   c->vh = c->alloc((size_t)c->KVH * cfg->max_tokens * c->hd * es);
+  if (c->bf16) {  // every sequence starts at a column that is a multiple of 8
+    c->vt_ld = (long long)cdiv((long long)cfg->max_tokens + 8LL * cfg->max_batch, 64) * 64;
+    c->vt = c->alloc((size_t)c->KVH * c->hd * c->vt_ld * es);
+  }
   c->u = c->alloc(R * c->Fp * es);
   if (!c->bf16) c->gu32 = (float*)c->alloc(R * 2 * c->Fp * 4);
   int hmax = 1;
@@ -921,10 +927,27 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
     c->part = (float*)c->alloc(c->part_floats * 4);
   }
   if (c->oom) return cleanup_fail(OUTLETS_ENOMEM);
-  for (auto& p : c->ring)
+  // metadata slots sized for the largest call up front (growing one later
+  // allocates and synchronizes): prefill attention items (8 ints per 128-row
+  // tile and head), per-sequence arrays, page lists
+  const size_t meta_ints = (size_t)8 * c->H * (cdiv(cfg->max_tokens, 128) + cfg->max_batch) +
+                           (size_t)8 * (cfg->max_batch + 1) + (size_t)2 * (cdiv(cfg->max_tokens, 64) + cfg->max_batch) +
+                           (1u << 16);
+  for (auto& p : c->ring) {
     if (cudaEventCreateWithFlags(&p.ev, cudaEventDisableTiming) != cudaSuccess ||
         cudaEventCreateWithFlags(&p.done, cudaEventDisableTiming) != cudaSuccess)
       return cleanup_fail(OUTLETS_ECUDA);
+    if (cudaMallocHost(&p.h, meta_ints * sizeof(int)) != cudaSuccess) {
+      cudaGetLastError();
+      return cleanup_fail(OUTLETS_ENOMEM);
+    }
+    p.cap = meta_ints;
+    if (cudaMalloc(&p.dev, meta_ints * sizeof(int)) != cudaSuccess) {
+      cudaGetLastError();
+      return cleanup_fail(OUTLETS_ENOMEM);
+    }
+    p.dev_cap = meta_ints;
+  }
   if (cudaEventCreateWithFlags(&c->done_ev, cudaEventDisableTiming) != cudaSuccess) return cleanup_fail(OUTLETS_ECUDA);
 
   // ---- upload
@@ -1196,27 +1219,43 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
   std::vector<int> last(B);
   for (int b = 0; b < B; ++b) last[b] = cu[b + 1] - 1;
   const size_t off_last = mb.put(last);
-  size_t off_tiles = 0;
-  int n_tiles = 0;
+  size_t off_items = 0, off_vstart = 0;
+  int n_items = 0;
   if (c->bf16) {
-    std::vector<int> tiles;
-    std::vector<std::pair<int, int>> order;  // (key tiles, tile id): longest first
+    // tcgen05 attention work items: 128-row query tiles x query heads, the
+    // ones with the most key tiles first; V^T columns of each sequence start
+    // at a multiple of 8
+    std::vector<int> vstart(B);
+    long long col = 0;
+    for (int b = 0; b < B; ++b) {
+      vstart[b] = (int)col;
+      col += cdiv(cu[b + 1] - cu[b], 8) * 8;
+    }
+    if (col > c->vt_ld) return c->fail(OUTLETS_ECAPACITY, "V^T workspace too small");
+    off_vstart = mb.put(vstart);
+    std::vector<std::pair<int, int>> tiles;  // (n_kv, tile id)
+    std::vector<int> tq;                    // per tile: b, tile index
     for (int b = 0; b < B; ++b) {
       const int L = cu[b + 1] - cu[b];
-      for (int i = 0; i * 64 < L; ++i) {
-        order.push_back({i + 1, (int)(tiles.size() / 4)});
-        tiles.push_back(cu[b] + 64 * i);
-        tiles.push_back(std::min(64, L - 64 * i));
-        tiles.push_back(cu[b]);
-        tiles.push_back(L);
+      for (int i = 0; i * 128 < L; ++i) {
+        tiles.push_back({i + 1, (int)(tq.size() / 2)});
+        tq.push_back(b);
+        tq.push_back(i);
       }
     }
-    std::stable_sort(order.begin(), order.end(), [](const auto& x, const auto& y) { return x.first > y.first; });
-    std::vector<int> sorted;
-    sorted.reserve(tiles.size());
-    for (auto& o : order) sorted.insert(sorted.end(), tiles.begin() + 4 * o.second, tiles.begin() + 4 * o.second + 4);
-    n_tiles = (int)order.size();
-    off_tiles = mb.put(sorted);
+    std::stable_sort(tiles.begin(), tiles.end(), [](const auto& x, const auto& y) { return x.first > y.first; });
+    std::vector<int> items;
+    items.reserve(tiles.size() * c->H * 8);
+    for (auto& t : tiles) {
+      const int b = tq[2 * t.second], i = tq[2 * t.second + 1];
+      const int L = cu[b + 1] - cu[b];
+      for (int h = 0; h < c->H; ++h) {
+        const int v[8] = {cu[b] + 128 * i, std::min(128, L - 128 * i), cu[b], L, vstart[b], h, i + 1, 0};
+        items.insert(items.end(), v, v + 8);
+      }
+    }
+    n_items = (int)(items.size() / 8);
+    off_items = mb.put(items);
   }
   size_t off_pl = 0, off_po = 0;
   if (kv) {
@@ -1292,13 +1331,19 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
   // ---- attention
   c->stage_begin(OUTLETS_S_ATTN);
   if (c->bf16) {
+    // V^T for the tcgen05 attention (keys contiguous), then the attention
+    OUT_CK(c, v_transpose_launch(c->vh, cu_dev, m + off_vstart, B, T, c->cfg.max_tokens, c->KVH, c->hd, c->vt,
+                                 c->vt_ld, s));
     CUtensorMap qm, km, vm;
     const uint64_t kv_rows = (uint64_t)c->KVH * c->cfg.max_tokens;
-    if (!cached_map(c, &qm, c->q, c->attn_w, T, c->attn_w, 64) || !cached_map(c, &km, c->kh, c->hd, kv_rows, c->hd, 64) ||
-        !cached_map(c, &vm, c->vh, c->hd, kv_rows, c->hd, 64))
+    if (!cached_map(c, &qm, c->q, c->attn_w, T, c->attn_w, 128) ||
+        !cached_map(c, &km, c->kh, c->hd, kv_rows, c->hd, 128) ||
+        !cached_map(c, &vm, c->vt, c->vt_ld, (uint64_t)c->KVH * c->hd, c->vt_ld, c->hd))
       return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for attention");
-    OUT_CK(c, attn_prefill_bf16_launch(qm, km, vm, reinterpret_cast<const AttnTile*>(m + off_tiles), n_tiles,
-                                       c->cfg.max_tokens, c->H, c->KVH, c->hd, c->attn, c->gate_act, c->err_dev, s));
+    OUT_CK(c, attn_prefill_tc_launch(qm, km, vm, reinterpret_cast<const TcAttnItem*>(m + off_items), n_items,
+                                     c->cfg.max_tokens, c->H, c->KVH, c->hd, c->attn, c->gate_act, c->err_dev,
+                                     c->num_sms, s));
+    c->launches += 1;  // the transpose
   } else {
     OUT_CK(c, attn_prefill_simt_launch<float>((const float*)c->q, (const float*)c->kh, (const float*)c->vh, cu_dev,
                                               B, T, c->cfg.max_tokens, c->H, c->KVH, c->hd, (float*)c->attn,

@@ -244,6 +244,20 @@ __global__ void __launch_bounds__(192, 1)
           m_used = mx;
           resc = j > 0;
         }
+        // P = exp2(s - m) as bf16 pairs in registers, while the previous PV
+        // product (which still reads the shared P tile) runs; the row sum
+        // takes the bf16 values the PV product uses (O / l stays a convex
+        // combination of the value rows)
+        uint32_t pk[kBK / 2];
+        float ps = 0.f;
+#pragma unroll
+        for (int e = 0; e < kBK; e += 2) {
+          const float p0 = ex2_approx(__uint_as_float(v[e]) - m_used);
+          const float p1 = ex2_approx(__uint_as_float(v[e + 1]) - m_used);
+          pk[e >> 1] = pack_bf16x2(p0, p1);
+          const float2 pr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&pk[e >> 1]));
+          ps += pr.x + pr.y;
+        }
         // O and the P tile are free once the previous PV of this item is done
         if (j > 0 && !mbar_wait(pv_done, (g - 1) & 1, abort_flag, err)) {
           ok = false;
@@ -251,7 +265,7 @@ __global__ void __launch_bounds__(192, 1)
         }
         tc_fence_after();
         if (__any_sync(0xffffffffu, resc)) {
-          // rare: 32 columns at a time (the score row is still live in registers)
+          // rare: 32 columns at a time
           const float a = resc ? alpha : 1.f;
 #pragma unroll 1
           for (int c = 0; c < HD / 32; ++c) {
@@ -265,26 +279,15 @@ __global__ void __launch_bounds__(192, 1)
           }
           tmem_st_wait();
         }
-        // P = exp2(s - m) as bf16 into the swizzled A tile, and the row sum of
-        // the bf16 values the PV product uses (O / l stays a convex combination)
-        float ps = 0.f;
+        // keys 32c .. 32c+31 of the row: block c/2, 16-byte chunks 4(c%2) .. 4(c%2)+3
 #pragma unroll
         for (int c = 0; c < kBK / 32; ++c) {
-          uint32_t pk[16];
-#pragma unroll
-          for (int e = 0; e < 32; e += 2) {
-            const float p0 = ex2_approx(__uint_as_float(v[32 * c + e]) - m_used);
-            const float p1 = ex2_approx(__uint_as_float(v[32 * c + e + 1]) - m_used);
-            pk[e >> 1] = pack_bf16x2(p0, p1);
-            const float2 pr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&pk[e >> 1]));
-            ps += pr.x + pr.y;
-          }
-          // keys 32c .. 32c+31: block c/2, 16-byte chunks 4(c%2) .. 4(c%2)+3 of the row
           uint8_t* blk = prow + (c >> 1) * (kBQ * 128);
 #pragma unroll
           for (int t = 0; t < 4; ++t) {
             const int chunk = ((c & 1) * 4 + t) ^ (r & 7);
-            *reinterpret_cast<uint4*>(blk + chunk * 16) = make_uint4(pk[4 * t], pk[4 * t + 1], pk[4 * t + 2], pk[4 * t + 3]);
+            const uint32_t* q4 = pk + 16 * c + 4 * t;
+            *reinterpret_cast<uint4*>(blk + chunk * 16) = make_uint4(q4[0], q4[1], q4[2], q4[3]);
           }
         }
         l += ps;

@@ -6,16 +6,20 @@
 // Persistent kernel, one CTA per SM, 6 warps.  A work item is one 128-row
 // query tile of one sequence x one query head; items are taken longest first
 // (most key tiles) with a grid stride.
-//   warp 0      TMA producer: Q tile (two buffers), then K and V^T tiles of 128
-//               keys (two stages), continuously across items
+//   warp 0      TMA producer: Q tile (one or two buffers), then K and V^T
+//               tiles of 128 keys (three or more stages), continuously across
+//               items
 //   warp 1      TMEM owner and single-thread MMA issuer:
 //                 S_j = Q K_j^T     M=128 N=128 K=hd, into one of two TMEM S buffers
 //                 O  += P_j V_j     M=128 N=hd K=128, into the TMEM O accumulator
 //               S_{j+1} is issued before waiting for P_j, so the next scores
 //               are computed while the softmax of the current tile runs
-//   warps 2..5  softmax, one query row per thread (TMEM lane): row max of the
-//               masked, scaled scores, P = exp2(s - m) written as bf16 into a
-//               128-byte-swizzled shared tile (the A operand of the PV MMA),
+//   warps 2..5  softmax, one query row per thread (TMEM lane): the score row
+//               is read from TMEM once into registers; row max of the masked,
+//               scaled scores; P = exp2(s - m) written as bf16 pairs back
+//               into the S buffer it came from (the PV MMA reads its A
+//               operand from TMEM, so P is double-buffered with S and PV_j
+//               overlaps the softmax of the next tile),
 //               O and l rescaled in place only when a row max grows by more
 //               than 2^8 over the one in use (the result is exact either way);
 //               at the end of an item O / l (x gate) is stored as bf16
@@ -47,8 +51,13 @@ struct TcAttnCfg {
   static constexpr uint32_t Q_BYTES = kBQ * HD * 2;    // [NB][128 rows][64]
   static constexpr uint32_t K_BYTES = kBK * HD * 2;    // [NB][128 keys][64]
   static constexpr uint32_t V_BYTES = HD * kBK * 2;    // V^T: [2][hd rows][64 keys]
-  static constexpr uint32_t P_BYTES = kBQ * kBK * 2;   // [2][128 rows][64 keys]
-  static constexpr size_t SMEM = 1024 + 2 * Q_BYTES + 2 * K_BYTES + 2 * V_BYTES + P_BYTES + 256;
+  // Q buffers and K/V stages share the 227 KB: K/V latency wants stages, and a
+  // second Q buffer only hides the Q load between items
+  static constexpr int NQ = HD >= 128 ? 1 : 2;
+  static constexpr int NS_FIT = (int)((232448u - 1024u - 512u - NQ * Q_BYTES) / (K_BYTES + V_BYTES));
+  static constexpr int NS = NS_FIT > 6 ? 6 : NS_FIT;
+  static constexpr size_t SMEM = 1024 + NQ * Q_BYTES + NS * (K_BYTES + V_BYTES) + 512;
+  static_assert(NS >= 3, "K/V stages");
   static constexpr uint32_t O_COL = 2 * kBK;           // TMEM: S0 [0,128), S1 [128,256), O [256, 256+hd)
   static_assert(SMEM <= 232448, "shared memory");
 };
@@ -62,15 +71,15 @@ __global__ void __launch_bounds__(192, 1)
   using C = TcAttnCfg<HD>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = smem;                    // two buffers
-  uint8_t* sK = sQ + 2 * C::Q_BYTES;     // two stages
-  uint8_t* sV = sK + 2 * C::K_BYTES;     // two stages
-  uint8_t* sP = sV + 2 * C::V_BYTES;
-  uint64_t* q_full = reinterpret_cast<uint64_t*>(sP + C::P_BYTES);
-  uint64_t* q_empty = q_full + 2;
-  uint64_t* kv_full = q_empty + 2;
-  uint64_t* kv_empty = kv_full + 2;
-  uint64_t* s_full = kv_empty + 2;
+  constexpr int NQ = C::NQ, NS = C::NS;
+  uint8_t* sQ = smem;                     // NQ buffers
+  uint8_t* sK = sQ + NQ * C::Q_BYTES;     // NS stages
+  uint8_t* sV = sK + NS * C::K_BYTES;     // NS stages
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(sV + NS * C::V_BYTES);
+  uint64_t* q_empty = q_full + NQ;
+  uint64_t* kv_full = q_empty + NQ;
+  uint64_t* kv_empty = kv_full + NS;
+  uint64_t* s_full = kv_empty + NS;
   uint64_t* p_full = s_full + 2;
   uint64_t* pv_done = p_full + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pv_done + 1);
@@ -79,13 +88,15 @@ __global__ void __launch_bounds__(192, 1)
   const int lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < NQ; ++i) {
       mbar_init(&q_full[i], 1);
       mbar_init(&q_empty[i], 1);
+    }
+    for (int i = 0; i < NS; ++i) {
       mbar_init(&kv_full[i], 1);
       mbar_init(&kv_empty[i], 1);
-      mbar_init(&s_full[i], 1);
     }
+    for (int i = 0; i < 2; ++i) mbar_init(&s_full[i], 1);
     mbar_init(p_full, 4 * 32);
     mbar_init(pv_done, 1);
     *abort_flag = 0;
@@ -114,16 +125,16 @@ __global__ void __launch_bounds__(192, 1)
       for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
         const TcAttnItem w = items[it];
         const int kvh = (w.head * KVH) / H;
-        const int qb = k & 1;
-        if (k >= 2 && !mbar_wait(&q_empty[qb], ((k - 2) >> 1) & 1, abort_flag, err)) break;
+        const int qb = k % NQ;
+        if (k >= NQ && !mbar_wait(&q_empty[qb], ((k - NQ) / NQ) & 1, abort_flag, err)) break;
         mbar_arrive_expect_tx(&q_full[qb], C::Q_BYTES);
 #pragma unroll
         for (int b = 0; b < C::NB; ++b)
           tma_load_2d(sQ + qb * C::Q_BYTES + b * (kBQ * 128), &q_map, &q_full[qb], w.head * HD + 64 * b, w.q_start);
         bool ok = true;
         for (int j = 0; j < w.n_kv; ++j, ++g) {
-          const int st = g & 1;
-          if (g >= 2 && !mbar_wait(&kv_empty[st], ((g - 2) >> 1) & 1, abort_flag, err)) {
+          const int st = g % NS;
+          if (g >= NS && !mbar_wait(&kv_empty[st], ((g - NS) / NS) & 1, abort_flag, err)) {
             ok = false;
             break;
           }
@@ -149,20 +160,21 @@ __global__ void __launch_bounds__(192, 1)
       int s_nkv = s_it < n_items ? items[s_it].n_kv : 0;
       auto issue_s = [&]() -> bool {
         if (s_it >= n_items) return true;
-        const int qb = s_k & 1;
-        if (s_j == 0 && !mbar_wait(&q_full[qb], (s_k >> 1) & 1, abort_flag, err)) return false;
-        const int st = s_g & 1;
-        if (!mbar_wait(&kv_full[st], (s_g >> 1) & 1, abort_flag, err)) return false;
+        const int qb = s_k % NQ;
+        if (s_j == 0 && !mbar_wait(&q_full[qb], (s_k / NQ) & 1, abort_flag, err)) return false;
+        const int st = s_g % NS;  // K/V stage
+        const int sb = s_g & 1;   // TMEM S buffer
+        if (!mbar_wait(&kv_full[st], (s_g / NS) & 1, abort_flag, err)) return false;
         tc_fence_after();
         const uint32_t qa = smem_u32(sQ + qb * C::Q_BYTES);
         const uint32_t ka = smem_u32(sK + st * C::K_BYTES);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
           const uint32_t off = (kk >> 2) * (128 * 128);
-          tc_mma_bf16(tmem_base + st * kBK, sw128_kmajor_desc(qa + off) + 2u * (kk & 3),
+          tc_mma_bf16(tmem_base + sb * kBK, sw128_kmajor_desc(qa + off) + 2u * (kk & 3),
                       sw128_kmajor_desc(ka + off) + 2u * (kk & 3), id_s, kk > 0 ? 1u : 0u);
         }
-        tc_commit(&s_full[st]);
+        tc_commit(&s_full[sb]);
         if (s_j == s_nkv - 1) tc_commit(&q_empty[qb]);  // last S of the item: its Q buffer is free
         ++s_g;
         if (++s_j == s_nkv) {
@@ -187,14 +199,15 @@ __global__ void __launch_bounds__(192, 1)
             break;
           }
           tc_fence_after();
-          const int st = p_g & 1;
-          const uint32_t pa = smem_u32(sP);
+          const int st = p_g % NS;  // K/V stage
+          const int sb = p_g & 1;   // TMEM buffer holding P_j
           const uint32_t va = smem_u32(sV + st * C::V_BYTES);
+          // A = P_j in TMEM (the S buffer it was computed in: 16 keys = 8 columns per MMA)
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk)
-            tc_mma_bf16(tmem_base + C::O_COL, sw128_kmajor_desc(pa + (kk >> 2) * (kBQ * 128)) + 2u * (kk & 3),
-                        sw128_kmajor_desc(va + (kk >> 2) * (HD * 128)) + 2u * (kk & 3), id_o,
-                        (j > 0 || kk > 0) ? 1u : 0u);
+            tc_mma_bf16_ta(tmem_base + C::O_COL, tmem_base + sb * kBK + 8 * kk,
+                           sw128_kmajor_desc(va + (kk >> 2) * (HD * 128)) + 2u * (kk & 3), id_o,
+                           (j > 0 || kk > 0) ? 1u : 0u);
           tc_commit(pv_done);
           tc_commit(&kv_empty[st]);  // S_j and PV_j have read this stage's K and V
         }
@@ -206,7 +219,6 @@ __global__ void __launch_bounds__(192, 1)
     const int r = quarter * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
     const float sl2 = rsqrtf((float)HD) * kLog2e;
-    uint8_t* prow = sP + r * 128;
     int g = 0;
     bool ok = true;
     for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
@@ -228,14 +240,20 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
         for (int c = 0; c < kBK / 32; ++c) tmem_ld_32x32b_x32(s_addr + 32 * c, v + 32 * c);
         tmem_ld_wait();
+        // row max on the raw scores (the scale is positive); the causal mask
+        // only applies on the diagonal tile (key > query position)
         float mx = -INFINITY;
+        if (diag) {
 #pragma unroll
-        for (int e = 0; e < kBK; ++e) {
-          float x = __uint_as_float(v[e]) * sl2;
-          if (diag && key0 + e > qp) x = -INFINITY;  // causal mask (diagonal tile only)
-          v[e] = __float_as_uint(x);
-          mx = fmaxf(mx, x);
+          for (int e = 0; e < kBK; ++e) {
+            if (key0 + e > qp) v[e] = __float_as_uint(-INFINITY);
+            mx = fmaxf(mx, __uint_as_float(v[e]));
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < kBK; ++e) mx = fmaxf(mx, __uint_as_float(v[e]));
         }
+        mx *= sl2;  // in the log2 domain of the exponentials
         float alpha = 1.f;
         bool resc = false;
         if (mx > m_used + kRescaleLog2) {
@@ -244,21 +262,24 @@ __global__ void __launch_bounds__(192, 1)
           m_used = mx;
           resc = j > 0;
         }
-        // P = exp2(s - m) as bf16 pairs in registers, while the previous PV
-        // product (which still reads the shared P tile) runs; the row sum
-        // takes the bf16 values the PV product uses (O / l stays a convex
-        // combination of the value rows)
+        // P = exp2(s - m) as bf16 pairs, written back over the scores of this
+        // buffer (columns 0..63); the row sum takes the bf16 values the PV
+        // product uses (O / l stays a convex combination of the value rows)
         uint32_t pk[kBK / 2];
         float ps = 0.f;
 #pragma unroll
         for (int e = 0; e < kBK; e += 2) {
-          const float p0 = ex2_approx(__uint_as_float(v[e]) - m_used);
-          const float p1 = ex2_approx(__uint_as_float(v[e + 1]) - m_used);
+          const float p0 = ex2_approx(fmaf(__uint_as_float(v[e]), sl2, -m_used));
+          const float p1 = ex2_approx(fmaf(__uint_as_float(v[e + 1]), sl2, -m_used));
           pk[e >> 1] = pack_bf16x2(p0, p1);
           const float2 pr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&pk[e >> 1]));
           ps += pr.x + pr.y;
         }
-        // O and the P tile are free once the previous PV of this item is done
+        tmem_st_32x32b_x32(s_addr, pk);
+        tmem_st_32x32b_x32(s_addr + 32, pk + 32);
+        // the previous PV must be complete before this tile's P is released (the
+        // PV barrier then never runs two phases ahead of this thread) and
+        // before O is rescaled
         if (j > 0 && !mbar_wait(pv_done, (g - 1) & 1, abort_flag, err)) {
           ok = false;
           break;
@@ -277,21 +298,9 @@ __global__ void __launch_bounds__(192, 1)
             for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * a);
             tmem_st_32x32b_x32(o_addr, o);
           }
-          tmem_st_wait();
         }
-        // keys 32c .. 32c+31 of the row: block c/2, 16-byte chunks 4(c%2) .. 4(c%2)+3
-#pragma unroll
-        for (int c = 0; c < kBK / 32; ++c) {
-          uint8_t* blk = prow + (c >> 1) * (kBQ * 128);
-#pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            const int chunk = ((c & 1) * 4 + t) ^ (r & 7);
-            const uint32_t* q4 = pk + 16 * c + 4 * t;
-            *reinterpret_cast<uint4*>(blk + chunk * 16) = make_uint4(q4[0], q4[1], q4[2], q4[3]);
-          }
-        }
+        tmem_st_wait();
         l += ps;
-        fence_proxy_async_smem();  // the P tile is read by the tensor cores (async proxy)
         tc_fence_before();
         mbar_arrive(p_full);
       }

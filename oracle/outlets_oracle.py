@@ -35,7 +35,12 @@ Readings where the paper is silent (the same list is kept in the design notes):
     has position = number of tokens already cached for its request;
   * Linear layers of the decoder have no bias; the length head has biases;
   * static pooling takes the last prompt position;
-  * length_hat = max(0, expm1(z_hat)) (clamped because expm1 < 0 for z < 0).
+  * length_hat = max(0, expm1(z_hat)) (clamped because expm1 < 0 for z < 0);
+  * dual head (Sec. 4.2, Eq. 2): the draft branch reads the same final-normed
+    state h^draft as the length head; its output is the log of the softmax of
+    W_lm h^draft over the vocabulary, reported as the k most probable tokens
+    (ties: smaller token id first), their log-probabilities and the row's
+    logsumexp.  Used when the weights carry "w_lm" and draft_k is given.
 
 Parity pins: every function here is checked by ``tests/test_oracle_pins.py``
 against closed forms, special cases, brute force on tiny inputs, invariants and
@@ -199,13 +204,55 @@ def head_weights(w):
     return ws, bs
 
 
+# ------------------------------------------------------------------ draft head (Sec. 4.2, Eq. 2)
+def draft_logits(h, w_lm):
+    """W_lm h^draft for every row: the vector Eq. 2 passes to the softmax.
+    w_lm: [V, d] (one row per vocabulary entry)."""
+    return _f64(h) @ _f64(w_lm).T
+
+
+def log_softmax_rows(logits):
+    """log of the softmax of Eq. 2 over the vocabulary axis, and the logsumexp.
+
+    logsumexp = m + log(sum_v exp(l_v - m)) with m the row maximum (the shift
+    keeps every exponent <= 0); log P(v) = l_v - logsumexp.
+    """
+    l = _f64(logits)
+    m = np.max(l, axis=-1, keepdims=True)
+    lse = m + np.log(np.sum(np.exp(l - m), axis=-1, keepdims=True))
+    return l - lse, lse[..., 0]
+
+
+def top_k_tokens(values, k):
+    """Indices of the k largest entries of each row, largest first; equal
+    values are ordered by smaller index (a total order, so the answer is unique)."""
+    values = _f64(values)
+    ids = np.arange(values.shape[-1])
+    out = np.empty((values.shape[0], k), dtype=np.int64)
+    for r in range(values.shape[0]):
+        out[r] = np.lexsort((ids, -values[r]))[:k]
+    return out
+
+
+def draft_head(h, w_lm, k):
+    """Draft branch of the dual head: P_draft = softmax(W_lm h^draft) (Eq. 2),
+    reported as the top-k tokens with their log-probabilities."""
+    logits = draft_logits(h, w_lm)
+    logp, lse = log_softmax_rows(logits)
+    ids = top_k_tokens(logits, k)
+    return dict(logits=logits, logprob=logp, lse=lse, topk_ids=ids,
+                topk_logprob=np.take_along_axis(logp, ids, axis=1))
+
+
 # ------------------------------------------------------------------ forward
-def predict_prefill(w, shape, taps, cu, all_tokens=False):
+def predict_prefill(w, shape, taps, cu, all_tokens=False, draft_k=None):
     """Static prediction over a packed varlen batch (Sec. 3.2, Sec. 4).
 
     Returns a dict with the hidden states of every step (for parity tests),
     the post-RoPE keys/values of every token (the draft KV cache), z_hat and
     length_hat at each sequence's last token (or every token if all_tokens).
+    With draft_k and weights carrying "w_lm", "draft" holds the draft head's
+    output (draft_head) on the same rows.
     """
     H, KVH, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
     eps, theta = shape.rms_eps, shape.rope_theta
@@ -230,8 +277,11 @@ def predict_prefill(w, shape, taps, cu, all_tokens=False):
     hd_state = rms_norm(y[rows], w["g_final"], eps)          # h^draft
     ws, bs = head_weights(w)
     z = length_head(hd_state, ws, bs)
-    return dict(f=f, x=x, q=q, k=k, v=v, attn=o, a=a, y=y, rows=rows,
-                h_draft=hd_state, z=z, length=z_to_length(z))
+    out = dict(f=f, x=x, q=q, k=k, v=v, attn=o, a=a, y=y, rows=rows,
+               h_draft=hd_state, z=z, length=z_to_length(z))
+    if draft_k:
+        out["draft"] = draft_head(hd_state, w["w_lm"], draft_k)
+    return out
 
 
 def caches_from_prefill(out, cu):
@@ -241,13 +291,13 @@ def caches_from_prefill(out, cu):
             for b in range(len(cu) - 1)]
 
 
-def predict_step(w, shape, taps_rows, caches):
+def predict_step(w, shape, taps_rows, caches, draft_k=None):
     """Dynamic prediction for one new token per request (Sec. 3.2, t >= 1).
 
     taps_rows: three [B, d] arrays; caches: list of B (k [L, KVH, hd],
     v [L, KVH, hd]) already-cached post-RoPE keys/values.  The new token sits
     at position L of its request.  Returns z_hat, length_hat, intermediates and
-    the caches extended by the new token.
+    the caches extended by the new token (and "draft" as in predict_prefill).
     """
     H, KVH, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
     eps, theta = shape.rms_eps, shape.rope_theta
@@ -273,11 +323,14 @@ def predict_step(w, shape, taps_rows, caches):
     hd_state = rms_norm(y, w["g_final"], eps)
     ws, bs = head_weights(w)
     z = length_head(hd_state, ws, bs)
-    return dict(f=f, x=x, q=q, k=k, v=v, attn=o, a=a, y=y, h_draft=hd_state,
-                z=z, length=z_to_length(z), caches=new_caches)
+    out = dict(f=f, x=x, q=q, k=k, v=v, attn=o, a=a, y=y, h_draft=hd_state,
+               z=z, length=z_to_length(z), caches=new_caches)
+    if draft_k:
+        out["draft"] = draft_head(hd_state, w["w_lm"], draft_k)
+    return out
 
 
-def sample_prefill_rows(w, shape, taps, cu, seqs):
+def sample_prefill_rows(w, shape, taps, cu, seqs, draft_k=None):
     """Oracle for a subset of sequences of a large packed batch.
 
     Every sequence is independent (attention never crosses sequences), so the
@@ -289,4 +342,4 @@ def sample_prefill_rows(w, shape, taps, cu, seqs):
     sub_len = np.array([cu[b + 1] - cu[b] for b in seqs], dtype=np.int64)
     sub_cu = np.zeros(len(seqs) + 1, dtype=np.int64)
     np.cumsum(sub_len, out=sub_cu[1:])
-    return predict_prefill(w, shape, sub_taps, sub_cu)
+    return predict_prefill(w, shape, sub_taps, sub_cu, draft_k=draft_k)

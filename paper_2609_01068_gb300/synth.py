@@ -8,7 +8,8 @@ Shapes follow the draft backbones the method is evaluated with (Sec. 5.1,
 (three hidden states of width d from layers {2, floor(N/2), N-2}).
 
 Recipe (all draws from numpy PCG64 streams spawned from one SeedSequence):
-  * stream 0 -> sequence / cache lengths;  stream 1 -> taps;  stream 2 -> weights.
+  * stream 0 -> sequence / cache lengths;  stream 1 -> taps;  stream 2 -> weights;
+    stream 3 -> draft LM head W_lm (Eq. 2) and stand-in draft states.
   * lengths: rint(lognormal(ln(median), sigma=1)) clipped to the stated range.
   * taps ~ N(0, 1); every Linear weight ~ N(0, 0.02); RMSNorm gains = 1;
     head hidden biases ~ N(0, 0.02); output bias = ln(1 + 256).
@@ -28,6 +29,7 @@ __all__ = [
     "lengths_tiny", "lengths_8b_prefill", "lengths_8b_step_cache",
     "lengths_70b_prefill", "lengths_sweep", "cu_seqlens",
     "make_weights", "make_taps", "weight_names",
+    "LLAMA3_VOCAB", "make_lm_head", "make_draft_states",
 ]
 
 
@@ -172,6 +174,33 @@ def make_weights(shape: ModelShape, seed: int = 0, std: float = 0.02,
     if gated:
         w["w_attn_gate"] = lin(H * hd, d)
     return w
+
+
+LLAMA3_VOCAB = 128256  # vocabulary of the Llama-3 targets (the draft head's output width)
+
+
+def make_lm_head(shape: ModelShape, vocab: int, seed: int = 0, std: float = 0.02) -> np.ndarray:
+    """Draft LM head W_lm [vocab, d] ~ N(0, std) (Eq. 2), from its own stream
+    (stream 3), so drawing it leaves every other weight unchanged."""
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence(seed).spawn(4)[3]))
+    rnd = round_bf16 if shape.dtype == "bf16" else (lambda a: np.ascontiguousarray(a, np.float32))
+    out = np.empty((vocab, shape.d), np.float32)
+    step = max(1, (1 << 24) // shape.d)
+    for r0 in range(0, vocab, step):  # bounded temporaries at vocab ~128k
+        r1 = min(vocab, r0 + step)
+        out[r0:r1] = rnd(rng.standard_normal((r1 - r0, shape.d), dtype=np.float32) * np.float32(std))
+    return out
+
+
+def make_draft_states(shape: ModelShape, rows: int, seed: int = 0, stream_offset: int = 0) -> np.ndarray:
+    """Stand-in final-normed draft states h^draft [rows, d] for testing the
+    draft head on its own: N(0, 1) entries (unit RMS, like an RMSNorm output
+    with unit gains), bf16-rounded on the bf16 path."""
+    ss = np.random.SeedSequence(seed).spawn(4)[3]
+    ss = np.random.SeedSequence(entropy=ss.entropy, spawn_key=ss.spawn_key + (1000 + stream_offset,))
+    rng = np.random.Generator(np.random.PCG64(ss))
+    rnd = round_bf16 if shape.dtype == "bf16" else (lambda a: a)
+    return rnd(rng.standard_normal((rows, shape.d), dtype=np.float32))
 
 
 def make_taps(shape: ModelShape, n_tokens: int, seed: int = 0, stream_offset: int = 0):

@@ -419,3 +419,101 @@ def test_default_weights_have_no_gate():
     assert "w_attn_gate" not in w
     for k in w:
         np.testing.assert_array_equal(w[k], wg[k])
+
+
+# ---------------------------------------------------------------- dual head, draft branch (Eq. 2)
+def _draft_case(V=37, rows=5, seed=3):
+    rng = np.random.default_rng(seed)
+    h = rng.standard_normal((rows, SMALL.d))
+    w_lm = rng.standard_normal((V, SMALL.d)) * 0.2
+    return h, w_lm
+
+
+def test_draft_softmax_is_a_distribution():
+    h, w_lm = _draft_case()
+    out = O.draft_head(h, w_lm, 4)
+    np.testing.assert_allclose(np.exp(out["logprob"]).sum(axis=1), 1.0, rtol=0, atol=1e-12)
+    assert np.all(out["logprob"] <= 0.0)
+
+
+def test_draft_logsumexp_and_log_softmax_match_library():
+    special = pytest.importorskip("scipy.special")
+    rng = np.random.default_rng(4)
+    logits = rng.standard_normal((6, 1000)) * 30.0  # large spread: the max shift matters
+    logp, lse = O.log_softmax_rows(logits)
+    np.testing.assert_allclose(lse, special.logsumexp(logits, axis=1), rtol=1e-13)
+    np.testing.assert_allclose(logp, special.log_softmax(logits, axis=1), rtol=1e-12, atol=1e-12)
+
+
+def test_draft_permutation_head_closed_form():
+    """W_lm = a permutation matrix (V = d): logit v = h[perm[v]] exactly; a
+    transposed operand would give h[perm^-1[v]] instead."""
+    rng = np.random.default_rng(5)
+    d = SMALL.d
+    perm = rng.permutation(d)
+    assert np.any(perm[perm] != np.arange(d))  # not an involution, so P != P^T
+    w_lm = np.zeros((d, d))
+    w_lm[np.arange(d), perm] = 1.0
+    h = rng.standard_normal((3, d))
+    out = O.draft_head(h, w_lm, 5)
+    np.testing.assert_array_equal(out["logits"], h[:, perm])
+    for r in range(3):
+        vals = list(h[r, perm])
+        expect = []
+        for _ in range(5):  # brute force: repeatedly take the largest remaining
+            best = max(range(d), key=lambda v: (vals[v], -v) if v not in expect else (-np.inf, 0))
+            expect.append(best)
+        assert list(out["topk_ids"][r]) == expect
+
+
+def test_draft_zero_head_is_uniform_and_ties_go_to_smaller_ids():
+    V = 50
+    out = O.draft_head(np.ones((2, SMALL.d)), np.zeros((V, SMALL.d)), 6)
+    np.testing.assert_allclose(out["logprob"], -math.log(V), rtol=0, atol=1e-14)
+    np.testing.assert_allclose(out["lse"], math.log(V), rtol=1e-15)
+    assert out["topk_ids"].tolist() == [list(range(6))] * 2
+
+
+def test_draft_topk_brute_force_with_planted_ties():
+    logits = np.array([[0.5, 2.0, -1.0, 2.0, 0.5, 3.0, 2.0, -4.0, 0.5, 3.0, 1.0]])
+    ids = O.top_k_tokens(logits, 7)
+    rows = sorted(range(logits.shape[1]), key=lambda v: (-logits[0, v], v))
+    assert ids[0].tolist() == rows[:7] == [5, 9, 1, 3, 6, 10, 0]
+
+
+def test_draft_row_shift_invariance():
+    """Adding the same vector u to every row of W_lm adds h.u to every logit of
+    the row: log-probabilities and top-k are unchanged, logsumexp moves by h.u."""
+    h, w_lm = _draft_case()
+    u = np.random.default_rng(6).standard_normal(SMALL.d)
+    a = O.draft_head(h, w_lm, 5)
+    b = O.draft_head(h, w_lm + u[None, :], 5)
+    np.testing.assert_allclose(b["logprob"], a["logprob"], rtol=0, atol=1e-10)
+    np.testing.assert_allclose(b["lse"], a["lse"] + h @ u, rtol=0, atol=1e-10)
+    np.testing.assert_array_equal(b["topk_ids"], a["topk_ids"])
+
+
+def test_dual_head_reads_the_length_heads_state():
+    """Both branches of the dual head read the same h^draft (Sec. 4.2): the
+    draft output of a prediction is the draft head of its h_draft, and asking
+    for it changes nothing else."""
+    w = _weights()
+    w["w_lm"] = synth.make_lm_head(SMALL, 29, 0)
+    cu = synth.cu_seqlens([4, 7])
+    taps = _taps(SMALL, 11)
+    plain = O.predict_prefill(w, SMALL, taps, cu)
+    dual = O.predict_prefill(w, SMALL, taps, cu, draft_k=3)
+    np.testing.assert_array_equal(dual["z"], plain["z"])
+    ref = O.draft_head(plain["h_draft"], w["w_lm"], 3)
+    np.testing.assert_array_equal(dual["draft"]["topk_ids"], ref["topk_ids"])
+    np.testing.assert_array_equal(dual["draft"]["lse"], ref["lse"])
+
+
+def test_lm_head_draw_leaves_other_weights_unchanged():
+    a = synth.make_weights(SMALL, 0)
+    w1 = synth.make_lm_head(SMALL, 40, 0)
+    b = synth.make_weights(SMALL, 0)
+    for k in a:
+        np.testing.assert_array_equal(a[k], b[k])
+    np.testing.assert_array_equal(w1, synth.make_lm_head(SMALL, 40, 0))
+    assert w1.shape == (40, SMALL.d) and abs(float(w1.std()) - 0.02) < 0.004

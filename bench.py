@@ -43,6 +43,9 @@ def model_setup(args):
     from paper_2609_01068_gb300 import synth
     gate = ", gated attention" if getattr(args, "gated", False) else ""
     gkey = "-gated" if getattr(args, "gated", False) else ""
+    if getattr(args, "dual", 0):
+        gate += ", dual head (draft LM head over the 128256-token Llama-3 vocabulary, top-%d)" % args.dual
+        gkey += "-dual%d" % args.dual
     if args.model == "70b":
         lengths = synth.lengths_70b_prefill(0)
         return synth.LLAMA70B, lengths[:args.prompts] if args.prompts else lengths, WORKLOAD_70B + gate, "70b" + gkey
@@ -62,6 +65,9 @@ def parse():
                     help="first N prompts of the workload (profiling cases; default: all)")
     ap.add_argument("--gated", action="store_true",
                     help="gated attention (Sec. 4.1): sigmoid gate on the attention output, gate weights [H*hd, d]")
+    ap.add_argument("--dual", type=int, default=0, metavar="K",
+                    help="dual head (Sec. 4.2, Eq. 2): also run the draft LM head (Llama-3 vocabulary, "
+                         "128256 tokens) and return its top-K tokens (1..8); 0 = length head only")
     ap.add_argument("--model", default="8b", choices=["8b", "70b"],
                     help="draft-layer shape; 70b (Llama-3.3-70B-shaped, 32 prompts) runs the static mode only")
     ap.add_argument("--step-requests", type=int, default=256, help="live requests of the dynamic-prediction run")
@@ -72,6 +78,7 @@ def parse():
 
 TRAFFIC_SOURCES = {  # files whose content decides the kernel's DRAM traffic (incl. the tile raster)
     "gateup_swiglu_gemm": ["gemm_tc.cu", "common.cuh", "kernels.h", "outlets.cu"],
+    "draft_head": ["gemm_tc.cu", "lm_head.cu", "lm_topk.cuh", "common.cuh", "kernels.h", "outlets.cu"],
     "decode_attention": ["attn_decode.cu", "mma_sync.cuh", "common.cuh", "kernels.h", "outlets.cu"],
 }
 
@@ -192,8 +199,9 @@ def cpu_threads():
     return os.cpu_count()
 
 
-def oracle_sample(shape, w, taps, cu, lengths, budget_tokens):
-    """Oracle on whole prompts taken in order until the token budget is used."""
+def oracle_sample(shape, w, taps, cu, lengths, budget_tokens, draft_k=None):
+    """Oracle on whole prompts taken in order until the token budget is used
+    (with the draft head when draft_k is given)."""
     from oracle import outlets_oracle as OR
     picks, tot = [], 0
     for b in np.argsort(np.abs(lengths - np.median(lengths))):
@@ -202,7 +210,7 @@ def oracle_sample(shape, w, taps, cu, lengths, budget_tokens):
         picks.append(int(b))
         tot += int(lengths[b])
     t0 = time.perf_counter()
-    OR.sample_prefill_rows(w, shape, taps, cu, picks)
+    OR.sample_prefill_rows(w, shape, taps, cu, picks, draft_k=draft_k)
     dt = time.perf_counter() - t0
     return len(picks), tot, dt
 
@@ -242,14 +250,17 @@ def run_reference(args):
     from paper_2609_01068_gb300 import synth
     shape, lengths, workload, _ = model_setup(args)
     w = synth.make_weights(shape, 0, gated=args.gated)
+    if args.dual:
+        w["w_lm"] = synth.make_lm_head(shape, synth.LLAMA3_VOCAB, 0)
     cu = synth.cu_seqlens(lengths)
     taps = synth.make_taps(shape, int(cu[-1]), 0)
     budget = 400
+    dk = args.dual or None
     for _ in range(args.warmup):
-        oracle_sample(shape, w, taps, cu, lengths, budget)
+        oracle_sample(shape, w, taps, cu, lengths, budget, dk)
     n_pred, n_tok, secs = 0, 0, 0.0
     for _ in range(args.steps):
-        p, t, dt = oracle_sample(shape, w, taps, cu, lengths, budget)
+        p, t, dt = oracle_sample(shape, w, taps, cu, lengths, budget, dk)
         n_pred, n_tok, secs = n_pred + p, n_tok + t, secs + dt
     value = n_pred / secs
     out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "predictions/s", "n_gpus": args.gpus,
@@ -283,6 +294,8 @@ def run_ours(args):
     shape, lengths, workload, tkey = model_setup(args)
     args.workload, args.traffic_key = workload, tkey
     w = synth.make_weights(shape, 0, gated=args.gated)
+    if args.dual:
+        w["w_lm"] = synth.make_lm_head(shape, synth.LLAMA3_VOCAB, 0)
     cu = synth.cu_seqlens(lengths)
     T, Bq = int(cu[-1]), len(lengths)
     taps = synth.make_taps(shape, T, 0, rank)
@@ -308,7 +321,8 @@ def run_ours(args):
     if args.mode in ("both", "step"):
         sm = run_step_mode(args, pred, shape, peaks, step_B, world, barrier, max_over_ranks, stream, max_tokens)
         if args.mode == "step":
-            out.update({k: sm[k] for k in ("value", "unit", "ms_per_step", "e2e", "gpu_launches", "clocks")})
+            out.update({k: sm[k] for k in ("value", "unit", "ms_per_step", "e2e", "gpu_launches", "clocks",
+                                           "roofline")})
             out["config"] = {"workload": sm["workload"], "parallelism": f"replicas x{world}"}
         out["step_mode"] = sm
     if args.mode == "sweep":
@@ -333,11 +347,20 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
                      max_over_ranks, stream):
     import torch
     T, Bq = int(cu[-1]), len(lengths)
+    K = args.dual
+    dout = draft_buffers(K, Bq) if K else None
+
+    def run(tp, zo, lo, out=None):
+        if K:
+            pred.prefill_dual(tp, cu, K, out=out if out is not None else dout, z_out=zo, len_out=lo)
+        else:
+            pred.prefill(tp, cu, z_out=zo, len_out=lo)
+
     # ---------------- device-timed static prediction
     z = torch.empty(Bq, dtype=torch.float32, device="cuda")
     ln = torch.empty(Bq, dtype=torch.float32, device="cuda")
     for _ in range(args.warmup):
-        pred.prefill(taps_d, cu, z_out=z, len_out=ln)
+        run(taps_d, z, ln)
     pred.check()
     pred.profile(True, ["gateup_swiglu_gemm"])  # the dominant kernel, timed live on its stream
     launches0 = pred.launch_count
@@ -347,7 +370,7 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
     for _ in range(args.steps):
-        pred.prefill(taps_d, cu, z_out=z, len_out=ln)
+        run(taps_d, z, ln)
     ev1.record(stream)
     ev1.synchronize()
     barrier()
@@ -360,12 +383,12 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     # per-stage breakdown in a separate (untimed) pass: stage events serialize the kernels
     pred.profile(True)
     for _ in range(3):
-        pred.prefill(taps_d, cu, z_out=z, len_out=ln)
+        run(taps_d, z, ln)
     prof = pred.profile_read()
     pred.profile(False)
     ms_step = ms / args.steps
     value = world * Bq * args.steps / (ms / 1e3)
-    flops = prefill_flops(shape, lengths, Bq, args.gated)
+    flops = prefill_flops(shape, lengths, Bq, args.gated) + (2.0 * Bq * pred.vocab * shape.d if K else 0.0)
     gu_ms, gu_n = prof_live["gateup_swiglu_gemm"]
     gu_flops = 2.0 * T * (2 * shape.ffn) * shape.d
     gu_tflops = gu_flops / (gu_ms / gu_n / 1e3) / 1e12
@@ -383,18 +406,19 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
         host_taps = [t.cpu().pin_memory() for t in taps_d]
         zh = torch.empty(Bq, dtype=torch.float32).pin_memory()
         lh = torch.empty(Bq, dtype=torch.float32).pin_memory()
+        dh = draft_buffers(K, Bq, pin=True) if K else None
         for _ in range(max(2, args.warmup // 2)):
-            pred.prefill(host_taps, cu, z_out=zh, len_out=lh)
+            run(host_taps, zh, lh, dh)
             stream.synchronize()
         barrier()
         t0 = time.perf_counter()
         for _ in range(args.steps):
-            pred.prefill(host_taps, cu, z_out=zh, len_out=lh)
+            run(host_taps, zh, lh, dh)
             stream.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - t0)
         e2e = {"value": world * Bq * args.steps / e2e_s, "unit": "predictions/s",
                "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps)),
-               "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4)}
+               "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4 + buffer_bytes(dh))}
 
     out = {"value": value, "unit": "predictions/s", "ms_per_step": ms_step,
            "config": {"workload": args.workload, "prompts_per_gpu": Bq, "tokens_per_gpu": T,
@@ -407,7 +431,7 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
            "roofline": roofline, "stages": stages, "clocks": clocks, "e2e": e2e,
            "gpu_launches": launches}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        n_pred, n_tok, secs = oracle_sample(shape, w, taps, cu, lengths, 1200)
+        n_pred, n_tok, secs = oracle_sample(shape, w, taps, cu, lengths, 1200, args.dual or None)
         out["cpu_baseline"] = {"value": n_pred / secs, "unit": "predictions/s", "cores": cpu_threads(),
                                "kind": "oracle",
                                "sample": f"{n_pred} whole prompts ({n_tok} tokens) of the same workload, {secs:.1f} s"}
@@ -435,11 +459,21 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     st_taps = [torch.randn(B, shape.d, device="cuda", generator=gen).to(torch.bfloat16) for _ in range(3)]
     z = torch.empty(B, dtype=torch.float32, device="cuda")
     ln = torch.empty(B, dtype=torch.float32, device="cuda")
+    K = args.dual
+    dout = draft_buffers(K, B) if K else None
+
+    def run(tp, zo, lo, out=None):
+        if K:
+            pred.step_dual(tp, kv, slots, K, out=out if out is not None else dout, z_out=zo, len_out=lo)
+        else:
+            pred.step(tp, kv, slots, z_out=zo, len_out=lo)
+
     for _ in range(args.warmup):
-        pred.step(st_taps, kv, slots, z_out=z, len_out=ln)
+        run(st_taps, z, ln)
     pred.check()
     cache0 = sum(kv.slot_length(int(s)) for s in slots)
-    pred.profile(True, ["attention"])  # the dominant kernel, timed live on its stream
+    # the dominant kernel(s), timed live on their stream
+    pred.profile(True, ["attention", "draft_head"] if K else ["attention"])
     launches0 = pred.launch_count
     sampler = ClockSampler(torch.cuda.current_device())
     sampler.start()
@@ -448,7 +482,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     ev0.record(stream)
     h0 = time.perf_counter()
     for _ in range(args.steps):
-        pred.step(st_taps, kv, slots, z_out=z, len_out=ln)
+        run(st_taps, z, ln)
     host_ms = (time.perf_counter() - h0) * 1e3 / args.steps
     ev1.record(stream)
     ev1.synchronize()
@@ -462,7 +496,7 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     pred.profile(True)  # per-stage breakdown, separate pass (stage events serialize kernels)
     n_prof = 3
     for _ in range(n_prof):
-        pred.step(st_taps, kv, slots, z_out=z, len_out=ln)
+        run(st_taps, z, ln)
     prof = pred.profile_read()
     pred.profile(False)
     # end to end through the C ABI: host taps in, host predictions out, every step
@@ -471,18 +505,19 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
         host_taps = [t.cpu().pin_memory() for t in st_taps]
         zh = torch.empty(B, dtype=torch.float32).pin_memory()
         lh = torch.empty(B, dtype=torch.float32).pin_memory()
+        dh = draft_buffers(K, B, pin=True) if K else None
         for _ in range(2):
-            pred.step(host_taps, kv, slots, z_out=zh, len_out=lh)
+            run(host_taps, zh, lh, dh)
             stream.synchronize()
         barrier()
         t0 = time.perf_counter()
         for _ in range(args.steps):
-            pred.step(host_taps, kv, slots, z_out=zh, len_out=lh)
+            run(host_taps, zh, lh, dh)
             stream.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - t0)
         e2e = {"value": world * B * args.steps / e2e_s, "unit": "predictions/s",
                "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps)),
-               "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4)}
+               "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4 + buffer_bytes(dh))}
     d, KVH, hd, F = shape.d, shape.n_kv_heads, shape.head_dim, shape.ffn
     # keys read per step: every cached position plus the new one, K and V, bf16
     keys_avg = cache0 + B * (args.steps + 1) / 2.0
@@ -491,25 +526,53 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     w_bytes = 2 * (3 * d * d + d * shape.qkv_out + shape.n_heads * hd * d + 3 * d * F + widths[0] * widths[1])
     if args.gated:
         w_bytes += 2 * shape.n_heads * hd * d  # gate rows of the QKV weight
-    step_bytes = kv_bytes + w_bytes + 3 * B * d * 2
+    lm_bytes = pred.vocab * d * 2 + B * d * 2 if K else 0  # W_lm and the draft states, read once
+    step_bytes = kv_bytes + w_bytes + 3 * B * d * 2 + lm_bytes
     at_ms, at_n = prof_live["attention"]
     at_gbs = kv_bytes / (at_ms / at_n / 1e3) / 1e9
     ms_step = ms / args.steps
     kv.close()
+    roofline = {"bound": "hbm", "kernel": "decode attention (k_attn_decode_bf16 + combine)",
+                "achieved": at_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": at_gbs / peaks["hbm_gbs"],
+                "traffic": measured_traffic("decode_attention", f"8b-step-{B}r-L{int(lens.sum())}"
+                                            + ("-gated" if args.gated else "")),
+                "algorithmic_per_launch": f"{kv_bytes:.4g} B of K/V (cached + new)"}
+    extra = {}
+    if K:
+        lm_ms, lm_n = prof_live["draft_head"]
+        lm_t = lm_ms / lm_n / 1e3
+        lm_gbs = lm_bytes / lm_t / 1e9
+        extra["attention_roofline"] = roofline
+        roofline = {"bound": "hbm", "kernel": "draft LM head (k_gemm_small<EPI_LM8> + k_lm_merge)",
+                    "achieved": lm_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": lm_gbs / peaks["hbm_gbs"],
+                    "traffic": measured_traffic("draft_head", f"8b-step-{B}r-V{pred.vocab}"),
+                    "algorithmic_per_launch": f"{lm_bytes:.4g} B = W_lm [{pred.vocab}, {d}] bf16 + states",
+                    "tensor_frac": 2.0 * B * pred.vocab * d / lm_t / 1e12 / peaks["bf16_sus"]}
+    dual_txt = (", dual head (draft LM head over the 128256-token Llama-3 vocabulary, top-%d)" % K) if K else ""
     return {"workload": "dynamic prediction, %d live requests x 1 new token, cache lengths lognormal "
-                        "median 512 clipped 1-4096 (sum %d), Llama-3.1-8B-shaped draft layer%s"
-                        % (B, int(lens.sum()), ", gated attention" if args.gated else ""),
+                        "median 512 clipped 1-4096 (sum %d), Llama-3.1-8B-shaped draft layer%s%s"
+                        % (B, int(lens.sum()), ", gated attention" if args.gated else "", dual_txt),
             "value": world * B * args.steps / (ms / 1e3), "unit": "predictions/s", "ms_per_step": ms_step,
             "hbm_frac_step": step_bytes / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"],
             "algorithmic_bytes_per_step": step_bytes,
-            "roofline": {"bound": "hbm", "kernel": "decode attention (k_attn_decode_bf16 + combine)",
-                         "achieved": at_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                         "frac": at_gbs / peaks["hbm_gbs"],
-                         "traffic": measured_traffic("decode_attention", f"8b-step-{B}r-L{int(lens.sum())}"
-                                                     + ("-gated" if args.gated else "")),
-                         "algorithmic_per_launch": f"{kv_bytes:.4g} B of K/V (cached + new)"},
+            "roofline": roofline, **extra,
             "stages": {k: v[0] / max(v[1], 1) for k, v in prof.items() if v[1]},
             "clocks": clocks, "gpu_launches": launches, "host_issue_ms_per_step": host_ms, "e2e": e2e}
+
+
+def draft_buffers(k, n, pin=False):
+    """Outputs of the draft head for n rows (device, or pinned host)."""
+    import torch
+
+    def mk(shape, dt):
+        return torch.empty(shape, dtype=dt).pin_memory() if pin else torch.empty(shape, dtype=dt, device="cuda")
+
+    return {"ids": mk((n, k), torch.int32), "logprob": mk((n, k), torch.float32), "lse": mk(n, torch.float32)}
+
+
+def buffer_bytes(bufs):
+    return sum(t.numel() * t.element_size() for t in bufs.values()) if bufs else 0
 
 
 def pack_batches(lengths, cap):

@@ -13,6 +13,9 @@
  *   Sec. 3.2           static prediction r_hat_0 after prefill (last prompt
  *                      position); dynamic prediction r_hat_t at decode step t,
  *                      one new token per request against the draft KV cache.
+ *   Sec. 4.2, Eq. 2    dual head: the same h^draft also feeds the draft LM
+ *                      head, P_draft = softmax(W_lm h^draft) over the
+ *                      vocabulary (the *_dual calls and outlets_draft_head).
  *
  * The returned length is the REMAINING length r_hat_t (Sec. 3.1); a scheduler
  * forms the projected total t + r_hat_t itself.
@@ -82,6 +85,9 @@ typedef struct outlets_config {
   int32_t max_batch;      /* most sequences per prefill call / requests per step call */
   int32_t max_position;   /* positions 0 .. max_position-1 are supported (RoPE table) */
   int32_t device;         /* CUDA device ordinal */
+  int32_t vocab;          /* V: rows of the draft LM head W_lm (Eq. 2), 8 .. 262144;
+                             0 = no draft head (the *_dual calls and
+                             outlets_draft_head then return OUTLETS_EUNSUPPORTED) */
 } outlets_config;
 
 /* Host pointers to f32 weights, nn.Linear layout [out, in], row-major.
@@ -97,6 +103,8 @@ typedef struct outlets_config {
  *     o [rows, H*hd] is multiplied elementwise by sigmoid(x_hat w_attn_gate^T)
  *     (x_hat: the RMS-normalized layer input that also feeds QKV) before W_o;
  *     NULL gives standard attention.
+ *   w_lm [V, d]              the draft LM head of Eq. 2 (required when vocab > 0,
+ *     ignored otherwise).
  * The library copies everything during outlets_create; the caller may free
  * its arrays afterwards. */
 typedef struct outlets_weights {
@@ -114,6 +122,7 @@ typedef struct outlets_weights {
   const float* head_w[OUTLETS_MAX_HEAD_HIDDEN + 1];
   const float* head_b[OUTLETS_MAX_HEAD_HIDDEN + 1];
   const float* w_attn_gate;
+  const float* w_lm;
 } outlets_weights;
 
 typedef struct outlets_ctx outlets_ctx;
@@ -179,6 +188,46 @@ outlets_status outlets_predict_prefill(outlets_ctx* ctx, const void* const taps[
 outlets_status outlets_predict_step(outlets_ctx* ctx, const void* const taps[3], int32_t B, outlets_kv* kv,
                                     const int32_t* slots, float* z_out, float* len_out, void* stream);
 
+/* ---- Dual head: the draft LM head (Sec. 4.2, Eq. 2).
+ * P_draft(v) = softmax(W_lm h^draft)_v over the V vocabulary entries, for
+ * every predicted row (the rows whose z_hat a prediction call returns).  The
+ * library reports the k most probable tokens of each row, most probable first
+ * (equal logits: smaller token id first), their log-probabilities
+ * log P_draft(v) = l_v - logsumexp_v'(l_v'), l = W_lm h^draft, and optionally
+ * the logsumexp and the logits themselves.  The [rows, V] logits are never
+ * materialized unless `logits` is given: the tensor-core GEMM reduces each
+ * tile of logits to its softmax statistics and best tokens on chip.
+ * Arithmetic: bf16 operands (h^draft as the length head reads it, W_lm
+ * rounded on upload), f32 accumulation and softmax statistics. */
+#define OUTLETS_MAX_TOPK 8
+
+typedef struct outlets_draft_out {
+  int32_t k;              /* tokens per row, 1 .. OUTLETS_MAX_TOPK and <= vocab */
+  int32_t* topk_ids;      /* device or host int32 [rows, k]: token ids */
+  float* topk_logprob;    /* device or host f32 [rows, k]: their log P_draft */
+  float* logsumexp;       /* device or host f32 [rows], or NULL */
+  float* logits;          /* device or host f32 [rows, vocab] (W_lm h^draft), or NULL */
+} outlets_draft_out;
+
+/* outlets_predict_prefill plus the draft head on the same rows (one pass of
+ * the backbone serves both heads).  draft must not be NULL.  Extra errors:
+ * EUNSUPPORTED (vocab == 0), EINVAL (bad k or NULL topk pointers). */
+outlets_status outlets_predict_prefill_dual(outlets_ctx* ctx, const void* const taps[3], const int32_t* cu_seqlens,
+                                            int32_t B, int32_t T, outlets_kv* kv, const int32_t* slots,
+                                            uint32_t flags, float* z_out, float* len_out,
+                                            const outlets_draft_out* draft, void* stream);
+
+/* outlets_predict_step plus the draft head on the same rows. */
+outlets_status outlets_predict_step_dual(outlets_ctx* ctx, const void* const taps[3], int32_t B, outlets_kv* kv,
+                                         const int32_t* slots, float* z_out, float* len_out,
+                                         const outlets_draft_out* draft, void* stream);
+
+/* The draft head alone on caller-given states.
+ *   h_draft  device [rows, d] (bf16 or f32 like the context), 16-byte aligned.
+ *   draft    outputs as above, rows rows. */
+outlets_status outlets_draft_head(outlets_ctx* ctx, const void* h_draft, int32_t rows, const outlets_draft_out* draft,
+                                  void* stream);
+
 /* Synchronizes the stream, then reports (and clears) the device error word. */
 outlets_status outlets_check(outlets_ctx* ctx, void* stream);
 
@@ -222,7 +271,8 @@ typedef enum outlets_stage {
   OUTLETS_S_DOWN = 8,        /* down projection GEMM + residual */
   OUTLETS_S_FINAL_NORM = 9,  /* final RMSNorm of the predicted rows (h^draft) */
   OUTLETS_S_HEAD = 10,       /* length head (Sec. 4.2): Linear+ReLU layers and output row */
-  OUTLETS_N_STAGES = 11
+  OUTLETS_S_DRAFT = 11,      /* draft LM head (Eq. 2): GEMM with on-chip softmax/top-k, merge */
+  OUTLETS_N_STAGES = 12
 } outlets_stage;
 
 /* Times the stages whose bit (1 << outlets_stage) is set in stage_mask for

@@ -20,7 +20,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "liboutlets_gb300.so")
-SOURCES = ["outlets.cu", "gemm_tc.cu", "attn_prefill.cu", "attn_prefill_tc.cu", "attn_decode.cu", "elementwise.cu"]
+SOURCES = ["outlets.cu", "gemm_tc.cu", "attn_prefill.cu", "attn_prefill_tc.cu", "attn_decode.cu", "elementwise.cu",
+           "lm_head.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 

@@ -16,12 +16,13 @@
 // f32 slice that the consuming kernel adds up.
 //
 // Used for Eq. 1 (three-tap fusion: A is split along K over the three taps),
-// the QKV / O / gate-up / down projections of the draft decoder layer, and
-// the first Linear of the length head (Sec. 4.2).
+// the QKV / O / gate-up / down projections of the draft decoder layer, the
+// first Linear of the length head and the draft LM head (Sec. 4.2, Eq. 2).
 #include <stdlib.h>
 
 #include "common.cuh"
 #include "kernels.h"
+#include "lm_topk.cuh"
 
 namespace outlets {
 namespace {
@@ -439,6 +440,128 @@ cudaError_t launch_one(const CUtensorMap a_maps[3], const GemmArgs& args, int nu
 // ring barriers (AS and WS slots; the producer may run the weight ring
 // WS - AS blocks ahead); with AS == WS this is one ring holding both tiles of
 // a K block, which is what the latency of both operands needs.
+// ---------------------------------------------------------------- draft LM head epilogue (Eq. 2)
+// Candidate places per epilogue thread in the idle operand ring.
+constexpr int kLmCap = 64;
+
+__device__ __forceinline__ float lm_ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void lm_store32(float* dst, const uint32_t (&r)[32], int n, bool vec) {
+  if (vec && n >= 32) {
+#pragma unroll
+    for (int j = 0; j < 32; j += 4)
+      *reinterpret_cast<float4*>(dst + j) = make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]),
+                                                        __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3]));
+  } else {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < n) dst[j] = __uint_as_float(r[j]);
+  }
+}
+
+// One row of a draft LM head tile: the calling thread owns TMEM lane `tb`'s
+// row (global row m, columns n0 .. n0 + BN - 1, of which the first lim are
+// inside the vocabulary when MASK) and writes the row's partials (kernels.h).
+//  pass 1 reads the row from TMEM and takes the maximum of each of 8 column
+//         groups (column mod 8); the smallest group maximum is reached by 8
+//         distinct columns, so it bounds the tile's 8th best logit from below;
+//  pass 2 re-reads the row, sums exp(logit - max) and moves the logits that
+//         reach the bound (a few percent of a smooth row) to this thread's
+//         candidate list in shared memory (column-major over the 128 threads);
+//  then only the candidates go through the sorted insertion, after the scan,
+//  so the lanes of a warp do not diverge on every logit.  A list that fills
+//  up inserts its overflow directly (the order of insertion does not matter).
+template <int BN, int KT, bool MASK>
+__device__ __forceinline__ void lm_row(const GemmArgs& p, uint32_t tb, int m, int n0, int lim, int num_n,
+                                       int n_blk, float* cval, int* cidx, int et) {
+  constexpr int NCH = BN / 32;
+  float gmax[8];
+#pragma unroll
+  for (int g = 0; g < 8; ++g) gmax[g] = -INFINITY;
+  float best = -INFINITY;
+  int best_c = INT_MAX;
+#pragma unroll 1
+  for (int ch = 0; ch < NCH; ++ch) {
+    uint32_t r[32];
+    tmem_ld_32x32b_x32(tb + ch * 32, r);
+    tmem_ld_wait();
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int col = ch * 32 + j;
+      float v = __uint_as_float(r[j]);
+      if (MASK && col >= lim) v = -INFINITY;
+      if constexpr (KT == 1) {
+        if (v > best) {  // strict: the first (smallest) column keeps a tie
+          best = v;
+          best_c = col;
+        }
+      } else {
+        gmax[j & 7] = fmaxf(gmax[j & 7], v);
+      }
+    }
+  }
+  float mx = best, thr = gmax[0];
+  if constexpr (KT > 1) {
+    mx = gmax[0];
+#pragma unroll
+    for (int g = 1; g < 8; ++g) {
+      mx = fmaxf(mx, gmax[g]);
+      thr = fminf(thr, gmax[g]);
+    }
+  }
+  const float mxl = mx * kLog2e;
+  float tv[KT];
+  int ti[KT];
+  lm_init<KT>(tv, ti);
+  float se = 0.f;
+  int cnt = 0;
+  float* lrow = (p.lm_logits && m < p.M) ? p.lm_logits + (long long)m * p.ldo + n0 : nullptr;
+  const bool vec = (reinterpret_cast<uintptr_t>(lrow) & 15) == 0;
+#pragma unroll 1
+  for (int ch = 0; ch < NCH; ++ch) {
+    uint32_t r[32];
+    tmem_ld_32x32b_x32(tb + ch * 32, r);
+    tmem_ld_wait();
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int col = ch * 32 + j;
+      const bool in = !MASK || col < lim;
+      const float v = in ? __uint_as_float(r[j]) : -INFINITY;
+      se += lm_ex2(fmaf(v, kLog2e, -mxl));
+      if constexpr (KT > 1) {
+        if (in && v >= thr) {
+          if (cnt < kLmCap) {
+            cval[cnt * 128 + et] = v;
+            cidx[cnt * 128 + et] = col;
+            ++cnt;
+          } else {
+            lm_insert<KT>(tv, ti, v, n0 + col);
+          }
+        }
+      }
+    }
+    if (lrow) lm_store32(lrow + ch * 32, r, MASK ? lim - ch * 32 : 32, vec);
+  }
+  if constexpr (KT == 1) {
+    tv[0] = best;
+    ti[0] = n0 + best_c;
+  } else {
+#pragma unroll 1
+    for (int i = 0; i < cnt; ++i) lm_insert<KT>(tv, ti, cval[i * 128 + et], n0 + cidx[i * 128 + et]);
+  }
+  if (m < p.M) {
+    const long long e = (long long)m * num_n + n_blk;
+    p.lm_stats[e] = make_float2(mx, se);
+    int2* tp = p.lm_top + e * KT;
+#pragma unroll
+    for (int i = 0; i < KT; ++i) tp[i] = make_int2(__float_as_int(tv[i]), ti[i]);
+  }
+}
+
 template <int BN, int MT>
 struct SmCfg {
   static constexpr uint32_t A_BYTES = MT * BM * BK * 2;
@@ -622,6 +745,25 @@ __global__ void __launch_bounds__(192, 1)
         }
       }
     }
+  } else if constexpr (EPI == EPI_LM1 || EPI == EPI_LM8) {
+    constexpr int KT = EPI == EPI_LM1 ? 1 : 8;
+    static_assert((size_t)kLmCap * 128 * 8 <= C::RING_BYTES, "candidate lists fit in the ring");
+    if (warp >= 2 && have) {
+      const int et = threadIdx.x - 64;
+      float* cval = reinterpret_cast<float*>(smem);
+      int* cidx = reinterpret_cast<int*>(smem + kLmCap * 128 * 4);
+      const int n0 = n_blk * BN;
+      const int lim = p.N - n0;
+#pragma unroll 1
+      for (int mt = 0; mt < MT; ++mt) {
+        const int m = m_blk * TM + mt * BM + quarter * 32 + lane;
+        const uint32_t tb = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(mt * BN);
+        if (lim >= BN)
+          lm_row<BN, KT, false>(p, tb, m, n0, lim, num_n, n_blk, cval, cidx, et);
+        else
+          lm_row<BN, KT, true>(p, tb, m, n0, lim, num_n, n_blk, cval, cidx, et);
+      }
+    }
   } else {
     // Split-K partial: the f32 tile of this K split goes to slice `split`
     // (out + split * group_stride); the consuming kernel adds the slices in
@@ -724,6 +866,8 @@ bool pdl_enabled() {
 cudaError_t gemm_small_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args,
                               cudaStream_t stream) {
   if (args.splits < 1 || (epi == EPI_SLICES && args.N % 4)) return cudaErrorInvalidValue;
+  if ((epi == EPI_LM1 || epi == EPI_LM8) && (args.splits != 1 || !args.lm_stats || !args.lm_top))
+    return cudaErrorInvalidValue;
 #define OUTLETS_SM_CASE(BNV, EV, MTV) \
   if (bn == BNV && epi == EV && mt == MTV) return launch_small<BNV, EV, MTV>(a_maps, args, stream);
   OUTLETS_SM_CASE(256, EPI_SLICES, 2)
@@ -736,6 +880,19 @@ cudaError_t gemm_small_launch(const CUtensorMap a_maps[3], int bn, int epi, int 
   OUTLETS_SM_CASE(192, EPI_SWIGLU, 1)
   OUTLETS_SM_CASE(128, EPI_SWIGLU, 2)
   OUTLETS_SM_CASE(128, EPI_SWIGLU, 1)
+  // draft LM head: tile widths the host's wave model chooses from
+  OUTLETS_SM_CASE(256, EPI_LM8, 2)
+  OUTLETS_SM_CASE(256, EPI_LM8, 1)
+  OUTLETS_SM_CASE(224, EPI_LM8, 2)
+  OUTLETS_SM_CASE(224, EPI_LM8, 1)
+  OUTLETS_SM_CASE(128, EPI_LM8, 2)
+  OUTLETS_SM_CASE(128, EPI_LM8, 1)
+  OUTLETS_SM_CASE(256, EPI_LM1, 2)
+  OUTLETS_SM_CASE(256, EPI_LM1, 1)
+  OUTLETS_SM_CASE(224, EPI_LM1, 2)
+  OUTLETS_SM_CASE(224, EPI_LM1, 1)
+  OUTLETS_SM_CASE(128, EPI_LM1, 2)
+  OUTLETS_SM_CASE(128, EPI_LM1, 1)
 #undef OUTLETS_SM_CASE
   return cudaErrorInvalidValue;
 }

@@ -56,7 +56,14 @@ enum Epi : int {
   EPI_SWIGLU = 2,     // B rows interleaved in blocks of 32 [gate | up]; out act = silu(g) * u
   EPI_BIAS_RELU = 3,  // out f32 = max(acc + bias, 0)
   EPI_SLICES = 6,     // small M: split-K, K split s writes its f32 partial to slice s (summed by the consumer)
+  EPI_LM1 = 7,        // draft LM head (Eq. 2): per (row, N tile) softmax statistics and best column
+  EPI_LM8 = 8,        // same with the 8 best columns
 };
+
+// Draft LM head partials, one entry per (row, N tile), row-major [rows][tiles]:
+//   stats: (max logit m_t, sum over the tile's columns of exp(logit - m_t))
+//   top:   the tile's KT best (logit bits, token id) pairs, best first
+// (order: larger logit, then smaller id; empty places hold (-inf, INT_MAX)).
 
 // B operands (weights) live in a k-block-major, pre-swizzled layout owned by the
 // library: element (n, k) of a [N, K] weight is stored at
@@ -80,6 +87,9 @@ struct GemmArgs {
   long long ldr;
   const float* bias;      // EPI_BIAS_RELU
   int* err;
+  float* lm_logits;       // EPI_LM*: optional f32 logits [M, N] with row stride ldo (null: not stored)
+  float2* lm_stats;       // EPI_LM*: partials [M][tiles], layout above
+  int2* lm_top;           // EPI_LM*: partials [M][tiles][KT]
 };
 
 // tcgen05 path (bf16 operands).  a_maps: 3 tensor maps over the A pieces (box
@@ -93,6 +103,17 @@ cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt,
 //     its f32 partial [M, N] to out + s * group_stride (N % 4 == 0).
 cudaError_t gemm_small_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt, const GemmArgs& args,
                               cudaStream_t stream);
+
+// Draft LM head, CUDA-core path: partials of tiles of tile_w columns from f32
+// logits [rows, V] (row stride ld); kt is 1 or 8.
+cudaError_t lm_tile_stats_f32_launch(const float* logits, long long ld, int rows, int V, int tile_w, int kt,
+                                     float2* stats, int2* top, cudaStream_t stream);
+
+// Draft LM head: combines the n_tiles partials of each row into the row's
+// logsumexp and its k (<= kt) best tokens with their log-probabilities
+// (ids, logprob: [rows, k]; lse: [rows] or null).  n_tiles <= 2048.
+cudaError_t lm_merge_launch(const float2* stats, const int2* top, int n_tiles, int kt, int rows, int k, int* ids,
+                            float* logprob, float* lse, cudaStream_t stream);
 
 // CUDA-core path of the f32 configuration.  a[0..2]: A pieces with row stride k_per_map.
 cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int epi, const GemmArgs& args,

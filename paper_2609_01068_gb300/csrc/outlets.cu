@@ -36,6 +36,9 @@ constexpr int kMinTapChunkRows = 2048;
 constexpr int kSplitLen = 512;        // shortest split-KV work item (keys)
 constexpr int kDecodeCtasPerSm = 3;   // resident decode-attention CTAs per SM
 constexpr int kRing = 4;
+constexpr int kMaxVocab = 262144;     // draft head: at most 2048 tiles of 128 columns per row
+constexpr int kLmRowsPerPass = 256;   // draft head rows per GEMM + merge pass (one 256-row tile)
+constexpr int kLmTileF32 = 256;       // draft head tile width of the f32 path
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -119,6 +122,17 @@ struct outlets_ctx {
   size_t esz = 2;
   int d = 0, H = 0, KVH = 0, hd = 0, F = 0, Fp = 0, qkv_n = 0, attn_w = 0, max_rows = 0;
   bool gated = false;        // gated attention: QKV carries H*hd gate columns after q, k, v
+  // draft LM head (Eq. 2): weights, per (row, tile) partials, outputs of host callers
+  int V = 0;
+  void* w_lm = nullptr;
+  long long np_lm = 0;
+  int lm_rows_cap = 0;       // rows per GEMM + merge pass
+  float2* lm_stats = nullptr;
+  int2* lm_top = nullptr;
+  int* lm_ids = nullptr;
+  float *lm_lp = nullptr, *lm_lse = nullptr;
+  float* lm_logits_ws = nullptr;  // f32 path: logits of one pass
+  float* lm_logits_stage = nullptr;  // host `logits` callers: one pass, copied out (allocated on first use)
   void* vt = nullptr;        // V^T [KVH * hd, vt_ld] for the tcgen05 prefill attention (bf16)
   long long vt_ld = 0;
   void* gate_act = nullptr;  // [max_rows, H*hd] sigmoid(gate), act dtype
@@ -294,6 +308,7 @@ outlets_status validate_config(const outlets_config* cfg, std::string& why) {
   if (cfg->head_dim <= 0 || cfg->head_dim % 16) return bad("head_dim must be a positive multiple of 16");
   if ((cfg->n_heads * cfg->head_dim) % 64) return bad("n_heads * head_dim must be a multiple of 64");
   if (cfg->ffn_dim <= 0) return bad("ffn_dim must be positive");
+  if (cfg->vocab != 0 && (cfg->vocab < 8 || cfg->vocab > kMaxVocab)) return bad("vocab must be 0 or in 8..262144");
   if (cfg->n_head_hidden < 1 || cfg->n_head_hidden > OUTLETS_MAX_HEAD_HIDDEN)
     return bad("n_head_hidden must be in 1..OUTLETS_MAX_HEAD_HIDDEN");
   for (int i = 0; i < cfg->n_head_hidden; ++i)
@@ -685,6 +700,109 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   return OUTLETS_OK;
 }
 
+// Draft LM head tile width (tensor-core path): the one of 256, 224, 128 with
+// the smallest estimated time, waves x per-tile time.  A tile streams K/64
+// blocks of A and W_lm tiles (about 90 GB/s per SM) or is bound by its MMAs
+// (about 11.5 TFLOP/s per SM), whichever is slower, and then reduces its
+// logits on chip (the epilogue, about 45 ps per logit).  Narrower tiles fill
+// the last wave better (V = 128256 on 152 SMs: 224 gives 3.8 waves).
+int lm_tile_width(const outlets_ctx* c, int rows) {
+  const double tm = rows <= 128 ? 128.0 : 256.0;
+  const double kb = (double)cdiv(c->d, 64);
+  int best = 256;
+  double best_t = -1.0;
+  for (int bn : {256, 224, 128}) {
+    const double waves = (double)cdiv(cdiv(c->V, bn), c->num_sms);
+    const double ingest = (tm + bn) * 128.0 / 90e3;
+    const double mma = 2.0 * tm * bn * 64.0 / 11.5e6;
+    const double t = waves * (kb * std::max(ingest, mma) + tm * bn * 4.5e-5);
+    if (best_t < 0 || t < best_t) {
+      best_t = t;
+      best = bn;
+    }
+  }
+  return best;
+}
+
+outlets_status check_draft(outlets_ctx* c, const outlets_draft_out* o) {
+  if (!o) return c->fail(OUTLETS_EINVAL, "draft outputs must not be NULL");
+  if (c->V == 0) return c->fail(OUTLETS_EUNSUPPORTED, "the context has no draft head (vocab == 0)");
+  if (o->k < 1 || o->k > OUTLETS_MAX_TOPK || o->k > c->V)
+    return c->fail(OUTLETS_EINVAL, "draft k must be in 1 .. min(OUTLETS_MAX_TOPK, vocab)");
+  if (!o->topk_ids || !o->topk_logprob) return c->fail(OUTLETS_EINVAL, "topk_ids and topk_logprob must not be NULL");
+  return OUTLETS_OK;
+}
+
+// Draft LM head (Sec. 4.2, Eq. 2) on rows states h [rows, d] (act dtype, on the
+// device), in passes of lm_rows_cap rows: GEMM with the on-chip softmax/top-k
+// epilogue (CUDA-core path: logits, then tile statistics), then the merge.
+// Device outputs are written in place; host outputs go through the context's
+// buffers and are copied on the stream.
+outlets_status run_draft(outlets_ctx* c, const void* h, int rows, const outlets_draft_out& o, cudaStream_t s) {
+  if (rows == 0) return OUTLETS_OK;
+  const int V = c->V, d = c->d, k = o.k, kt = k == 1 ? 1 : 8;
+  int* ids = is_device_ptr(o.topk_ids) ? o.topk_ids : c->lm_ids;
+  float* lp = is_device_ptr(o.topk_logprob) ? o.topk_logprob : c->lm_lp;
+  float* lse = o.logsumexp ? (is_device_ptr(o.logsumexp) ? o.logsumexp : c->lm_lse) : nullptr;
+  const bool host_logits = o.logits && !is_device_ptr(o.logits);
+  if ((ids == c->lm_ids || lp == c->lm_lp || lse == c->lm_lse) && rows > c->max_rows)
+    return c->fail(OUTLETS_ECAPACITY, "rows exceed the context's output buffers (max_tokens / max_batch)");
+  if (host_logits && !c->lm_logits_stage) {
+    c->lm_logits_stage = (float*)c->alloc((size_t)c->lm_rows_cap * V * 4);
+    if (!c->lm_logits_stage) return c->fail(OUTLETS_ENOMEM, "draft logits staging allocation failed");
+  }
+  c->stage_begin(OUTLETS_S_DRAFT);
+  int n_launch = 0;
+  for (int g0 = 0; g0 < rows; g0 += c->lm_rows_cap) {
+    const int gr = std::min(c->lm_rows_cap, rows - g0);
+    const void* hg = static_cast<const char*>(h) + (size_t)g0 * d * c->esz;
+    float* lg = o.logits ? (host_logits ? c->lm_logits_stage : o.logits + (size_t)g0 * V) : nullptr;
+    const void* a1[3] = {hg, hg, hg};
+    int n_tiles = 0;
+    if (c->bf16) {
+      const int bn = lm_tile_width(c, gr);
+      n_tiles = (int)cdiv(V, bn);
+      CUtensorMap am[3];
+      OUT_TRY(a_maps(c, a1, 1, d, d, gr, am));
+      GemmArgs g{};
+      g.M = gr;
+      g.N = V;
+      g.K = d;
+      g.b = c->w_lm;
+      g.b_np = c->np_lm;
+      g.k_per_map = d;
+      g.splits = 1;
+      g.group_m = 1;
+      g.ldo = V;
+      g.err = c->err_dev;
+      g.lm_logits = lg;
+      g.lm_stats = c->lm_stats;
+      g.lm_top = c->lm_top;
+      OUT_CK(c, gemm_small_launch(am, bn, kt == 1 ? EPI_LM1 : EPI_LM8, gr <= 128 ? 1 : 2, g, s));
+      n_launch += 1;
+    } else {
+      float* lw = lg ? lg : c->lm_logits_ws;
+      OUT_TRY(gemm_f32(c, a1, d, gr, c->w_lm, V, d, EPI_F32, lw, V, nullptr, 0, nullptr, s));
+      n_tiles = (int)cdiv(V, kLmTileF32);
+      OUT_CK(c, lm_tile_stats_f32_launch(lw, V, gr, V, kLmTileF32, kt, c->lm_stats, c->lm_top, s));
+      n_launch += 2;
+    }
+    OUT_CK(c, lm_merge_launch(c->lm_stats, c->lm_top, n_tiles, kt, gr, k, ids + (size_t)g0 * k,
+                              lp + (size_t)g0 * k, lse ? lse + g0 : nullptr, s));
+    n_launch += 1;
+    if (host_logits)
+      OUT_CK(c, cudaMemcpyAsync(o.logits + (size_t)g0 * V, lg, (size_t)gr * V * 4, cudaMemcpyDeviceToHost, s));
+  }
+  c->stage_end(n_launch);
+  if (ids != o.topk_ids)
+    OUT_CK(c, cudaMemcpyAsync(o.topk_ids, ids, (size_t)rows * k * sizeof(int), cudaMemcpyDeviceToHost, s));
+  if (lp != o.topk_logprob)
+    OUT_CK(c, cudaMemcpyAsync(o.topk_logprob, lp, (size_t)rows * k * 4, cudaMemcpyDeviceToHost, s));
+  if (lse && lse != o.logsumexp)
+    OUT_CK(c, cudaMemcpyAsync(o.logsumexp, lse, (size_t)rows * 4, cudaMemcpyDeviceToHost, s));
+  return OUTLETS_OK;
+}
+
 // FC (Eq. 1) -> input RMSNorm -> QKV projection.  Fills the input side of the
 // RoPE arguments (fused qkv rows, or split slices on the small-M path).
 struct QkvSrc {
@@ -834,6 +952,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
     if (!p) return OUTLETS_EINVAL;
   for (int i = 0; i <= cfg->n_head_hidden; ++i)
     if (!w->head_w[i] || !w->head_b[i]) return OUTLETS_EINVAL;
+  if (cfg->vocab > 0 && !w->w_lm) return OUTLETS_EINVAL;
   if (cudaSetDevice(cfg->device) != cudaSuccess) {
     cudaGetLastError();
     return OUTLETS_ECUDA;
@@ -856,6 +975,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->gated = w->w_attn_gate != nullptr;
   c->qkv_n = (c->H + 2 * c->KVH) * c->hd + (c->gated ? c->attn_w : 0);
   c->max_rows = std::max(cfg->max_tokens, cfg->max_batch);
+  c->V = cfg->vocab;
   c->head_dims.push_back(c->d);
   for (int i = 0; i < cfg->n_head_hidden; ++i) c->head_dims.push_back(cfg->head_hidden[i]);
   c->head_dims.push_back(1);
@@ -876,6 +996,9 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->np_gu = np_of(2 * c->Fp);
   c->np_down = np_of(d);
   c->np_h0 = np_of(c->head_dims[1]);
+  // draft LM head: rows padded so that a tile of any of its widths (256, 224, 128) stays in bounds
+  if (c->V > 0 && c->bf16)
+    c->np_lm = std::max({cdiv(c->V, 256) * 256, cdiv(c->V, 224) * 224, cdiv(c->V, 128) * 128});
   auto rows_of = [&](long long np, int n) -> size_t { return (size_t)(np ? np : n); };
   c->w_proj = c->alloc(rows_of(c->np_proj, d) * 3 * d * es);
   c->w_qkv = c->alloc(rows_of(c->np_qkv, c->qkv_n) * d * es);
@@ -891,6 +1014,17 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->head_w0 = c->alloc(rows_of(c->np_h0, c->head_dims[1]) * d * es);
   for (int i = 1; i < nl; ++i) c->head_wf[i] = (float*)c->alloc((size_t)c->head_dims[i + 1] * c->head_dims[i] * 4);
   for (int i = 0; i < nl; ++i) c->head_b[i] = (float*)c->alloc((size_t)c->head_dims[i + 1] * 4);
+  if (c->V > 0) {
+    c->w_lm = c->alloc(rows_of(c->np_lm, c->V) * d * es);
+    c->lm_rows_cap = std::min(c->max_rows, kLmRowsPerPass);
+    const size_t tiles = (size_t)cdiv(c->V, c->bf16 ? 128 : kLmTileF32);
+    c->lm_stats = (float2*)c->alloc((size_t)c->lm_rows_cap * tiles * sizeof(float2));
+    c->lm_top = (int2*)c->alloc((size_t)c->lm_rows_cap * tiles * OUTLETS_MAX_TOPK * sizeof(int2));
+    c->lm_ids = (int*)c->alloc((size_t)c->max_rows * OUTLETS_MAX_TOPK * sizeof(int));
+    c->lm_lp = (float*)c->alloc((size_t)c->max_rows * OUTLETS_MAX_TOPK * 4);
+    c->lm_lse = (float*)c->alloc((size_t)c->max_rows * 4);
+    if (!c->bf16) c->lm_logits_ws = (float*)c->alloc((size_t)c->lm_rows_cap * c->V * 4);
+  }
   c->rope_cos = (float*)c->alloc((size_t)cfg->max_position * (c->hd / 2) * 4);
   c->rope_sin = (float*)c->alloc((size_t)cfg->max_position * (c->hd / 2) * 4);
   // ---- workspace
@@ -974,6 +1108,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   up(w->w_up, c->F, d, c->w_gu, d, 2, 0, c->np_gu);
   up(w->w_down, d, c->F, c->w_down, c->Fp, 0, 0, c->np_down);
   up(w->head_w[0], c->head_dims[1], d, c->head_w0, d, 0, 0, c->np_h0);
+  if (c->V > 0) up(w->w_lm, c->V, d, c->w_lm, d, 0, 0, c->np_lm);
   cudaFree(stage);
   if (st != OUTLETS_OK) return cleanup_fail(st);
   auto h2d = [&](void* dst, const void* src, size_t bytes) {
@@ -1071,7 +1206,8 @@ outlets_status outlets_profile_read(outlets_ctx* c, double* ms, int32_t* count) 
 const char* outlets_stage_name(int32_t s) {
   static const char* names[OUTLETS_N_STAGES] = {"fc_gemm",      "rmsnorm_in",     "qkv_gemm",    "rope_scatter",
                                                 "attention",    "o_gemm",         "rmsnorm_post", "gateup_swiglu_gemm",
-                                                "down_gemm",    "final_rmsnorm",  "length_head"};
+                                                "down_gemm",    "final_rmsnorm",  "length_head",
+                                                "draft_head"};
   return (s >= 0 && s < OUTLETS_N_STAGES) ? names[s] : "";
 }
 
@@ -1160,11 +1296,13 @@ outlets_status outlets_check(outlets_ctx* c, void* stream) {
   return OUTLETS_OK;
 }
 
-outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3], const int32_t* cu, int32_t B,
-                                       int32_t T, outlets_kv* kv, const int32_t* slots, uint32_t flags,
-                                       float* z_out, float* len_out, void* stream) {
-  if (!c) return OUTLETS_EINVAL;
-  c->err.clear();
+}  // extern "C"
+
+namespace {
+
+outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const int32_t* cu, int32_t B, int32_t T,
+                               outlets_kv* kv, const int32_t* slots, uint32_t flags, float* z_out, float* len_out,
+                               const outlets_draft_out* draft, void* stream) {
   cudaStream_t s = (cudaStream_t)stream;
   if (!taps || !cu || !z_out) return c->fail(OUTLETS_EINVAL, "taps, cu_seqlens and z_out must not be NULL");
   if (flags & ~OUTLETS_ALL_TOKENS) return c->fail(OUTLETS_EINVAL, "unknown flag");
@@ -1351,15 +1489,15 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
   }
   c->stage_end(1);
   OUT_TRY(run_tail(c, T, out_rows, all_tokens ? nullptr : m + off_last, c->z, c->len, s));
+  if (draft) OUT_TRY(run_draft(c, c->hn, out_rows, *draft, s));
   c->last_rows = T;
   c->last_out_rows = out_rows;
   return end_call(c, out_rows, z_out, len_out, s);
 }
 
-outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], int32_t B, outlets_kv* kv,
-                                    const int32_t* slots, float* z_out, float* len_out, void* stream) {
-  if (!c) return OUTLETS_EINVAL;
-  c->err.clear();
+outlets_status predict_step(outlets_ctx* c, const void* const taps[3], int32_t B, outlets_kv* kv,
+                            const int32_t* slots, float* z_out, float* len_out, const outlets_draft_out* draft,
+                            void* stream) {
   cudaStream_t s = (cudaStream_t)stream;
   if (!taps || !kv || !slots || !z_out) return c->fail(OUTLETS_EINVAL, "taps, kv, slots and z_out must not be NULL");
   if (kv->ctx != c) return c->fail(OUTLETS_EINVAL, "kv belongs to another context");
@@ -1498,9 +1636,65 @@ outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], i
     }
   }
   OUT_TRY(run_tail(c, B, B, nullptr, c->z, c->len, s));
+  if (draft) OUT_TRY(run_draft(c, c->hn, B, *draft, s));
   c->last_rows = B;
   c->last_out_rows = B;
   return end_call(c, B, z_out, len_out, s);
+}
+
+}  // namespace
+
+extern "C" {
+
+outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3], const int32_t* cu, int32_t B,
+                                       int32_t T, outlets_kv* kv, const int32_t* slots, uint32_t flags,
+                                       float* z_out, float* len_out, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  return predict_prefill(c, taps, cu, B, T, kv, slots, flags, z_out, len_out, nullptr, stream);
+}
+
+outlets_status outlets_predict_prefill_dual(outlets_ctx* c, const void* const taps[3], const int32_t* cu,
+                                            int32_t B, int32_t T, outlets_kv* kv, const int32_t* slots,
+                                            uint32_t flags, float* z_out, float* len_out,
+                                            const outlets_draft_out* draft, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  OUT_TRY(check_draft(c, draft));
+  return predict_prefill(c, taps, cu, B, T, kv, slots, flags, z_out, len_out, draft, stream);
+}
+
+outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], int32_t B, outlets_kv* kv,
+                                    const int32_t* slots, float* z_out, float* len_out, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  return predict_step(c, taps, B, kv, slots, z_out, len_out, nullptr, stream);
+}
+
+outlets_status outlets_predict_step_dual(outlets_ctx* c, const void* const taps[3], int32_t B, outlets_kv* kv,
+                                         const int32_t* slots, float* z_out, float* len_out,
+                                         const outlets_draft_out* draft, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  OUT_TRY(check_draft(c, draft));
+  return predict_step(c, taps, B, kv, slots, z_out, len_out, draft, stream);
+}
+
+outlets_status outlets_draft_head(outlets_ctx* c, const void* h_draft, int32_t rows, const outlets_draft_out* draft,
+                                  void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  OUT_TRY(check_draft(c, draft));
+  if (rows < 0) return c->fail(OUTLETS_EINVAL, "rows must be >= 0");
+  if (rows == 0) return OUTLETS_OK;
+  if (!h_draft || !is_device_ptr(h_draft) || reinterpret_cast<uintptr_t>(h_draft) % 16)
+    return c->fail(OUTLETS_EINVAL, "h_draft must be 16-byte aligned device memory");
+  cudaStream_t s = (cudaStream_t)stream;
+  OUT_TRY(begin_call(c, s));
+  OUT_TRY(run_draft(c, h_draft, rows, *draft, s));
+  OUT_CK(c, cudaEventRecord(c->done_ev, s));
+  c->have_prev = true;
+  return OUTLETS_OK;
 }
 
 outlets_status outlets_get_intermediate(outlets_ctx* c, int32_t which, void* dst, size_t dst_bytes,

@@ -20,7 +20,8 @@ STATUS_NAMES = ["OK", "EINVAL", "ENOMEM", "ECUDA", "EUNSUPPORTED", "ECAPACITY", 
 F32, BF16 = 0, 1
 ALL_TOKENS = 1
 T_FCTX, T_XIN, T_Q, T_ATTN, T_A, T_Y, T_HDRAFT = range(7)
-N_STAGES = 11
+N_STAGES = 12
+MAX_TOPK = 8
 
 c_i32, c_f32, c_vp = ctypes.c_int32, ctypes.c_float, ctypes.c_void_p
 
@@ -29,7 +30,7 @@ class Config(ctypes.Structure):
     _fields_ = [("d_model", c_i32), ("n_heads", c_i32), ("n_kv_heads", c_i32), ("head_dim", c_i32),
                 ("ffn_dim", c_i32), ("n_head_hidden", c_i32), ("head_hidden", c_i32 * MAX_HEAD_HIDDEN),
                 ("rope_theta", c_f32), ("rms_eps", c_f32), ("dtype", c_i32), ("max_tokens", c_i32),
-                ("max_batch", c_i32), ("max_position", c_i32), ("device", c_i32)]
+                ("max_batch", c_i32), ("max_position", c_i32), ("device", c_i32), ("vocab", c_i32)]
 
 
 _WNAMES = ["w_proj", "w_q", "w_k", "w_v", "w_o", "g_in", "g_post", "g_final", "w_gate", "w_up", "w_down"]
@@ -38,7 +39,11 @@ _WNAMES = ["w_proj", "w_q", "w_k", "w_v", "w_o", "g_in", "g_post", "g_final", "w
 class Weights(ctypes.Structure):
     _fields_ = [(n, c_vp) for n in _WNAMES] + [("head_w", c_vp * (MAX_HEAD_HIDDEN + 1)),
                                                ("head_b", c_vp * (MAX_HEAD_HIDDEN + 1)),
-                                               ("w_attn_gate", c_vp)]
+                                               ("w_attn_gate", c_vp), ("w_lm", c_vp)]
+
+
+class DraftOut(ctypes.Structure):
+    _fields_ = [("k", c_i32), ("topk_ids", c_vp), ("topk_logprob", c_vp), ("logsumexp", c_vp), ("logits", c_vp)]
 
 
 class TensorInfo(ctypes.Structure):
@@ -76,6 +81,10 @@ def load():
         "outlets_predict_prefill": (c_i32, [c_vp, P(c_vp), c_vp, c_i32, c_i32, c_vp, c_vp, ctypes.c_uint32,
                                             c_vp, c_vp, c_vp]),
         "outlets_predict_step": (c_i32, [c_vp, P(c_vp), c_i32, c_vp, c_vp, c_vp, c_vp, c_vp]),
+        "outlets_predict_prefill_dual": (c_i32, [c_vp, P(c_vp), c_vp, c_i32, c_i32, c_vp, c_vp, ctypes.c_uint32,
+                                                 c_vp, c_vp, P(DraftOut), c_vp]),
+        "outlets_predict_step_dual": (c_i32, [c_vp, P(c_vp), c_i32, c_vp, c_vp, c_vp, c_vp, P(DraftOut), c_vp]),
+        "outlets_draft_head": (c_i32, [c_vp, c_vp, c_i32, P(DraftOut), c_vp]),
         "outlets_check": (c_i32, [c_vp, c_vp]),
         "outlets_get_intermediate": (c_i32, [c_vp, c_i32, c_vp, ctypes.c_size_t, P(TensorInfo), c_vp]),
         "outlets_profile_enable": (c_i32, [c_vp, c_i32]),
@@ -149,6 +158,12 @@ class Predictor:
             ga = np.ascontiguousarray(weights["w_attn_gate"], dtype=np.float32)
             keep["w_attn_gate"] = ga
             w.w_attn_gate = ga.ctypes.data
+        if weights.get("w_lm") is not None:  # draft LM head of the dual head (Eq. 2)
+            la = np.ascontiguousarray(weights["w_lm"], dtype=np.float32)
+            keep["w_lm"] = la
+            w.w_lm = la.ctypes.data
+            cfg.vocab = la.shape[0]
+        self.vocab = cfg.vocab
         h = c_vp()
         st = self.lib.outlets_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h))
         if st != OK:
@@ -212,6 +227,64 @@ class Predictor:
         if st != OK:
             self._raise(st)
         return z_out, len_out
+
+    # -- dual head (Sec. 4.2, Eq. 2)
+    def _draft_out(self, n, k, like, logits, out=None):
+        """DraftOut for n rows: torch outputs on like's device unless `out` supplies them."""
+        import torch
+        if out is None:
+            dev = like.device if hasattr(like, "device") else torch.device("cpu")
+            out = {"ids": torch.empty((n, k), dtype=torch.int32, device=dev),
+                   "logprob": torch.empty((n, k), dtype=torch.float32, device=dev),
+                   "lse": torch.empty(n, dtype=torch.float32, device=dev)}
+            if logits:
+                out["logits"] = torch.empty((n, self.vocab), dtype=torch.float32, device=dev)
+        d = DraftOut()
+        d.k = k
+        d.topk_ids, d.topk_logprob = _ptr(out["ids"]), _ptr(out["logprob"])
+        d.logsumexp, d.logits = _ptr(out.get("lse")), _ptr(out.get("logits"))
+        return d, out
+
+    def prefill_dual(self, taps, cu_seqlens, k, kv=None, slots=None, all_tokens=False, logits=False, out=None,
+                     z_out=None, len_out=None, stream=None):
+        """Static prediction plus the draft head on the same rows:
+        (z_hat, length_hat, {"ids", "logprob", "lse"[, "logits"]})."""
+        cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+        B, T = len(cu) - 1, int(cu[-1]) if len(cu) else 0
+        n_out = T if all_tokens else B
+        z_out, len_out = self._outputs(n_out, taps[0], z_out, len_out)
+        d, draft = self._draft_out(n_out, k, taps[0], logits, out)
+        tp = (c_vp * 3)(*[_ptr(t) for t in taps])
+        sl = None if slots is None else np.ascontiguousarray(slots, dtype=np.int32)
+        st = self.lib.outlets_predict_prefill_dual(self.h, tp, cu.ctypes.data, B, T, kv.h if kv else None,
+                                                   None if sl is None else sl.ctypes.data,
+                                                   ALL_TOKENS if all_tokens else 0, _ptr(z_out), _ptr(len_out),
+                                                   ctypes.byref(d), _stream_handle(stream))
+        if st != OK:
+            self._raise(st)
+        return z_out, len_out, draft
+
+    def step_dual(self, taps, kv, slots, k, logits=False, out=None, z_out=None, len_out=None, stream=None):
+        """Dynamic prediction plus the draft head: (z_hat, length_hat, draft outputs)."""
+        sl = np.ascontiguousarray(slots, dtype=np.int32)
+        B = len(sl)
+        z_out, len_out = self._outputs(B, taps[0], z_out, len_out)
+        d, draft = self._draft_out(B, k, taps[0], logits, out)
+        tp = (c_vp * 3)(*[_ptr(t) for t in taps])
+        st = self.lib.outlets_predict_step_dual(self.h, tp, B, kv.h, sl.ctypes.data, _ptr(z_out), _ptr(len_out),
+                                                ctypes.byref(d), _stream_handle(stream))
+        if st != OK:
+            self._raise(st)
+        return z_out, len_out, draft
+
+    def draft_head(self, h_draft, k, logits=False, out=None, stream=None):
+        """The draft head alone on device states h_draft [rows, d]."""
+        rows = int(h_draft.shape[0])
+        d, draft = self._draft_out(rows, k, h_draft, logits, out)
+        st = self.lib.outlets_draft_head(self.h, _ptr(h_draft), rows, ctypes.byref(d), _stream_handle(stream))
+        if st != OK:
+            self._raise(st)
+        return draft
 
     def selftest_bounded_wait(self, timeout_ns=1_000_000, stream=None):
         """Enqueue a kernel whose bounded wait runs out (see outlets_check)."""

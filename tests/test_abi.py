@@ -35,7 +35,8 @@ def built_lib():
 def test_header_declares_the_entry_points():
     names = _declared_functions()
     for must in ("outlets_create", "outlets_predict_prefill", "outlets_predict_step", "outlets_kv_create",
-                 "outlets_destroy", "outlets_last_error"):
+                 "outlets_destroy", "outlets_last_error", "outlets_predict_prefill_dual",
+                 "outlets_predict_step_dual", "outlets_draft_head"):
         assert must in names
 
 
@@ -62,6 +63,20 @@ def test_create_rejects_invalid_config_on_host(built_lib):
     cfg.dtype = O.BF16
     cfg.head_dim = 96  # bf16 attention supports 64 / 128
     assert built_lib.outlets_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h)) == O.EINVAL
+    cfg.head_dim = 64
+    # every weight pointer set (never read: the config is checked first), so
+    # only the draft head width makes these configurations invalid
+    dummy = (ctypes.c_float * 4)()
+    for name, _ in O.Weights._fields_:
+        if name in ("head_w", "head_b"):
+            for i in range(cfg.n_head_hidden + 1):
+                getattr(w, name)[i] = ctypes.addressof(dummy)
+        else:
+            setattr(w, name, ctypes.addressof(dummy))
+    for vocab in (5, -1, 262145):  # outside 8 .. 262144
+        cfg.vocab = vocab
+        assert built_lib.outlets_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h)) == O.EINVAL
+        assert not h.value
 
 
 def test_null_handles_are_rejected(built_lib):
@@ -70,6 +85,11 @@ def test_null_handles_are_rejected(built_lib):
     taps = (ctypes.c_void_p * 3)()
     assert built_lib.outlets_predict_prefill(None, taps, cu, 1, 4, None, None, 0, z, None, None) == O.EINVAL
     assert built_lib.outlets_predict_step(None, taps, 1, None, None, z, None, None) == O.EINVAL
+    d = O.DraftOut()
+    assert built_lib.outlets_predict_prefill_dual(None, taps, cu, 1, 4, None, None, 0, z, None, ctypes.byref(d),
+                                                  None) == O.EINVAL
+    assert built_lib.outlets_predict_step_dual(None, taps, 1, None, None, z, None, ctypes.byref(d), None) == O.EINVAL
+    assert built_lib.outlets_draft_head(None, None, 1, ctypes.byref(d), None) == O.EINVAL
     assert built_lib.outlets_kv_reset_slot(None, 0) == O.EINVAL
     assert built_lib.outlets_kv_slot_length(None, 0) == -1
     assert built_lib.outlets_kv_free_pages(None) == -1

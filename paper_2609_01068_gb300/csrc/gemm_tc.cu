@@ -441,6 +441,10 @@ cudaError_t launch_one(const CUtensorMap a_maps[3], const GemmArgs& args, int nu
 // WS - AS blocks ahead); with AS == WS this is one ring holding both tiles of
 // a K block, which is what the latency of both operands needs.
 // ---------------------------------------------------------------- draft LM head epilogue (Eq. 2)
+// Epilogue warps of the draft LM head kernel: 8 (two per TMEM lane quarter;
+// the two warps of a quarter take the two column halves of the tile).
+constexpr int kLmEpiWarps = 8;
+constexpr int kLmEpiThreads = kLmEpiWarps * 32;
 // Candidate places per epilogue thread in the idle operand ring.
 constexpr int kLmCap = 64;
 
@@ -463,29 +467,60 @@ __device__ __forceinline__ void lm_store32(float* dst, const uint32_t (&r)[32], 
   }
 }
 
-// One row of a draft LM head tile: the calling thread owns TMEM lane `tb`'s
-// row (global row m, columns n0 .. n0 + BN - 1, of which the first lim are
-// inside the vocabulary when MASK) and writes the row's partials (kernels.h).
-//  pass 1 reads the row from TMEM and takes the maximum of each of 8 column
-//         groups (column mod 8); the smallest group maximum is reached by 8
-//         distinct columns, so it bounds the tile's 8th best logit from below;
-//  pass 2 re-reads the row, sums exp(logit - max) and moves the logits that
-//         reach the bound (a few percent of a smooth row) to this thread's
-//         candidate list in shared memory (column-major over the 128 threads);
-//  then only the candidates go through the sorted insertion, after the scan,
-//  so the lanes of a warp do not diverge on every logit.  A list that fills
-//  up inserts its overflow directly (the order of insertion does not matter).
+// Inserts candidate list entries 0 .. cnt-1 of thread et into the sorted list.
+template <int KT>
+__device__ __forceinline__ void lm_flush(float (&tv)[KT], int (&ti)[KT], const float* cval, const int* cidx, int et,
+                                         int n0, int cnt) {
+#pragma unroll 1
+  for (int i = 0; i < cnt; ++i)
+    lm_insert<KT>(tv, ti, cval[i * kLmEpiThreads + et], n0 + cidx[i * kLmEpiThreads + et]);
+}
+
+// One row of one column half of a draft LM head tile.  The calling thread
+// owns TMEM lane `tb`'s row (global row m) and chunks ch0 .. ch1-1 of 32
+// columns (tile columns n0 + 32 ch ..; the first lim tile columns are inside
+// the vocabulary when MASK), and writes the partials (kernels.h) of partial
+// tile pt (num_pt partial tiles per row).
+//  pass 1 reads the columns from TMEM and takes the maximum of each of 8
+//         column groups (column mod 8); the smallest group maximum is reached
+//         by 8 distinct columns, so it bounds the half's 8th best logit from
+//         below.  A bound over the whole row comes from the row's 8 slots:
+//         slot pt mod 8 keeps the largest maximum of the partial tiles it has
+//         seen, so the slots hold logits of 8 distinct columns and their
+//         minimum never exceeds the row's 8th best logit.  The slots are read
+//         before pass 1 (the loads overlap it) and this half's maximum is
+//         added after it.  Once every slot has seen a few tiles the bound is
+//         close to the row's 8th best and later tiles keep almost no
+//         candidates; which tile sees which bound depends on timing, the
+//         merged top-k does not.
+//  pass 2 re-reads the columns and sums exp(logit - max) in one branch-free
+//         block per chunk; only a chunk in which some lane of the warp has a
+//         logit at or above the bound goes through candidate collection,
+//         which moves those logits to the thread's list in shared memory.
+//  The list goes through the sorted insertion after the scan (and before a
+//  chunk whenever fewer than 32 places are left, raising the bound to the
+//  current KT-th best), so the lanes of a warp do not diverge on every logit.
 template <int BN, int KT, bool MASK>
-__device__ __forceinline__ void lm_row(const GemmArgs& p, uint32_t tb, int m, int n0, int lim, int num_n,
-                                       int n_blk, float* cval, int* cidx, int et) {
-  constexpr int NCH = BN / 32;
+__device__ __forceinline__ void lm_row(const GemmArgs& p, uint32_t tb, int m, int n0, int lim, int ch0, int ch1,
+                                       int pt, int num_pt, float* cval, int* cidx, int et) {
+  static_assert(kLmCap >= 64, "a flushed list takes a whole chunk");
+  // rows past M read zero-filled A: nothing to do there (tcgen05.ld is
+  // warp-collective, so a warp with any live row runs the scan as a whole)
+  const bool live = m < p.M;
+  if (!__any_sync(0xffffffffu, live)) return;
+  int* slot = p.lm_bound + (long long)(live ? m : 0) * kLmBoundSlots;
+  int4 sa = make_int4(kLmBoundInit, kLmBoundInit, kLmBoundInit, kLmBoundInit), sb = sa;
+  if (KT > 1 && live) {
+    sa = __ldcg(reinterpret_cast<const int4*>(slot));
+    sb = __ldcg(reinterpret_cast<const int4*>(slot) + 1);
+  }
   float gmax[8];
 #pragma unroll
   for (int g = 0; g < 8; ++g) gmax[g] = -INFINITY;
   float best = -INFINITY;
   int best_c = INT_MAX;
 #pragma unroll 1
-  for (int ch = 0; ch < NCH; ++ch) {
+  for (int ch = ch0; ch < ch1; ++ch) {
     uint32_t r[32];
     tmem_ld_32x32b_x32(tb + ch * 32, r);
     tmem_ld_wait();
@@ -512,35 +547,58 @@ __device__ __forceinline__ void lm_row(const GemmArgs& p, uint32_t tb, int m, in
       mx = fmaxf(mx, gmax[g]);
       thr = fminf(thr, gmax[g]);
     }
+    if (live) {
+      atomicMax(slot + (pt & (kLmBoundSlots - 1)), lm_key(mx));
+      const int kmin = min(min(min(sa.x, sa.y), min(sa.z, sa.w)), min(min(sb.x, sb.y), min(sb.z, sb.w)));
+      thr = fmaxf(thr, lm_unkey(kmin));
+    }
   }
-  const float mxl = mx * kLog2e;
+  const float mxl = mx == -INFINITY ? 0.f : mx * kLog2e;  // a half past the vocabulary: sum 0
   float tv[KT];
   int ti[KT];
   lm_init<KT>(tv, ti);
   float se = 0.f;
   int cnt = 0;
-  float* lrow = (p.lm_logits && m < p.M) ? p.lm_logits + (long long)m * p.ldo + n0 : nullptr;
+  float* lrow = (p.lm_logits && live) ? p.lm_logits + (long long)m * p.ldo + n0 : nullptr;
   const bool vec = (reinterpret_cast<uintptr_t>(lrow) & 15) == 0;
 #pragma unroll 1
-  for (int ch = 0; ch < NCH; ++ch) {
+  for (int ch = ch0; ch < ch1; ++ch) {
+    if constexpr (KT > 1) {
+      if (cnt > kLmCap - 32) {
+        lm_flush<KT>(tv, ti, cval, cidx, et, n0, cnt);
+        cnt = 0;
+        thr = fmaxf(thr, tv[KT - 1]);
+      }
+    }
     uint32_t r[32];
     tmem_ld_32x32b_x32(tb + ch * 32, r);
     tmem_ld_wait();
+    if (MASK) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (ch * 32 + j >= lim) r[j] = __float_as_uint(-INFINITY);
+    }
+    // softmax sum: one branch-free block (four partial sums), the chunk's max on the side
+    float s4[4] = {0.f, 0.f, 0.f, 0.f};
+    float cmx = -INFINITY;
 #pragma unroll
     for (int j = 0; j < 32; ++j) {
-      const int col = ch * 32 + j;
-      const bool in = !MASK || col < lim;
-      const float v = in ? __uint_as_float(r[j]) : -INFINITY;
-      se += lm_ex2(fmaf(v, kLog2e, -mxl));
-      if constexpr (KT > 1) {
-        if (in && v >= thr) {
-          if (cnt < kLmCap) {
-            cval[cnt * 128 + et] = v;
-            cidx[cnt * 128 + et] = col;
-            ++cnt;
-          } else {
-            lm_insert<KT>(tv, ti, v, n0 + col);
+      const float v = __uint_as_float(r[j]);
+      s4[j & 3] += lm_ex2(fmaf(v, kLog2e, -mxl));
+      cmx = fmaxf(cmx, v);
+    }
+    se += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+    if constexpr (KT > 1) {
+      if (__any_sync(0xffffffffu, live && cmx >= thr)) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const float v = __uint_as_float(r[j]);
+          const bool take = live && v >= thr;
+          if (take) {
+            cval[cnt * kLmEpiThreads + et] = v;
+            cidx[cnt * kLmEpiThreads + et] = ch * 32 + j;
           }
+          cnt += take ? 1 : 0;
         }
       }
     }
@@ -548,13 +606,12 @@ __device__ __forceinline__ void lm_row(const GemmArgs& p, uint32_t tb, int m, in
   }
   if constexpr (KT == 1) {
     tv[0] = best;
-    ti[0] = n0 + best_c;
+    ti[0] = best_c == INT_MAX ? INT_MAX : n0 + best_c;
   } else {
-#pragma unroll 1
-    for (int i = 0; i < cnt; ++i) lm_insert<KT>(tv, ti, cval[i * 128 + et], n0 + cidx[i * 128 + et]);
+    lm_flush<KT>(tv, ti, cval, cidx, et, n0, cnt);
   }
-  if (m < p.M) {
-    const long long e = (long long)m * num_n + n_blk;
+  if (live) {
+    const long long e = (long long)m * num_pt + pt;
     p.lm_stats[e] = make_float2(mx, se);
     int2* tp = p.lm_top + e * KT;
 #pragma unroll
@@ -579,8 +636,15 @@ struct SmCfg {
   static_assert(TMEM_USED <= 512, "TMEM columns");
 };
 
+// Threads of a small-M GEMM CTA: producer warp, MMA warp, epilogue warps
+// (4; 8 for the draft LM head, whose epilogue is the longer part of a tile).
+template <int EPI>
+constexpr int small_threads() {
+  return (EPI == EPI_LM1 || EPI == EPI_LM8) ? 64 + kLmEpiThreads : 192;
+}
+
 template <int BN, int EPI, int MT>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(small_threads<EPI>(), 1)
     k_gemm_small(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_a1,
                  const __grid_constant__ CUtensorMap map_a2, const GemmArgs p) {
   using C = SmCfg<BN, MT>;
@@ -746,22 +810,27 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else if constexpr (EPI == EPI_LM1 || EPI == EPI_LM8) {
+    // warps 2..9: lane quarter warp % 4, column half (warp - 2) / 4; each half
+    // is its own partial tile (2 per N tile), so nothing is combined here
     constexpr int KT = EPI == EPI_LM1 ? 1 : 8;
-    static_assert((size_t)kLmCap * 128 * 8 <= C::RING_BYTES, "candidate lists fit in the ring");
+    constexpr int NCH = BN / 32, SPLIT = (NCH + 1) / 2;
+    static_assert((size_t)kLmCap * kLmEpiThreads * 8 <= C::RING_BYTES, "candidate lists fit in the ring");
     if (warp >= 2 && have) {
       const int et = threadIdx.x - 64;
+      const int half = (warp - 2) >> 2;
       float* cval = reinterpret_cast<float*>(smem);
-      int* cidx = reinterpret_cast<int*>(smem + kLmCap * 128 * 4);
+      int* cidx = reinterpret_cast<int*>(smem + kLmCap * kLmEpiThreads * 4);
       const int n0 = n_blk * BN;
       const int lim = p.N - n0;
+      const int ch0 = half ? SPLIT : 0, ch1 = half ? NCH : SPLIT;
 #pragma unroll 1
       for (int mt = 0; mt < MT; ++mt) {
         const int m = m_blk * TM + mt * BM + quarter * 32 + lane;
         const uint32_t tb = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(mt * BN);
         if (lim >= BN)
-          lm_row<BN, KT, false>(p, tb, m, n0, lim, num_n, n_blk, cval, cidx, et);
+          lm_row<BN, KT, false>(p, tb, m, n0, lim, ch0, ch1, 2 * n_blk + half, 2 * num_n, cval, cidx, et);
         else
-          lm_row<BN, KT, true>(p, tb, m, n0, lim, num_n, n_blk, cval, cidx, et);
+          lm_row<BN, KT, true>(p, tb, m, n0, lim, ch0, ch1, 2 * n_blk + half, 2 * num_n, cval, cidx, et);
       }
     }
   } else {
@@ -838,7 +907,7 @@ cudaError_t launch_small(const CUtensorMap a_maps[3], const GemmArgs& args, cuda
   const int tiles = ((args.M + BM * MT - 1) / (BM * MT)) * ((args.N + BN - 1) / BN);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(tiles * args.splits);
-  cfg.blockDim = dim3(192);
+  cfg.blockDim = dim3(small_threads<EPI>());
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = stream;
   cudaLaunchAttribute at[1];
@@ -868,6 +937,7 @@ cudaError_t gemm_small_launch(const CUtensorMap a_maps[3], int bn, int epi, int 
   if (args.splits < 1 || (epi == EPI_SLICES && args.N % 4)) return cudaErrorInvalidValue;
   if ((epi == EPI_LM1 || epi == EPI_LM8) && (args.splits != 1 || !args.lm_stats || !args.lm_top))
     return cudaErrorInvalidValue;
+  if (epi == EPI_LM8 && !args.lm_bound) return cudaErrorInvalidValue;
 #define OUTLETS_SM_CASE(BNV, EV, MTV) \
   if (bn == BNV && epi == EV && mt == MTV) return launch_small<BNV, EV, MTV>(a_maps, args, stream);
   OUTLETS_SM_CASE(256, EPI_SLICES, 2)

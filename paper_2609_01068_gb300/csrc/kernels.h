@@ -60,10 +60,20 @@ enum Epi : int {
   EPI_LM8 = 8,        // same with the 8 best columns
 };
 
-// Draft LM head partials, one entry per (row, N tile), row-major [rows][tiles]:
+// Draft LM head partials, one entry per (row, partial tile), row-major
+// [rows][tiles]; the tensor-core epilogue splits every N tile into two column
+// halves, each its own partial tile (partial tile 2t + h: half h of N tile t):
 //   stats: (max logit m_t, sum over the tile's columns of exp(logit - m_t))
-//   top:   the tile's KT best (logit bits, token id) pairs, best first
-// (order: larger logit, then smaller id; empty places hold (-inf, INT_MAX)).
+//   top:   the tile's best (logit bits, token id) pairs, best first, up to KT
+//          of them (order: larger logit, then smaller id; empty places hold
+//          (-inf, INT_MAX)).  A tile may keep fewer than KT pairs: it drops
+//          pairs below a lower bound of the row's KT-th best logit over the
+//          whole vocabulary, which no pair of the row's top-KT falls below.
+// Row bounds: kLmBoundSlots int keys per row (floats mapped so that int order
+// is float order; kLmBoundInit is below every finite logit); the merge kernel
+// puts its rows back to kLmBoundInit.
+constexpr int kLmBoundSlots = 8;
+constexpr int kLmBoundInit = (int)0x80808080;  // byte pattern 0x80: cudaMemset can write it
 
 // B operands (weights) live in a k-block-major, pre-swizzled layout owned by the
 // library: element (n, k) of a [N, K] weight is stored at
@@ -90,6 +100,7 @@ struct GemmArgs {
   float* lm_logits;       // EPI_LM*: optional f32 logits [M, N] with row stride ldo (null: not stored)
   float2* lm_stats;       // EPI_LM*: partials [M][tiles], layout above
   int2* lm_top;           // EPI_LM*: partials [M][tiles][KT]
+  int* lm_bound;          // EPI_LM8: [M][kLmBoundSlots] per-row slots bounding the row's 8th best logit (int keys)
 };
 
 // tcgen05 path (bf16 operands).  a_maps: 3 tensor maps over the A pieces (box
@@ -111,9 +122,10 @@ cudaError_t lm_tile_stats_f32_launch(const float* logits, long long ld, int rows
 
 // Draft LM head: combines the n_tiles partials of each row into the row's
 // logsumexp and its k (<= kt) best tokens with their log-probabilities
-// (ids, logprob: [rows, k]; lse: [rows] or null).  n_tiles <= 2048.
+// (ids, logprob: [rows, k]; lse: [rows] or null) and resets the rows' bound
+// slots to kLmBoundInit (bound may be null).  n_tiles <= 4096.
 cudaError_t lm_merge_launch(const float2* stats, const int2* top, int n_tiles, int kt, int rows, int k, int* ids,
-                            float* logprob, float* lse, cudaStream_t stream);
+                            float* logprob, float* lse, int* bound, cudaStream_t stream);
 
 // CUDA-core path of the f32 configuration.  a[0..2]: A pieces with row stride k_per_map.
 cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int epi, const GemmArgs& args,

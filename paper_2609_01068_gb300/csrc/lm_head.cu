@@ -6,7 +6,8 @@
 // columns, and its best KT (logit, token id) pairs.  This file holds
 //   k_lm_merge          one CTA per row: logsumexp = m + log(sum_t s_t exp(m_t - m)),
 //                       m = max_t m_t, and the k best tokens of the row, taken one
-//                       at a time as the best head of the tiles' sorted lists;
+//                       at a time as the best head of the tiles' sorted lists
+//                       (every token of the row's top-k is in its tile's list);
 //   k_lm_tile_stats_f32 the same partials from f32 logits (CUDA-core path).
 #include "common.cuh"
 #include "kernels.h"
@@ -16,7 +17,7 @@ namespace outlets {
 namespace {
 
 constexpr int kMergeThreads = 256;
-constexpr int kMaxTilesPerThread = 8;  // n_tiles <= 2048
+constexpr int kMaxTilesPerThread = 16;  // n_tiles <= 4096
 
 // Best (value, id, owner) over the block; every thread gets the result.
 __device__ __forceinline__ void block_best(float& v, int& i, float* sv, int* si) {
@@ -66,7 +67,7 @@ template <int KT>
 __global__ void __launch_bounds__(kMergeThreads) k_lm_merge(const float2* __restrict__ stats,
                                                             const int2* __restrict__ top, int n_tiles, int k,
                                                             int* __restrict__ ids, float* __restrict__ logprob,
-                                                            float* __restrict__ lse_out) {
+                                                            float* __restrict__ lse_out, int* __restrict__ bound) {
   __shared__ float sv[kMergeThreads / 32];
   __shared__ int si[kMergeThreads / 32];
   pdl_trigger();
@@ -119,6 +120,8 @@ __global__ void __launch_bounds__(kMergeThreads) k_lm_merge(const float2* __rest
     }
   }
   if (threadIdx.x == 0 && lse_out) lse_out[row] = lse;
+  if (bound && threadIdx.x < kLmBoundSlots)
+    bound[(long long)row * kLmBoundSlots + threadIdx.x] = kLmBoundInit;  // ready for the next pass over these rows
 }
 
 template <int KT>
@@ -151,15 +154,15 @@ __global__ void __launch_bounds__(128) k_lm_tile_stats_f32(const float* __restri
 }  // namespace
 
 cudaError_t lm_merge_launch(const float2* stats, const int2* top, int n_tiles, int kt, int rows, int k, int* ids,
-                            float* logprob, float* lse, cudaStream_t stream) {
+                            float* logprob, float* lse, int* bound, cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
   if (n_tiles < 1 || n_tiles > kMergeThreads * kMaxTilesPerThread || k < 1 || k > kt) return cudaErrorInvalidValue;
   if (kt == 1)
     return launch_k(k_lm_merge<1>, dim3(rows), dim3(kMergeThreads), 0, stream, stats, top, n_tiles, k, ids, logprob,
-                    lse);
+                    lse, bound);
   if (kt == 8)
     return launch_k(k_lm_merge<8>, dim3(rows), dim3(kMergeThreads), 0, stream, stats, top, n_tiles, k, ids, logprob,
-                    lse);
+                    lse, bound);
   return cudaErrorInvalidValue;
 }
 

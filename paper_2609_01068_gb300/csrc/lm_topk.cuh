@@ -14,6 +14,13 @@ namespace outlets {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
+// Order-preserving map between floats and signed ints (for atomicMax on logits).
+__device__ __forceinline__ int lm_key(float f) {
+  const int i = __float_as_int(f);
+  return i >= 0 ? i : i ^ 0x7FFFFFFF;
+}
+__device__ __forceinline__ float lm_unkey(int k) { return __int_as_float(k >= 0 ? k : k ^ 0x7FFFFFFF); }
+
 __device__ __forceinline__ bool lm_better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);
 }

@@ -129,6 +129,8 @@ struct outlets_ctx {
   int lm_rows_cap = 0;       // rows per GEMM + merge pass
   float2* lm_stats = nullptr;
   int2* lm_top = nullptr;
+  int* lm_bound = nullptr;   // per-row slots bounding the 8th best logit (reset by the merge kernel)
+  bool lm_bound_dirty = true;  // a pass may have stopped before its merge: reset before the next GEMM
   int* lm_ids = nullptr;
   float *lm_lp = nullptr, *lm_lse = nullptr;
   float* lm_logits_ws = nullptr;  // f32 path: logits of one pass
@@ -753,6 +755,11 @@ outlets_status run_draft(outlets_ctx* c, const void* h, int rows, const outlets_
   }
   c->stage_begin(OUTLETS_S_DRAFT);
   int n_launch = 0;
+  if (c->lm_bound_dirty) {
+    OUT_CK(c, cudaMemsetAsync(c->lm_bound, kLmBoundInit & 0xFF, (size_t)c->lm_rows_cap * kLmBoundSlots * sizeof(int),
+                              s));
+    c->lm_bound_dirty = false;
+  }
   for (int g0 = 0; g0 < rows; g0 += c->lm_rows_cap) {
     const int gr = std::min(c->lm_rows_cap, rows - g0);
     const void* hg = static_cast<const char*>(h) + (size_t)g0 * d * c->esz;
@@ -761,7 +768,7 @@ outlets_status run_draft(outlets_ctx* c, const void* h, int rows, const outlets_
     int n_tiles = 0;
     if (c->bf16) {
       const int bn = lm_tile_width(c, gr);
-      n_tiles = (int)cdiv(V, bn);
+      n_tiles = 2 * (int)cdiv(V, bn);  // two column halves per tile
       CUtensorMap am[3];
       OUT_TRY(a_maps(c, a1, 1, d, d, gr, am));
       GemmArgs g{};
@@ -778,6 +785,8 @@ outlets_status run_draft(outlets_ctx* c, const void* h, int rows, const outlets_
       g.lm_logits = lg;
       g.lm_stats = c->lm_stats;
       g.lm_top = c->lm_top;
+      g.lm_bound = c->lm_bound;
+      c->lm_bound_dirty = true;  // until its merge is enqueued
       OUT_CK(c, gemm_small_launch(am, bn, kt == 1 ? EPI_LM1 : EPI_LM8, gr <= 128 ? 1 : 2, g, s));
       n_launch += 1;
     } else {
@@ -788,7 +797,8 @@ outlets_status run_draft(outlets_ctx* c, const void* h, int rows, const outlets_
       n_launch += 2;
     }
     OUT_CK(c, lm_merge_launch(c->lm_stats, c->lm_top, n_tiles, kt, gr, k, ids + (size_t)g0 * k,
-                              lp + (size_t)g0 * k, lse ? lse + g0 : nullptr, s));
+                              lp + (size_t)g0 * k, lse ? lse + g0 : nullptr, c->lm_bound, s));
+    c->lm_bound_dirty = false;
     n_launch += 1;
     if (host_logits)
       OUT_CK(c, cudaMemcpyAsync(o.logits + (size_t)g0 * V, lg, (size_t)gr * V * 4, cudaMemcpyDeviceToHost, s));
@@ -1017,9 +1027,11 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   if (c->V > 0) {
     c->w_lm = c->alloc(rows_of(c->np_lm, c->V) * d * es);
     c->lm_rows_cap = std::min(c->max_rows, kLmRowsPerPass);
-    const size_t tiles = (size_t)cdiv(c->V, c->bf16 ? 128 : kLmTileF32);
+    // partial tiles per row: two column halves of every 128-wide tile (tensor-core path)
+    const size_t tiles = c->bf16 ? 2 * (size_t)cdiv(c->V, 128) : (size_t)cdiv(c->V, kLmTileF32);
     c->lm_stats = (float2*)c->alloc((size_t)c->lm_rows_cap * tiles * sizeof(float2));
     c->lm_top = (int2*)c->alloc((size_t)c->lm_rows_cap * tiles * OUTLETS_MAX_TOPK * sizeof(int2));
+    c->lm_bound = (int*)c->alloc((size_t)c->lm_rows_cap * kLmBoundSlots * sizeof(int));
     c->lm_ids = (int*)c->alloc((size_t)c->max_rows * OUTLETS_MAX_TOPK * sizeof(int));
     c->lm_lp = (float*)c->alloc((size_t)c->max_rows * OUTLETS_MAX_TOPK * 4);
     c->lm_lse = (float*)c->alloc((size_t)c->max_rows * 4);

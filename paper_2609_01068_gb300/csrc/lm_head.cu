@@ -5,9 +5,11 @@
 // the tile's maximum logit m_t, the sum s_t of exp(logit - m_t) over its
 // columns, and its best KT (logit, token id) pairs.  This file holds
 //   k_lm_merge          one CTA per row: logsumexp = m + log(sum_t s_t exp(m_t - m)),
-//                       m = max_t m_t, and the k best tokens of the row, taken one
-//                       at a time as the best head of the tiles' sorted lists
-//                       (every token of the row's top-k is in its tile's list);
+//                       m = max_t m_t, and the k best tokens of the row (every
+//                       token of the row's top-k is in its tile's list, at or
+//                       above the row's bound): the list entries that reach the
+//                       bound are gathered in shared memory and the k best
+//                       taken from there, one at a time;
 //   k_lm_tile_stats_f32 the same partials from f32 logits (CUDA-core path).
 #include "common.cuh"
 #include "kernels.h"
@@ -63,6 +65,10 @@ __device__ __forceinline__ float block_reduce(float v, bool is_max, float* sv) {
   return v;
 }
 
+// Candidates of a row the merge collects in shared memory (beyond this the
+// merge takes the k rounds over the tiles' lists in global memory instead).
+constexpr int kMergeCap = 2048;
+
 template <int KT>
 __global__ void __launch_bounds__(kMergeThreads) k_lm_merge(const float2* __restrict__ stats,
                                                             const int2* __restrict__ top, int n_tiles, int k,
@@ -70,53 +76,113 @@ __global__ void __launch_bounds__(kMergeThreads) k_lm_merge(const float2* __rest
                                                             float* __restrict__ lse_out, int* __restrict__ bound) {
   __shared__ float sv[kMergeThreads / 32];
   __shared__ int si[kMergeThreads / 32];
+  __shared__ float cv[kMergeCap];
+  __shared__ int ci[kMergeCap];
+  __shared__ int ncand;
   pdl_trigger();
   pdl_wait();
   const int row = blockIdx.x;
   const float2* st = stats + (long long)row * n_tiles;
   const int2* tp = top + (long long)row * n_tiles * KT;
-  float m = -INFINITY;
-  for (int t = threadIdx.x; t < n_tiles; t += kMergeThreads) m = fmaxf(m, st[t].x);
-  m = block_reduce(m, true, sv);
-  float s = 0.f;
+  // logsumexp in one pass: each thread keeps (max, sum relative to it)
+  float m = -INFINITY, sm = 0.f;
   for (int t = threadIdx.x; t < n_tiles; t += kMergeThreads) {
     const float2 e = st[t];
-    s += e.y * exp2f((e.x - m) * kLog2e);
+    if (e.y == 0.f) continue;  // a partial tile past the vocabulary
+    if (e.x > m) {
+      sm = sm * exp2f((m - e.x) * kLog2e) + e.y;
+      m = e.x;
+    } else {
+      sm += e.y * exp2f((e.x - m) * kLog2e);
+    }
   }
-  s = block_reduce(s, false, sv);
-  const float lse = m + logf(s);
-  // head of each owned tile's list (tiles threadIdx.x + j * kMergeThreads)
-  int head[kMaxTilesPerThread];
+  const float M = block_reduce(m, true, sv);
+  const float S = block_reduce(m == -INFINITY ? 0.f : sm * exp2f((m - M) * kLog2e), false, sv);
+  const float lse = M + logf(S);
+
+  // The row's bound slots (written by the GEMM epilogue) bound the row's 8th
+  // best logit from below, so every token of the top-k is at or above it:
+  // collect the tiles' list entries that reach it (the lists are sorted, so a
+  // thread stops at the first entry below it), then take the k best of those.
+  float thr = -INFINITY;
+  if (KT > 1 && bound) {
+    int kmin = INT_MAX;
 #pragma unroll
-  for (int j = 0; j < kMaxTilesPerThread; ++j) head[j] = 0;
-  for (int r = 0; r < k; ++r) {
-    float bv = -INFINITY;
-    int bi = INT_MAX, bj = -1;
-#pragma unroll
-    for (int j = 0; j < kMaxTilesPerThread; ++j) {
-      const int t = threadIdx.x + j * kMergeThreads;
-      if (t < n_tiles && head[j] < KT) {
-        const int2 e = tp[(long long)t * KT + head[j]];
+    for (int q = 0; q < kLmBoundSlots; ++q) kmin = min(kmin, __ldcg(bound + (long long)row * kLmBoundSlots + q));
+    thr = lm_unkey(kmin);
+  }
+  if (threadIdx.x == 0) ncand = 0;
+  __syncthreads();
+  if (KT > 1) {
+    for (int t = threadIdx.x; t < n_tiles; t += kMergeThreads) {
+#pragma unroll 1
+      for (int q = 0; q < KT; ++q) {
+        const int2 e = tp[(long long)t * KT + q];
         const float v = __int_as_float(e.x);
-        if (lm_better(v, e.y, bv, bi)) {
-          bv = v;
-          bi = e.y;
-          bj = j;
+        if (e.y == INT_MAX || v < thr) break;
+        const int pos = atomicAdd(&ncand, 1);
+        if (pos < kMergeCap) {
+          cv[pos] = v;
+          ci[pos] = e.y;
         }
       }
     }
-    const float mv = bv;
-    const int mi = bi;
-    block_best(bv, bi, sv, si);
-    // token ids are unique, so exactly one thread owns the winner
-    if (bj >= 0 && mi == bi && mv == bv) {
-#pragma unroll
-      for (int j = 0; j < kMaxTilesPerThread; ++j)
-        if (j == bj) ++head[j];
+  }
+  __syncthreads();
+  const int nc = ncand;
+  if (KT > 1 && nc <= kMergeCap) {
+    for (int r = 0; r < k; ++r) {
+      float bv = -INFINITY;
+      int bi = INT_MAX, bp = -1;
+      for (int c = threadIdx.x; c < nc; c += kMergeThreads)
+        if (lm_better(cv[c], ci[c], bv, bi)) {
+          bv = cv[c];
+          bi = ci[c];
+          bp = c;
+        }
+      const float mv = bv;
+      const int mi = bi;
+      block_best(bv, bi, sv, si);
+      if (bp >= 0 && mi == bi && mv == bv) cv[bp] = -INFINITY, ci[bp] = INT_MAX;  // taken
+      if (threadIdx.x == 0) {
+        ids[(long long)row * k + r] = bi;
+        logprob[(long long)row * k + r] = bv - lse;
+      }
     }
-    if (threadIdx.x == 0) {
-      ids[(long long)row * k + r] = bi;
-      logprob[(long long)row * k + r] = bv - lse;
+  } else {
+    // k rounds over the heads of the tiles' sorted lists in global memory
+    int head[kMaxTilesPerThread];
+#pragma unroll
+    for (int j = 0; j < kMaxTilesPerThread; ++j) head[j] = 0;
+    for (int r = 0; r < k; ++r) {
+      float bv = -INFINITY;
+      int bi = INT_MAX, bj = -1;
+#pragma unroll
+      for (int j = 0; j < kMaxTilesPerThread; ++j) {
+        const int t = threadIdx.x + j * kMergeThreads;
+        if (t < n_tiles && head[j] < KT) {
+          const int2 e = tp[(long long)t * KT + head[j]];
+          const float v = __int_as_float(e.x);
+          if (lm_better(v, e.y, bv, bi)) {
+            bv = v;
+            bi = e.y;
+            bj = j;
+          }
+        }
+      }
+      const float mv = bv;
+      const int mi = bi;
+      block_best(bv, bi, sv, si);
+      // token ids are unique, so exactly one thread owns the winner
+      if (bj >= 0 && mi == bi && mv == bv) {
+#pragma unroll
+        for (int j = 0; j < kMaxTilesPerThread; ++j)
+          if (j == bj) ++head[j];
+      }
+      if (threadIdx.x == 0) {
+        ids[(long long)row * k + r] = bi;
+        logprob[(long long)row * k + r] = bv - lse;
+      }
     }
   }
   if (threadIdx.x == 0 && lse_out) lse_out[row] = lse;

@@ -196,3 +196,25 @@ def test_llama3_vocab_full_size_sampled(rows):
     got = {key: torch.as_tensor(out[key])[sample] for key in ("ids", "logprob", "lse")}
     check_draft(got, OR.draft_logits(h[sample], w["w_lm"]), 8, TOL_GIVEN["bf16"], f"llama3 vocab rows={rows}")
     pred.close()
+
+
+def test_uniform_distribution_ties_go_to_smallest_ids():
+    """W_lm = 0: every logit ties at 0 (the uniform case of Eq. 2).  With
+    V = 40000 every partial tile keeps 8 tied entries, more than the merge
+    gathers in shared memory, so this also covers its fallback path."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = MID128
+    w = synth.make_weights(shape, 0)
+    V = 40000
+    w["w_lm"] = np.zeros((V, shape.d), np.float32)
+    pred = OT.Predictor(shape, w, max_tokens=256, max_batch=64, max_position=1024)
+    h = synth.make_draft_states(shape, 37, 0, 5)
+    for k in (1, 8):
+        out = pred.draft_head(to_device(h, "bf16"), k)
+        torch.cuda.synchronize()
+        pred.check()
+        assert torch.as_tensor(out["ids"]).cpu().numpy().tolist() == [list(range(k))] * 37
+        np.testing.assert_allclose(to_np(torch.as_tensor(out["logprob"])), -np.log(V), rtol=0, atol=1e-4)
+        ref = OR.draft_head(h, w["w_lm"], k)
+        np.testing.assert_array_equal(ref["topk_ids"], np.tile(np.arange(k), (37, 1)))
+    pred.close()

@@ -36,6 +36,12 @@ Readings where the paper is silent (the same list is kept in the design notes):
   * Linear layers of the decoder have no bias; the length head has biases;
   * static pooling takes the last prompt position;
   * length_hat = max(0, expm1(z_hat)) (clamped because expm1 < 0 for z < 0);
+  * input-embedding branch of the EAGLE-3-style backbone (an ablated
+    component in Sec. 5.4, no formula given): the layer input is
+    Concat(RMSNorm(E[token]; g_emb), RMSNorm(f_ctx; g_in)), width 2d, so the
+    QKV projections (and the attention gate) take 2d inputs; the residual
+    stream stays f_ctx.  Used when the weights carry "w_embed" and the call
+    gives one token id per row;
   * dual head (Sec. 4.2, Eq. 2): the draft branch reads the same final-normed
     state h^draft as the length head; its output is the log of the softmax of
     W_lm h^draft over the vocabulary, reported as the k most probable tokens
@@ -155,6 +161,22 @@ def attend_single(q_row, k_all, v_all):
     return out
 
 
+# ------------------------------------------------------------------ input embeddings (Sec. 5.4)
+def layer_input(w, f, tokens, eps):
+    """Normalized input of the draft decoder layer.
+
+    Without the input-embedding branch: RMSNorm(f_ctx; g_in).  With it
+    (weights carry "w_embed" [V, d] and "g_emb" [d]): the token's embedding
+    row, normalized on its own, followed by the normalized fused feature:
+    Concat(RMSNorm(E[token]; g_emb), RMSNorm(f_ctx; g_in)), width 2d.
+    """
+    x = rms_norm(f, w["g_in"], eps)
+    if w.get("w_embed") is None:
+        return x
+    e = _f64(w["w_embed"])[np.asarray(tokens, dtype=np.int64)]
+    return np.concatenate([rms_norm(e, w["g_emb"], eps), x], axis=1)
+
+
 # ------------------------------------------------------------------ gated attention (Sec. 4.1)
 def sigmoid(x):
     x = _f64(x)
@@ -245,14 +267,15 @@ def draft_head(h, w_lm, k):
 
 
 # ------------------------------------------------------------------ forward
-def predict_prefill(w, shape, taps, cu, all_tokens=False, draft_k=None):
+def predict_prefill(w, shape, taps, cu, all_tokens=False, draft_k=None, tokens=None):
     """Static prediction over a packed varlen batch (Sec. 3.2, Sec. 4).
 
     Returns a dict with the hidden states of every step (for parity tests),
     the post-RoPE keys/values of every token (the draft KV cache), z_hat and
     length_hat at each sequence's last token (or every token if all_tokens).
     With draft_k and weights carrying "w_lm", "draft" holds the draft head's
-    output (draft_head) on the same rows.
+    output (draft_head) on the same rows.  tokens: [T] token ids, required
+    with the input-embedding branch (layer_input).
     """
     H, KVH, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
     eps, theta = shape.rms_eps, shape.rope_theta
@@ -261,7 +284,7 @@ def predict_prefill(w, shape, taps, cu, all_tokens=False, draft_k=None):
     pos = positions_from_cu(cu)
 
     f = fuse_taps(taps, w["w_proj"])                         # Eq. 1
-    x = rms_norm(f, w["g_in"], eps)
+    x = layer_input(w, f, tokens, eps)
     q = (x @ _f64(w["w_q"]).T).reshape(T, H, hd)
     k = (x @ _f64(w["w_k"]).T).reshape(T, KVH, hd)
     v = (x @ _f64(w["w_v"]).T).reshape(T, KVH, hd)
@@ -291,13 +314,14 @@ def caches_from_prefill(out, cu):
             for b in range(len(cu) - 1)]
 
 
-def predict_step(w, shape, taps_rows, caches, draft_k=None):
+def predict_step(w, shape, taps_rows, caches, draft_k=None, tokens=None):
     """Dynamic prediction for one new token per request (Sec. 3.2, t >= 1).
 
     taps_rows: three [B, d] arrays; caches: list of B (k [L, KVH, hd],
     v [L, KVH, hd]) already-cached post-RoPE keys/values.  The new token sits
     at position L of its request.  Returns z_hat, length_hat, intermediates and
     the caches extended by the new token (and "draft" as in predict_prefill).
+    tokens: [B] ids of the new tokens (input-embedding branch).
     """
     H, KVH, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
     eps, theta = shape.rms_eps, shape.rope_theta
@@ -305,7 +329,7 @@ def predict_step(w, shape, taps_rows, caches, draft_k=None):
     pos = np.array([c[0].shape[0] for c in caches], dtype=np.int64)
 
     f = fuse_taps(taps_rows, w["w_proj"])
-    x = rms_norm(f, w["g_in"], eps)
+    x = layer_input(w, f, tokens, eps)
     q = apply_rope((x @ _f64(w["w_q"]).T).reshape(B, H, hd), pos, theta)
     k = apply_rope((x @ _f64(w["w_k"]).T).reshape(B, KVH, hd), pos, theta)
     v = (x @ _f64(w["w_v"]).T).reshape(B, KVH, hd)
@@ -330,7 +354,7 @@ def predict_step(w, shape, taps_rows, caches, draft_k=None):
     return out
 
 
-def sample_prefill_rows(w, shape, taps, cu, seqs, draft_k=None):
+def sample_prefill_rows(w, shape, taps, cu, seqs, draft_k=None, tokens=None):
     """Oracle for a subset of sequences of a large packed batch.
 
     Every sequence is independent (attention never crosses sequences), so the
@@ -339,7 +363,8 @@ def sample_prefill_rows(w, shape, taps, cu, seqs, draft_k=None):
     """
     cu = np.asarray(cu, dtype=np.int64)
     sub_taps = [np.concatenate([t[cu[b]:cu[b + 1]] for b in seqs]) for t in taps]
+    sub_tok = None if tokens is None else np.concatenate([np.asarray(tokens)[cu[b]:cu[b + 1]] for b in seqs])
     sub_len = np.array([cu[b + 1] - cu[b] for b in seqs], dtype=np.int64)
     sub_cu = np.zeros(len(seqs) + 1, dtype=np.int64)
     np.cumsum(sub_len, out=sub_cu[1:])
-    return predict_prefill(w, shape, sub_taps, sub_cu, draft_k=draft_k)
+    return predict_prefill(w, shape, sub_taps, sub_cu, draft_k=draft_k, tokens=sub_tok)

@@ -9,7 +9,8 @@ Shapes follow the draft backbones the method is evaluated with (Sec. 5.1,
 
 Recipe (all draws from numpy PCG64 streams spawned from one SeedSequence):
   * stream 0 -> sequence / cache lengths;  stream 1 -> taps;  stream 2 -> weights;
-    stream 3 -> draft LM head W_lm (Eq. 2) and stand-in draft states.
+    stream 3 -> draft LM head W_lm (Eq. 2) and stand-in draft states;
+    stream 4 -> input-embedding branch (embedding table, its QKV columns, token ids).
   * lengths: rint(lognormal(ln(median), sigma=1)) clipped to the stated range.
   * taps ~ N(0, 1); every Linear weight ~ N(0, 0.02); RMSNorm gains = 1;
     head hidden biases ~ N(0, 0.02); output bias = ln(1 + 256).
@@ -29,7 +30,7 @@ __all__ = [
     "lengths_tiny", "lengths_8b_prefill", "lengths_8b_step_cache",
     "lengths_70b_prefill", "lengths_sweep", "cu_seqlens",
     "make_weights", "make_taps", "weight_names",
-    "LLAMA3_VOCAB", "make_lm_head", "make_draft_states",
+    "LLAMA3_VOCAB", "make_lm_head", "make_draft_states", "make_tokens",
 ]
 
 
@@ -138,12 +139,17 @@ def weight_names(shape: ModelShape):
 
 
 def make_weights(shape: ModelShape, seed: int = 0, std: float = 0.02,
-                 out_bias: float = math.log(257.0), gated: bool = False) -> dict:
+                 out_bias: float = math.log(257.0), gated: bool = False, embed_vocab: int = 0) -> dict:
     """All draft weights, nn.Linear [out, in] row-major, float32 arrays.
 
     On the bf16 path the matrices and head parameters are bf16-representable.
     gated=True adds the attention gate "w_attn_gate" [H*hd, d] (gated
     attention), drawn after every other weight so the rest are unchanged.
+    embed_vocab > 0 adds the input-embedding branch: the embedding table
+    "w_embed" [embed_vocab, d] ~ N(0, std), its RMSNorm gain "g_emb" = 1, and
+    d input columns in front of w_q, w_k, w_v (and w_attn_gate) for the
+    normalized embedding, all from stream 4, so the columns that read the
+    fused feature are the weights drawn without the branch.
     """
     rng = _streams(seed)[2]
     d, H, KVH, hd, F = shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
@@ -173,7 +179,29 @@ def make_weights(shape: ModelShape, seed: int = 0, std: float = 0.02,
             w[f"head_b{i}"] = rnd(np.full(1, out_bias, np.float32))
     if gated:
         w["w_attn_gate"] = lin(H * hd, d)
+    if embed_vocab:
+        erng = np.random.Generator(np.random.PCG64(np.random.SeedSequence(seed).spawn(5)[4]))
+
+        def elin(o, i):
+            return rnd(erng.standard_normal((o, i), dtype=np.float32) * np.float32(std))
+
+        w["g_emb"] = np.ones(d, np.float32)
+        for name in ("w_q", "w_k", "w_v") + (("w_attn_gate",) if gated else ()):
+            w[name] = np.ascontiguousarray(np.concatenate([elin(w[name].shape[0], d), w[name]], axis=1))
+        table = np.empty((embed_vocab, d), np.float32)
+        step = max(1, (1 << 24) // d)
+        for r0 in range(0, embed_vocab, step):
+            r1 = min(embed_vocab, r0 + step)
+            table[r0:r1] = elin(r1 - r0, d)
+        w["w_embed"] = table
     return w
+
+
+def make_tokens(n: int, vocab: int, seed: int = 0, stream_offset: int = 0) -> np.ndarray:
+    """Token ids [n] uniform in [0, vocab) (int32), for the input-embedding branch."""
+    ss = np.random.SeedSequence(seed).spawn(5)[4]
+    ss = np.random.SeedSequence(entropy=ss.entropy, spawn_key=ss.spawn_key + (2000 + stream_offset,))
+    return np.random.Generator(np.random.PCG64(ss)).integers(0, vocab, size=n, dtype=np.int64).astype(np.int32)
 
 
 LLAMA3_VOCAB = 128256  # vocabulary of the Llama-3 targets (the draft head's output width)

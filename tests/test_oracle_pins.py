@@ -517,3 +517,100 @@ def test_lm_head_draw_leaves_other_weights_unchanged():
         np.testing.assert_array_equal(a[k], b[k])
     np.testing.assert_array_equal(w1, synth.make_lm_head(SMALL, 40, 0))
     assert w1.shape == (40, SMALL.d) and abs(float(w1.std()) - 0.02) < 0.004
+
+
+# ---------------------------------------------------------------- input-embedding branch (Sec. 5.4)
+EV = 40  # embedding rows of the pin cases
+
+
+def _embed_case(lengths=(5, 3), gated=False, seed=0, off=0):
+    w = synth.make_weights(SMALL, seed, gated=gated, embed_vocab=EV)
+    cu = synth.cu_seqlens(list(lengths))
+    T = int(cu[-1])
+    return w, cu, _taps(SMALL, T, seed, off), synth.make_tokens(T, EV, seed, off)
+
+
+def test_embedding_columns_zero_reduce_to_the_plain_layer():
+    """With the embedding columns of W_q, W_k, W_v (and W_ag) set to zero the
+    branch contributes nothing: every output equals the layer without it."""
+    for gated in (False, True):
+        w, cu, taps, tok = _embed_case(gated=gated)
+        d = SMALL.d
+        for name in ("w_q", "w_k", "w_v") + (("w_attn_gate",) if gated else ()):
+            w[name] = w[name].copy()
+            w[name][:, :d] = 0.0
+        plain = synth.make_weights(SMALL, 0, gated=gated)
+        a = O.predict_prefill(w, SMALL, taps, cu, tokens=tok)
+        b = O.predict_prefill(plain, SMALL, taps, cu)
+        np.testing.assert_allclose(a["y"], b["y"], rtol=0, atol=1e-13)
+        np.testing.assert_allclose(a["z"], b["z"], rtol=0, atol=1e-13)
+
+
+def test_embedding_is_a_row_lookup():
+    """Permuting the table rows and relabelling the tokens the same way changes nothing."""
+    w, cu, taps, tok = _embed_case()
+    perm = np.random.default_rng(8).permutation(EV)
+    w2 = dict(w)
+    w2["w_embed"] = w["w_embed"][perm]          # new row r holds old row perm[r]
+    inv = np.argsort(perm)                       # old token t sits at new row inv[t]
+    a = O.predict_prefill(w, SMALL, taps, cu, tokens=tok)
+    b = O.predict_prefill(w2, SMALL, taps, cu, tokens=inv[tok])
+    np.testing.assert_array_equal(a["z"], b["z"])
+    np.testing.assert_array_equal(a["x"], b["x"])
+
+
+def test_embedding_layer_input_brute_force():
+    """q of one row by explicit loops: the normalized embedding fills input
+    columns 0..d-1, the normalized fused feature columns d..2d-1."""
+    w, cu, taps, tok = _embed_case(lengths=(4,))
+    out = O.predict_prefill(w, SMALL, taps, cu, tokens=tok)
+    d, r, eps = SMALL.d, 2, SMALL.rms_eps
+    e = [float(v) for v in w["w_embed"][tok[r]]]
+    f = [sum(float(taps[j][r, i]) * float(w["w_proj"][c, j * d + i]) for j in range(3) for i in range(d))
+         for c in range(d)]
+    re = math.sqrt(sum(v * v for v in e) / d + eps)
+    rf = math.sqrt(sum(v * v for v in f) / d + eps)
+    x = [e[i] / re * float(w["g_emb"][i]) for i in range(d)] + [f[i] / rf * float(w["g_in"][i]) for i in range(d)]
+    q = [sum(float(w["w_q"][j, i]) * x[i] for i in range(2 * d)) for j in range(SMALL.n_heads * SMALL.head_dim)]
+    # the oracle's layer input (the rotation comes after the projection, so compare before it)
+    np.testing.assert_allclose(out["x"][r], x, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(out["x"][r] @ w["w_q"].astype(np.float64).T, q, rtol=1e-11, atol=1e-12)
+
+
+def test_embedding_token_change_is_causal():
+    """Changing the token at position p of a sequence changes that sequence's
+    outputs at positions >= p only, and no other sequence."""
+    w, cu, taps, tok = _embed_case(lengths=(6, 4))
+    a = O.predict_prefill(w, SMALL, taps, cu, all_tokens=True, tokens=tok)
+    tok2 = tok.copy()
+    tok2[3] = (tok2[3] + 1) % EV
+    b = O.predict_prefill(w, SMALL, taps, cu, all_tokens=True, tokens=tok2)
+    diff = np.abs(a["y"] - b["y"]).max(axis=1)
+    assert np.all(diff[:3] == 0) and np.all(diff[3:6] > 0) and np.all(diff[6:] == 0)
+
+
+def test_embedding_prefill_equals_prefix_then_steps():
+    w, cu, taps, tok = _embed_case(lengths=(5, 3), gated=True)
+    full = O.predict_prefill(w, SMALL, taps, cu, all_tokens=True, tokens=tok)
+    kpre = [2, 1]
+    pre_rows = np.concatenate([np.arange(cu[b], cu[b] + kpre[b]) for b in range(2)])
+    pre_cu = synth.cu_seqlens(kpre)
+    caches = O.caches_from_prefill(
+        O.predict_prefill(w, SMALL, [t[pre_rows] for t in taps], pre_cu, tokens=tok[pre_rows]), pre_cu)
+    for step in range(2):
+        rows = [cu[b] + kpre[b] + step for b in range(2)]
+        st = O.predict_step(w, SMALL, [t[rows] for t in taps], caches, tokens=tok[rows])
+        np.testing.assert_allclose(st["z"], full["z"][rows], rtol=1e-11, atol=1e-11)
+        caches = st["caches"]
+
+
+def test_embedding_draw_keeps_the_fused_feature_columns():
+    w = synth.make_weights(SMALL, 0, gated=True, embed_vocab=EV)
+    p = synth.make_weights(SMALL, 0, gated=True)
+    d = SMALL.d
+    for name in ("w_q", "w_k", "w_v", "w_attn_gate"):
+        assert w[name].shape == (p[name].shape[0], 2 * d)
+        np.testing.assert_array_equal(w[name][:, d:], p[name])
+    for name in p:
+        if name not in ("w_q", "w_k", "w_v", "w_attn_gate"):
+            np.testing.assert_array_equal(w[name], p[name])

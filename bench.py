@@ -43,6 +43,9 @@ def model_setup(args):
     from paper_2609_01068_gb300 import synth
     gate = ", gated attention" if getattr(args, "gated", False) else ""
     gkey = "-gated" if getattr(args, "gated", False) else ""
+    if getattr(args, "embed", False):
+        gate += ", input-embedding branch (128256-row Llama-3 embedding table)"
+        gkey += "-embed"
     if getattr(args, "dual", 0):
         gate += ", dual head (draft LM head over the 128256-token Llama-3 vocabulary, top-%d)" % args.dual
         gkey += "-dual%d" % args.dual
@@ -68,6 +71,9 @@ def parse():
     ap.add_argument("--dual", type=int, default=0, metavar="K",
                     help="dual head (Sec. 4.2, Eq. 2): also run the draft LM head (Llama-3 vocabulary, "
                          "128256 tokens) and return its top-K tokens (1..8); 0 = length head only")
+    ap.add_argument("--embed", action="store_true",
+                    help="input-embedding branch of the EAGLE-3-style layer (Sec. 5.4): token embeddings "
+                         "(128256-row table) normalized and concatenated to the layer input, QKV K = 2d")
     ap.add_argument("--model", default="8b", choices=["8b", "70b"],
                     help="draft-layer shape; 70b (Llama-3.3-70B-shaped, 32 prompts) runs the static mode only")
     ap.add_argument("--step-requests", type=int, default=256, help="live requests of the dynamic-prediction run")
@@ -177,11 +183,12 @@ def weight_bytes(shape):
     return 2 * (3 * d * d + d * (H + 2 * KVH) * hd + H * hd * d + 3 * d * F + d * shape.head_widths[0])
 
 
-def prefill_flops(shape, lengths, n_out, gated=False):
+def prefill_flops(shape, lengths, n_out, gated=False, embed=False):
     """Algorithmic FLOPs of one static-prediction pass (dense GEMMs + causal attention + head)."""
     d, H, KVH, hd, F = shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
     T = int(np.sum(lengths))
-    per_tok = 2 * (3 * d * d + d * (H + 2 * KVH + (H if gated else 0)) * hd + H * hd * d + 3 * d * F)
+    qkv_k = 2 * d if embed else d
+    per_tok = 2 * (3 * d * d + qkv_k * (H + 2 * KVH + (H if gated else 0)) * hd + H * hd * d + 3 * d * F)
     attn = 4 * H * hd * float(np.sum(lengths * (lengths + 1) / 2))
     widths = (d,) + tuple(shape.head_widths) + (1,)
     head = 2 * sum(widths[i] * widths[i + 1] for i in range(len(widths) - 1)) * n_out
@@ -199,7 +206,7 @@ def cpu_threads():
     return os.cpu_count()
 
 
-def oracle_sample(shape, w, taps, cu, lengths, budget_tokens, draft_k=None):
+def oracle_sample(shape, w, taps, cu, lengths, budget_tokens, draft_k=None, tokens=None):
     """Oracle on whole prompts taken in order until the token budget is used
     (with the draft head when draft_k is given)."""
     from oracle import outlets_oracle as OR
@@ -210,7 +217,7 @@ def oracle_sample(shape, w, taps, cu, lengths, budget_tokens, draft_k=None):
         picks.append(int(b))
         tot += int(lengths[b])
     t0 = time.perf_counter()
-    OR.sample_prefill_rows(w, shape, taps, cu, picks, draft_k=draft_k)
+    OR.sample_prefill_rows(w, shape, taps, cu, picks, draft_k=draft_k, tokens=tokens)
     dt = time.perf_counter() - t0
     return len(picks), tot, dt
 
@@ -249,18 +256,19 @@ def run_reference(args):
         return
     from paper_2609_01068_gb300 import synth
     shape, lengths, workload, _ = model_setup(args)
-    w = synth.make_weights(shape, 0, gated=args.gated)
+    w = synth.make_weights(shape, 0, gated=args.gated, embed_vocab=synth.LLAMA3_VOCAB if args.embed else 0)
     if args.dual:
         w["w_lm"] = synth.make_lm_head(shape, synth.LLAMA3_VOCAB, 0)
     cu = synth.cu_seqlens(lengths)
     taps = synth.make_taps(shape, int(cu[-1]), 0)
+    tok = synth.make_tokens(int(cu[-1]), synth.LLAMA3_VOCAB, 0, 0) if args.embed else None
     budget = 400
     dk = args.dual or None
     for _ in range(args.warmup):
-        oracle_sample(shape, w, taps, cu, lengths, budget, dk)
+        oracle_sample(shape, w, taps, cu, lengths, budget, dk, tok)
     n_pred, n_tok, secs = 0, 0, 0.0
     for _ in range(args.steps):
-        p, t, dt = oracle_sample(shape, w, taps, cu, lengths, budget, dk)
+        p, t, dt = oracle_sample(shape, w, taps, cu, lengths, budget, dk, tok)
         n_pred, n_tok, secs = n_pred + p, n_tok + t, secs + dt
     value = n_pred / secs
     out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "predictions/s", "n_gpus": args.gpus,
@@ -291,14 +299,17 @@ def run_ours(args):
     peaks = load_peaks()
     if args.model == "70b" and args.mode != "prefill":
         raise SystemExit("--model 70b runs the static (prefill) mode only")
+    if args.embed and args.mode == "sweep":
+        raise SystemExit("--embed runs the static and dynamic modes (the sweep uses the plain layer input)")
     shape, lengths, workload, tkey = model_setup(args)
     args.workload, args.traffic_key = workload, tkey
-    w = synth.make_weights(shape, 0, gated=args.gated)
+    w = synth.make_weights(shape, 0, gated=args.gated, embed_vocab=synth.LLAMA3_VOCAB if args.embed else 0)
     if args.dual:
         w["w_lm"] = synth.make_lm_head(shape, synth.LLAMA3_VOCAB, 0)
     cu = synth.cu_seqlens(lengths)
     T, Bq = int(cu[-1]), len(lengths)
     taps = synth.make_taps(shape, T, 0, rank)
+    args.tokens = synth.make_tokens(T, synth.LLAMA3_VOCAB, 0, rank) if args.embed else None
 
     def dev(a):
         return torch.from_numpy(synth.bf16_bits(a).view(np.int16)).view(torch.bfloat16).cuda()
@@ -349,12 +360,15 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     T, Bq = int(cu[-1]), len(lengths)
     K = args.dual
     dout = draft_buffers(K, Bq) if K else None
+    tok_host = args.tokens  # token ids (input-embedding branch): device copy for the device-timed passes
+    tok_dev = torch.from_numpy(tok_host).cuda() if tok_host is not None else None
 
-    def run(tp, zo, lo, out=None):
+    def run(tp, zo, lo, out=None, tok=None):
+        tok = tok_dev if tok is None else tok
         if K:
-            pred.prefill_dual(tp, cu, K, out=out if out is not None else dout, z_out=zo, len_out=lo)
+            pred.prefill_dual(tp, cu, K, out=out if out is not None else dout, z_out=zo, len_out=lo, tokens=tok)
         else:
-            pred.prefill(tp, cu, z_out=zo, len_out=lo)
+            pred.prefill(tp, cu, z_out=zo, len_out=lo, tokens=tok)
 
     # ---------------- device-timed static prediction
     z = torch.empty(Bq, dtype=torch.float32, device="cuda")
@@ -388,7 +402,8 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     pred.profile(False)
     ms_step = ms / args.steps
     value = world * Bq * args.steps / (ms / 1e3)
-    flops = prefill_flops(shape, lengths, Bq, args.gated) + (2.0 * Bq * pred.vocab * shape.d if K else 0.0)
+    flops = (prefill_flops(shape, lengths, Bq, args.gated, args.embed)
+             + (2.0 * Bq * pred.vocab * shape.d if K else 0.0))
     gu_ms, gu_n = prof_live["gateup_swiglu_gemm"]
     gu_flops = 2.0 * T * (2 * shape.ffn) * shape.d
     gu_tflops = gu_flops / (gu_ms / gu_n / 1e3) / 1e12
@@ -408,16 +423,17 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
         lh = torch.empty(Bq, dtype=torch.float32).pin_memory()
         dh = draft_buffers(K, Bq, pin=True) if K else None
         for _ in range(max(2, args.warmup // 2)):
-            run(host_taps, zh, lh, dh)
+            run(host_taps, zh, lh, dh, tok_host)  # host buffers in, host ids too
             stream.synchronize()
         barrier()
         t0 = time.perf_counter()
         for _ in range(args.steps):
-            run(host_taps, zh, lh, dh)
+            run(host_taps, zh, lh, dh, tok_host)
             stream.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - t0)
         e2e = {"value": world * Bq * args.steps / e2e_s, "unit": "predictions/s",
-               "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps)),
+               "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps))
+               + (int(tok_host.nbytes) if tok_host is not None else 0),
                "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4 + buffer_bytes(dh))}
 
     out = {"value": value, "unit": "predictions/s", "ms_per_step": ms_step,
@@ -431,7 +447,7 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
            "roofline": roofline, "stages": stages, "clocks": clocks, "e2e": e2e,
            "gpu_launches": launches}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        n_pred, n_tok, secs = oracle_sample(shape, w, taps, cu, lengths, 1200, args.dual or None)
+        n_pred, n_tok, secs = oracle_sample(shape, w, taps, cu, lengths, 1200, args.dual or None, args.tokens)
         out["cpu_baseline"] = {"value": n_pred / secs, "unit": "predictions/s", "cores": cpu_threads(),
                                "kind": "oracle",
                                "sample": f"{n_pred} whole prompts ({n_tok} tokens) of the same workload, {secs:.1f} s"}
@@ -453,7 +469,9 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
             tot += int(lens[e])
             e += 1
         taps = [torch.randn(tot, shape.d, device="cuda", generator=gen).to(torch.bfloat16) for _ in range(3)]
-        pred.prefill(taps, synth.cu_seqlens(lens[b:e]), kv=kv, slots=np.arange(b, e, dtype=np.int32))
+        ftok = (torch.randint(0, synth.LLAMA3_VOCAB, (tot,), device="cuda", generator=gen, dtype=torch.int32)
+                if args.embed else None)
+        pred.prefill(taps, synth.cu_seqlens(lens[b:e]), kv=kv, slots=np.arange(b, e, dtype=np.int32), tokens=ftok)
         b = e
     slots = np.arange(B, dtype=np.int32)
     st_taps = [torch.randn(B, shape.d, device="cuda", generator=gen).to(torch.bfloat16) for _ in range(3)]
@@ -461,12 +479,15 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     ln = torch.empty(B, dtype=torch.float32, device="cuda")
     K = args.dual
     dout = draft_buffers(K, B) if K else None
+    st_tok = synth.make_tokens(B, synth.LLAMA3_VOCAB, 0, 7) if args.embed else None
+    st_tok_dev = torch.from_numpy(st_tok).cuda() if st_tok is not None else None
 
-    def run(tp, zo, lo, out=None):
+    def run(tp, zo, lo, out=None, tok=None):
+        tok = st_tok_dev if tok is None else tok
         if K:
-            pred.step_dual(tp, kv, slots, K, out=out if out is not None else dout, z_out=zo, len_out=lo)
+            pred.step_dual(tp, kv, slots, K, out=out if out is not None else dout, z_out=zo, len_out=lo, tokens=tok)
         else:
-            pred.step(tp, kv, slots, z_out=zo, len_out=lo)
+            pred.step(tp, kv, slots, z_out=zo, len_out=lo, tokens=tok)
 
     for _ in range(args.warmup):
         run(st_taps, z, ln)
@@ -507,16 +528,17 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
         lh = torch.empty(B, dtype=torch.float32).pin_memory()
         dh = draft_buffers(K, B, pin=True) if K else None
         for _ in range(2):
-            run(host_taps, zh, lh, dh)
+            run(host_taps, zh, lh, dh, st_tok)
             stream.synchronize()
         barrier()
         t0 = time.perf_counter()
         for _ in range(args.steps):
-            run(host_taps, zh, lh, dh)
+            run(host_taps, zh, lh, dh, st_tok)
             stream.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - t0)
         e2e = {"value": world * B * args.steps / e2e_s, "unit": "predictions/s",
-               "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps)),
+               "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps))
+               + (int(st_tok.nbytes) if st_tok is not None else 0),
                "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4 + buffer_bytes(dh))}
     d, KVH, hd, F = shape.d, shape.n_kv_heads, shape.head_dim, shape.ffn
     # keys read per step: every cached position plus the new one, K and V, bf16
@@ -526,6 +548,8 @@ def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, s
     w_bytes = 2 * (3 * d * d + d * shape.qkv_out + shape.n_heads * hd * d + 3 * d * F + widths[0] * widths[1])
     if args.gated:
         w_bytes += 2 * shape.n_heads * hd * d  # gate rows of the QKV weight
+    if args.embed:  # embedding columns of the QKV (and gate) weight, and the B gathered embedding rows
+        w_bytes += 2 * d * (shape.qkv_out + (shape.n_heads * hd if args.gated else 0)) + B * d * 2
     lm_bytes = pred.vocab * d * 2 + B * d * 2 if K else 0  # W_lm and the draft states, read once
     step_bytes = kv_bytes + w_bytes + 3 * B * d * 2 + lm_bytes
     at_ms, at_n = prof_live["attention"]

@@ -88,6 +88,10 @@ typedef struct outlets_config {
   int32_t vocab;          /* V: rows of the draft LM head W_lm (Eq. 2), 8 .. 262144;
                              0 = no draft head (the *_dual calls and
                              outlets_draft_head then return OUTLETS_EUNSUPPORTED) */
+  int32_t embed_vocab;    /* rows of the token-embedding table of the input-embedding
+                             branch (EAGLE-3-style layer input, Sec. 5.4); 0 = no
+                             branch.  With the branch every prediction needs token
+                             ids (the *_ex calls). */
 } outlets_config;
 
 /* Host pointers to f32 weights, nn.Linear layout [out, in], row-major.
@@ -105,6 +109,12 @@ typedef struct outlets_config {
  *     NULL gives standard attention.
  *   w_lm [V, d]              the draft LM head of Eq. 2 (required when vocab > 0,
  *     ignored otherwise).
+ *   w_embed [embed_vocab, d], g_emb [d]: the input-embedding branch (required
+ *     when embed_vocab > 0).  The layer input is then
+ *     Concat(RMSNorm(w_embed[token]; g_emb), RMSNorm(f_ctx; g_in)), width 2d:
+ *     w_q, w_k, w_v (and w_attn_gate) are [out, 2d], their columns 0 .. d-1
+ *     read the normalized embedding and d .. 2d-1 the normalized fused
+ *     feature.  The residual stream stays f_ctx.
  * The library copies everything during outlets_create; the caller may free
  * its arrays afterwards. */
 typedef struct outlets_weights {
@@ -123,6 +133,8 @@ typedef struct outlets_weights {
   const float* head_b[OUTLETS_MAX_HEAD_HIDDEN + 1];
   const float* w_attn_gate;
   const float* w_lm;
+  const float* w_embed;
+  const float* g_emb;
 } outlets_weights;
 
 typedef struct outlets_ctx outlets_ctx;
@@ -221,6 +233,24 @@ outlets_status outlets_predict_prefill_dual(outlets_ctx* ctx, const void* const 
 outlets_status outlets_predict_step_dual(outlets_ctx* ctx, const void* const taps[3], int32_t B, outlets_kv* kv,
                                          const int32_t* slots, float* z_out, float* len_out,
                                          const outlets_draft_out* draft, void* stream);
+
+/* ---- Input-embedding branch (contexts with embed_vocab > 0).
+ * The same calls with one token id per row: tokens is device or host int32,
+ * [T] for prefill (every packed prompt token) and [B] for a step (each
+ * request's new token), ids in 0 .. embed_vocab-1 (host ids are checked on
+ * the host, EINVAL; device ids a kernel refuses set the device error word,
+ * OUTLETS_EDEVICE from outlets_check).  draft may be NULL (length head only)
+ * or request the draft head as in the *_dual calls.  Contexts without the
+ * branch take tokens == NULL; contexts with it reject the calls without
+ * tokens (EINVAL). */
+outlets_status outlets_predict_prefill_ex(outlets_ctx* ctx, const void* const taps[3], const int32_t* tokens,
+                                          const int32_t* cu_seqlens, int32_t B, int32_t T, outlets_kv* kv,
+                                          const int32_t* slots, uint32_t flags, float* z_out, float* len_out,
+                                          const outlets_draft_out* draft, void* stream);
+
+outlets_status outlets_predict_step_ex(outlets_ctx* ctx, const void* const taps[3], const int32_t* tokens, int32_t B,
+                                       outlets_kv* kv, const int32_t* slots, float* z_out, float* len_out,
+                                       const outlets_draft_out* draft, void* stream);
 
 /* The draft head alone on caller-given states.
  *   h_draft  device [rows, d] (bf16 or f32 like the context), 16-byte aligned.

@@ -173,7 +173,7 @@ def layer_input(w, f, tokens, eps):
     x = rms_norm(f, w["g_in"], eps)
     if w.get("w_embed") is None:
         return x
-    e = _f64(w["w_embed"])[np.asarray(tokens, dtype=np.int64)]
+    e = _f64(np.asarray(w["w_embed"])[np.asarray(tokens, dtype=np.int64)])  # row lookup, then widen
     return np.concatenate([rms_norm(e, w["g_emb"], eps), x], axis=1)
 
 

@@ -190,6 +190,40 @@ __device__ __forceinline__ void store8<float>(float* p, const float* v) {
   *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
 }
 
+// Input-embedding branch (EAGLE-3-style layer input): y[r] = RMSNorm(E[tok[r]]) * g,
+// one CTA per row, 8 elements per thread step (d is a multiple of 64).  A token
+// outside [0, V) raises ERR_BAD_INDEX and reads row 0 instead.
+template <typename Act>
+__global__ void __launch_bounds__(256) k_embed_rmsnorm(const int* __restrict__ tok, const Act* __restrict__ E, int V,
+                                                       const float* __restrict__ g, Act* __restrict__ y, int d,
+                                                       float eps, int* __restrict__ err) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float red[33];
+  const int r = blockIdx.x;
+  int t = tok[r];
+  if (t < 0 || t >= V) {
+    if (threadIdx.x == 0) atomicOr(err, ERR_BAD_INDEX);
+    t = 0;
+  }
+  const long long base = (long long)t * d;
+  float ss = 0.f;
+  for (int i = threadIdx.x * 8; i < d; i += blockDim.x * 8) {
+    float v[8];
+    load8<Act>(E, base + i, 1, 0, v);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) ss += v[k] * v[k];
+  }
+  const float inv = rsqrtf(block_sum(ss, red) / (float)d + eps);
+  for (int i = threadIdx.x * 8; i < d; i += blockDim.x * 8) {
+    float v[8];
+    load8<Act>(E, base + i, 1, 0, v);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] *= inv * g[i + k];
+    store8<Act>(y + (long long)r * d + i, v);
+  }
+}
+
 // One CTA per row; a thread rotates 8 pairs (i..i+7 with i+hd/2..i+hd/2+7) of
 // one head and copies 8 values of V.  hd is a multiple of 16.
 // Block shape of the RoPE/scatter kernel.  f32 input (split-K slices, small
@@ -511,6 +545,16 @@ cudaError_t swiglu_launch(const float* gu, Act* u, int rows, int f_pad, cudaStre
   return cudaGetLastError();
 }
 
+template <typename Act>
+cudaError_t embed_rmsnorm_launch(const int* tokens, const Act* table, int vocab, const float* g, Act* y, int rows,
+                                 int d, float eps, int* err, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  const int threads = std::min(256, std::max(32, ((d / 8 + 31) / 32) * 32));
+  OUTLETS_TRY_LAUNCH(launch_k(k_embed_rmsnorm<Act>, dim3(rows), dim3(threads), 0, stream, tokens, table, vocab, g, y, d,
+                              eps, err));
+  return cudaGetLastError();
+}
+
 cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_stride, const float* b_prev,
                              const float* w_last, const float* b_last, int rows, int width, float* z, float* len,
                              cudaStream_t stream) {
@@ -550,6 +594,8 @@ cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int ep
   template cudaError_t rmsnorm_gather_launch<Act>(const float*, const int*, const float*, Act*, int, int, float, \
                                                   cudaStream_t);                                               \
   template cudaError_t swiglu_launch<Act>(const float*, Act*, int, int, cudaStream_t);                         \
+  template cudaError_t embed_rmsnorm_launch<Act>(const int*, const Act*, int, const float*, Act*, int, int, float, \
+                                                 int*, cudaStream_t);                                          \
   template cudaError_t convert_rows_launch<Act>(const float*, Act*, int, int, long long, int, int, long long,       \
                                                 cudaStream_t);                                                  \
   template cudaError_t rope_scatter_launch<float, Act>(const float*, const RopeArgs&, cudaStream_t);           \
@@ -561,6 +607,8 @@ template cudaError_t rmsnorm_launch<float>(const float*, const float*, float*, f
 template cudaError_t rmsnorm_gather_launch<float>(const float*, const int*, const float*, float*, int, int, float,
                                                   cudaStream_t);
 template cudaError_t swiglu_launch<float>(const float*, float*, int, int, cudaStream_t);
+template cudaError_t embed_rmsnorm_launch<float>(const int*, const float*, int, const float*, float*, int, int, float,
+                                                 int*, cudaStream_t);
 template cudaError_t convert_rows_launch<float>(const float*, float*, int, int, long long, int, int, long long,
                                                 cudaStream_t);
 template cudaError_t rope_scatter_launch<float, float>(const float*, const RopeArgs&, cudaStream_t);

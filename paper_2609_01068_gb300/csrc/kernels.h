@@ -149,6 +149,12 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
                                   const int* row_index, const float* g, Act* y, float* copy_out, int rows, int d,
                                   float eps, cudaStream_t stream);
 
+// Input-embedding branch: y[r] = RMSNorm(table[tokens[r]]) * g (table [vocab, d],
+// row-major, act dtype); an id outside [0, vocab) sets ERR_BAD_INDEX in *err.
+template <typename Act>
+cudaError_t embed_rmsnorm_launch(const int* tokens, const Act* table, int vocab, const float* g, Act* y, int rows,
+                                 int d, float eps, int* err, cudaStream_t stream);
+
 struct RopeArgs {
   int T;                 // rows of this launch (rows row0 .. row0 + T - 1 of the call)
   int row0;              // first row (a prefill call may run its rows in chunks)

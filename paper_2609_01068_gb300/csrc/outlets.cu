@@ -122,6 +122,12 @@ struct outlets_ctx {
   size_t esz = 2;
   int d = 0, H = 0, KVH = 0, hd = 0, F = 0, Fp = 0, qkv_n = 0, attn_w = 0, max_rows = 0;
   bool gated = false;        // gated attention: QKV carries H*hd gate columns after q, k, v
+  // input-embedding branch: table [EV, d] (act dtype, row-major), its gain, the
+  // normalized embedding of each row; the QKV GEMM then has K = 2d (qkv_k)
+  int EV = 0, qkv_k = 0;
+  void* w_embed = nullptr;
+  float* g_emb = nullptr;
+  void* ehat = nullptr;
   // draft LM head (Eq. 2): weights, per (row, tile) partials, outputs of host callers
   int V = 0;
   void* w_lm = nullptr;
@@ -311,6 +317,7 @@ outlets_status validate_config(const outlets_config* cfg, std::string& why) {
   if ((cfg->n_heads * cfg->head_dim) % 64) return bad("n_heads * head_dim must be a multiple of 64");
   if (cfg->ffn_dim <= 0) return bad("ffn_dim must be positive");
   if (cfg->vocab != 0 && (cfg->vocab < 8 || cfg->vocab > kMaxVocab)) return bad("vocab must be 0 or in 8..262144");
+  if (cfg->embed_vocab < 0) return bad("embed_vocab must be >= 0");
   if (cfg->n_head_hidden < 1 || cfg->n_head_hidden > OUTLETS_MAX_HEAD_HIDDEN)
     return bad("n_head_hidden must be in 1..OUTLETS_MAX_HEAD_HIDDEN");
   for (int i = 0; i < cfg->n_head_hidden; ++i)
@@ -825,7 +832,7 @@ struct QkvSrc {
 // FC (Eq. 1) -> input RMSNorm -> QKV for rows row0 .. row0 + rows - 1 (tp
 // points at row row0 of each tap; row0 > 0 only on the large-M path).
 outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvSrc* q, cudaStream_t s,
-                         int row0 = 0) {
+                         int row0, const int* tok_dev) {
   const int d = c->d;
   const float eps = c->cfg.rms_eps;
   const bool small = small_path(c, rows);
@@ -846,19 +853,38 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
                                    d, eps, s));
   else
     OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
-  c->stage_end(1);
-  c->stage_begin(OUTLETS_S_QKV);
+  int n_norm = 1;
   const void* xr = (const char*)c->xhat + (size_t)row0 * d * c->esz;
   const void* a1[3] = {xr, xr, xr};
+  int pieces = 1;
+  if (c->EV > 0) {
+    // input-embedding branch: the normalized embeddings are the first d input
+    // columns of the QKV GEMM (a second A piece; nothing is concatenated)
+    OUT_TRY(wait_meta(c, s));  // host token ids travel with the call's metadata
+    void* er = (char*)c->ehat + (size_t)row0 * d * c->esz;
+    if (c->bf16)
+      OUT_CK(c, embed_rmsnorm_launch<bf16>(tok_dev + row0, (const bf16*)c->w_embed, c->EV, c->g_emb, (bf16*)er, rows,
+                                           d, eps, c->err_dev, s));
+    else
+      OUT_CK(c, embed_rmsnorm_launch<float>(tok_dev + row0, (const float*)c->w_embed, c->EV, c->g_emb, (float*)er,
+                                            rows, d, eps, c->err_dev, s));
+    a1[0] = er;
+    a1[1] = xr;
+    pieces = 2;
+    n_norm = 2;
+  }
+  c->stage_end(n_norm);
+  c->stage_begin(OUTLETS_S_QKV);
+  const int K = c->qkv_k;
   if (small) {
-    OUT_TRY(gemm_split(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, c->part, &sl, s));
+    OUT_TRY(gemm_split(c, a1, pieces, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, K, c->part, &sl, s));
     *q = {c->part, true, sl, (long long)rows * c->qkv_n};
   } else if (c->bf16) {
-    OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, d, EPI_ACT,
+    OUT_TRY(gemm_tc(c, a1, pieces, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, K, EPI_ACT,
                     (char*)c->qkv + (size_t)row0 * c->qkv_n * c->esz, c->qkv_n, nullptr, 0, nullptr, s));
     *q = {c->qkv, false, 1, 0};
   } else {
-    OUT_TRY(gemm_f32(c, a1, d, rows, c->w_qkv, c->qkv_n, d, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
+    OUT_TRY(gemm_f32(c, a1, d, rows, c->w_qkv, c->qkv_n, K, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
     *q = {c->qkv, true, 1, 0};
   }
   c->stage_end(1);
@@ -963,6 +989,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   for (int i = 0; i <= cfg->n_head_hidden; ++i)
     if (!w->head_w[i] || !w->head_b[i]) return OUTLETS_EINVAL;
   if (cfg->vocab > 0 && !w->w_lm) return OUTLETS_EINVAL;
+  if (cfg->embed_vocab > 0 && (!w->w_embed || !w->g_emb)) return OUTLETS_EINVAL;
   if (cudaSetDevice(cfg->device) != cudaSuccess) {
     cudaGetLastError();
     return OUTLETS_ECUDA;
@@ -984,6 +1011,8 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->attn_w = c->H * c->hd;
   c->gated = w->w_attn_gate != nullptr;
   c->qkv_n = (c->H + 2 * c->KVH) * c->hd + (c->gated ? c->attn_w : 0);
+  c->EV = cfg->embed_vocab;
+  c->qkv_k = c->EV > 0 ? 2 * cfg->d_model : cfg->d_model;
   c->max_rows = std::max(cfg->max_tokens, cfg->max_batch);
   c->V = cfg->vocab;
   c->head_dims.push_back(c->d);
@@ -1011,7 +1040,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
     c->np_lm = std::max({cdiv(c->V, 256) * 256, cdiv(c->V, 224) * 224, cdiv(c->V, 128) * 128});
   auto rows_of = [&](long long np, int n) -> size_t { return (size_t)(np ? np : n); };
   c->w_proj = c->alloc(rows_of(c->np_proj, d) * 3 * d * es);
-  c->w_qkv = c->alloc(rows_of(c->np_qkv, c->qkv_n) * d * es);
+  c->w_qkv = c->alloc(rows_of(c->np_qkv, c->qkv_n) * c->qkv_k * es);
   c->w_o = c->alloc(rows_of(c->np_o, d) * c->attn_w * es);
   c->w_gu = c->alloc(rows_of(c->np_gu, 2 * c->Fp) * d * es);
   c->w_down = c->alloc(rows_of(c->np_down, d) * c->Fp * es);
@@ -1024,6 +1053,10 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->head_w0 = c->alloc(rows_of(c->np_h0, c->head_dims[1]) * d * es);
   for (int i = 1; i < nl; ++i) c->head_wf[i] = (float*)c->alloc((size_t)c->head_dims[i + 1] * c->head_dims[i] * 4);
   for (int i = 0; i < nl; ++i) c->head_b[i] = (float*)c->alloc((size_t)c->head_dims[i + 1] * 4);
+  if (c->EV > 0) {
+    c->w_embed = c->alloc((size_t)c->EV * d * es);
+    c->g_emb = (float*)c->alloc((size_t)d * 4);
+  }
   if (c->V > 0) {
     c->w_lm = c->alloc(rows_of(c->np_lm, c->V) * d * es);
     c->lm_rows_cap = std::min(c->max_rows, kLmRowsPerPass);
@@ -1047,6 +1080,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->xhat = c->alloc(R * d * es);
   c->ahat = c->alloc(R * d * es);
   c->hn = c->alloc(R * d * es);
+  if (c->EV > 0) c->ehat = c->alloc(R * d * es);
   c->qkv = c->alloc(R * c->qkv_n * es);
   c->q = c->alloc(R * c->attn_w * es);
   if (c->gated) c->gate_act = c->alloc(R * c->attn_w * es);
@@ -1078,7 +1112,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   // tile and head), per-sequence arrays, page lists
   const size_t meta_ints = (size_t)8 * c->H * (cdiv(cfg->max_tokens, 128) + cfg->max_batch) +
                            (size_t)8 * (cfg->max_batch + 1) + (size_t)2 * (cdiv(cfg->max_tokens, 64) + cfg->max_batch) +
-                           (1u << 16);
+                           (c->EV > 0 ? R : 0) + (1u << 16);
   for (auto& p : c->ring) {
     if (cudaEventCreateWithFlags(&p.ev, cudaEventDisableTiming) != cudaSuccess ||
         cudaEventCreateWithFlags(&p.done, cudaEventDisableTiming) != cudaSuccess)
@@ -1111,10 +1145,12 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
       st = upload_rows(c, src, rows, cols, dst, ld, mode, base, np, stage, mode == 0 ? stage_floats : il_floats);
   };
   up(w->w_proj, d, 3 * d, c->w_proj, 3 * d, 0, 0, c->np_proj);
-  up(w->w_q, c->H * c->hd, d, c->w_qkv, d, 0, 0, c->np_qkv);
-  up(w->w_k, c->KVH * c->hd, d, c->w_qkv, d, 0, c->H * c->hd, c->np_qkv);
-  up(w->w_v, c->KVH * c->hd, d, c->w_qkv, d, 0, (c->H + c->KVH) * c->hd, c->np_qkv);
-  if (c->gated) up(w->w_attn_gate, c->attn_w, d, c->w_qkv, d, 0, (c->H + 2 * c->KVH) * c->hd, c->np_qkv);
+  const int qk = c->qkv_k;
+  up(w->w_q, c->H * c->hd, qk, c->w_qkv, qk, 0, 0, c->np_qkv);
+  up(w->w_k, c->KVH * c->hd, qk, c->w_qkv, qk, 0, c->H * c->hd, c->np_qkv);
+  up(w->w_v, c->KVH * c->hd, qk, c->w_qkv, qk, 0, (c->H + c->KVH) * c->hd, c->np_qkv);
+  if (c->gated) up(w->w_attn_gate, c->attn_w, qk, c->w_qkv, qk, 0, (c->H + 2 * c->KVH) * c->hd, c->np_qkv);
+  if (c->EV > 0) up(w->w_embed, c->EV, d, c->w_embed, d, 0, 0, 0);
   up(w->w_o, d, c->attn_w, c->w_o, c->attn_w, 0, 0, c->np_o);
   up(w->w_gate, c->F, d, c->w_gu, d, 1, 0, c->np_gu);
   up(w->w_up, c->F, d, c->w_gu, d, 2, 0, c->np_gu);
@@ -1129,6 +1165,7 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   h2d(c->g_in, w->g_in, (size_t)d * 4);
   h2d(c->g_post, w->g_post, (size_t)d * 4);
   h2d(c->g_final, w->g_final, (size_t)d * 4);
+  if (c->EV > 0) h2d(c->g_emb, w->g_emb, (size_t)d * 4);
   for (int i = 1; i < nl; ++i) h2d(c->head_wf[i], w->head_w[i], (size_t)c->head_dims[i + 1] * c->head_dims[i] * 4);
   for (int i = 0; i < nl; ++i) h2d(c->head_b[i], w->head_b[i], (size_t)c->head_dims[i + 1] * 4);
   // RoPE table, angles in fp64: pos * theta^(-2i/hd)
@@ -1312,9 +1349,24 @@ outlets_status outlets_check(outlets_ctx* c, void* stream) {
 
 namespace {
 
-outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const int32_t* cu, int32_t B, int32_t T,
-                               outlets_kv* kv, const int32_t* slots, uint32_t flags, float* z_out, float* len_out,
-                               const outlets_draft_out* draft, void* stream) {
+// Token ids of the input-embedding branch: required exactly when the context
+// has the branch; host ids are range-checked here (device ids by the kernel).
+outlets_status check_tokens(outlets_ctx* c, const int32_t* tokens, long long n) {
+  if (c->EV == 0) {
+    if (tokens) return c->fail(OUTLETS_EINVAL, "token ids given, but the context has no input-embedding branch");
+    return OUTLETS_OK;
+  }
+  if (!tokens)
+    return c->fail(OUTLETS_EINVAL, "the context has the input-embedding branch: pass token ids (the *_ex calls)");
+  if (!is_device_ptr(tokens))
+    for (long long i = 0; i < n; ++i)
+      if (tokens[i] < 0 || tokens[i] >= c->EV) return c->fail(OUTLETS_EINVAL, "token id outside 0 .. embed_vocab-1");
+  return OUTLETS_OK;
+}
+
+outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const int32_t* tokens, const int32_t* cu,
+                               int32_t B, int32_t T, outlets_kv* kv, const int32_t* slots, uint32_t flags,
+                               float* z_out, float* len_out, const outlets_draft_out* draft, void* stream) {
   cudaStream_t s = (cudaStream_t)stream;
   if (!taps || !cu || !z_out) return c->fail(OUTLETS_EINVAL, "taps, cu_seqlens and z_out must not be NULL");
   if (flags & ~OUTLETS_ALL_TOKENS) return c->fail(OUTLETS_EINVAL, "unknown flag");
@@ -1333,6 +1385,7 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   }
   if (cu[B] != T) return c->fail(OUTLETS_EINVAL, "cu_seqlens[B] must equal T");
   if (T > c->cfg.max_tokens) return c->fail(OUTLETS_ECAPACITY, "T exceeds max_tokens");
+  OUT_TRY(check_tokens(c, tokens, T));
   if (B > c->cfg.max_batch) return c->fail(OUTLETS_ECAPACITY, "B exceeds max_batch");
   if (max_len > c->cfg.max_position) return c->fail(OUTLETS_ECAPACITY, "a sequence is longer than max_position");
   if (kv) {
@@ -1366,6 +1419,8 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   // ---- host metadata
   MetaBuilder mb;
   const size_t off_cu = mb.put(cu, B + 1);
+  const bool tok_host = tokens && !is_device_ptr(tokens);
+  const size_t off_tok = tok_host ? mb.put(tokens, T) : 0;
   std::vector<int> last(B);
   for (int b = 0; b < B; ++b) last[b] = cu[b + 1] - 1;
   const size_t off_last = mb.put(last);
@@ -1435,6 +1490,7 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   else OUT_TRY(prepare_taps(c, taps, T, tp, s));
   const int* m = c->meta_dev;
   const int* cu_dev = m + off_cu;
+  const int* tok_dev = tok_host ? m + off_tok : tokens;
 
   // ---- per row chunk: FC (Eq. 1) -> input RMSNorm -> QKV -> RoPE (q,
   // head-major k/v, cache)
@@ -1469,7 +1525,7 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
       const size_t off = (size_t)r0 * c->d * c->esz;
       const void* tpc[3] = {(const char*)tp[0] + off, (const char*)tp[1] + off, (const char*)tp[2] + off};
       QkvSrc qsrc;
-      OUT_TRY(run_front(c, tpc, rows, &qsrc, s, r0));
+      OUT_TRY(run_front(c, tpc, rows, &qsrc, s, r0, tok_dev));
       OUT_TRY(wait_meta(c, s));
       c->stage_begin(OUTLETS_S_ROPE);
       ra.row0 = r0;
@@ -1507,15 +1563,16 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   return end_call(c, out_rows, z_out, len_out, s);
 }
 
-outlets_status predict_step(outlets_ctx* c, const void* const taps[3], int32_t B, outlets_kv* kv,
-                            const int32_t* slots, float* z_out, float* len_out, const outlets_draft_out* draft,
-                            void* stream) {
+outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int32_t* tokens, int32_t B,
+                            outlets_kv* kv, const int32_t* slots, float* z_out, float* len_out,
+                            const outlets_draft_out* draft, void* stream) {
   cudaStream_t s = (cudaStream_t)stream;
   if (!taps || !kv || !slots || !z_out) return c->fail(OUTLETS_EINVAL, "taps, kv, slots and z_out must not be NULL");
   if (kv->ctx != c) return c->fail(OUTLETS_EINVAL, "kv belongs to another context");
   if (B < 0) return c->fail(OUTLETS_EINVAL, "B must be >= 0");
   if (B == 0) return OUTLETS_OK;
   if (B > c->cfg.max_batch) return c->fail(OUTLETS_ECAPACITY, "B exceeds max_batch");
+  OUT_TRY(check_tokens(c, tokens, B));
   std::vector<char> seen(kv->max_slots, 0);
   int need = 0;
   for (int b = 0; b < B; ++b) {
@@ -1578,11 +1635,13 @@ outlets_status predict_step(outlets_ctx* c, const void* const taps[3], int32_t B
   const size_t off_w = mb.put(work);
   const size_t off_wo = mb.put(work_off);
   const size_t off_ord = mb.put(order);
+  const bool tok_host = tokens && !is_device_ptr(tokens);
+  const size_t off_tok = tok_host ? mb.put(tokens, B) : 0;
   OUT_TRY(upload_meta(c, mb.v, s));
   const int* m = c->meta_dev;
 
   QkvSrc qsrc;
-  OUT_TRY(run_front(c, tp, B, &qsrc, s));
+  OUT_TRY(run_front(c, tp, B, &qsrc, s, 0, tok_host ? m + off_tok : tokens));
   OUT_TRY(wait_meta(c, s));  // RoPE is the first kernel that reads the metadata
   c->stage_begin(OUTLETS_S_ROPE);
   {
@@ -1663,7 +1722,7 @@ outlets_status outlets_predict_prefill(outlets_ctx* c, const void* const taps[3]
                                        float* z_out, float* len_out, void* stream) {
   if (!c) return OUTLETS_EINVAL;
   c->err.clear();
-  return predict_prefill(c, taps, cu, B, T, kv, slots, flags, z_out, len_out, nullptr, stream);
+  return predict_prefill(c, taps, nullptr, cu, B, T, kv, slots, flags, z_out, len_out, nullptr, stream);
 }
 
 outlets_status outlets_predict_prefill_dual(outlets_ctx* c, const void* const taps[3], const int32_t* cu,
@@ -1673,14 +1732,24 @@ outlets_status outlets_predict_prefill_dual(outlets_ctx* c, const void* const ta
   if (!c) return OUTLETS_EINVAL;
   c->err.clear();
   OUT_TRY(check_draft(c, draft));
-  return predict_prefill(c, taps, cu, B, T, kv, slots, flags, z_out, len_out, draft, stream);
+  return predict_prefill(c, taps, nullptr, cu, B, T, kv, slots, flags, z_out, len_out, draft, stream);
+}
+
+outlets_status outlets_predict_prefill_ex(outlets_ctx* c, const void* const taps[3], const int32_t* tokens,
+                                          const int32_t* cu, int32_t B, int32_t T, outlets_kv* kv,
+                                          const int32_t* slots, uint32_t flags, float* z_out, float* len_out,
+                                          const outlets_draft_out* draft, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  if (draft) OUT_TRY(check_draft(c, draft));
+  return predict_prefill(c, taps, tokens, cu, B, T, kv, slots, flags, z_out, len_out, draft, stream);
 }
 
 outlets_status outlets_predict_step(outlets_ctx* c, const void* const taps[3], int32_t B, outlets_kv* kv,
                                     const int32_t* slots, float* z_out, float* len_out, void* stream) {
   if (!c) return OUTLETS_EINVAL;
   c->err.clear();
-  return predict_step(c, taps, B, kv, slots, z_out, len_out, nullptr, stream);
+  return predict_step(c, taps, nullptr, B, kv, slots, z_out, len_out, nullptr, stream);
 }
 
 outlets_status outlets_predict_step_dual(outlets_ctx* c, const void* const taps[3], int32_t B, outlets_kv* kv,
@@ -1689,7 +1758,16 @@ outlets_status outlets_predict_step_dual(outlets_ctx* c, const void* const taps[
   if (!c) return OUTLETS_EINVAL;
   c->err.clear();
   OUT_TRY(check_draft(c, draft));
-  return predict_step(c, taps, B, kv, slots, z_out, len_out, draft, stream);
+  return predict_step(c, taps, nullptr, B, kv, slots, z_out, len_out, draft, stream);
+}
+
+outlets_status outlets_predict_step_ex(outlets_ctx* c, const void* const taps[3], const int32_t* tokens, int32_t B,
+                                       outlets_kv* kv, const int32_t* slots, float* z_out, float* len_out,
+                                       const outlets_draft_out* draft, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  if (draft) OUT_TRY(check_draft(c, draft));
+  return predict_step(c, taps, tokens, B, kv, slots, z_out, len_out, draft, stream);
 }
 
 outlets_status outlets_draft_head(outlets_ctx* c, const void* h_draft, int32_t rows, const outlets_draft_out* draft,

@@ -30,7 +30,8 @@ class Config(ctypes.Structure):
     _fields_ = [("d_model", c_i32), ("n_heads", c_i32), ("n_kv_heads", c_i32), ("head_dim", c_i32),
                 ("ffn_dim", c_i32), ("n_head_hidden", c_i32), ("head_hidden", c_i32 * MAX_HEAD_HIDDEN),
                 ("rope_theta", c_f32), ("rms_eps", c_f32), ("dtype", c_i32), ("max_tokens", c_i32),
-                ("max_batch", c_i32), ("max_position", c_i32), ("device", c_i32), ("vocab", c_i32)]
+                ("max_batch", c_i32), ("max_position", c_i32), ("device", c_i32), ("vocab", c_i32),
+                ("embed_vocab", c_i32)]
 
 
 _WNAMES = ["w_proj", "w_q", "w_k", "w_v", "w_o", "g_in", "g_post", "g_final", "w_gate", "w_up", "w_down"]
@@ -39,7 +40,8 @@ _WNAMES = ["w_proj", "w_q", "w_k", "w_v", "w_o", "g_in", "g_post", "g_final", "w
 class Weights(ctypes.Structure):
     _fields_ = [(n, c_vp) for n in _WNAMES] + [("head_w", c_vp * (MAX_HEAD_HIDDEN + 1)),
                                                ("head_b", c_vp * (MAX_HEAD_HIDDEN + 1)),
-                                               ("w_attn_gate", c_vp), ("w_lm", c_vp)]
+                                               ("w_attn_gate", c_vp), ("w_lm", c_vp), ("w_embed", c_vp),
+                                               ("g_emb", c_vp)]
 
 
 class DraftOut(ctypes.Structure):
@@ -85,6 +87,9 @@ def load():
                                                  c_vp, c_vp, P(DraftOut), c_vp]),
         "outlets_predict_step_dual": (c_i32, [c_vp, P(c_vp), c_i32, c_vp, c_vp, c_vp, c_vp, P(DraftOut), c_vp]),
         "outlets_draft_head": (c_i32, [c_vp, c_vp, c_i32, P(DraftOut), c_vp]),
+        "outlets_predict_prefill_ex": (c_i32, [c_vp, P(c_vp), c_vp, c_vp, c_i32, c_i32, c_vp, c_vp, ctypes.c_uint32,
+                                               c_vp, c_vp, c_vp, c_vp]),
+        "outlets_predict_step_ex": (c_i32, [c_vp, P(c_vp), c_vp, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]),
         "outlets_check": (c_i32, [c_vp, c_vp]),
         "outlets_get_intermediate": (c_i32, [c_vp, c_i32, c_vp, ctypes.c_size_t, P(TensorInfo), c_vp]),
         "outlets_profile_enable": (c_i32, [c_vp, c_i32]),
@@ -113,6 +118,14 @@ def _ptr(x):
     if not x.is_contiguous():
         raise ValueError("tensors must be contiguous")
     return x.data_ptr()
+
+
+def _tokens(tokens):
+    """Token ids as a contiguous int32 array/tensor (device tensors stay on the device)."""
+    if isinstance(tokens, np.ndarray) or not hasattr(tokens, "data_ptr"):
+        return np.ascontiguousarray(tokens, dtype=np.int32)
+    import torch
+    return tokens.to(torch.int32).contiguous()
 
 
 def _stream_handle(stream):
@@ -164,6 +177,13 @@ class Predictor:
             w.w_lm = la.ctypes.data
             cfg.vocab = la.shape[0]
         self.vocab = cfg.vocab
+        if weights.get("w_embed") is not None:  # input-embedding branch
+            ea = np.ascontiguousarray(weights["w_embed"], dtype=np.float32)
+            ga = np.ascontiguousarray(weights["g_emb"], dtype=np.float32)
+            keep["w_embed"], keep["g_emb"] = ea, ga
+            w.w_embed, w.g_emb = ea.ctypes.data, ga.ctypes.data
+            cfg.embed_vocab = ea.shape[0]
+        self.embed_vocab = cfg.embed_vocab
         h = c_vp()
         st = self.lib.outlets_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h))
         if st != OK:
@@ -200,30 +220,39 @@ class Predictor:
 
     # -- prediction
     def prefill(self, taps, cu_seqlens, kv=None, slots=None, all_tokens=False, z_out=None, len_out=None,
-                stream=None):
-        """Static prediction (z_hat, length_hat) for a packed varlen batch."""
+                stream=None, tokens=None):
+        """Static prediction (z_hat, length_hat) for a packed varlen batch.
+        tokens: [T] int32 ids (numpy or torch), for the input-embedding branch."""
         cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
         B, T = len(cu) - 1, int(cu[-1]) if len(cu) else 0
         n_out = T if all_tokens else B
         z_out, len_out = self._outputs(n_out, taps[0], z_out, len_out)
         tp = (c_vp * 3)(*[_ptr(t) for t in taps])
         sl = None if slots is None else np.ascontiguousarray(slots, dtype=np.int32)
-        st = self.lib.outlets_predict_prefill(self.h, tp, cu.ctypes.data, B, T, kv.h if kv else None,
-                                              None if sl is None else sl.ctypes.data,
-                                              ALL_TOKENS if all_tokens else 0, _ptr(z_out), _ptr(len_out),
-                                              _stream_handle(stream))
+        args = (cu.ctypes.data, B, T, kv.h if kv else None, None if sl is None else sl.ctypes.data,
+                ALL_TOKENS if all_tokens else 0, _ptr(z_out), _ptr(len_out))
+        if tokens is None:
+            st = self.lib.outlets_predict_prefill(self.h, tp, *args, _stream_handle(stream))
+        else:
+            tok = _tokens(tokens)
+            st = self.lib.outlets_predict_prefill_ex(self.h, tp, _ptr(tok), *args, None, _stream_handle(stream))
         if st != OK:
             self._raise(st)
         return z_out, len_out
 
-    def step(self, taps, kv, slots, z_out=None, len_out=None, stream=None):
-        """Dynamic prediction for one new token per request."""
+    def step(self, taps, kv, slots, z_out=None, len_out=None, stream=None, tokens=None):
+        """Dynamic prediction for one new token per request (tokens: their ids, [B])."""
         sl = np.ascontiguousarray(slots, dtype=np.int32)
         B = len(sl)
         z_out, len_out = self._outputs(B, taps[0], z_out, len_out)
         tp = (c_vp * 3)(*[_ptr(t) for t in taps])
-        st = self.lib.outlets_predict_step(self.h, tp, B, kv.h, sl.ctypes.data, _ptr(z_out), _ptr(len_out),
-                                           _stream_handle(stream))
+        if tokens is None:
+            st = self.lib.outlets_predict_step(self.h, tp, B, kv.h, sl.ctypes.data, _ptr(z_out), _ptr(len_out),
+                                               _stream_handle(stream))
+        else:
+            tok = _tokens(tokens)
+            st = self.lib.outlets_predict_step_ex(self.h, tp, _ptr(tok), B, kv.h, sl.ctypes.data, _ptr(z_out),
+                                                  _ptr(len_out), None, _stream_handle(stream))
         if st != OK:
             self._raise(st)
         return z_out, len_out
@@ -246,7 +275,7 @@ class Predictor:
         return d, out
 
     def prefill_dual(self, taps, cu_seqlens, k, kv=None, slots=None, all_tokens=False, logits=False, out=None,
-                     z_out=None, len_out=None, stream=None):
+                     z_out=None, len_out=None, stream=None, tokens=None):
         """Static prediction plus the draft head on the same rows:
         (z_hat, length_hat, {"ids", "logprob", "lse"[, "logits"]})."""
         cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
@@ -256,23 +285,32 @@ class Predictor:
         d, draft = self._draft_out(n_out, k, taps[0], logits, out)
         tp = (c_vp * 3)(*[_ptr(t) for t in taps])
         sl = None if slots is None else np.ascontiguousarray(slots, dtype=np.int32)
-        st = self.lib.outlets_predict_prefill_dual(self.h, tp, cu.ctypes.data, B, T, kv.h if kv else None,
-                                                   None if sl is None else sl.ctypes.data,
-                                                   ALL_TOKENS if all_tokens else 0, _ptr(z_out), _ptr(len_out),
-                                                   ctypes.byref(d), _stream_handle(stream))
+        args = (cu.ctypes.data, B, T, kv.h if kv else None, None if sl is None else sl.ctypes.data,
+                ALL_TOKENS if all_tokens else 0, _ptr(z_out), _ptr(len_out), ctypes.byref(d))
+        if tokens is None:
+            st = self.lib.outlets_predict_prefill_dual(self.h, tp, *args, _stream_handle(stream))
+        else:
+            tok = _tokens(tokens)
+            st = self.lib.outlets_predict_prefill_ex(self.h, tp, _ptr(tok), *args, _stream_handle(stream))
         if st != OK:
             self._raise(st)
         return z_out, len_out, draft
 
-    def step_dual(self, taps, kv, slots, k, logits=False, out=None, z_out=None, len_out=None, stream=None):
+    def step_dual(self, taps, kv, slots, k, logits=False, out=None, z_out=None, len_out=None, stream=None,
+                  tokens=None):
         """Dynamic prediction plus the draft head: (z_hat, length_hat, draft outputs)."""
         sl = np.ascontiguousarray(slots, dtype=np.int32)
         B = len(sl)
         z_out, len_out = self._outputs(B, taps[0], z_out, len_out)
         d, draft = self._draft_out(B, k, taps[0], logits, out)
         tp = (c_vp * 3)(*[_ptr(t) for t in taps])
-        st = self.lib.outlets_predict_step_dual(self.h, tp, B, kv.h, sl.ctypes.data, _ptr(z_out), _ptr(len_out),
-                                                ctypes.byref(d), _stream_handle(stream))
+        if tokens is None:
+            st = self.lib.outlets_predict_step_dual(self.h, tp, B, kv.h, sl.ctypes.data, _ptr(z_out), _ptr(len_out),
+                                                    ctypes.byref(d), _stream_handle(stream))
+        else:
+            tok = _tokens(tokens)
+            st = self.lib.outlets_predict_step_ex(self.h, tp, _ptr(tok), B, kv.h, sl.ctypes.data, _ptr(z_out),
+                                                  _ptr(len_out), ctypes.byref(d), _stream_handle(stream))
         if st != OK:
             self._raise(st)
         return z_out, len_out, draft

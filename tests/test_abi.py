@@ -36,7 +36,8 @@ def test_header_declares_the_entry_points():
     names = _declared_functions()
     for must in ("outlets_create", "outlets_predict_prefill", "outlets_predict_step", "outlets_kv_create",
                  "outlets_destroy", "outlets_last_error", "outlets_predict_prefill_dual",
-                 "outlets_predict_step_dual", "outlets_draft_head"):
+                 "outlets_predict_step_dual", "outlets_draft_head", "outlets_predict_prefill_ex",
+                 "outlets_predict_step_ex"):
         assert must in names
 
 
@@ -77,6 +78,10 @@ def test_create_rejects_invalid_config_on_host(built_lib):
         cfg.vocab = vocab
         assert built_lib.outlets_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h)) == O.EINVAL
         assert not h.value
+    cfg.vocab = 0
+    cfg.embed_vocab = -3
+    assert built_lib.outlets_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(h)) == O.EINVAL
+    assert not h.value
 
 
 def test_null_handles_are_rejected(built_lib):
@@ -90,6 +95,9 @@ def test_null_handles_are_rejected(built_lib):
                                                   None) == O.EINVAL
     assert built_lib.outlets_predict_step_dual(None, taps, 1, None, None, z, None, ctypes.byref(d), None) == O.EINVAL
     assert built_lib.outlets_draft_head(None, None, 1, ctypes.byref(d), None) == O.EINVAL
+    assert built_lib.outlets_predict_prefill_ex(None, taps, None, cu, 1, 4, None, None, 0, z, None, None,
+                                                None) == O.EINVAL
+    assert built_lib.outlets_predict_step_ex(None, taps, None, 1, None, None, z, None, None, None) == O.EINVAL
     assert built_lib.outlets_kv_reset_slot(None, 0) == O.EINVAL
     assert built_lib.outlets_kv_slot_length(None, 0) == -1
     assert built_lib.outlets_kv_free_pages(None) == -1

@@ -62,8 +62,9 @@ def parse():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--mode", default="both", choices=["both", "prefill", "step", "sweep"],
-                    help="static prediction (headline), dynamic prediction, both, or the serving sweep")
+    ap.add_argument("--mode", default="both", choices=["both", "prefill", "step", "sweep", "sched"],
+                    help="static prediction (headline), dynamic prediction, both, the serving sweep, or the "
+                         "length-aware scheduling model (host code, Sec. 5.5)")
     ap.add_argument("--prompts", type=int, default=None,
                     help="first N prompts of the workload (profiling cases; default: all)")
     ap.add_argument("--gated", action="store_true",
@@ -279,6 +280,79 @@ def run_reference(args):
            "cpu_baseline": {"value": value, "unit": "predictions/s", "cores": cpu_threads(), "kind": "oracle",
                             "sample": f"{n_pred} prompts / {n_tok} tokens over {args.steps} steps"},
            "e2e": {"value": value, "unit": "predictions/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+
+
+SCHED_CFG = dict(n_decode=3, max_running=128, pf_base=0.005, pf_per_token=2e-5, step_base=0.02,
+                 step_per_seq=1e-4, step_per_kv=1e-8)
+SCHED_TRACE = dict(n=6000, qps=13.0)
+
+
+def serving_metrics(arrival, output, finish):
+    """Throughput (output tokens / makespan), mean latency, P99 latency (nearest rank) of
+    short (< 800), medium and long (>= 1300 tokens) requests: the categories of Sec. 5.5."""
+    lat = finish - arrival
+    out = {"throughput_tok_s": float(output.sum() / (finish.max() - arrival.min())),
+           "mean_latency_s": float(lat.mean())}
+    for name, sel in (("short", output < 800), ("medium", (output >= 800) & (output < 1300)),
+                      ("long", output >= 1300)):
+        out[f"p99_{name}_s"] = float(np.percentile(lat[sel], 99, method="inverted_cdf")) if sel.any() else None
+    return {k: (round(v, 3) if isinstance(v, float) else v) for k, v in out.items()}
+
+
+def run_sched(args):
+    """Length-aware serving model (include/outlets_sched.h): one prefill and three
+    decode instances at saturation; RR+FCFS vs RR+SJF vs LB+SJF driven by the
+    static prediction (stand-in predictions: true length x lognormal noise).
+    value = requests the C++ model simulates per second (LB+SJF, whole trace)."""
+    from oracle import sched_oracle as S
+    from paper_2609_01068_gb300 import build as B
+    from paper_2609_01068_gb300 import outlets, synth
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    B.build()
+    n, qps = SCHED_TRACE["n"], SCHED_TRACE["qps"]
+    traces = {"exact": synth.make_serving_requests(n, qps, 0, pred_sigma=0.0),
+              "noisy (sigma 0.5)": synth.make_serving_requests(n, qps, 0, pred_sigma=0.5)}
+    none = dict(traces["exact"])
+    none["predicted"] = np.full(n, float(np.median(none["output"])), np.float32)
+    traces["none (constant)"] = none
+    policies = {"RR+FCFS": (0, 0), "RR+SJF": (0, 1), "LB+SJF": (1, 1)}
+    results = {}
+    for pname, (route, order) in policies.items():
+        for tname, w in traces.items():
+            if pname == "RR+FCFS" and tname != "exact":
+                continue  # uses no prediction
+            cfg = dict(SCHED_CFG, route=route, order=order)
+            fin, _ = outlets.simulate_serving(cfg, w["arrival"], w["prompt"], w["output"], w["predicted"])
+            results[pname if pname == "RR+FCFS" else f"{pname}, {tname} predictions"] = serving_metrics(
+                w["arrival"], w["output"], fin)
+    w = traces["noisy (sigma 0.5)"]
+    cfg = dict(SCHED_CFG, route=1, order=1)
+    for _ in range(args.warmup):
+        outlets.simulate_serving(cfg, w["arrival"], w["prompt"], w["output"], w["predicted"])
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        outlets.simulate_serving(cfg, w["arrival"], w["prompt"], w["output"], w["predicted"])
+    secs = time.perf_counter() - t0
+    value = n * args.steps / secs
+    ns = 2000  # oracle on a bounded sample (the first 2000 requests)
+    t0 = time.perf_counter()
+    S.simulate(cfg, [float(x) for x in w["arrival"][:ns]], [int(x) for x in w["prompt"][:ns]],
+               [int(x) for x in w["output"][:ns]], [float(x) for x in w["predicted"][:ns]])
+    osecs = time.perf_counter() - t0
+    out = {"metric": "length-aware scheduling model: simulated requests/s", "value": value,
+           "unit": "simulated requests/s", "n_gpus": 0, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": 1000 * secs / args.steps, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": f"{n} requests, Poisson {qps} QPS, prompts LN(ln 256, 1), outputs LN(ln 700, 0.8); "
+                                  "1 prefill + 3 decode instances, 128-request continuous batches (host model)",
+                      "model": SCHED_CFG},
+           "roofline": None, "gpu_launches": 0,
+           "policies": results,
+           "cpu_baseline": {"value": ns / osecs, "unit": "simulated requests/s", "cores": 1, "kind": "oracle",
+                            "sample": f"first {ns} requests of the trace, LB+SJF, {osecs:.1f} s"}}
     print(json.dumps(out))
 
 
@@ -690,7 +764,9 @@ def run_sweep(args, shape, w, world, local, barrier, max_over_ranks, stream):
 
 def main():
     args = parse()
-    if args.impl == "reference":
+    if args.mode == "sched":
+        run_sched(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

@@ -21,7 +21,9 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "liboutlets_gb300.so")
 SOURCES = ["outlets.cu", "gemm_tc.cu", "attn_prefill.cu", "attn_prefill_tc.cu", "attn_decode.cu", "elementwise.cu",
-           "lm_head.cu"]
+           "lm_head.cu", "sched.cpp"]
+# host-only sources: IEEE double results that do not depend on the host (no contracted multiply-adds)
+HOST_FLAGS = ["-Xcompiler", "-ffp-contract=off"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 
@@ -56,7 +58,8 @@ def build(force: bool = False, verbose: bool = False) -> str:
 
     def compile_one(src):
         obj = os.path.join(BUILD_DIR, os.path.splitext(src)[0] + ".o")
-        cmd = [nvcc, *ARCH, *NVCC_FLAGS, "-c", os.path.join(CSRC, src), "-o", obj]
+        cmd = [nvcc, *ARCH, *NVCC_FLAGS, *(HOST_FLAGS if src.endswith(".cpp") else []), "-c",
+               os.path.join(CSRC, src), "-o", obj]
         if verbose:
             cmd.insert(1, "-Xptxas=-v")
         r = subprocess.run(cmd, capture_output=True, text=True)

@@ -48,6 +48,17 @@ class DraftOut(ctypes.Structure):
     _fields_ = [("k", c_i32), ("topk_ids", c_vp), ("topk_logprob", c_vp), ("logsumexp", c_vp), ("logits", c_vp)]
 
 
+class SchedConfig(ctypes.Structure):
+    _fields_ = [("n_decode", c_i32), ("max_running", c_i32), ("route", c_i32), ("order", c_i32),
+                ("pf_base_s", ctypes.c_double), ("pf_per_token_s", ctypes.c_double),
+                ("step_base_s", ctypes.c_double), ("step_per_seq_s", ctypes.c_double),
+                ("step_per_kv_token_s", ctypes.c_double)]
+
+
+ROUTE_RR, ROUTE_LB = 0, 1
+ORDER_FCFS, ORDER_SJF = 0, 1
+
+
 class TensorInfo(ctypes.Structure):
     _fields_ = [("dtype", c_i32), ("rows", c_i32), ("cols", c_i32)]
 
@@ -98,6 +109,7 @@ def load():
         "outlets_launch_count": (ctypes.c_uint64, [c_vp]),
         "outlets_length_head_noalloc": (c_i32, [c_vp, c_vp, c_i32, c_vp, c_vp, c_vp]),
         "outlets_selftest_bounded_wait": (c_i32, [c_vp, ctypes.c_uint64, c_vp]),
+        "outlets_sched_simulate": (c_i32, [P(SchedConfig), c_i32, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -412,3 +424,31 @@ class KVCache:
             self.close()
         except Exception:
             pass
+
+
+def simulate_serving(cfg: dict, arrival, prompt_len, output_len, predicted_len):
+    """Length-aware serving model of include/outlets_sched.h (host code).
+
+    cfg keys: n_decode, max_running, route (ROUTE_RR / ROUTE_LB), order
+    (ORDER_FCFS / ORDER_SJF), pf_base, pf_per_token, step_base, step_per_seq,
+    step_per_kv (seconds).  Returns (finish time [n] f64, decode instance [n] i32).
+    """
+    lib = load()
+    c = SchedConfig()
+    c.n_decode, c.max_running, c.route, c.order = cfg["n_decode"], cfg["max_running"], cfg["route"], cfg["order"]
+    c.pf_base_s, c.pf_per_token_s = cfg["pf_base"], cfg["pf_per_token"]
+    c.step_base_s, c.step_per_seq_s, c.step_per_kv_token_s = cfg["step_base"], cfg["step_per_seq"], cfg["step_per_kv"]
+    a = np.ascontiguousarray(arrival, dtype=np.float64)
+    p = np.ascontiguousarray(prompt_len, dtype=np.int32)
+    o = np.ascontiguousarray(output_len, dtype=np.int32)
+    r = np.ascontiguousarray(predicted_len, dtype=np.float32)
+    n = len(a)
+    if not (len(p) == len(o) == len(r) == n):
+        raise ValueError("arrays must have the same length")
+    fin = np.zeros(n, np.float64)
+    inst = np.zeros(n, np.int32)
+    st = lib.outlets_sched_simulate(ctypes.byref(c), n, a.ctypes.data, p.ctypes.data, o.ctypes.data, r.ctypes.data,
+                                    fin.ctypes.data, inst.ctypes.data)
+    if st != OK:
+        raise OutletsError(st, "outlets_sched_simulate rejected its arguments")
+    return fin, inst

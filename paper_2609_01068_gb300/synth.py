@@ -10,7 +10,8 @@ Shapes follow the draft backbones the method is evaluated with (Sec. 5.1,
 Recipe (all draws from numpy PCG64 streams spawned from one SeedSequence):
   * stream 0 -> sequence / cache lengths;  stream 1 -> taps;  stream 2 -> weights;
     stream 3 -> draft LM head W_lm (Eq. 2) and stand-in draft states;
-    stream 4 -> input-embedding branch (embedding table, its QKV columns, token ids).
+    stream 4 -> input-embedding branch (embedding table, its QKV columns, token ids);
+    stream 5 -> serving workloads (arrivals, prompt and output lengths, prediction noise).
   * lengths: rint(lognormal(ln(median), sigma=1)) clipped to the stated range.
   * taps ~ N(0, 1); every Linear weight ~ N(0, 0.02); RMSNorm gains = 1;
     head hidden biases ~ N(0, 0.02); output bias = ln(1 + 256).
@@ -30,7 +31,7 @@ __all__ = [
     "lengths_tiny", "lengths_8b_prefill", "lengths_8b_step_cache",
     "lengths_70b_prefill", "lengths_sweep", "cu_seqlens",
     "make_weights", "make_taps", "weight_names",
-    "LLAMA3_VOCAB", "make_lm_head", "make_draft_states", "make_tokens",
+    "LLAMA3_VOCAB", "make_lm_head", "make_draft_states", "make_tokens", "make_serving_requests",
 ]
 
 
@@ -239,3 +240,19 @@ def make_taps(shape: ModelShape, n_tokens: int, seed: int = 0, stream_offset: in
     rng = np.random.Generator(np.random.PCG64(ss))
     rnd = round_bf16 if shape.dtype == "bf16" else (lambda a: a)
     return [rnd(rng.standard_normal((n_tokens, shape.d), dtype=np.float32)) for _ in range(3)]
+
+
+def make_serving_requests(n: int, qps: float, seed: int = 0, pred_sigma: float = 0.5,
+                          prompt_median: float = 256, output_median: float = 700):
+    """A serving trace for the scheduling model: Poisson arrivals at qps,
+    prompt lengths lognormal (median prompt_median, sigma 1, clipped 16-4096),
+    output lengths lognormal (median output_median, sigma 0.8, clipped 1-8192),
+    and stand-in static predictions output * exp(pred_sigma * N(0, 1)) as f32
+    (pred_sigma = 0: exact predictions).  Returns a dict of numpy arrays."""
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence(seed).spawn(6)[5]))
+    arrival = np.cumsum(rng.exponential(1.0 / qps, size=n))
+    prompt = np.clip(np.rint(rng.lognormal(math.log(prompt_median), 1.0, n)), 16, 4096).astype(np.int32)
+    output = np.clip(np.rint(rng.lognormal(math.log(output_median), 0.8, n)), 1, 8192).astype(np.int32)
+    noise = np.exp(pred_sigma * rng.standard_normal(n))
+    predicted = (output * noise).astype(np.float32)
+    return {"arrival": arrival, "prompt": prompt, "output": output, "predicted": predicted}

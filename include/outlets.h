@@ -252,6 +252,26 @@ outlets_status outlets_predict_step_ex(outlets_ctx* ctx, const void* const taps[
                                        outlets_kv* kv, const int32_t* slots, float* z_out, float* len_out,
                                        const outlets_draft_out* draft, void* stream);
 
+/* ---- Draft rollouts (EAGLE-3-style multi-token drafting).
+ * One more draft position per request: the feature input is the draft
+ * layer's own output state y (the residual stream before the final norm) of
+ * the request's previous position, in place of Eq. 1's fused taps, so no
+ * target hidden states are needed.  It must follow a step (tapped or draft)
+ * of this context over the same slots in the same order (EINVAL otherwise);
+ * each request's position is its slot length, which grows by one.  tokens:
+ * device or host int32 [B], the drafted tokens (e.g. the previous call's
+ * top-1 draft ids, left on the device), required iff the context has the
+ * input-embedding branch.  draft: optional, as in the *_dual calls.
+ * The outputs are the length prediction at the draft position. */
+outlets_status outlets_predict_draft_step(outlets_ctx* ctx, const int32_t* tokens, int32_t B, outlets_kv* kv,
+                                          const int32_t* slots, float* z_out, float* len_out,
+                                          const outlets_draft_out* draft, void* stream);
+
+/* Keeps the first `length` cached positions of a slot (0 <= length <= its
+ * length), e.g. to drop draft positions the target rejected.  Host
+ * bookkeeping only, ordered after earlier calls like outlets_kv_reset_slot. */
+outlets_status outlets_kv_truncate(outlets_kv* kv, int32_t slot, int32_t length);
+
 /* The draft head alone on caller-given states.
  *   h_draft  device [rows, d] (bf16 or f32 like the context), 16-byte aligned.
  *   draft    outputs as above, rows rows. */

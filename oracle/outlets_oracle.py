@@ -42,6 +42,12 @@ Readings where the paper is silent (the same list is kept in the design notes):
     QKV projections (and the attention gate) take 2d inputs; the residual
     stream stays f_ctx.  Used when the weights carry "w_embed" and the call
     gives one token id per row;
+  * draft rollouts (EAGLE-3-style multi-token drafting, Sec. 2): a draft
+    position after the first takes the draft layer's output state y (the
+    residual stream before the final norm) of the previous position as its
+    feature input in place of the fused taps, with the drafted token's
+    embedding; its K/V are cached like any position (and dropped again when
+    the target rejects it);
   * dual head (Sec. 4.2, Eq. 2): the draft branch reads the same final-normed
     state h^draft as the length head; its output is the log of the softmax of
     W_lm h^draft over the vocabulary, reported as the k most probable tokens
@@ -314,7 +320,7 @@ def caches_from_prefill(out, cu):
             for b in range(len(cu) - 1)]
 
 
-def predict_step(w, shape, taps_rows, caches, draft_k=None, tokens=None):
+def predict_step(w, shape, taps_rows, caches, draft_k=None, tokens=None, f_rows=None):
     """Dynamic prediction for one new token per request (Sec. 3.2, t >= 1).
 
     taps_rows: three [B, d] arrays; caches: list of B (k [L, KVH, hd],
@@ -322,13 +328,16 @@ def predict_step(w, shape, taps_rows, caches, draft_k=None, tokens=None):
     at position L of its request.  Returns z_hat, length_hat, intermediates and
     the caches extended by the new token (and "draft" as in predict_prefill).
     tokens: [B] ids of the new tokens (input-embedding branch).
+    f_rows: [B, d] feature input in place of Eq. 1's fused taps: a draft
+    rollout step (EAGLE-3-style multi-token drafting) feeds the draft layer's
+    own output state y of the request's previous position back in.
     """
     H, KVH, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
     eps, theta = shape.rms_eps, shape.rope_theta
-    B = taps_rows[0].shape[0]
+    B = len(caches)
     pos = np.array([c[0].shape[0] for c in caches], dtype=np.int64)
 
-    f = fuse_taps(taps_rows, w["w_proj"])
+    f = fuse_taps(taps_rows, w["w_proj"]) if f_rows is None else _f64(f_rows)
     x = layer_input(w, f, tokens, eps)
     q = apply_rope((x @ _f64(w["w_q"]).T).reshape(B, H, hd), pos, theta)
     k = apply_rope((x @ _f64(w["w_k"]).T).reshape(B, KVH, hd), pos, theta)

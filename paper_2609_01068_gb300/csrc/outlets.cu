@@ -190,6 +190,8 @@ struct outlets_ctx {
   bool have_prev = false;
 
   int last_rows = 0, last_out_rows = 0;
+  int last_kind = 0;              // 0: none, 1: prefill, 2: step or draft step (its y rows feed a draft step)
+  std::vector<int> last_slots;    // slots of the last step, in row order
   bool oom = false;
   std::unordered_map<MapKey, CUtensorMap, MapKeyHash> map_cache;  // library-owned buffers only
 
@@ -831,13 +833,25 @@ struct QkvSrc {
 
 // FC (Eq. 1) -> input RMSNorm -> QKV for rows row0 .. row0 + rows - 1 (tp
 // points at row row0 of each tap; row0 > 0 only on the large-M path).
+outlets_status run_qkv(outlets_ctx* c, int rows, QkvSrc* q, cudaStream_t s, int row0, const int* tok_dev, int sl,
+                       int n_norm);
+
 outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvSrc* q, cudaStream_t s,
                          int row0, const int* tok_dev) {
   const int d = c->d;
   const float eps = c->cfg.rms_eps;
   const bool small = small_path(c, rows);
-  c->stage_begin(OUTLETS_S_FC);
   int sl = 1;
+  if (!tp) {
+    // draft rollout step: the feature input is the draft layer's own output
+    // state y of the previous step (same rows), in place of Eq. 1's fused taps
+    c->stage_begin(OUTLETS_S_NORM_IN);
+    OUT_CK(c, cudaMemcpyAsync(c->f, c->y, (size_t)rows * d * 4, cudaMemcpyDeviceToDevice, s));
+    if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xhat, nullptr, rows, d, eps, s));
+    else OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
+    return run_qkv(c, rows, q, s, row0, tok_dev, sl, 1);
+  }
+  c->stage_begin(OUTLETS_S_FC);
   if (small) OUT_TRY(gemm_split(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, c->part, &sl, s));
   else if (c->bf16)
     OUT_TRY(gemm_tc(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, EPI_F32, c->f + (size_t)row0 * d, d, nullptr,
@@ -853,7 +867,16 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
                                    d, eps, s));
   else
     OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
-  int n_norm = 1;
+  return run_qkv(c, rows, q, s, row0, tok_dev, sl, 1);
+}
+
+// Input-embedding branch (if any) and the QKV projection; the input-norm stage
+// (n_norm kernels so far) is still open.
+outlets_status run_qkv(outlets_ctx* c, int rows, QkvSrc* q, cudaStream_t s, int row0, const int* tok_dev, int sl,
+                       int n_norm) {
+  const int d = c->d;
+  const float eps = c->cfg.rms_eps;
+  const bool small = small_path(c, rows);
   const void* xr = (const char*)c->xhat + (size_t)row0 * d * c->esz;
   const void* a1[3] = {xr, xr, xr};
   int pieces = 1;
@@ -1314,6 +1337,17 @@ void outlets_kv_destroy(outlets_kv* kv) {
   delete kv;
 }
 
+outlets_status outlets_kv_truncate(outlets_kv* kv, int32_t slot, int32_t length) {
+  if (!kv || slot < 0 || slot >= kv->max_slots || length < 0 || length > kv->len[slot]) return OUTLETS_EINVAL;
+  const size_t keep = (size_t)cdiv(length, kPageTokens);
+  while (kv->pages[slot].size() > keep) {
+    kv->free_list.push_back(kv->pages[slot].back());
+    kv->pages[slot].pop_back();
+  }
+  kv->len[slot] = length;
+  return OUTLETS_OK;
+}
+
 outlets_status outlets_kv_reset_slot(outlets_kv* kv, int32_t slot) {
   if (!kv || slot < 0 || slot >= kv->max_slots) return OUTLETS_EINVAL;
   for (int p : kv->pages[slot]) kv->free_list.push_back(p);
@@ -1406,6 +1440,7 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
 
   OUT_TRY(begin_call(c, s));
   CallSlot slot_guard{c, s};
+  c->last_kind = 0;
   // Large calls with host taps overlap the copy with the front of the pipeline
   // (FC, input norm, QKV, RoPE are row-wise): rows run in chunks of whole
   // 128-row tiles as their taps land.
@@ -1560,14 +1595,24 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   if (draft) OUT_TRY(run_draft(c, c->hn, out_rows, *draft, s));
   c->last_rows = T;
   c->last_out_rows = out_rows;
+  c->last_kind = 1;
+  c->last_slots.clear();
   return end_call(c, out_rows, z_out, len_out, s);
 }
 
 outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int32_t* tokens, int32_t B,
                             outlets_kv* kv, const int32_t* slots, float* z_out, float* len_out,
-                            const outlets_draft_out* draft, void* stream) {
+                            const outlets_draft_out* draft, void* stream, bool self_feed = false) {
   cudaStream_t s = (cudaStream_t)stream;
-  if (!taps || !kv || !slots || !z_out) return c->fail(OUTLETS_EINVAL, "taps, kv, slots and z_out must not be NULL");
+  if ((!taps && !self_feed) || !kv || !slots || !z_out)
+    return c->fail(OUTLETS_EINVAL, "taps, kv, slots and z_out must not be NULL");
+  if (self_feed) {
+    bool same = c->last_kind == 2 && (int)c->last_slots.size() == B;
+    for (int b = 0; same && b < B; ++b) same = c->last_slots[b] == slots[b];
+    if (!same)
+      return c->fail(OUTLETS_EINVAL,
+                     "a draft step follows a step or draft step of this context over the same slots, in the same order");
+  }
   if (kv->ctx != c) return c->fail(OUTLETS_EINVAL, "kv belongs to another context");
   if (B < 0) return c->fail(OUTLETS_EINVAL, "B must be >= 0");
   if (B == 0) return OUTLETS_OK;
@@ -1587,8 +1632,9 @@ outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int
 
   OUT_TRY(begin_call(c, s));
   CallSlot slot_guard{c, s};
-  const void* tp[3];
-  OUT_TRY(prepare_taps(c, taps, B, tp, s));
+  c->last_kind = 0;  // y is rewritten from here on: a later draft step needs this call to complete
+  const void* tp[3] = {nullptr, nullptr, nullptr};
+  if (!self_feed) OUT_TRY(prepare_taps(c, taps, B, tp, s));
 
   // ---- commit the append and build metadata
   std::vector<int> pos(B), seq_len(B), po(B + 1, 0), pl, work, work_off(B + 1, 0);
@@ -1641,7 +1687,7 @@ outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int
   const int* m = c->meta_dev;
 
   QkvSrc qsrc;
-  OUT_TRY(run_front(c, tp, B, &qsrc, s, 0, tok_host ? m + off_tok : tokens));
+  OUT_TRY(run_front(c, self_feed ? nullptr : tp, B, &qsrc, s, 0, tok_host ? m + off_tok : tokens));
   OUT_TRY(wait_meta(c, s));  // RoPE is the first kernel that reads the metadata
   c->stage_begin(OUTLETS_S_ROPE);
   {
@@ -1710,6 +1756,8 @@ outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int
   if (draft) OUT_TRY(run_draft(c, c->hn, B, *draft, s));
   c->last_rows = B;
   c->last_out_rows = B;
+  c->last_kind = 2;
+  c->last_slots.assign(slots, slots + B);
   return end_call(c, B, z_out, len_out, s);
 }
 
@@ -1768,6 +1816,15 @@ outlets_status outlets_predict_step_ex(outlets_ctx* c, const void* const taps[3]
   c->err.clear();
   if (draft) OUT_TRY(check_draft(c, draft));
   return predict_step(c, taps, tokens, B, kv, slots, z_out, len_out, draft, stream);
+}
+
+outlets_status outlets_predict_draft_step(outlets_ctx* c, const int32_t* tokens, int32_t B, outlets_kv* kv,
+                                          const int32_t* slots, float* z_out, float* len_out,
+                                          const outlets_draft_out* draft, void* stream) {
+  if (!c) return OUTLETS_EINVAL;
+  c->err.clear();
+  if (draft) OUT_TRY(check_draft(c, draft));
+  return predict_step(c, nullptr, tokens, B, kv, slots, z_out, len_out, draft, stream, true);
 }
 
 outlets_status outlets_draft_head(outlets_ctx* c, const void* h_draft, int32_t rows, const outlets_draft_out* draft,

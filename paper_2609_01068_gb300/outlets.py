@@ -101,6 +101,8 @@ def load():
         "outlets_predict_prefill_ex": (c_i32, [c_vp, P(c_vp), c_vp, c_vp, c_i32, c_i32, c_vp, c_vp, ctypes.c_uint32,
                                                c_vp, c_vp, c_vp, c_vp]),
         "outlets_predict_step_ex": (c_i32, [c_vp, P(c_vp), c_vp, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]),
+        "outlets_predict_draft_step": (c_i32, [c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]),
+        "outlets_kv_truncate": (c_i32, [c_vp, c_i32, c_i32]),
         "outlets_check": (c_i32, [c_vp, c_vp]),
         "outlets_get_intermediate": (c_i32, [c_vp, c_i32, c_vp, ctypes.c_size_t, P(TensorInfo), c_vp]),
         "outlets_profile_enable": (c_i32, [c_vp, c_i32]),
@@ -336,6 +338,26 @@ class Predictor:
             self._raise(st)
         return draft
 
+    def draft_step(self, kv, slots, tokens=None, k=None, logits=False, out=None, z_out=None, len_out=None,
+                   stream=None):
+        """One draft rollout position per request, fed by the previous step's own output
+        state: (z_hat, length_hat) or, with k, (z_hat, length_hat, draft outputs)."""
+        sl = np.ascontiguousarray(slots, dtype=np.int32)
+        B = len(sl)
+        like = tokens if tokens is not None and hasattr(tokens, "device") else z_out
+        if like is None:
+            import torch
+            like = torch.empty(0, device=f"cuda:{self.device}")
+        z_out, len_out = self._outputs(B, like, z_out, len_out)
+        d, draft = (self._draft_out(B, k, like, logits, out) if k else (None, None))
+        tok = None if tokens is None else _tokens(tokens)
+        st = self.lib.outlets_predict_draft_step(self.h, _ptr(tok), B, kv.h, sl.ctypes.data, _ptr(z_out),
+                                                 _ptr(len_out), ctypes.byref(d) if d is not None else None,
+                                                 _stream_handle(stream))
+        if st != OK:
+            self._raise(st)
+        return (z_out, len_out, draft) if k else (z_out, len_out)
+
     def selftest_bounded_wait(self, timeout_ns=1_000_000, stream=None):
         """Enqueue a kernel whose bounded wait runs out (see outlets_check)."""
         st = self.lib.outlets_selftest_bounded_wait(self.h, timeout_ns, _stream_handle(stream))
@@ -406,6 +428,12 @@ class KVCache:
         st = self.lib.outlets_kv_reset_slot(self.h, slot)
         if st != OK:
             raise OutletsError(st, "bad slot")
+
+    def truncate(self, slot, length):
+        """Keep the first `length` cached positions of a slot (drop rejected draft positions)."""
+        st = self.lib.outlets_kv_truncate(self.h, slot, length)
+        if st != OK:
+            raise OutletsError(st, "bad slot or length")
 
     def slot_length(self, slot):
         return self.lib.outlets_kv_slot_length(self.h, slot)

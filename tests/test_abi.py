@@ -37,7 +37,7 @@ def test_header_declares_the_entry_points():
     for must in ("outlets_create", "outlets_predict_prefill", "outlets_predict_step", "outlets_kv_create",
                  "outlets_destroy", "outlets_last_error", "outlets_predict_prefill_dual",
                  "outlets_predict_step_dual", "outlets_draft_head", "outlets_predict_prefill_ex",
-                 "outlets_predict_step_ex"):
+                 "outlets_predict_step_ex", "outlets_predict_draft_step", "outlets_kv_truncate"):
         assert must in names
 
 
@@ -98,6 +98,8 @@ def test_null_handles_are_rejected(built_lib):
     assert built_lib.outlets_predict_prefill_ex(None, taps, None, cu, 1, 4, None, None, 0, z, None, None,
                                                 None) == O.EINVAL
     assert built_lib.outlets_predict_step_ex(None, taps, None, 1, None, None, z, None, None, None) == O.EINVAL
+    assert built_lib.outlets_predict_draft_step(None, None, 1, None, None, z, None, None, None) == O.EINVAL
+    assert built_lib.outlets_kv_truncate(None, 0, 0) == O.EINVAL
     assert built_lib.outlets_kv_reset_slot(None, 0) == O.EINVAL
     assert built_lib.outlets_kv_slot_length(None, 0) == -1
     assert built_lib.outlets_kv_free_pages(None) == -1

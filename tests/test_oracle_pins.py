@@ -614,3 +614,36 @@ def test_embedding_draw_keeps_the_fused_feature_columns():
     for name in p:
         if name not in ("w_q", "w_k", "w_v", "w_attn_gate"):
             np.testing.assert_array_equal(w[name], p[name])
+
+
+# ---------------------------------------------------------------- draft rollouts
+def test_draft_step_with_the_fused_feature_is_a_normal_step():
+    """Feeding f_ctx itself as the feature input reproduces the tapped step."""
+    w, cu, taps, tok = _embed_case(lengths=(4, 6))
+    caches = O.caches_from_prefill(O.predict_prefill(w, SMALL, taps, cu, tokens=tok), cu)
+    st = _taps(SMALL, 2, 0, 9)
+    stok = synth.make_tokens(2, EV, 0, 9)
+    a = O.predict_step(w, SMALL, st, caches, tokens=stok)
+    b = O.predict_step(w, SMALL, None, caches, tokens=stok, f_rows=O.fuse_taps(st, w["w_proj"]))
+    np.testing.assert_array_equal(a["z"], b["z"])
+    np.testing.assert_array_equal(a["caches"][1][0], b["caches"][1][0])
+
+
+def test_rollout_then_rollback_equals_never_drafting():
+    """Two draft positions appended and dropped again (the target rejected
+    them): the next tapped step sees exactly the cache it would have seen."""
+    w, cu, taps, tok = _embed_case(lengths=(5, 3))
+    caches = O.caches_from_prefill(O.predict_prefill(w, SMALL, taps, cu, tokens=tok), cu)
+    st = _taps(SMALL, 2, 0, 11)
+    s1 = O.predict_step(w, SMALL, st, caches, tokens=synth.make_tokens(2, EV, 0, 11))
+    d1 = O.predict_step(w, SMALL, None, s1["caches"], tokens=synth.make_tokens(2, EV, 0, 12), f_rows=s1["y"])
+    d2 = O.predict_step(w, SMALL, None, d1["caches"], tokens=synth.make_tokens(2, EV, 0, 13), f_rows=d1["y"])
+    assert d2["caches"][0][0].shape[0] == s1["caches"][0][0].shape[0] + 2
+    rolled = [(k[:-2], v[:-2]) for k, v in d2["caches"]]
+    for (ka, va), (kb, vb) in zip(rolled, s1["caches"]):
+        np.testing.assert_array_equal(ka, kb)
+        np.testing.assert_array_equal(va, vb)
+    nxt = _taps(SMALL, 2, 0, 14)
+    t2 = synth.make_tokens(2, EV, 0, 14)
+    np.testing.assert_array_equal(O.predict_step(w, SMALL, nxt, rolled, tokens=t2)["z"],
+                                  O.predict_step(w, SMALL, nxt, s1["caches"], tokens=t2)["z"])

@@ -983,10 +983,23 @@ outlets_status begin_call(outlets_ctx* c, cudaStream_t s) {
   return OUTLETS_OK;
 }
 
-outlets_status end_call(outlets_ctx* c, int out_rows, float* z_out, float* len_out, cudaStream_t s) {
-  if (z_out != c->z) OUT_CK(c, cudaMemcpyAsync(z_out, c->z, (size_t)out_rows * 4, cudaMemcpyDefault, s));
-  if (len_out && len_out != c->len)
-    OUT_CK(c, cudaMemcpyAsync(len_out, c->len, (size_t)out_rows * 4, cudaMemcpyDefault, s));
+// Where the head writes z_hat and the length: straight into the caller's
+// buffers when they are device memory (no copy after the head, so the next
+// call's first kernel can start under this call's last one), else into the
+// context's buffers, copied out by end_call.
+struct OutDst {
+  float* z;
+  float* len;
+};
+OutDst out_dst(outlets_ctx* c, float* z_out, float* len_out) {
+  return {is_device_ptr(z_out) ? z_out : c->z, (len_out && is_device_ptr(len_out)) ? len_out : c->len};
+}
+
+outlets_status end_call(outlets_ctx* c, int out_rows, float* z_out, float* len_out, const OutDst& od,
+                        cudaStream_t s) {
+  if (z_out != od.z) OUT_CK(c, cudaMemcpyAsync(z_out, od.z, (size_t)out_rows * 4, cudaMemcpyDefault, s));
+  if (len_out && len_out != od.len)
+    OUT_CK(c, cudaMemcpyAsync(len_out, od.len, (size_t)out_rows * 4, cudaMemcpyDefault, s));
   OUT_CK(c, cudaEventRecord(c->done_ev, s));
   c->have_prev = true;
   return OUTLETS_OK;
@@ -1591,13 +1604,14 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
                                               (const float*)c->gate_act, s));
   }
   c->stage_end(1);
-  OUT_TRY(run_tail(c, T, out_rows, all_tokens ? nullptr : m + off_last, c->z, c->len, s));
+  const OutDst od = out_dst(c, z_out, len_out);
+  OUT_TRY(run_tail(c, T, out_rows, all_tokens ? nullptr : m + off_last, od.z, od.len, s));
   if (draft) OUT_TRY(run_draft(c, c->hn, out_rows, *draft, s));
   c->last_rows = T;
   c->last_out_rows = out_rows;
   c->last_kind = 1;
   c->last_slots.clear();
-  return end_call(c, out_rows, z_out, len_out, s);
+  return end_call(c, out_rows, z_out, len_out, od, s);
 }
 
 outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int32_t* tokens, int32_t B,
@@ -1752,13 +1766,14 @@ outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int
       c->stage_end(1);
     }
   }
-  OUT_TRY(run_tail(c, B, B, nullptr, c->z, c->len, s));
+  const OutDst od = out_dst(c, z_out, len_out);
+  OUT_TRY(run_tail(c, B, B, nullptr, od.z, od.len, s));
   if (draft) OUT_TRY(run_draft(c, c->hn, B, *draft, s));
   c->last_rows = B;
   c->last_out_rows = B;
   c->last_kind = 2;
   c->last_slots.assign(slots, slots + B);
-  return end_call(c, B, z_out, len_out, s);
+  return end_call(c, B, z_out, len_out, od, s);
 }
 
 }  // namespace

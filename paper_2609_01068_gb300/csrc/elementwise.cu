@@ -232,7 +232,7 @@ __global__ void __launch_bounds__(256) k_embed_rmsnorm(const int* __restrict__ t
 template <typename In>
 struct RopeBlock {
   static constexpr int kThreads = std::is_same<In, float>::value ? 320 : 128;
-  static constexpr int kMinBlocks = std::is_same<In, float>::value ? 2 : 12;
+  static constexpr int kMinBlocks = std::is_same<In, float>::value ? 2 : 10;  // bf16: 51 registers, no spills
 };
 
 template <typename In, typename Act>

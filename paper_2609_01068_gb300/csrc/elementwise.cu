@@ -387,7 +387,8 @@ __global__ void __launch_bounds__(512) k_head_tail(const float* __restrict__ h, 
 
 template <typename Act>
 __global__ void k_convert_rows(const float* __restrict__ src, Act* __restrict__ dst, int rows, int cols,
-                               long long dst_ld, int row_mode, int row_base, long long kb_np) {
+                               long long dst_ld, int row_mode, int row_base, long long kb_np,
+                               const float* __restrict__ col_scale) {
   const long long n = (long long)rows * cols;
   for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n;
        idx += (long long)gridDim.x * blockDim.x) {
@@ -405,7 +406,7 @@ __global__ void k_convert_rows(const float* __restrict__ src, Act* __restrict__ 
     } else {
       o = dr * dst_ld + c;
     }
-    dst[o] = from_f<Act>(src[idx]);
+    dst[o] = from_f<Act>(col_scale ? src[idx] * col_scale[c] : src[idx]);
   }
 }
 
@@ -566,10 +567,10 @@ cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_st
 
 template <typename Act>
 cudaError_t convert_rows_launch(const float* src, Act* dst, int rows, int cols, long long dst_ld, int row_mode,
-                                int row_base, long long kb_np, cudaStream_t stream) {
+                                int row_base, long long kb_np, const float* col_scale, cudaStream_t stream) {
   if (rows == 0 || cols == 0) return cudaSuccess;
   OUTLETS_TRY_LAUNCH(launch_k(k_convert_rows<Act>, dim3(grid_for((long long)rows * cols, 256)), dim3(256), 0, stream, src, dst, rows, cols, dst_ld,
-                                                                                row_mode, row_base, kb_np));
+                                                                                row_mode, row_base, kb_np, col_scale));
   return cudaGetLastError();
 }
 
@@ -597,7 +598,7 @@ cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int ep
   template cudaError_t embed_rmsnorm_launch<Act>(const int*, const Act*, int, const float*, Act*, int, int, float, \
                                                  int*, cudaStream_t);                                          \
   template cudaError_t convert_rows_launch<Act>(const float*, Act*, int, int, long long, int, int, long long,       \
-                                                cudaStream_t);                                                  \
+                                                const float*, cudaStream_t);                                    \
   template cudaError_t rope_scatter_launch<float, Act>(const float*, const RopeArgs&, cudaStream_t);           \
   template cudaError_t rope_scatter_launch<Act, Act>(const Act*, const RopeArgs&, cudaStream_t);
 OUTLETS_INST_ACT(bf16)
@@ -610,7 +611,7 @@ template cudaError_t swiglu_launch<float>(const float*, float*, int, int, cudaSt
 template cudaError_t embed_rmsnorm_launch<float>(const int*, const float*, int, const float*, float*, int, int, float,
                                                  int*, cudaStream_t);
 template cudaError_t convert_rows_launch<float>(const float*, float*, int, int, long long, int, int, long long,
-                                                cudaStream_t);
+                                                const float*, cudaStream_t);
 template cudaError_t rope_scatter_launch<float, float>(const float*, const RopeArgs&, cudaStream_t);
 #undef OUTLETS_INST_ACT
 

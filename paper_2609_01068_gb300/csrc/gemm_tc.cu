@@ -78,6 +78,33 @@ __device__ __forceinline__ Tile decode_tile(int t, int num_m, int num_n, int gro
 // silu(x) = x * sigmoid(x); the fast division is exact to ~2 ulp (the result is rounded to bf16)
 __device__ __forceinline__ float silu_f(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
 
+// RMSNorm folded into the GEMMs: row m's scale rsqrt(mean(x^2) + eps) from the
+// per-N-tile sums of squares its producer left (summed in tile order).
+__device__ __forceinline__ float fold_row_scale(const GemmArgs& p, int m) {
+  if (!p.row_ss || m >= p.M) return 1.0f;
+  const float* ss = p.row_ss + (long long)m * p.nrm_tiles;
+  float t = 0.f;
+  for (int i = 0; i < p.nrm_tiles; ++i) t += ss[i];
+  return rsqrtf(t / (float)p.nrm_d + p.nrm_eps);
+}
+
+// Producer side: the 8 lanes (lane & 7) that share a row add up their
+// columns' squares; the first writes the row's sum for this 64-column group.
+// Groups of 64 columns whatever the tile width, so the consumer's sum over the
+// groups (in group order) does not depend on how the producer was tiled.
+__device__ __forceinline__ void fold_store_ss(const GemmArgs& p, float (&ssr)[8], int row0, int group, int lane) {
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    float v = ssr[k];
+    v += __shfl_xor_sync(0xffffffffu, v, 1);
+    v += __shfl_xor_sync(0xffffffffu, v, 2);
+    v += __shfl_xor_sync(0xffffffffu, v, 4);
+    const int mm = row0 + k * 4 + (lane >> 3);
+    if ((lane & 7) == 0 && mm < p.M) p.nrm_ss[(long long)mm * p.nrm_tiles + group] = v;
+    ssr[k] = 0.f;
+  }
+}
+
 template <typename T>
 __device__ __forceinline__ void store_row32(T* dst, const float* v, int valid);
 
@@ -273,6 +300,7 @@ __global__ void __launch_bounds__(192, 1)
         // B rows are interleaved in blocks of 32: tile columns [64j, 64j+32) are
         // gate and [64j+32, 64j+64) up for the same 32 outputs
         const int n_out = p.N / 2;
+        const float rs = fold_row_scale(p, m);  // 1 unless the norm is folded in
         for (int c = 0; c < BN; c += 64) {
           uint32_t g[32], u[32];
           tmem_ld_32x32b_x32(tbase + c, g);
@@ -282,7 +310,8 @@ __global__ void __launch_bounds__(192, 1)
           if (row_ok && n0 < n_out) {
             float v[32];
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = silu_f(__uint_as_float(g[j])) * __uint_as_float(u[j]);
+            for (int j = 0; j < 32; ++j)
+              v[j] = silu_f(__uint_as_float(g[j]) * rs) * (__uint_as_float(u[j]) * rs);
             store_row32(reinterpret_cast<bf16*>(p.out) + (long long)m * p.ldo + n0, v, min(32, n_out - n0));
           }
         }
@@ -308,6 +337,7 @@ __global__ void __launch_bounds__(192, 1)
         };
 #pragma unroll
         for (int i = 0; i < LA; ++i) load_res(i, res[i]);
+        float ssr[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int ci = 0; ci < NC; ++ci) {
           uint32_t r[32];
@@ -326,15 +356,25 @@ __global__ void __launch_bounds__(192, 1)
               if (row0 + rr < p.M) {
                 const float4 v = *reinterpret_cast<const float4*>(stg + rr * 36 + cq);
                 const float4 q = res[ci % LA][k];
-                *reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (long long)(row0 + rr) * p.ldo + n) =
-                    make_float4(v.x + q.x, v.y + q.y, v.z + q.z, v.w + q.w);
+                const float4 o = make_float4(v.x + q.x, v.y + q.y, v.z + q.z, v.w + q.w);
+                *reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (long long)(row0 + rr) * p.ldo + n) = o;
+                if (p.nrm_out) {
+                  uint2 packed;
+                  packed.x = pack_bf16x2(o.x, o.y);
+                  packed.y = pack_bf16x2(o.z, o.w);
+                  *reinterpret_cast<uint2*>(p.nrm_out + (long long)(row0 + rr) * p.ldo + n) = packed;
+                  ssr[k] += o.x * o.x + o.y * o.y + o.z * o.z + o.w * o.w;
+                }
               }
             }
           }
           if (ci + LA < NC) load_res(ci + LA, res[ci % LA]);
           __syncwarp();
+          if ((ci & 1) && p.nrm_out) fold_store_ss(p, ssr, row0, (tl.n_blk * BN + ci * 32) / 64, lane);
         }
       } else {
+        float ssr[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // EPI_F32 producer of a folded norm
+        const float rs_mine = EPI == EPI_ACT ? fold_row_scale(p, m) : 1.0f;  // EPI_ACT consumer
         for (int c = 0; c < BN; c += 32) {
           uint32_t r[32];
           tmem_ld_32x32b_x32(tbase + c, r);
@@ -353,6 +393,10 @@ __global__ void __launch_bounds__(192, 1)
             const int row0 = tl.m_blk * TM + mt * BM + quarter * 32;
             const int cq = (lane & 7) * 4;  // this lane's 4 columns of the chunk
             const int n = n0 + cq;
+            float rsk[8];                   // EPI_ACT: the scales of the 8 rows this lane writes
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+              rsk[k] = EPI == EPI_ACT ? __shfl_sync(0xffffffffu, rs_mine, k * 4 + (lane >> 3)) : 1.0f;
             if (n < p.N) {                  // N % 4 == 0: a lane's 4 columns are all in or all out
               if constexpr (EPI == EPI_F32) {
                 float4 res[8];
@@ -368,24 +412,35 @@ __global__ void __launch_bounds__(192, 1)
                   const int rr = k * 4 + (lane >> 3);
                   if (row0 + rr < p.M) {
                     const float4 v = *reinterpret_cast<const float4*>(stg + rr * 36 + cq);
-                    *reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (long long)(row0 + rr) * p.ldo + n) =
-                        make_float4(v.x + res[k].x, v.y + res[k].y, v.z + res[k].z, v.w + res[k].w);
+                    const float4 o = make_float4(v.x + res[k].x, v.y + res[k].y, v.z + res[k].z, v.w + res[k].w);
+                    *reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (long long)(row0 + rr) * p.ldo + n) = o;
+                    if (p.nrm_out) {
+                      uint2 packed;
+                      packed.x = pack_bf16x2(o.x, o.y);
+                      packed.y = pack_bf16x2(o.z, o.w);
+                      *reinterpret_cast<uint2*>(p.nrm_out + (long long)(row0 + rr) * p.ldo + n) = packed;
+                      ssr[k] += o.x * o.x + o.y * o.y + o.z * o.z + o.w * o.w;
+                    }
                   }
                 }
               } else {
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
                   const int rr = k * 4 + (lane >> 3);
+                  const float rs = rsk[k];
                   if (row0 + rr < p.M) {
                     const float4 v = *reinterpret_cast<const float4*>(stg + rr * 36 + cq);
                     uint2 packed;
-                    packed.x = pack_bf16x2(v.x, v.y);
-                    packed.y = pack_bf16x2(v.z, v.w);
+                    packed.x = pack_bf16x2(v.x * rs, v.y * rs);
+                    packed.y = pack_bf16x2(v.z * rs, v.w * rs);
                     *reinterpret_cast<uint2*>(reinterpret_cast<bf16*>(p.out) + (long long)(row0 + rr) * p.ldo + n) =
                         packed;
                   }
                 }
               }
+            }
+            if constexpr (EPI == EPI_F32) {  // after every second 32-column chunk (all lanes together)
+              if ((c & 32) && p.nrm_out) fold_store_ss(p, ssr, row0, n0 / 64, lane);
             }
             __syncwarp();
           } else if (row_ok && n0 < p.N) {  // EPI_BIAS_RELU

@@ -100,6 +100,16 @@ struct GemmArgs {
   float* lm_logits;       // EPI_LM*: optional f32 logits [M, N] with row stride ldo (null: not stored)
   float2* lm_stats;       // EPI_LM*: partials [M][tiles], layout above
   int2* lm_top;           // EPI_LM*: partials [M][tiles][KT]
+  // RMSNorm folded into the GEMMs (large-M path): a producer (EPI_F32) also
+  // writes its output rows as bf16 (nrm_out, row stride ldo) and each row's
+  // sum of squares per 64-column group (nrm_ss [M][nrm_tiles]); a consumer (EPI_ACT,
+  // EPI_SWIGLU) whose A operand is such a bf16 copy and whose weights carry
+  // the norm gain scales row r by rsqrt(sum_t row_ss[r][t] / nrm_d + nrm_eps).
+  bf16* nrm_out;
+  float* nrm_ss;
+  const float* row_ss;
+  int nrm_tiles, nrm_d;
+  float nrm_eps;
   int* lm_bound;          // EPI_LM8: [M][kLmBoundSlots] per-row slots bounding the row's 8th best logit (int keys)
 };
 
@@ -199,7 +209,7 @@ cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_st
 // weight layout of GemmArgs with b_np = kb_np.
 template <typename Act>
 cudaError_t convert_rows_launch(const float* src, Act* dst, int rows, int cols, long long dst_ld, int row_mode,
-                                int row_base, long long kb_np, cudaStream_t stream);
+                                int row_base, long long kb_np, const float* col_scale, cudaStream_t stream);
 
 // One CTA whose bounded mbarrier wait can never complete: raises ERR_TIMEOUT in err.
 cudaError_t wait_selftest_launch(int* err, unsigned long long timeout_ns, cudaStream_t stream);

@@ -125,6 +125,17 @@ struct outlets_ctx {
   // input-embedding branch: table [EV, d] (act dtype, row-major), its gain, the
   // normalized embedding of each row; the QKV GEMM then has K = 2d (qkv_k)
   int EV = 0, qkv_k = 0;
+  // RMSNorm folded into the GEMMs (bf16 path): g_in / g_post are folded into
+  // the QKV / gate-up weights at upload, so explicit norms of f and a use unit
+  // gains; on the large-M path the FC and O GEMMs also write bf16 copies and
+  // per-tile sums of squares, and QKV / gate-up scale their rows
+  bool fold = false;
+  float* ones = nullptr;
+  float *ss_f = nullptr, *ss_a = nullptr;  // [max_rows][ss_stride]
+  int ss_stride = 0;
+  bool xin_raw = false;          // xhat holds bf16(f), not the normalized x_hat (last call)
+  int fold_tiles_f = 0;          // 64-column groups of the FC output in ss_f (its consumer needs the count)
+  void* xin_scratch = nullptr;   // x_hat on request (outlets_get_intermediate)
   void* w_embed = nullptr;
   float* g_emb = nullptr;
   void* ehat = nullptr;
@@ -292,14 +303,17 @@ bool owned_by(const outlets_ctx* c, const void* p) {
 // converts it (f32 -> act) into dst with the given row mapping and layout
 // (kb_np > 0: k-block-major swizzled weight layout, else row-major, stride dst_ld).
 outlets_status upload_rows(outlets_ctx* c, const float* src, int rows, int cols, void* dst, long long dst_ld,
-                           int row_mode, int row_base, long long kb_np, float* stage, size_t stage_floats) {
+                           int row_mode, int row_base, long long kb_np, float* stage, size_t stage_floats,
+                           const float* col_scale = nullptr) {
   const int chunk = (int)std::max<size_t>(1, stage_floats / (size_t)cols);
   for (int r0 = 0; r0 < rows; r0 += chunk) {
     const int n = std::min(chunk, rows - r0);
     OUT_CK(c, cudaMemcpy(stage, src + (size_t)r0 * cols, (size_t)n * cols * 4, cudaMemcpyHostToDevice));
     const cudaError_t e =
-        c->bf16 ? convert_rows_launch<bf16>(stage, (bf16*)dst, n, cols, dst_ld, row_mode, row_base + r0, kb_np, 0)
-                : convert_rows_launch<float>(stage, (float*)dst, n, cols, dst_ld, row_mode, row_base + r0, kb_np, 0);
+        c->bf16 ? convert_rows_launch<bf16>(stage, (bf16*)dst, n, cols, dst_ld, row_mode, row_base + r0, kb_np,
+                                            col_scale, 0)
+                : convert_rows_launch<float>(stage, (float*)dst, n, cols, dst_ld, row_mode, row_base + r0, kb_np,
+                                             col_scale, 0);
     OUT_CK(c, e);
     OUT_CK(c, cudaDeviceSynchronize());
   }
@@ -462,9 +476,20 @@ outlets_status a_maps(outlets_ctx* c, const void* const* a, int n_pieces, int k_
 
 // bf16 GEMM through tcgen05 with an explicit tile plan.  A pieces: row-major
 // [M, k_piece] with row stride lda.
+// RMSNorm folded into a large-M GEMM pair (see GemmArgs): a producer writes
+// out_bf16 and ss (row stride ss_stride; tiles = its 64-column groups, set
+// here); a consumer reads row_ss with the producer's group count.
+struct NormFold {
+  bf16* out_bf16 = nullptr;
+  float* ss = nullptr;
+  const float* row_ss = nullptr;
+  int tiles = 0;
+};
+
 outlets_status gemm_tc_ex(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
                           const void* b, long long b_np, int N, int K, int epi, int bn, int mt, int splits, void* out,
-                          long long ldo, const float* residual, long long ldr, const float* bias, cudaStream_t s) {
+                          long long ldo, const float* residual, long long ldr, const float* bias, cudaStream_t s,
+                          NormFold* nf = nullptr) {
   if (M == 0) return OUTLETS_OK;
   CUtensorMap am[3];
   OUT_TRY(a_maps(c, a, n_pieces, k_piece, lda, M, am));
@@ -486,6 +511,19 @@ outlets_status gemm_tc_ex(outlets_ctx* c, const void* const* a, int n_pieces, in
   g.ldr = ldr;
   g.bias = bias;
   g.err = c->err_dev;
+  if (nf) {
+    g.nrm_d = c->d;
+    g.nrm_eps = c->cfg.rms_eps;
+    if (nf->out_bf16) {  // producer
+      nf->tiles = (int)cdiv(N, 64);  // sums of squares per 64-column group
+      if (nf->tiles > c->ss_stride) return c->fail(OUTLETS_ECAPACITY, "folded-norm tile count");
+      g.nrm_out = nf->out_bf16;
+      g.nrm_ss = nf->ss;
+    } else {  // consumer
+      g.row_ss = nf->row_ss;
+    }
+    g.nrm_tiles = nf->tiles;
+  }
   OUT_CK(c, gemm_tc_launch(am, bn, epi, mt, g, c->num_sms, s));
   return OUTLETS_OK;
 }
@@ -493,7 +531,8 @@ outlets_status gemm_tc_ex(outlets_ctx* c, const void* const* a, int n_pieces, in
 // Large-M GEMM (prefill): 128-row tiles, tile width chosen to fill the SMs.
 outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k_piece, long long lda, int M,
                        const void* b, long long b_np, int N, int K, int epi, void* out, long long ldo,
-                       const float* residual, long long ldr, const float* bias, cudaStream_t s) {
+                       const float* residual, long long ldr, const float* bias, cudaStream_t s,
+                       NormFold* nf = nullptr) {
   int bn = 256;
   if (epi != EPI_SWIGLU) {
     auto tiles = [&](int bnv) { return cdiv(M, 128) * cdiv(N, bnv); };
@@ -501,7 +540,7 @@ outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k
     else if (tiles(128) >= c->num_sms) bn = 128;
     else bn = 64;
   }
-  return gemm_tc_ex(c, a, n_pieces, k_piece, lda, M, b, b_np, N, K, epi, bn, 1, 1, out, ldo, residual, ldr, bias, s);
+  return gemm_tc_ex(c, a, n_pieces, k_piece, lda, M, b, b_np, N, K, epi, bn, 1, 1, out, ldo, residual, ldr, bias, s, nf);
 }
 
 // Small-M GEMM (M <= 256): every weight tile is streamed once.  K is split so
@@ -587,28 +626,32 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   const float eps = c->cfg.rms_eps;
   const bool small = small_path(c, rows);
   int sl = 1;
+  NormFold nf_a;  // large-M bf16: the O GEMM leaves bf16(a) and its sums of squares for gate/up
+  nf_a.out_bf16 = (bf16*)c->ahat;
+  nf_a.ss = c->ss_a;
   // O projection + residual: a = f + attn W_o^T; post-attention RMSNorm
   c->stage_begin(OUTLETS_S_O);
   {
     const void* a1[3] = {c->attn, c->attn, c->attn};
     if (small)
       OUT_TRY(gemm_split(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, c->part, &sl, s));
-    else if (c->bf16)
+    else if (c->bf16)  // a = f + attn W_o^T, its bf16 copy and per-tile sums of squares (norm folded)
       OUT_TRY(gemm_tc(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d,
-                      nullptr, s));
+                      nullptr, s, &nf_a));
     else
       OUT_TRY(gemm_f32(c, a1, c->attn_w, rows, c->w_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d, nullptr, s));
   }
   c->stage_end(1);
-  c->stage_begin(OUTLETS_S_NORM_POST);
-  if (small)
-    OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, c->f, nullptr, c->g_post, (bf16*)c->ahat,
+  if (small) {
+    c->stage_begin(OUTLETS_S_NORM_POST);
+    OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, c->f, nullptr, c->ones, (bf16*)c->ahat,
                                           c->a, rows, d, eps, s));
-  else if (c->bf16)
-    OUT_CK(c, rmsnorm_launch<bf16>(c->a, c->g_post, (bf16*)c->ahat, nullptr, rows, d, eps, s));
-  else
+    c->stage_end(1);
+  } else if (!c->bf16) {
+    c->stage_begin(OUTLETS_S_NORM_POST);
     OUT_CK(c, rmsnorm_launch<float>(c->a, c->g_post, (float*)c->ahat, nullptr, rows, d, eps, s));
-  c->stage_end(1);
+    c->stage_end(1);
+  }
   // gate/up + SwiGLU
   c->stage_begin(OUTLETS_S_GATEUP);
   {
@@ -639,8 +682,10 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
       g.ldo = c->Fp;
       g.err = c->err_dev;
       OUT_CK(c, gemm_small_launch(am, best_bn, EPI_SWIGLU, rows <= 128 ? 1 : 2, g, s));
-    } else if (c->bf16) {
-      OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_gu, c->np_gu, 2 * c->Fp, d, EPI_SWIGLU, c->u, c->Fp, nullptr, 0, nullptr, s));
+    } else if (c->bf16) {  // A = bf16(a); the rows are scaled by their RMSNorm factor before SwiGLU
+      NormFold use{nullptr, nullptr, c->ss_a, nf_a.tiles};
+      OUT_TRY(gemm_tc(c, a1, 1, d, d, rows, c->w_gu, c->np_gu, 2 * c->Fp, d, EPI_SWIGLU, c->u, c->Fp, nullptr, 0, nullptr,
+                      s, &use));
     } else {
       OUT_TRY(gemm_f32(c, a1, d, rows, c->w_gu, 2 * c->Fp, d, EPI_F32, c->gu32, 2 * c->Fp, nullptr, 0, nullptr, s));
       OUT_CK(c, swiglu_launch<float>(c->gu32, (float*)c->u, rows, c->Fp, s));
@@ -843,27 +888,40 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
   const bool small = small_path(c, rows);
   int sl = 1;
   if (!tp) {
+    c->xin_raw = false;
     // draft rollout step: the feature input is the draft layer's own output
     // state y of the previous step (same rows), in place of Eq. 1's fused taps
     c->stage_begin(OUTLETS_S_NORM_IN);
     OUT_CK(c, cudaMemcpyAsync(c->f, c->y, (size_t)rows * d * 4, cudaMemcpyDeviceToDevice, s));
-    if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xhat, nullptr, rows, d, eps, s));
+    if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->ones, (bf16*)c->xhat, nullptr, rows, d, eps, s));
     else OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
     return run_qkv(c, rows, q, s, row0, tok_dev, sl, 1);
   }
+  // large-M bf16 without the embedding branch: the input RMSNorm is folded
+  // into the FC (bf16 copy + sums of squares) and QKV (row scale) GEMMs
+  const bool fold_in = !small && c->bf16 && c->EV == 0;
+  c->xin_raw = fold_in;
   c->stage_begin(OUTLETS_S_FC);
-  if (small) OUT_TRY(gemm_split(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, c->part, &sl, s));
-  else if (c->bf16)
+  if (small) {
+    OUT_TRY(gemm_split(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, c->part, &sl, s));
+  } else if (c->bf16) {
+    NormFold nf;
+    nf.out_bf16 = (bf16*)c->xhat + (size_t)row0 * d;
+    nf.ss = c->ss_f + (size_t)row0 * c->ss_stride;
     OUT_TRY(gemm_tc(c, tp, 3, d, d, rows, c->w_proj, c->np_proj, d, 3 * d, EPI_F32, c->f + (size_t)row0 * d, d, nullptr,
-                    0, nullptr, s));
-  else OUT_TRY(gemm_f32(c, tp, d, rows, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
+                    0, nullptr, s, fold_in ? &nf : nullptr));
+    c->fold_tiles_f = nf.tiles;
+  } else {
+    OUT_TRY(gemm_f32(c, tp, d, rows, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
+  }
   c->stage_end(1);
+  if (fold_in) return run_qkv(c, rows, q, s, row0, tok_dev, sl, 0);
   c->stage_begin(OUTLETS_S_NORM_IN);
   if (small)
-    OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, nullptr, nullptr, c->g_in, (bf16*)c->xhat,
+    OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, nullptr, nullptr, c->ones, (bf16*)c->xhat,
                                           c->f, rows, d, eps, s));
   else if (c->bf16)
-    OUT_CK(c, rmsnorm_launch<bf16>(c->f + (size_t)row0 * d, c->g_in, (bf16*)c->xhat + (size_t)row0 * d, nullptr, rows,
+    OUT_CK(c, rmsnorm_launch<bf16>(c->f + (size_t)row0 * d, c->ones, (bf16*)c->xhat + (size_t)row0 * d, nullptr, rows,
                                    d, eps, s));
   else
     OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
@@ -903,8 +961,12 @@ outlets_status run_qkv(outlets_ctx* c, int rows, QkvSrc* q, cudaStream_t s, int 
     OUT_TRY(gemm_split(c, a1, pieces, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, K, c->part, &sl, s));
     *q = {c->part, true, sl, (long long)rows * c->qkv_n};
   } else if (c->bf16) {
+    NormFold use;  // folded input norm: scale the rows by the FC's sums of squares
+    use.row_ss = c->ss_f + (size_t)row0 * c->ss_stride;
+    use.tiles = c->fold_tiles_f;
     OUT_TRY(gemm_tc(c, a1, pieces, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, K, EPI_ACT,
-                    (char*)c->qkv + (size_t)row0 * c->qkv_n * c->esz, c->qkv_n, nullptr, 0, nullptr, s));
+                    (char*)c->qkv + (size_t)row0 * c->qkv_n * c->esz, c->qkv_n, nullptr, 0, nullptr, s,
+                    c->xin_raw ? &use : nullptr));
     *q = {c->qkv, false, 1, 0};
   } else {
     OUT_TRY(gemm_f32(c, a1, d, rows, c->w_qkv, c->qkv_n, K, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
@@ -1117,6 +1179,13 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   c->ahat = c->alloc(R * d * es);
   c->hn = c->alloc(R * d * es);
   if (c->EV > 0) c->ehat = c->alloc(R * d * es);
+  if (c->bf16) {  // RMSNorm gains folded into the consuming weights
+    c->fold = true;
+    c->ones = (float*)c->alloc((size_t)d * 4);
+    c->ss_stride = (int)cdiv(d, 64);
+    c->ss_f = (float*)c->alloc(R * c->ss_stride * 4);
+    c->ss_a = (float*)c->alloc(R * c->ss_stride * 4);
+  }
   c->qkv = c->alloc(R * c->qkv_n * es);
   c->q = c->alloc(R * c->attn_w * es);
   if (c->gated) c->gate_act = c->alloc(R * c->attn_w * es);
@@ -1176,24 +1245,47 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   // keep interleaved uploads chunked on 128-row boundaries
   const size_t il_floats = std::max<size_t>((stage_floats / d) / 128 * 128, 128) * d;
   outlets_status st = OUTLETS_OK;
-  auto up = [&](const float* src, int rows, int cols, void* dst, long long ld, int mode, int base, long long np) {
+  auto up = [&](const float* src, int rows, int cols, void* dst, long long ld, int mode, int base, long long np,
+                const float* col_scale = nullptr) {
     if (st == OUTLETS_OK)
-      st = upload_rows(c, src, rows, cols, dst, ld, mode, base, np, stage, mode == 0 ? stage_floats : il_floats);
+      st = upload_rows(c, src, rows, cols, dst, ld, mode, base, np, stage, mode == 0 ? stage_floats : il_floats,
+                       col_scale);
   };
+  // column scales folding the RMSNorm gains into the weights that read the
+  // normalized rows (bf16 path): QKV columns of the fused feature by g_in,
+  // gate/up columns by g_post (the embedding columns keep g_emb in their norm)
+  float *qkv_scale = nullptr, *gu_scale = nullptr;
+  if (c->fold) {
+    std::vector<float> one(d, 1.0f), qs((size_t)c->qkv_k, 1.0f);
+    std::memcpy(qs.data() + (c->qkv_k - d), w->g_in, (size_t)d * 4);
+    if (cudaMalloc(&qkv_scale, qs.size() * 4) != cudaSuccess || cudaMalloc(&gu_scale, (size_t)d * 4) != cudaSuccess) {
+      cudaGetLastError();
+      cudaFree(stage);
+      cudaFree(qkv_scale);
+      return cleanup_fail(OUTLETS_ENOMEM);
+    }
+    if (cudaMemcpy(qkv_scale, qs.data(), qs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(gu_scale, w->g_post, (size_t)d * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(c->ones, one.data(), (size_t)d * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      st = OUTLETS_ECUDA;
+  }
   up(w->w_proj, d, 3 * d, c->w_proj, 3 * d, 0, 0, c->np_proj);
   const int qk = c->qkv_k;
-  up(w->w_q, c->H * c->hd, qk, c->w_qkv, qk, 0, 0, c->np_qkv);
-  up(w->w_k, c->KVH * c->hd, qk, c->w_qkv, qk, 0, c->H * c->hd, c->np_qkv);
-  up(w->w_v, c->KVH * c->hd, qk, c->w_qkv, qk, 0, (c->H + c->KVH) * c->hd, c->np_qkv);
-  if (c->gated) up(w->w_attn_gate, c->attn_w, qk, c->w_qkv, qk, 0, (c->H + 2 * c->KVH) * c->hd, c->np_qkv);
+  up(w->w_q, c->H * c->hd, qk, c->w_qkv, qk, 0, 0, c->np_qkv, qkv_scale);
+  up(w->w_k, c->KVH * c->hd, qk, c->w_qkv, qk, 0, c->H * c->hd, c->np_qkv, qkv_scale);
+  up(w->w_v, c->KVH * c->hd, qk, c->w_qkv, qk, 0, (c->H + c->KVH) * c->hd, c->np_qkv, qkv_scale);
+  if (c->gated)
+    up(w->w_attn_gate, c->attn_w, qk, c->w_qkv, qk, 0, (c->H + 2 * c->KVH) * c->hd, c->np_qkv, qkv_scale);
   if (c->EV > 0) up(w->w_embed, c->EV, d, c->w_embed, d, 0, 0, 0);
   up(w->w_o, d, c->attn_w, c->w_o, c->attn_w, 0, 0, c->np_o);
-  up(w->w_gate, c->F, d, c->w_gu, d, 1, 0, c->np_gu);
-  up(w->w_up, c->F, d, c->w_gu, d, 2, 0, c->np_gu);
+  up(w->w_gate, c->F, d, c->w_gu, d, 1, 0, c->np_gu, gu_scale);
+  up(w->w_up, c->F, d, c->w_gu, d, 2, 0, c->np_gu, gu_scale);
   up(w->w_down, d, c->F, c->w_down, c->Fp, 0, 0, c->np_down);
   up(w->head_w[0], c->head_dims[1], d, c->head_w0, d, 0, 0, c->np_h0);
   if (c->V > 0) up(w->w_lm, c->V, d, c->w_lm, d, 0, 0, c->np_lm);
   cudaFree(stage);
+  cudaFree(qkv_scale);
+  cudaFree(gu_scale);
   if (st != OUTLETS_OK) return cleanup_fail(st);
   auto h2d = [&](void* dst, const void* src, size_t bytes) {
     if (st == OUTLETS_OK && cudaMemcpy(dst, src, bytes, cudaMemcpyHostToDevice) != cudaSuccess) st = OUTLETS_ECUDA;
@@ -1867,7 +1959,7 @@ outlets_status outlets_get_intermediate(outlets_ctx* c, int32_t which, void* dst
   outlets_tensor_info ti{};
   switch (which) {
     case OUTLETS_T_FCTX: ti = {OUTLETS_F32, c->last_rows, c->d}; src = c->f; break;
-    case OUTLETS_T_XIN: ti = {act, c->last_rows, c->d}; src = c->xhat; break;
+    case OUTLETS_T_XIN: ti = {act, c->last_rows, c->d}; src = c->xhat; break;  // bf16: recomputed below
     case OUTLETS_T_Q: ti = {act, c->last_rows, c->attn_w}; src = c->q; break;
     case OUTLETS_T_ATTN: ti = {act, c->last_rows, c->attn_w}; src = c->attn; break;
     case OUTLETS_T_A: ti = {OUTLETS_F32, c->last_rows, c->d}; src = c->a; break;
@@ -1880,6 +1972,17 @@ outlets_status outlets_get_intermediate(outlets_ctx* c, int32_t which, void* dst
   const size_t bytes = (size_t)ti.rows * ti.cols * (ti.dtype == OUTLETS_BF16 ? 2 : 4);
   if (dst_bytes < bytes) return c->fail(OUTLETS_EINVAL, "dst too small");
   OUT_CK(c, cudaSetDevice(c->cfg.device));
+  if (which == OUTLETS_T_XIN && c->fold) {
+    // the bf16 path keeps g_in in the QKV weights and never materializes
+    // x_hat = RMSNorm(f; g_in) itself: normalize f on request
+    if (!c->xin_scratch) {
+      c->xin_scratch = c->alloc((size_t)c->max_rows * c->d * c->esz);
+      if (!c->xin_scratch) return c->fail(OUTLETS_ENOMEM, "x_hat scratch allocation failed");
+    }
+    OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->g_in, (bf16*)c->xin_scratch, nullptr, c->last_rows, c->d,
+                                   c->cfg.rms_eps, (cudaStream_t)stream));
+    src = c->xin_scratch;
+  }
   OUT_CK(c, cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, (cudaStream_t)stream));
   return OUTLETS_OK;
 }

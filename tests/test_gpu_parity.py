@@ -365,3 +365,49 @@ def test_bounded_wait_timeout_is_reported_and_context_survives():
     ref = OR.predict_prefill(w, shape, taps, cu)
     check_z_len(z, ln, ref["z"], ref["length"], "bf16", "after timeout")
     pred.check()
+
+
+@pytest.mark.parametrize("name,gated,embed", [("tiny-f32", False, False), ("mid128", False, False),
+                                              ("mid128", True, True), ("mid64", False, False)])
+def test_nonunit_norm_gains(name, gated, embed):
+    """RMSNorm gains other than 1.  On the bf16 path g_in and g_post are folded
+    into the QKV and gate/up weights at upload and the large-M path folds the
+    norms into its GEMMs (bf16 copies, sums of squares, row scales), so unit
+    gains would not test any of it.  Prefill (large M) and steps (small M)."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = SHAPES[name]
+    ev = 500 if embed else 0
+    w = synth.make_weights(shape, 0, gated=gated, embed_vocab=ev)
+    rng = np.random.default_rng(17)
+    for g in ("g_in", "g_post", "g_final") + (("g_emb",) if embed else ()):
+        w[g] = (1.0 + 0.2 * rng.standard_normal(shape.d)).astype(np.float32)
+    pred = OT.Predictor(shape, w, max_tokens=4096, max_batch=16, max_position=8192)
+    lengths = PREFILL_LENGTHS[name]
+    B = len(lengths)
+    cu = synth.cu_seqlens(lengths)
+    T = int(cu[-1])
+    taps = synth.make_taps(shape, T, 0, 61)
+    tok = synth.make_tokens(T, ev, 0, 61) if embed else None
+    kv = OT.KVCache(pred, max_slots=B, max_tokens_total=T + 64 * B)
+    slots = np.arange(B, dtype=np.int32)
+    z, ln = pred.prefill([to_device(t, shape.dtype) for t in taps], cu, kv=kv, slots=slots, tokens=tok)
+    torch.cuda.synchronize()
+    pred.check()
+    ref = OR.predict_prefill(w, shape, taps, cu, tokens=tok)
+    d = shape.d
+    for which, r, what in [(OT.T_XIN, ref["x"][:, -d:], "x_in"), (OT.T_Q, ref["q"].reshape(T, -1), "q"),
+                           (OT.T_A, ref["a"], "a"), (OT.T_Y, ref["y"], "y"), (OT.T_HDRAFT, ref["h_draft"], "h_draft")]:
+        check_hidden(pred.intermediate(which), r, shape.dtype, f"gains {name} {what}")
+    check_z_len(z, ln, ref["z"], ref["length"], shape.dtype, f"gains {name} prefill")
+    caches = OR.caches_from_prefill(ref, cu)
+    st = synth.make_taps(shape, B, 0, 62)
+    stok = synth.make_tokens(B, ev, 0, 62) if embed else None
+    z2, ln2 = pred.step([to_device(t, shape.dtype) for t in st], kv, slots, tokens=stok)
+    torch.cuda.synchronize()
+    pred.check()
+    ref2 = OR.predict_step(w, shape, st, caches, tokens=stok)
+    check_hidden(pred.intermediate(OT.T_XIN), ref2["x"][:, -d:], shape.dtype, f"gains {name} step x_in")
+    check_hidden(pred.intermediate(OT.T_Y), ref2["y"], shape.dtype, f"gains {name} step y")
+    check_z_len(z2, ln2, ref2["z"], ref2["length"], shape.dtype, f"gains {name} step")
+    kv.close()
+    pred.close()

@@ -105,6 +105,13 @@ OUTLETS_DEV void bulk_prefetch_l2(const void* src, uint32_t bytes) {
                : "memory");
 }
 
+// Drops one 128-byte line (128-byte aligned) from L2 without writing it back;
+// the memory's contents become undefined.  Scratch that is read once would
+// otherwise be written back to DRAM when its dirty lines are evicted.
+OUTLETS_DEV void discard_l2_line(const void* p) {
+  asm volatile("discard.global.L2 [%0], 128;" ::"l"(static_cast<uint64_t>(__cvta_generic_to_global(p))) : "memory");
+}
+
 // ---------------------------------------------------------------- tcgen05
 OUTLETS_DEV void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),

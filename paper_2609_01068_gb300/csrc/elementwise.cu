@@ -82,6 +82,24 @@ __device__ __forceinline__ void ld_sum16(const float* p, const float* q, int n, 
   }
 }
 
+// Drops row `row` (ld floats) of every split-K slice from L2 once the block has
+// read it: the slices are scratch, rewritten before they are read again, and
+// their dirty lines would otherwise be written back to DRAM when evicted (in
+// the step, largely while the attention stage streams the K/V cache).  The
+// caller has passed a __syncthreads after its last read of the slices.  Only
+// whole, aligned 128-byte lines: nothing is done unless ld, the slice stride
+// and the base are multiples of 32 floats.
+__device__ __forceinline__ void discard_slice_rows(const float* x, int n_split, long long stride, long long row,
+                                                   int ld) {
+  if ((ld & 31) || (stride & 31) || (reinterpret_cast<uintptr_t>(x) & 127)) return;
+  const int lines = ld >> 5;
+  const float* r0 = x + row * ld;
+  for (int t = threadIdx.x; t < n_split * lines; t += blockDim.x) {
+    const int s = t / lines;
+    discard_l2_line(r0 + s * stride + (long long)(t - s * lines) * 32);
+  }
+}
+
 template <typename Act>
 __device__ __forceinline__ void store4(Act* p, float a, float b, float c, float d);
 template <>
@@ -103,7 +121,7 @@ template <typename Act, bool REDUCE>
 __global__ void __launch_bounds__(512, 2) k_rmsnorm(const float* __restrict__ x, int n_split, long long split_stride,
                           const float* __restrict__ residual, const int* __restrict__ row_index,
                           const float* __restrict__ g, Act* __restrict__ y, float* __restrict__ copy_out, int d,
-                          float eps) {
+                          float eps, bool discard) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[33];
@@ -122,7 +140,9 @@ __global__ void __launch_bounds__(512, 2) k_rmsnorm(const float* __restrict__ x,
     }
     ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
   }
-  const float inv = rsqrtf(block_sum(ss, red) / (float)d + eps);
+  const float inv = rsqrtf(block_sum(ss, red) / (float)d + eps);  // every slice read of the block is done
+  if constexpr (REDUCE)
+    if (discard && !row_index) discard_slice_rows(x, n_split, split_stride, r, d);
   Act* yr = y + (long long)r * d;
   for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
     float4 v;
@@ -331,6 +351,12 @@ __global__ void __launch_bounds__(RopeBlock<In>::kThreads, RopeBlock<In>::kMinBl
       store8<Act>(go + idx * 8, g);
     }
   }
+  if constexpr (std::is_same<In, float>::value) {
+    if (a.discard) {  // block-uniform
+      __syncthreads();  // every slice read of the block is done
+      discard_slice_rows(qkv, a.n_split, a.split_stride, row, a.qkv_ld);
+    }
+  }
 }
 
 template <typename Act>
@@ -352,7 +378,7 @@ __global__ void k_swiglu(const float* __restrict__ gu, Act* __restrict__ u, int 
 __global__ void __launch_bounds__(512) k_head_tail(const float* __restrict__ h, int n_split, long long split_stride,
                             const float* __restrict__ b_prev, const float* __restrict__ w_last,
                             const float* __restrict__ b_last, int rows, int width, float* __restrict__ z,
-                            float* __restrict__ len) {
+                            float* __restrict__ len, bool discard) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[33];
@@ -377,7 +403,8 @@ __global__ void __launch_bounds__(512) k_head_tail(const float* __restrict__ h, 
       acc += w_last[j] * x;
     }
   }
-  acc = block_sum(acc, red);
+  acc = block_sum(acc, red);  // every slice read of the block is done
+  if (discard) discard_slice_rows(h, n_split, split_stride, r, width);
   if (threadIdx.x == 0) {
     const float zz = acc + b_last[0];
     z[r] = zz;
@@ -495,19 +522,19 @@ inline int grid_for(long long n, int threads) {
 template <typename Act>
 cudaError_t rmsnorm_launch(const float* x, const float* g, Act* y, float* copy_out, int rows, int d, float eps,
                            cudaStream_t stream) {
-  return rmsnorm_reduce_launch<Act>(x, 1, 0, nullptr, nullptr, g, y, copy_out, rows, d, eps, stream);
+  return rmsnorm_reduce_launch<Act>(x, 1, 0, nullptr, nullptr, g, y, copy_out, rows, d, eps, stream, false);
 }
 
 template <typename Act>
 cudaError_t rmsnorm_gather_launch(const float* x, const int* row_index, const float* g, Act* y, int rows, int d,
                                   float eps, cudaStream_t stream) {
-  return rmsnorm_reduce_launch<Act>(x, 1, 0, nullptr, row_index, g, y, nullptr, rows, d, eps, stream);
+  return rmsnorm_reduce_launch<Act>(x, 1, 0, nullptr, row_index, g, y, nullptr, rows, d, eps, stream, false);
 }
 
 template <typename Act>
 cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_stride, const float* residual,
                                   const int* row_index, const float* g, Act* y, float* copy_out, int rows, int d,
-                                  float eps, cudaStream_t stream) {
+                                  float eps, cudaStream_t stream, bool discard) {
   if (rows == 0) return cudaSuccess;
   if (n_split > 1 || residual) {
     const size_t smem = (size_t)d * sizeof(float);
@@ -523,9 +550,9 @@ cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_s
     // two CTAs (rows) per SM fit beside each other: a one-wave grid for up to 2 x SMs rows
     const int threads = std::min(512, std::max(64, ((d / 4 + 31) / 32) * 32));
     OUTLETS_TRY_LAUNCH(launch_k(k_rmsnorm<Act, true>, dim3(rows), dim3(threads), smem, stream, x, n_split, split_stride, residual, row_index, g, y, copy_out,
-                                                      d, eps));
+                                                      d, eps, discard));
   } else {
-    OUTLETS_TRY_LAUNCH(launch_k(k_rmsnorm<Act, false>, dim3(rows), dim3(256), 0, stream, x, 1, 0, nullptr, row_index, g, y, copy_out, d, eps));
+    OUTLETS_TRY_LAUNCH(launch_k(k_rmsnorm<Act, false>, dim3(rows), dim3(256), 0, stream, x, 1, 0, nullptr, row_index, g, y, copy_out, d, eps, false));
   }
   return cudaGetLastError();
 }
@@ -558,10 +585,10 @@ cudaError_t embed_rmsnorm_launch(const int* tokens, const Act* table, int vocab,
 
 cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_stride, const float* b_prev,
                              const float* w_last, const float* b_last, int rows, int width, float* z, float* len,
-                             cudaStream_t stream) {
+                             cudaStream_t stream, bool discard) {
   if (rows == 0) return cudaSuccess;
   const int threads = std::min(512, std::max(64, ((width / 4 + 31) / 32) * 32));
-  OUTLETS_TRY_LAUNCH(launch_k(k_head_tail, dim3(rows), dim3(threads), 0, stream, h_pre, n_split, split_stride, b_prev, w_last, b_last, rows, width, z, len));
+  OUTLETS_TRY_LAUNCH(launch_k(k_head_tail, dim3(rows), dim3(threads), 0, stream, h_pre, n_split, split_stride, b_prev, w_last, b_last, rows, width, z, len, discard));
   return cudaGetLastError();
 }
 
@@ -589,7 +616,8 @@ cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int ep
 
 #define OUTLETS_INST_ACT(Act)                                                                                   \
   template cudaError_t rmsnorm_reduce_launch<Act>(const float*, int, long long, const float*, const int*,        \
-                                                  const float*, Act*, float*, int, int, float, cudaStream_t);   \
+                                                  const float*, Act*, float*, int, int, float, cudaStream_t,    \
+                                                  bool);                                                        \
   template cudaError_t rmsnorm_launch<Act>(const float*, const float*, Act*, float*, int, int, float,          \
                                            cudaStream_t);                                                      \
   template cudaError_t rmsnorm_gather_launch<Act>(const float*, const int*, const float*, Act*, int, int, float, \
@@ -603,7 +631,7 @@ cudaError_t gemm_simt_f32_launch(const float* const a[3], const float* b, int ep
   template cudaError_t rope_scatter_launch<Act, Act>(const Act*, const RopeArgs&, cudaStream_t);
 OUTLETS_INST_ACT(bf16)
 template cudaError_t rmsnorm_reduce_launch<float>(const float*, int, long long, const float*, const int*,
-                                                  const float*, float*, float*, int, int, float, cudaStream_t);
+                                                  const float*, float*, float*, int, int, float, cudaStream_t, bool);
 template cudaError_t rmsnorm_launch<float>(const float*, const float*, float*, float*, int, int, float, cudaStream_t);
 template cudaError_t rmsnorm_gather_launch<float>(const float*, const int*, const float*, float*, int, int, float,
                                                   cudaStream_t);

@@ -157,7 +157,7 @@ cudaError_t rmsnorm_gather_launch(const float* x, const int* row_index, const fl
 template <typename Act>
 cudaError_t rmsnorm_reduce_launch(const float* x, int n_split, long long split_stride, const float* residual,
                                   const int* row_index, const float* g, Act* y, float* copy_out, int rows, int d,
-                                  float eps, cudaStream_t stream);
+                                  float eps, cudaStream_t stream, bool discard = false);
 
 // Input-embedding branch: y[r] = RMSNorm(table[tokens[r]]) * g (table [vocab, d],
 // row-major, act dtype); an id outside [0, vocab) sets ERR_BAD_INDEX in *err.
@@ -189,6 +189,7 @@ struct RopeArgs {
   int qkv_ld;            // elements per qkv row: (H + 2 KVH) hd, + H hd gate columns when gated
   void* gate_out;        // gated attention: [T, H*hd] sigmoid of the gate columns, else null
   int* err;
+  bool discard;          // f32 slices: drop each row's slice lines from L2 after reading them
 };
 template <typename In, typename Act>
 cudaError_t rope_scatter_launch(const In* qkv, const RopeArgs& a, cudaStream_t stream);
@@ -201,7 +202,7 @@ cudaError_t swiglu_launch(const float* gu, Act* u, int rows, int f_pad, cudaStre
 // a(x) = relu(x + b_prev) (identity if b_prev is null); len[r] = max(0, expm1(z[r])).
 cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_stride, const float* b_prev,
                              const float* w_last, const float* b_last, int rows, int width, float* z, float* len,
-                             cudaStream_t stream);
+                             cudaStream_t stream, bool discard = false);
 
 // dst row map(row_base + r) <- src row r (f32 -> Act); map: row_mode 0 identity,
 // 1 gate rows, 2 up rows of the [gate 32 | up 32] interleave.  kb_np == 0:

@@ -112,6 +112,17 @@ int prefetch_blocks() {
   return n;
 }
 
+// Whether the kernels that add up split-K slices drop the slices' lines from
+// L2 after reading them (no write-back of scratch; OUTLETS_L2_DISCARD=0 keeps
+// them, for comparison).
+bool discard_slices() {
+  static const bool on = [] {
+    const char* v = getenv("OUTLETS_L2_DISCARD");
+    return !v || atoi(v) != 0;
+  }();
+  return on;
+}
+
 }  // namespace
 
 struct outlets_ctx {
@@ -645,7 +656,7 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   if (small) {
     c->stage_begin(OUTLETS_S_NORM_POST);
     OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, c->f, nullptr, c->ones, (bf16*)c->ahat,
-                                          c->a, rows, d, eps, s));
+                                          c->a, rows, d, eps, s, discard_slices()));
     c->stage_end(1);
   } else if (!c->bf16) {
     c->stage_begin(OUTLETS_S_NORM_POST);
@@ -711,12 +722,12 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
   if (small && !out_row_idx_dev) {
     // every row is predicted: add the slices and the residual, normalize, in one pass
     OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, c->a, nullptr, c->g_final, (bf16*)c->hn,
-                                          c->y, rows, d, eps, s));
+                                          c->y, rows, d, eps, s, discard_slices()));
   } else {
     if (small) {
       // y for every row (the normed copy goes to a dead buffer), then the predicted rows
       OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, c->a, nullptr, c->g_final,
-                                            (bf16*)c->ahat, c->y, rows, d, eps, s));
+                                            (bf16*)c->ahat, c->y, rows, d, eps, s, discard_slices()));
       n_final = 2;
     }
     if (c->bf16)
@@ -734,7 +745,7 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
     int hs = 1;
     OUT_TRY(gemm_split(c, ah, 1, d, d, out_rows, c->head_w0, c->np_h0, w1, d, c->part, &hs, s));
     OUT_CK(c, head_tail_launch(c->part, hs, (long long)out_rows * w1, c->head_b[0], c->head_wf[1], c->head_b[1],
-                               out_rows, w1, z_dev, len_dev, s));
+                               out_rows, w1, z_dev, len_dev, s, discard_slices()));
     c->stage_end(2);
     return OUTLETS_OK;
   }
@@ -919,7 +930,7 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
   c->stage_begin(OUTLETS_S_NORM_IN);
   if (small)
     OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, nullptr, nullptr, c->ones, (bf16*)c->xhat,
-                                          c->f, rows, d, eps, s));
+                                          c->f, rows, d, eps, s, discard_slices()));
   else if (c->bf16)
     OUT_CK(c, rmsnorm_launch<bf16>(c->f + (size_t)row0 * d, c->ones, (bf16*)c->xhat + (size_t)row0 * d, nullptr, rows,
                                    d, eps, s));
@@ -979,6 +990,7 @@ outlets_status run_qkv(outlets_ctx* c, int rows, QkvSrc* q, cudaStream_t s, int 
 outlets_status launch_rope(outlets_ctx* c, const QkvSrc& q, RopeArgs& ra, cudaStream_t s) {
   ra.n_split = q.n_split;
   ra.split_stride = q.stride;
+  ra.discard = q.f32 && q.p == c->part && discard_slices();
   if (c->bf16) {
     if (q.f32) OUT_CK(c, rope_scatter_launch<float, bf16>((const float*)q.p, ra, s));
     else OUT_CK(c, rope_scatter_launch<bf16, bf16>((const bf16*)q.p, ra, s));

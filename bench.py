@@ -75,6 +75,11 @@ def parse():
     ap.add_argument("--embed", action="store_true",
                     help="input-embedding branch of the EAGLE-3-style layer (Sec. 5.4): token embeddings "
                          "(128256-row table) normalized and concatenated to the layer input, QKV K = 2d")
+    ap.add_argument("--keep-rows", action="store_true",
+                    help="static prediction: run the whole draft layer on every prompt row (by default only the "
+                         "keys/values are projected for every row and the rest runs on each prompt's last row)")
+    ap.add_argument("--no-whole-layer", action="store_true",
+                    help="skip the extra whole-layer timing that the default static-prediction line carries")
     ap.add_argument("--model", default="8b", choices=["8b", "70b"],
                     help="draft-layer shape; 70b (Llama-3.3-70B-shaped, 32 prompts) runs the static mode only")
     ap.add_argument("--step-requests", type=int, default=256, help="live requests of the dynamic-prediction run")
@@ -84,6 +89,7 @@ def parse():
 
 
 TRAFFIC_SOURCES = {  # files whose content decides the kernel's DRAM traffic (incl. the tile raster)
+    "fc_gemm": ["gemm_tc.cu", "common.cuh", "kernels.h", "outlets.cu"],
     "gateup_swiglu_gemm": ["gemm_tc.cu", "common.cuh", "kernels.h", "outlets.cu"],
     "draft_head": ["gemm_tc.cu", "lm_head.cu", "lm_topk.cuh", "common.cuh", "kernels.h", "outlets.cu"],
     "decode_attention": ["attn_decode.cu", "mma_sync.cuh", "common.cuh", "kernels.h", "outlets.cu"],
@@ -184,16 +190,24 @@ def weight_bytes(shape):
     return 2 * (3 * d * d + d * (H + 2 * KVH) * hd + H * hd * d + 3 * d * F + d * shape.head_widths[0])
 
 
-def prefill_flops(shape, lengths, n_out, gated=False, embed=False):
-    """Algorithmic FLOPs of one static-prediction pass (dense GEMMs + causal attention + head)."""
+def prefill_flops(shape, lengths, n_out, gated=False, embed=False, whole_layer=True):
+    """Algorithmic FLOPs of one static-prediction pass (dense GEMMs + causal attention + head).
+    whole_layer=False: what the predicted rows need, the FC and the key/value
+    projection for every row, the rest for the n_out last rows (each query
+    against its prompt's keys)."""
     d, H, KVH, hd, F = shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
     T = int(np.sum(lengths))
     qkv_k = 2 * d if embed else d
-    per_tok = 2 * (3 * d * d + qkv_k * (H + 2 * KVH + (H if gated else 0)) * hd + H * hd * d + 3 * d * F)
-    attn = 4 * H * hd * float(np.sum(lengths * (lengths + 1) / 2))
     widths = (d,) + tuple(shape.head_widths) + (1,)
     head = 2 * sum(widths[i] * widths[i + 1] for i in range(len(widths) - 1)) * n_out
-    return per_tok * T + attn + head
+    if whole_layer:
+        per_tok = 2 * (3 * d * d + qkv_k * (H + 2 * KVH + (H if gated else 0)) * hd + H * hd * d + 3 * d * F)
+        attn = 4 * H * hd * float(np.sum(lengths * (lengths + 1) / 2))
+        return per_tok * T + attn + head
+    per_tok = 2 * (3 * d * d + qkv_k * 2 * KVH * hd)
+    per_row = 2 * (qkv_k * (H + (H if gated else 0)) * hd + H * hd * d + 3 * d * F)
+    attn = 4 * H * hd * float(np.sum(lengths))
+    return per_tok * T + per_row * n_out + attn + head
 
 
 def cpu_threads():
@@ -437,56 +451,77 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     tok_host = args.tokens  # token ids (input-embedding branch): device copy for the device-timed passes
     tok_dev = torch.from_numpy(tok_host).cuda() if tok_host is not None else None
 
-    def run(tp, zo, lo, out=None, tok=None):
+    def run(tp, zo, lo, out=None, tok=None, keep=args.keep_rows):
         tok = tok_dev if tok is None else tok
         if K:
-            pred.prefill_dual(tp, cu, K, out=out if out is not None else dout, z_out=zo, len_out=lo, tokens=tok)
+            pred.prefill_dual(tp, cu, K, out=out if out is not None else dout, z_out=zo, len_out=lo, tokens=tok,
+                              keep_rows=keep)
         else:
-            pred.prefill(tp, cu, z_out=zo, len_out=lo, tokens=tok)
+            pred.prefill(tp, cu, z_out=zo, len_out=lo, tokens=tok, keep_rows=keep)
 
     # ---------------- device-timed static prediction
     z = torch.empty(Bq, dtype=torch.float32, device="cuda")
     ln = torch.empty(Bq, dtype=torch.float32, device="cuda")
-    for _ in range(args.warmup):
-        run(taps_d, z, ln)
-    pred.check()
-    pred.profile(True, ["gateup_swiglu_gemm"])  # the dominant kernel, timed live on its stream
-    launches0 = pred.launch_count
-    sampler = ClockSampler(local)
-    sampler.start()
-    barrier()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    ev0.record(stream)
-    for _ in range(args.steps):
-        run(taps_d, z, ln)
-    ev1.record(stream)
-    ev1.synchronize()
-    barrier()
-    clocks = sampler.stop()
-    ms = max_over_ranks(ev0.elapsed_time(ev1))
-    launches = pred.launch_count - launches0
-    prof_live = pred.profile_read()
-    pred.profile(False)
-    pred.check()
+    pruned_rows = not args.keep_rows and T > 256  # bf16: past the K/V projection only the last rows run
+
+    def timed(keep):
+        """W warm-up and K timed passes; the dominant GEMM timed live on its stream."""
+        kern = "gateup_swiglu_gemm" if keep or not pruned_rows else "fc_gemm"
+        for _ in range(args.warmup):
+            run(taps_d, z, ln, keep=keep)
+        pred.check()
+        pred.profile(True, [kern])
+        launches0 = pred.launch_count
+        sampler = ClockSampler(local)
+        sampler.start()
+        barrier()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        for _ in range(args.steps):
+            run(taps_d, z, ln, keep=keep)
+        ev1.record(stream)
+        ev1.synchronize()
+        barrier()
+        clocks = sampler.stop()
+        ms = max_over_ranks(ev0.elapsed_time(ev1))
+        launches = pred.launch_count - launches0
+        prof_live = pred.profile_read()
+        pred.profile(False)
+        pred.check()
+        k_ms, k_n = prof_live[kern]
+        if kern == "fc_gemm":
+            k_flops = 2.0 * T * shape.d * 3 * shape.d
+            name, alg = "fc_gemm (k_gemm_tc<256, F32>, folded input norm)", f"2*T*d*3d, T={T}"
+        else:
+            k_flops = 2.0 * T * (2 * shape.ffn) * shape.d
+            name, alg = "gateup_swiglu_gemm (k_gemm_tc<256, SWIGLU>)", f"2*T*(2F)*d, T={T}"
+        k_tflops = k_flops / (k_ms / k_n / 1e3) / 1e12
+        roof = {"bound": "tensor", "kernel": name, "achieved": k_tflops, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
+                "frac": k_tflops / peaks["bf16_sus"], "peak_kind": f"bf16 sustained {peaks['src']}",
+                "traffic": measured_traffic(kern, f"{args.traffic_key}-static-{Bq}p-T{T}"),
+                "algorithmic_per_launch": f"{k_flops:.4g} FLOP = {alg}"}
+        flops = (prefill_flops(shape, lengths, Bq, args.gated, args.embed, whole_layer=keep or not pruned_rows)
+                 + (2.0 * Bq * pred.vocab * shape.d if K else 0.0))
+        return ms, launches, clocks, roof, flops
+
+    ms, launches, clocks, roofline, flops = timed(args.keep_rows)
+    whole = None
+    if pruned_rows and not args.no_whole_layer:
+        w_ms, _, w_clocks, w_roof, w_flops = timed(True)
+        whole = {"ms_per_step": w_ms / args.steps, "value": world * Bq * args.steps / (w_ms / 1e3),
+                 "tensor_peak_frac_step": w_flops * args.steps / (w_ms / 1e3) / 1e12 / peaks["bf16_sus"],
+                 "roofline": w_roof, "clocks": w_clocks,
+                 "note": "the same prediction with the whole layer run on every prompt row (OUTLETS_KEEP_ROWS)"}
     # per-stage breakdown in a separate (untimed) pass: stage events serialize the kernels
     pred.profile(True)
     for _ in range(3):
-        run(taps_d, z, ln)
+        run(taps_d, z, ln, keep=args.keep_rows)
     prof = pred.profile_read()
     pred.profile(False)
     ms_step = ms / args.steps
     value = world * Bq * args.steps / (ms / 1e3)
-    flops = (prefill_flops(shape, lengths, Bq, args.gated, args.embed)
-             + (2.0 * Bq * pred.vocab * shape.d if K else 0.0))
-    gu_ms, gu_n = prof_live["gateup_swiglu_gemm"]
-    gu_flops = 2.0 * T * (2 * shape.ffn) * shape.d
-    gu_tflops = gu_flops / (gu_ms / gu_n / 1e3) / 1e12
-    roofline = {"bound": "tensor", "kernel": "gateup_swiglu_gemm (k_gemm_tc<256, SWIGLU>)",
-                "achieved": gu_tflops, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
-                "frac": gu_tflops / peaks["bf16_sus"], "peak_kind": f"bf16 sustained {peaks['src']}",
-                "traffic": measured_traffic("gateup_swiglu_gemm", f"{args.traffic_key}-static-{Bq}p-T{T}"),
-                "algorithmic_per_launch": f"{gu_flops:.4g} FLOP = 2*T*(2F)*d, T={T}"}
-    stages = {k: {"ms_per_step": v[0] / max(v[1], 1), "share": v[0] / max(sum(x[0] for x in prof.values()), 1e-9)}
+    # a stage may run several kernels' event pairs per pass (pruned static prediction): per pass = total / 3
+    stages = {k: {"ms_per_step": v[0] / 3, "share": v[0] / max(sum(x[0] for x in prof.values()), 1e-9)}
               for k, v in prof.items() if v[1]}
 
     # ---------------- end to end through the C ABI with host buffers
@@ -520,6 +555,10 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
            "tensor_peak_frac_step": flops * args.steps / (ms / 1e3) / 1e12 / peaks["bf16_sus"],
            "roofline": roofline, "stages": stages, "clocks": clocks, "e2e": e2e,
            "gpu_launches": launches}
+    out["config"]["layer_rows"] = ("keys/values for every prompt row; queries, attention, O, MLP, final norm and "
+                                   "head for each prompt's last row" if pruned_rows else "whole layer on every row")
+    if whole:
+        out["whole_layer"] = whole
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n_pred, n_tok, secs = oracle_sample(shape, w, taps, cu, lengths, 1200, args.dual or None, args.tokens)
         out["cpu_baseline"] = {"value": n_pred / secs, "unit": "predictions/s", "cores": cpu_threads(),

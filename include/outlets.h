@@ -170,6 +170,14 @@ int32_t outlets_kv_slot_length(const outlets_kv* kv, int32_t slot);
 int32_t outlets_kv_free_pages(const outlets_kv* kv);
 
 #define OUTLETS_ALL_TOKENS 1u /* prefill flag: predict at every packed row, not only each sequence's last */
+/* Prefill flag: run the whole draft layer on every packed row even when only
+ * each sequence's last row is predicted.  Without it (bf16 contexts, T > 256)
+ * only the keys and values are projected for every row.  These feed the last
+ * rows' attention and the KV cache.  Queries, attention, O, the MLP, the
+ * final norm and the head run on the B predicted rows only.  The outputs are
+ * the same either way.  The flag keeps every row's q / attention / a / y for
+ * outlets_get_intermediate. */
+#define OUTLETS_KEEP_ROWS 2u
 
 /* Static prediction over a packed varlen batch (Sec. 3.2, t = 0).
  *   taps[3]     device or host, [T, d] each (bf16 or f32 like the context),
@@ -179,7 +187,7 @@ int32_t outlets_kv_free_pages(const outlets_kv* kv);
  *   kv, slots   optional (both or neither): slots is host int32 [B], distinct;
  *               each slot is reset and then holds its sequence's post-RoPE
  *               keys/values, ready for outlets_predict_step.
- *   flags       0 or OUTLETS_ALL_TOKENS.
+ *   flags       0, or OUTLETS_ALL_TOKENS and / or OUTLETS_KEEP_ROWS.
  *   z_out, len_out  device or host f32 [B] (or [T] with OUTLETS_ALL_TOKENS):
  *               z_hat and max(0, expm1(z_hat)) = predicted remaining length.
  *               len_out may be NULL.
@@ -281,7 +289,10 @@ outlets_status outlets_draft_head(outlets_ctx* ctx, const void* h_draft, int32_t
 /* Synchronizes the stream, then reports (and clears) the device error word. */
 outlets_status outlets_check(outlets_ctx* ctx, void* stream);
 
-/* Intermediates of the last prediction call, for parity testing. */
+/* Intermediates of the last prediction call, for parity testing.  Rows: every
+ * row of the call.  After a prefill that predicts only the last rows without
+ * OUTLETS_KEEP_ROWS, q, attention, a and y hold the B predicted rows instead.
+ * They are in sequence order, and the info's rows says which. */
 typedef enum outlets_tensor {
   OUTLETS_T_FCTX = 0,   /* f_ctx [rows, d] f32 (Eq. 1) */
   OUTLETS_T_XIN = 1,    /* input-normed x [rows, d] act */

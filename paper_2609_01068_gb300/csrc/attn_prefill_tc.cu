@@ -223,7 +223,7 @@ __global__ void __launch_bounds__(192, 1)
     bool ok = true;
     for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
       const TcAttnItem w = items[it];
-      const int qp = (w.q_start - w.seq_start) + r;  // position of this row in its sequence
+      const int qp = w.q_pos0 + r;  // position of this row in its sequence
       float m_used = -INFINITY, l = 0.f;
       for (int j = 0; j < w.n_kv; ++j, ++g) {
         const int sb = g & 1;

@@ -294,7 +294,7 @@ __global__ void __launch_bounds__(RopeBlock<In>::kThreads, RopeBlock<In>::kMinBl
     cache_base = ((long long)page * KVH) * a.page_tokens + pos % a.page_tokens;
   }
   const int cpr = half / 8;  // 8-element chunks per half head
-  for (int idx = threadIdx.x; idx < (H + KVH) * cpr; idx += blockDim.x) {
+  for (int idx = (q_out ? 0 : H * cpr) + threadIdx.x; idx < (H + KVH) * cpr; idx += blockDim.x) {
     const int head = idx / cpr;
     const int i = (idx - head * cpr) * 8;
     float x1[8], x2[8], y1[8], y2[8];
@@ -356,6 +356,18 @@ __global__ void __launch_bounds__(RopeBlock<In>::kThreads, RopeBlock<In>::kMinBl
       __syncthreads();  // every slice read of the block is done
       discard_slice_rows(qkv, a.n_split, a.split_stride, row, a.qkv_ld);
     }
+  }
+}
+
+// dst[r] = src[idx[r]], 16 bytes per thread step.
+__global__ void __launch_bounds__(256) k_gather_rows(const uint4* __restrict__ src, const int* __restrict__ idx,
+                                                     uint4* __restrict__ dst, int rows, long long row_vec) {
+  pdl_trigger();
+  pdl_wait();
+  const long long n = (long long)rows * row_vec;
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+    const long long r = i / row_vec, c = i - r * row_vec;
+    dst[i] = src[(long long)idx[r] * row_vec + c];
   }
 }
 
@@ -589,6 +601,17 @@ cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_st
   if (rows == 0) return cudaSuccess;
   const int threads = std::min(512, std::max(64, ((width / 4 + 31) / 32) * 32));
   OUTLETS_TRY_LAUNCH(launch_k(k_head_tail, dim3(rows), dim3(threads), 0, stream, h_pre, n_split, split_stride, b_prev, w_last, b_last, rows, width, z, len, discard));
+  return cudaGetLastError();
+}
+
+cudaError_t gather_rows_launch(const void* src, const int* idx, void* dst, int rows, long long row_bytes,
+                               cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  if (row_bytes % 16 || (reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) % 16)
+    return cudaErrorInvalidValue;
+  const long long vec = row_bytes / 16;
+  OUTLETS_TRY_LAUNCH(launch_k(k_gather_rows, dim3(grid_for((long long)rows * vec, 256)), dim3(256), 0, stream,
+                              reinterpret_cast<const uint4*>(src), idx, reinterpret_cast<uint4*>(dst), rows, vec));
   return cudaGetLastError();
 }
 

@@ -175,7 +175,7 @@ struct RopeArgs {
   const float* cos_tab;  // [max_pos, hd/2]
   const float* sin_tab;
   int max_pos;
-  void* q_out;           // [T, H, hd]
+  void* q_out;           // [T, H, hd], or null: q heads are skipped (keys/values only)
   void* k_out;           // head-major [KVH, kv_ld_rows, hd] or null
   void* v_out;
   long long kv_ld_rows;
@@ -204,6 +204,11 @@ cudaError_t head_tail_launch(const float* h_pre, int n_split, long long split_st
                              const float* w_last, const float* b_last, int rows, int width, float* z, float* len,
                              cudaStream_t stream, bool discard = false);
 
+// dst[r] = src[idx[r]] for r < rows: rows of row_bytes bytes (a multiple of 16,
+// 16-byte aligned rows).
+cudaError_t gather_rows_launch(const void* src, const int* idx, void* dst, int rows, long long row_bytes,
+                               cudaStream_t stream);
+
 // dst row map(row_base + r) <- src row r (f32 -> Act); map: row_mode 0 identity,
 // 1 gate rows, 2 up rows of the [gate 32 | up 32] interleave.  kb_np == 0:
 // row-major with row stride dst_ld; kb_np > 0: the k-block-major swizzled
@@ -228,8 +233,12 @@ cudaError_t attn_prefill_simt_launch(const Act* q, const Act* k, const Act* v, c
 // sequence [seq_start, seq_start + seq_len) for one query head; n_kv = number
 // of 128-key tiles it attends to (the last one is the diagonal tile);
 // v_start = the sequence's first column in V^T (a multiple of 8).
+// One work item: q_len query rows from row q_start of q (positions q_pos0 ..
+// q_pos0 + q_len - 1 of their sequence) against keys 0 .. 128 n_kv - 1 of the
+// sequence at rows seq_start.. of K; keys past a row's position are masked,
+// which the kernel does on the last key tile only.
 struct TcAttnItem {
-  int q_start, q_len, seq_start, seq_len, v_start, head, n_kv, pad;
+  int q_start, q_len, seq_start, seq_len, v_start, head, n_kv, q_pos0;
 };
 // q_map over q [rows, H*hd] (box 64 x 128), k_map over head-major K
 // [KVH * kv_ld, hd] (box 64 x 128), vt_map over V^T [KVH * hd, vt_ld] (box

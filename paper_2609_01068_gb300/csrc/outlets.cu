@@ -166,6 +166,10 @@ struct outlets_ctx {
   void* vt = nullptr;        // V^T [KVH * hd, vt_ld] for the tcgen05 prefill attention (bf16)
   long long vt_ld = 0;
   void* gate_act = nullptr;  // [max_rows, H*hd] sigmoid(gate), act dtype
+  // static prediction of the last rows only (bf16): x_hat, the embedding
+  // half of the layer input and f of each sequence's last row, [max_batch, d]
+  void *last_x = nullptr, *last_e = nullptr;
+  float* last_f = nullptr;
   std::vector<int> head_dims;  // d, hidden..., 1
   std::vector<void*> allocs;
   size_t dev_bytes = 0;
@@ -212,6 +216,7 @@ struct outlets_ctx {
   bool have_prev = false;
 
   int last_rows = 0, last_out_rows = 0;
+  int last_tail_rows = 0;         // rows of q / attention / a / y of the last call (all rows, or the predicted ones)
   int last_kind = 0;              // 0: none, 1: prefill, 2: step or draft step (its y rows feed a draft step)
   std::vector<int> last_slots;    // slots of the last step, in row order
   bool oom = false;
@@ -631,8 +636,10 @@ outlets_status gemm_f32(outlets_ctx* c, const void* const* a, int k_piece, int M
 
 // Everything after attention: O projection + residual, post-attention norm,
 // SwiGLU MLP + residual, final norm of the predicted rows, length head.
+// resid: the rows of f (the layer input's residual stream) that go with the
+// rows of c->attn.
 outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_row_idx_dev, float* z_dev,
-                        float* len_dev, cudaStream_t s) {
+                        float* len_dev, cudaStream_t s, const float* resid) {
   const int d = c->d;
   const float eps = c->cfg.rms_eps;
   const bool small = small_path(c, rows);
@@ -647,15 +654,15 @@ outlets_status run_tail(outlets_ctx* c, int rows, int out_rows, const int* out_r
     if (small)
       OUT_TRY(gemm_split(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, c->part, &sl, s));
     else if (c->bf16)  // a = f + attn W_o^T, its bf16 copy and per-tile sums of squares (norm folded)
-      OUT_TRY(gemm_tc(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d,
+      OUT_TRY(gemm_tc(c, a1, 1, c->attn_w, c->attn_w, rows, c->w_o, c->np_o, d, c->attn_w, EPI_F32, c->a, d, resid, d,
                       nullptr, s, &nf_a));
     else
-      OUT_TRY(gemm_f32(c, a1, c->attn_w, rows, c->w_o, d, c->attn_w, EPI_F32, c->a, d, c->f, d, nullptr, s));
+      OUT_TRY(gemm_f32(c, a1, c->attn_w, rows, c->w_o, d, c->attn_w, EPI_F32, c->a, d, resid, d, nullptr, s));
   }
   c->stage_end(1);
   if (small) {
     c->stage_begin(OUTLETS_S_NORM_POST);
-    OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, c->f, nullptr, c->ones, (bf16*)c->ahat,
+    OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, resid, nullptr, c->ones, (bf16*)c->ahat,
                                           c->a, rows, d, eps, s, discard_slices()));
     c->stage_end(1);
   } else if (!c->bf16) {
@@ -890,10 +897,12 @@ struct QkvSrc {
 // FC (Eq. 1) -> input RMSNorm -> QKV for rows row0 .. row0 + rows - 1 (tp
 // points at row row0 of each tap; row0 > 0 only on the large-M path).
 outlets_status run_qkv(outlets_ctx* c, int rows, QkvSrc* q, cudaStream_t s, int row0, const int* tok_dev, int sl,
-                       int n_norm);
+                       int n_norm, bool kv_only);
 
+// kv_only: the large-M QKV GEMM computes only the key and value columns (the
+// static prediction of the last rows computes their queries separately).
 outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvSrc* q, cudaStream_t s,
-                         int row0, const int* tok_dev) {
+                         int row0, const int* tok_dev, bool kv_only = false) {
   const int d = c->d;
   const float eps = c->cfg.rms_eps;
   const bool small = small_path(c, rows);
@@ -906,7 +915,7 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
     OUT_CK(c, cudaMemcpyAsync(c->f, c->y, (size_t)rows * d * 4, cudaMemcpyDeviceToDevice, s));
     if (c->bf16) OUT_CK(c, rmsnorm_launch<bf16>(c->f, c->ones, (bf16*)c->xhat, nullptr, rows, d, eps, s));
     else OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
-    return run_qkv(c, rows, q, s, row0, tok_dev, sl, 1);
+    return run_qkv(c, rows, q, s, row0, tok_dev, sl, 1, false);
   }
   // large-M bf16 without the embedding branch: the input RMSNorm is folded
   // into the FC (bf16 copy + sums of squares) and QKV (row scale) GEMMs
@@ -926,7 +935,7 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
     OUT_TRY(gemm_f32(c, tp, d, rows, c->w_proj, d, 3 * d, EPI_F32, c->f, d, nullptr, 0, nullptr, s));
   }
   c->stage_end(1);
-  if (fold_in) return run_qkv(c, rows, q, s, row0, tok_dev, sl, 0);
+  if (fold_in) return run_qkv(c, rows, q, s, row0, tok_dev, sl, 0, kv_only);
   c->stage_begin(OUTLETS_S_NORM_IN);
   if (small)
     OUT_CK(c, rmsnorm_reduce_launch<bf16>(c->part, sl, (long long)rows * d, nullptr, nullptr, c->ones, (bf16*)c->xhat,
@@ -936,13 +945,13 @@ outlets_status run_front(outlets_ctx* c, const void* const tp[3], int rows, QkvS
                                    d, eps, s));
   else
     OUT_CK(c, rmsnorm_launch<float>(c->f, c->g_in, (float*)c->xhat, nullptr, rows, d, eps, s));
-  return run_qkv(c, rows, q, s, row0, tok_dev, sl, 1);
+  return run_qkv(c, rows, q, s, row0, tok_dev, sl, 1, kv_only);
 }
 
 // Input-embedding branch (if any) and the QKV projection; the input-norm stage
 // (n_norm kernels so far) is still open.
 outlets_status run_qkv(outlets_ctx* c, int rows, QkvSrc* q, cudaStream_t s, int row0, const int* tok_dev, int sl,
-                       int n_norm) {
+                       int n_norm, bool kv_only) {
   const int d = c->d;
   const float eps = c->cfg.rms_eps;
   const bool small = small_path(c, rows);
@@ -975,9 +984,14 @@ outlets_status run_qkv(outlets_ctx* c, int rows, QkvSrc* q, cudaStream_t s, int 
     NormFold use;  // folded input norm: scale the rows by the FC's sums of squares
     use.row_ss = c->ss_f + (size_t)row0 * c->ss_stride;
     use.tiles = c->fold_tiles_f;
-    OUT_TRY(gemm_tc(c, a1, pieces, d, d, rows, c->w_qkv, c->np_qkv, c->qkv_n, K, EPI_ACT,
-                    (char*)c->qkv + (size_t)row0 * c->qkv_n * c->esz, c->qkv_n, nullptr, 0, nullptr, s,
-                    c->xin_raw ? &use : nullptr));
+    // keys and values only: output columns H*hd .. (H + 2 KVH)*hd, i.e. the
+    // weight rows from H*hd on in the k-block-major layout (row offset n0:
+    // n0 * 64 elements; n0 is a multiple of 8, so the swizzle phase holds)
+    const long long n0 = kv_only ? (long long)c->H * c->hd : 0;
+    const int n_cols = kv_only ? 2 * c->KVH * c->hd : c->qkv_n;
+    OUT_TRY(gemm_tc(c, a1, pieces, d, d, rows, (const char*)c->w_qkv + (size_t)n0 * 64 * c->esz, c->np_qkv, n_cols,
+                    K, EPI_ACT, (char*)c->qkv + ((size_t)row0 * c->qkv_n + n0) * c->esz, c->qkv_n, nullptr, 0,
+                    nullptr, s, c->xin_raw ? &use : nullptr));
     *q = {c->qkv, false, 1, 0};
   } else {
     OUT_TRY(gemm_f32(c, a1, d, rows, c->w_qkv, c->qkv_n, K, EPI_F32, c->qkv, c->qkv_n, nullptr, 0, nullptr, s));
@@ -1210,6 +1224,11 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
   }
   c->u = c->alloc(R * c->Fp * es);
   if (!c->bf16) c->gu32 = (float*)c->alloc(R * 2 * c->Fp * 4);
+  if (c->bf16) {
+    c->last_x = c->alloc((size_t)cfg->max_batch * d * es);
+    if (c->EV > 0) c->last_e = c->alloc((size_t)cfg->max_batch * d * es);
+    c->last_f = (float*)c->alloc((size_t)cfg->max_batch * d * 4);
+  }
   int hmax = 1;
   for (size_t i = 1; i < c->head_dims.size(); ++i) hmax = std::max(hmax, c->head_dims[i]);
   c->h1a = (float*)c->alloc(R * hmax * 4);
@@ -1515,12 +1534,64 @@ outlets_status check_tokens(outlets_ctx* c, const int32_t* tokens, long long n) 
   return OUTLETS_OK;
 }
 
+// Static prediction of the last rows only: x_hat (and the embedding half of
+// the layer input) of each sequence's last row, its q / k / v projection, and
+// RoPE of q at position L - 1 into rows 0 .. B-1 of c->q (the gate of gated
+// attention into rows 0 .. B-1 of c->gate_act).  The keys and values of
+// every row were written by the front.
+outlets_status run_last_q(outlets_ctx* c, int B, const int* last_dev, const int* pos_dev, cudaStream_t s) {
+  const int d = c->d;
+  c->stage_begin(OUTLETS_S_QKV);
+  // g_in is folded into W_qkv: the norm has unit gains
+  OUT_CK(c, rmsnorm_gather_launch<bf16>(c->f, last_dev, c->ones, (bf16*)c->last_x, B, d, c->cfg.rms_eps, s));
+  int n = 2;
+  const void* a1[3] = {c->last_x, c->last_x, c->last_x};
+  int pieces = 1;
+  if (c->EV > 0) {
+    OUT_CK(c, gather_rows_launch(c->ehat, last_dev, c->last_e, B, (long long)d * c->esz, s));
+    a1[0] = c->last_e;
+    a1[1] = c->last_x;
+    pieces = 2;
+    ++n;
+  }
+  QkvSrc q;
+  if (small_path(c, B)) {
+    int sl = 1;
+    OUT_TRY(gemm_split(c, a1, pieces, d, d, B, c->w_qkv, c->np_qkv, c->qkv_n, c->qkv_k, c->part, &sl, s));
+    q = {c->part, true, sl, (long long)B * c->qkv_n};
+  } else {
+    OUT_TRY(gemm_tc(c, a1, pieces, d, d, B, c->w_qkv, c->np_qkv, c->qkv_n, c->qkv_k, EPI_ACT, c->qkv, c->qkv_n, nullptr,
+                    0, nullptr, s));
+    q = {c->qkv, false, 1, 0};
+  }
+  c->stage_end(n);
+  c->stage_begin(OUTLETS_S_ROPE);
+  RopeArgs ra{};
+  ra.T = B;
+  ra.H = c->H;
+  ra.KVH = c->KVH;
+  ra.hd = c->hd;
+  ra.B = B;
+  ra.pos = pos_dev;
+  ra.cos_tab = c->rope_cos;
+  ra.sin_tab = c->rope_sin;
+  ra.max_pos = c->cfg.max_position;
+  ra.q_out = c->q;
+  ra.kv_ld_rows = c->cfg.max_tokens;
+  ra.qkv_ld = c->qkv_n;
+  ra.gate_out = c->gated ? c->gate_act : nullptr;
+  ra.err = c->err_dev;
+  OUT_TRY(launch_rope(c, q, ra, s));
+  c->stage_end(1);
+  return OUTLETS_OK;
+}
+
 outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const int32_t* tokens, const int32_t* cu,
                                int32_t B, int32_t T, outlets_kv* kv, const int32_t* slots, uint32_t flags,
                                float* z_out, float* len_out, const outlets_draft_out* draft, void* stream) {
   cudaStream_t s = (cudaStream_t)stream;
   if (!taps || !cu || !z_out) return c->fail(OUTLETS_EINVAL, "taps, cu_seqlens and z_out must not be NULL");
-  if (flags & ~OUTLETS_ALL_TOKENS) return c->fail(OUTLETS_EINVAL, "unknown flag");
+  if (flags & ~(OUTLETS_ALL_TOKENS | OUTLETS_KEEP_ROWS)) return c->fail(OUTLETS_EINVAL, "unknown flag");
   if (B < 0 || T < 0) return c->fail(OUTLETS_EINVAL, "B and T must be >= 0");
   if ((kv == nullptr) != (slots == nullptr)) return c->fail(OUTLETS_EINVAL, "kv and slots go together");
   if (kv && kv->ctx != c) return c->fail(OUTLETS_EINVAL, "kv belongs to another context");
@@ -1554,6 +1625,11 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   }
   const bool all_tokens = flags & OUTLETS_ALL_TOKENS;
   const int out_rows = all_tokens ? T : B;
+  // Only each sequence's last row is predicted, and the layer's output at a
+  // row feeds nothing but that row's prediction: every row needs its keys and
+  // values (attention of the last rows, the cache), only the last rows need
+  // queries, attention, O, the MLP, the final norm and the head.
+  const bool prune = c->bf16 && !all_tokens && !(flags & OUTLETS_KEEP_ROWS) && !small_path(c, T);
 
   OUT_TRY(begin_call(c, s));
   CallSlot slot_guard{c, s};
@@ -1576,6 +1652,9 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   std::vector<int> last(B);
   for (int b = 0; b < B; ++b) last[b] = cu[b + 1] - 1;
   const size_t off_last = mb.put(last);
+  std::vector<int> pos_last(B);
+  for (int b = 0; b < B; ++b) pos_last[b] = cu[b + 1] - cu[b] - 1;
+  const size_t off_pos_last = prune ? mb.put(pos_last) : 0;
   size_t off_items = 0, off_vstart = 0;
   int n_items = 0;
   if (c->bf16) {
@@ -1594,7 +1673,8 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
     std::vector<int> tq;                    // per tile: b, tile index
     for (int b = 0; b < B; ++b) {
       const int L = cu[b + 1] - cu[b];
-      for (int i = 0; i * 128 < L; ++i) {
+      // pruned: one query row per sequence (its last), against all its keys
+      for (int i = prune ? (L - 1) / 128 : 0; i * 128 < L; ++i) {
         tiles.push_back({i + 1, (int)(tq.size() / 2)});
         tq.push_back(b);
         tq.push_back(i);
@@ -1607,7 +1687,9 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
       const int b = tq[2 * t.second], i = tq[2 * t.second + 1];
       const int L = cu[b + 1] - cu[b];
       for (int h = 0; h < c->H; ++h) {
-        const int v[8] = {cu[b] + 128 * i, std::min(128, L - 128 * i), cu[b], L, vstart[b], h, i + 1, 0};
+        // pruned: the query is row b of the compact q (position L - 1)
+        const int v[8] = {prune ? b : cu[b] + 128 * i, prune ? 1 : std::min(128, L - 128 * i), cu[b], L, vstart[b],
+                          h, i + 1, prune ? L - 1 : 128 * i};
         items.insert(items.end(), v, v + 8);
       }
     }
@@ -1669,15 +1751,16 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
       ra.page_tokens = kPageTokens;
     }
     ra.qkv_ld = c->qkv_n;
-    ra.gate_out = c->gated ? c->gate_act : nullptr;
+    ra.gate_out = c->gated && !prune ? c->gate_act : nullptr;
     ra.err = c->err_dev;
+    if (prune) ra.q_out = nullptr;  // keys and values of every row; queries of the last rows below
     for (int k = 0; k < n_chunks; ++k) {
       const int r0 = k * chunk_rows, rows = std::min(T, r0 + chunk_rows) - r0;
       if (n_chunks > 1) OUT_CK(c, cudaStreamWaitEvent(s, c->chunk_ev[k], 0));
       const size_t off = (size_t)r0 * c->d * c->esz;
       const void* tpc[3] = {(const char*)tp[0] + off, (const char*)tp[1] + off, (const char*)tp[2] + off};
       QkvSrc qsrc;
-      OUT_TRY(run_front(c, tpc, rows, &qsrc, s, r0, tok_dev));
+      OUT_TRY(run_front(c, tpc, rows, &qsrc, s, r0, tok_dev, prune));
       OUT_TRY(wait_meta(c, s));
       c->stage_begin(OUTLETS_S_ROPE);
       ra.row0 = r0;
@@ -1686,6 +1769,8 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
       c->stage_end(1);
     }
   }
+  if (prune) OUT_TRY(run_last_q(c, B, m + off_last, m + off_pos_last, s));
+  const int q_rows = prune ? B : T;
   // ---- attention
   c->stage_begin(OUTLETS_S_ATTN);
   if (c->bf16) {
@@ -1694,7 +1779,7 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
                                  c->vt_ld, s));
     CUtensorMap qm, km, vm;
     const uint64_t kv_rows = (uint64_t)c->KVH * c->cfg.max_tokens;
-    if (!cached_map(c, &qm, c->q, c->attn_w, T, c->attn_w, 128) ||
+    if (!cached_map(c, &qm, c->q, c->attn_w, q_rows, c->attn_w, 128) ||
         !cached_map(c, &km, c->kh, c->hd, kv_rows, c->hd, 128) ||
         !cached_map(c, &vm, c->vt, c->vt_ld, (uint64_t)c->KVH * c->hd, c->vt_ld, c->hd))
       return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for attention");
@@ -1709,8 +1794,17 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   }
   c->stage_end(1);
   const OutDst od = out_dst(c, z_out, len_out);
-  OUT_TRY(run_tail(c, T, out_rows, all_tokens ? nullptr : m + off_last, od.z, od.len, s));
+  if (prune) {
+    // the residual f of the last rows, then O, the MLP, the norm and the head on those rows
+    c->stage_begin(OUTLETS_S_O);
+    OUT_CK(c, gather_rows_launch(c->f, m + off_last, c->last_f, B, (long long)c->d * 4, s));
+    c->stage_end(1);
+    OUT_TRY(run_tail(c, B, B, nullptr, od.z, od.len, s, c->last_f));
+  } else {
+    OUT_TRY(run_tail(c, T, out_rows, all_tokens ? nullptr : m + off_last, od.z, od.len, s, c->f));
+  }
   if (draft) OUT_TRY(run_draft(c, c->hn, out_rows, *draft, s));
+  c->last_tail_rows = prune ? B : T;
   c->last_rows = T;
   c->last_out_rows = out_rows;
   c->last_kind = 1;
@@ -1871,10 +1965,11 @@ outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int
     }
   }
   const OutDst od = out_dst(c, z_out, len_out);
-  OUT_TRY(run_tail(c, B, B, nullptr, od.z, od.len, s));
+  OUT_TRY(run_tail(c, B, B, nullptr, od.z, od.len, s, c->f));
   if (draft) OUT_TRY(run_draft(c, c->hn, B, *draft, s));
   c->last_rows = B;
   c->last_out_rows = B;
+  c->last_tail_rows = B;
   c->last_kind = 2;
   c->last_slots.assign(slots, slots + B);
   return end_call(c, B, z_out, len_out, od, s);
@@ -1972,10 +2067,10 @@ outlets_status outlets_get_intermediate(outlets_ctx* c, int32_t which, void* dst
   switch (which) {
     case OUTLETS_T_FCTX: ti = {OUTLETS_F32, c->last_rows, c->d}; src = c->f; break;
     case OUTLETS_T_XIN: ti = {act, c->last_rows, c->d}; src = c->xhat; break;  // bf16: recomputed below
-    case OUTLETS_T_Q: ti = {act, c->last_rows, c->attn_w}; src = c->q; break;
-    case OUTLETS_T_ATTN: ti = {act, c->last_rows, c->attn_w}; src = c->attn; break;
-    case OUTLETS_T_A: ti = {OUTLETS_F32, c->last_rows, c->d}; src = c->a; break;
-    case OUTLETS_T_Y: ti = {OUTLETS_F32, c->last_rows, c->d}; src = c->y; break;
+    case OUTLETS_T_Q: ti = {act, c->last_tail_rows, c->attn_w}; src = c->q; break;
+    case OUTLETS_T_ATTN: ti = {act, c->last_tail_rows, c->attn_w}; src = c->attn; break;
+    case OUTLETS_T_A: ti = {OUTLETS_F32, c->last_tail_rows, c->d}; src = c->a; break;
+    case OUTLETS_T_Y: ti = {OUTLETS_F32, c->last_tail_rows, c->d}; src = c->y; break;
     case OUTLETS_T_HDRAFT: ti = {act, c->last_out_rows, c->d}; src = c->hn; break;
     default: return c->fail(OUTLETS_EINVAL, "unknown intermediate");
   }

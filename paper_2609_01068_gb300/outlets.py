@@ -19,6 +19,7 @@ OK, EINVAL, ENOMEM, ECUDA, EUNSUPPORTED, ECAPACITY, ETIMEOUT, EDEVICE = range(8)
 STATUS_NAMES = ["OK", "EINVAL", "ENOMEM", "ECUDA", "EUNSUPPORTED", "ECAPACITY", "ETIMEOUT", "EDEVICE"]
 F32, BF16 = 0, 1
 ALL_TOKENS = 1
+KEEP_ROWS = 2
 T_FCTX, T_XIN, T_Q, T_ATTN, T_A, T_Y, T_HDRAFT = range(7)
 N_STAGES = 12
 MAX_TOPK = 8
@@ -234,9 +235,11 @@ class Predictor:
 
     # -- prediction
     def prefill(self, taps, cu_seqlens, kv=None, slots=None, all_tokens=False, z_out=None, len_out=None,
-                stream=None, tokens=None):
+                stream=None, tokens=None, keep_rows=False):
         """Static prediction (z_hat, length_hat) for a packed varlen batch.
-        tokens: [T] int32 ids (numpy or torch), for the input-embedding branch."""
+        tokens: [T] int32 ids (numpy or torch), for the input-embedding branch.
+        keep_rows: run the whole layer on every row (keeps every row's
+        intermediates); otherwise only the predicted rows go past the K/V."""
         cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
         B, T = len(cu) - 1, int(cu[-1]) if len(cu) else 0
         n_out = T if all_tokens else B
@@ -244,7 +247,7 @@ class Predictor:
         tp = (c_vp * 3)(*[_ptr(t) for t in taps])
         sl = None if slots is None else np.ascontiguousarray(slots, dtype=np.int32)
         args = (cu.ctypes.data, B, T, kv.h if kv else None, None if sl is None else sl.ctypes.data,
-                ALL_TOKENS if all_tokens else 0, _ptr(z_out), _ptr(len_out))
+                (ALL_TOKENS if all_tokens else 0) | (KEEP_ROWS if keep_rows else 0), _ptr(z_out), _ptr(len_out))
         if tokens is None:
             st = self.lib.outlets_predict_prefill(self.h, tp, *args, _stream_handle(stream))
         else:
@@ -289,7 +292,7 @@ class Predictor:
         return d, out
 
     def prefill_dual(self, taps, cu_seqlens, k, kv=None, slots=None, all_tokens=False, logits=False, out=None,
-                     z_out=None, len_out=None, stream=None, tokens=None):
+                     z_out=None, len_out=None, stream=None, tokens=None, keep_rows=False):
         """Static prediction plus the draft head on the same rows:
         (z_hat, length_hat, {"ids", "logprob", "lse"[, "logits"]})."""
         cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
@@ -300,7 +303,8 @@ class Predictor:
         tp = (c_vp * 3)(*[_ptr(t) for t in taps])
         sl = None if slots is None else np.ascontiguousarray(slots, dtype=np.int32)
         args = (cu.ctypes.data, B, T, kv.h if kv else None, None if sl is None else sl.ctypes.data,
-                ALL_TOKENS if all_tokens else 0, _ptr(z_out), _ptr(len_out), ctypes.byref(d))
+                (ALL_TOKENS if all_tokens else 0) | (KEEP_ROWS if keep_rows else 0), _ptr(z_out), _ptr(len_out),
+                ctypes.byref(d))
         if tokens is None:
             st = self.lib.outlets_predict_prefill_dual(self.h, tp, *args, _stream_handle(stream))
         else:

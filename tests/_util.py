@@ -42,3 +42,19 @@ def check_hidden(g, r, dtype, what):
     e = maxrel(to_np(g) if not isinstance(g, np.ndarray) else g, r)
     assert e <= HIDDEN_TOL[dtype], f"{what}: max relative error {e}"
     return e
+
+
+def pruned(dtype, T, keep_rows=False, all_tokens=False):
+    """Whether a static prediction runs past the K/V projection on the
+    predicted rows only: bf16, more than 256 rows, last rows predicted, and
+    keep_rows not asked for."""
+    return dtype == "bf16" and T > 256 and not keep_rows and not all_tokens
+
+
+def check_rows(g, r_all, cu, dtype, what, is_pruned):
+    """A per-row intermediate against the oracle: every row, or each
+    sequence's last row (in sequence order) after a pruned prediction."""
+    r = np.asarray(r_all)[np.asarray(cu[1:]) - 1] if is_pruned else r_all
+    g = to_np(g) if not isinstance(g, np.ndarray) else g
+    assert g.shape[0] == r.shape[0], f"{what}: {g.shape[0]} rows, expected {r.shape[0]}"
+    return check_hidden(g, r, dtype, what)

@@ -11,7 +11,7 @@ import pytest
 
 from oracle import outlets_oracle as OR
 from paper_2609_01068_gb300 import synth
-from _util import check_hidden, check_z_len, to_device
+from _util import check_hidden, check_rows, check_z_len, pruned, to_device
 
 pytestmark = pytest.mark.gpu
 torch = pytest.importorskip("torch")
@@ -49,9 +49,11 @@ def test_gated_prefill_matches_oracle_every_intermediate(name):
     torch.cuda.synchronize()
     pred.check()
     T = int(cu[-1])
+    pr = pruned(shape.dtype, T)
     for which, r, what in [(OT.T_Q, ref["q"].reshape(T, -1), "q"), (OT.T_ATTN, ref["attn"], "gated attn"),
-                           (OT.T_A, ref["a"], "a"), (OT.T_HDRAFT, ref["h_draft"], "h_draft")]:
-        check_hidden(pred.intermediate(which), r, shape.dtype, f"gated {name} {what}")
+                           (OT.T_A, ref["a"], "a")]:
+        check_rows(pred.intermediate(which), r, cu, shape.dtype, f"gated {name} {what}", pr)
+    check_hidden(pred.intermediate(OT.T_HDRAFT), ref["h_draft"], shape.dtype, f"gated {name} h_draft")
     check_z_len(z, ln, ref["z"], ref["length"], shape.dtype, f"gated {name}")
 
 

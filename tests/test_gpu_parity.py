@@ -9,7 +9,7 @@ import pytest
 
 from oracle import outlets_oracle as OR
 from paper_2609_01068_gb300 import synth
-from _util import HIDDEN_TOL, check_hidden, check_z_len, maxrel, to_device, to_np
+from _util import pruned, check_rows, HIDDEN_TOL, check_hidden, check_z_len, maxrel, to_device, to_np
 
 pytestmark = pytest.mark.gpu
 
@@ -46,24 +46,62 @@ def _taps(shape, T, off=0):
     return synth.make_taps(shape, T, 0, off)
 
 
+@pytest.mark.parametrize("keep_rows", [True, False])
 @pytest.mark.parametrize("name", list(SHAPES))
-def test_prefill_matches_oracle_every_intermediate(name):
+def test_prefill_matches_oracle_every_intermediate(name, keep_rows):
+    """keep_rows: the whole layer on every row; otherwise (bf16, T > 256) q,
+    attention, a and y exist for each sequence's last row only."""
     from paper_2609_01068_gb300 import outlets as OT
     shape = SHAPES[name]
     pred, w = predictor(name)
     cu = synth.cu_seqlens(PREFILL_LENGTHS[name])
     taps = _taps(shape, int(cu[-1]))
     ref = OR.predict_prefill(w, shape, taps, cu)
-    z, ln = pred.prefill([to_device(t, shape.dtype) for t in taps], cu)
+    z, ln = pred.prefill([to_device(t, shape.dtype) for t in taps], cu, keep_rows=keep_rows)
     torch.cuda.synchronize()
     pred.check()
     T = int(cu[-1])
-    pairs = [(OT.T_FCTX, ref["f"], "f_ctx"), (OT.T_XIN, ref["x"], "x_in"),
-             (OT.T_Q, ref["q"].reshape(T, -1), "q"), (OT.T_ATTN, ref["attn"], "attn"),
-             (OT.T_A, ref["a"], "a"), (OT.T_Y, ref["y"], "y"), (OT.T_HDRAFT, ref["h_draft"], "h_draft")]
-    for which, r, what in pairs:
+    pr = pruned(shape.dtype, T, keep_rows)
+    for which, r, what in [(OT.T_FCTX, ref["f"], "f_ctx"), (OT.T_XIN, ref["x"], "x_in"),
+                           (OT.T_HDRAFT, ref["h_draft"], "h_draft")]:
         check_hidden(pred.intermediate(which), r, shape.dtype, f"{name} {what}")
+    for which, r, what in [(OT.T_Q, ref["q"].reshape(T, -1), "q"), (OT.T_ATTN, ref["attn"], "attn"),
+                           (OT.T_A, ref["a"], "a"), (OT.T_Y, ref["y"], "y")]:
+        check_rows(pred.intermediate(which), r, cu, shape.dtype, f"{name} {what}", pr)
     check_z_len(z, ln, ref["z"], ref["length"], shape.dtype, name)
+
+
+@pytest.mark.parametrize("name", ["mid128", "mid64"])
+def test_pruned_prefill_writes_the_same_cache_as_the_whole_layer(name):
+    """The static prediction of the last rows only projects keys and values
+    for every row with the same GEMM tiles as the whole layer: the KV caches
+    agree bit for bit (the steps after them do), and both predictions match
+    the oracle."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = SHAPES[name]
+    pred, w = predictor(name)
+    lengths = PREFILL_LENGTHS[name]
+    B = len(lengths)
+    cu = synth.cu_seqlens(lengths)
+    T = int(cu[-1])
+    assert pruned(shape.dtype, T)
+    taps_np = _taps(shape, T, off=81)
+    taps = [to_device(t, shape.dtype) for t in taps_np]
+    st = [to_device(t, shape.dtype) for t in synth.make_taps(shape, B, 0, 82)]
+    slots = np.arange(B, dtype=np.int32)
+    out = {}
+    for keep in (True, False):
+        kv = OT.KVCache(pred, max_slots=B, max_tokens_total=T + 64 * B)
+        z, ln = pred.prefill(taps, cu, kv=kv, slots=slots, keep_rows=keep)
+        z2, _ = pred.step(st, kv, slots)
+        torch.cuda.synchronize()
+        pred.check()
+        out[keep] = (z.clone(), ln.clone(), to_np(z2))
+        kv.close()
+    np.testing.assert_array_equal(out[False][2], out[True][2])
+    ref = OR.predict_prefill(w, shape, taps_np, cu)
+    for keep in (True, False):
+        check_z_len(out[keep][0], out[keep][1], ref["z"], ref["length"], shape.dtype, f"{name} keep_rows={keep}")
 
 
 @pytest.mark.parametrize("name", ["tiny-f32", "mid128"])
@@ -395,9 +433,11 @@ def test_nonunit_norm_gains(name, gated, embed):
     pred.check()
     ref = OR.predict_prefill(w, shape, taps, cu, tokens=tok)
     d = shape.d
-    for which, r, what in [(OT.T_XIN, ref["x"][:, -d:], "x_in"), (OT.T_Q, ref["q"].reshape(T, -1), "q"),
-                           (OT.T_A, ref["a"], "a"), (OT.T_Y, ref["y"], "y"), (OT.T_HDRAFT, ref["h_draft"], "h_draft")]:
+    pr = pruned(shape.dtype, T)
+    for which, r, what in [(OT.T_XIN, ref["x"][:, -d:], "x_in"), (OT.T_HDRAFT, ref["h_draft"], "h_draft")]:
         check_hidden(pred.intermediate(which), r, shape.dtype, f"gains {name} {what}")
+    for which, r, what in [(OT.T_Q, ref["q"].reshape(T, -1), "q"), (OT.T_A, ref["a"], "a"), (OT.T_Y, ref["y"], "y")]:
+        check_rows(pred.intermediate(which), r, cu, shape.dtype, f"gains {name} {what}", pr)
     check_z_len(z, ln, ref["z"], ref["length"], shape.dtype, f"gains {name} prefill")
     caches = OR.caches_from_prefill(ref, cu)
     st = synth.make_taps(shape, B, 0, 62)

@@ -3,7 +3,11 @@
 // request plus its own (already appended to the paged cache).
 //
 // Cache layout: pools [pages][KVH][page_tokens = 64][hd]; a request's keys are
-// the concatenation of its pages (page list uploaded per call).
+// the concatenation of its pages (page list uploaded per call).  The same
+// kernels read the head-major K/V of a static prediction ([KVH, kv_ld, hd],
+// "pages" of 64 rows from each prompt's first row) to attend from each
+// prompt's last row: the first row of a page is page * page_stride + kv head
+// * head_stride.
 //
 // bf16 path: split-KV.  One CTA = (request, split of <= split_len keys, kv
 // head).  The G = H / KVH query heads of the kv head form the rows of one
@@ -138,8 +142,7 @@ __global__ void __launch_bounds__(128, 3)
   __syncthreads();
 
   auto issue = [&](int pi, int stage) {
-    const int page = pages[page_begin + pi];
-    const int row = (page * a.KVH + g) * 64;
+    const int row = (int)((long long)pages[page_begin + pi] * a.page_stride + (long long)g * a.head_stride);
     uint8_t* dk = sKV + stage * 2 * C::PAGE_BYTES;
     mbar_arrive_expect_tx(&full[stage], 2 * C::PAGE_BYTES);
 #pragma unroll
@@ -364,7 +367,8 @@ __global__ void k_attn_decode_simt(const DecodeArgs a) {
   const float scale = rsqrtf((float)hd);
   float m = -INFINITY, l = 0.f;
   for (int j = 0; j < L; ++j) {
-    const long long base = (((long long)pages[j / a.page_tokens] * a.KVH + g) * a.page_tokens + j % a.page_tokens) * hd;
+    const long long base =
+        ((long long)pages[j / a.page_tokens] * a.page_stride + (long long)g * a.head_stride + j % a.page_tokens) * hd;
     float part = 0.f;
 #pragma unroll
     for (int i = 0; i < MAXD; ++i) {
@@ -415,7 +419,7 @@ cudaError_t launch_decode_tc(const CUtensorMap& k_map, const CUtensorMap& v_map,
 cudaError_t attn_decode_bf16_launch(const CUtensorMap& k_map, const CUtensorMap& v_map, const DecodeArgs& a,
                                     cudaStream_t stream) {
   if (a.B == 0) return cudaSuccess;
-  if (a.H / a.KVH > 16 || a.page_tokens != 64) return cudaErrorInvalidValue;
+  if (a.H / a.KVH > 16 || a.page_tokens != 64 || a.page_stride < 1 || a.head_stride < 1) return cudaErrorInvalidValue;
   if (a.hd == 128) return launch_decode_tc<128>(k_map, v_map, a, stream);
   if (a.hd == 64) return launch_decode_tc<64>(k_map, v_map, a, stream);
   return cudaErrorInvalidValue;
@@ -424,7 +428,7 @@ cudaError_t attn_decode_bf16_launch(const CUtensorMap& k_map, const CUtensorMap&
 template <typename Act>
 cudaError_t attn_decode_simt_launch(const DecodeArgs& a, cudaStream_t stream) {
   if (a.B == 0) return cudaSuccess;
-  if (a.hd > 256) return cudaErrorInvalidValue;
+  if (a.hd > 256 || a.page_stride < 1 || a.head_stride < 1) return cudaErrorInvalidValue;
   OUTLETS_TRY_LAUNCH(launch_k(k_attn_decode_simt<Act>, dim3(dim3(a.B, (a.H + 3) / 4)), dim3(128), 0, stream, a));
   return cudaGetLastError();
 }

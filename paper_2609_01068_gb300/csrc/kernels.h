@@ -259,6 +259,11 @@ struct DecodeArgs {
   int page_tokens;
   const int* page_list;   // concatenated page ids of every request
   const int* page_off;    // [B+1] offsets into page_list
+  // first K/V row of page p for kv head g: p * page_stride + g * head_stride
+  // (cache pools: KVH * 64 and 64; head-major [KVH, kv_ld, hd] buffers, with
+  // page ids that are row offsets: 1 and kv_ld)
+  long long page_stride;
+  int head_stride;
   const int* seq_len;     // [B] keys per request (cached + the new token)
   const int* work;        // [n_work] pairs (request, split), grouped by request
   const int* work_off;    // [B+1] first work item of each request

@@ -170,6 +170,10 @@ struct outlets_ctx {
   // half of the layer input and f of each sequence's last row, [max_batch, d]
   void *last_x = nullptr, *last_e = nullptr;
   float* last_f = nullptr;
+  // split-KV partials of the last rows' attention (decode attention over the
+  // head-major K/V of the call): [last_part_items, H, hd] and [.., H, 2]
+  float *last_part_o = nullptr, *last_part_ml = nullptr;
+  size_t last_part_items = 0;
   std::vector<int> head_dims;  // d, hidden..., 1
   std::vector<void*> allocs;
   size_t dev_bytes = 0;
@@ -1228,6 +1232,9 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
     c->last_x = c->alloc((size_t)cfg->max_batch * d * es);
     if (c->EV > 0) c->last_e = c->alloc((size_t)cfg->max_batch * d * es);
     c->last_f = (float*)c->alloc((size_t)cfg->max_batch * d * 4);
+    c->last_part_items = (size_t)cfg->max_batch + (size_t)cdiv(cfg->max_tokens, kSplitLen);
+    c->last_part_o = (float*)c->alloc(c->last_part_items * c->H * c->hd * 4);
+    c->last_part_ml = (float*)c->alloc(c->last_part_items * c->H * 2 * 4);
   }
   int hmax = 1;
   for (size_t i = 1; i < c->head_dims.size(); ++i) hmax = std::max(hmax, c->head_dims[i]);
@@ -1534,6 +1541,43 @@ outlets_status check_tokens(outlets_ctx* c, const int32_t* tokens, long long n) 
   return OUTLETS_OK;
 }
 
+// Split-KV work of decode attention over requests with seq_len[b] keys each.
+// Keys per work item: about a third of one resident CTA's share of all keys
+// (never below 512), so most requests need no split (and no merge) while the
+// longest items still fit several times into the whole pass.  Launch order:
+// longest items first (the short ones fill the tail).
+struct DecodeWork {
+  int split_len = 0, max_splits = 1, n_work = 0;
+  std::vector<int> work, work_off, order;  // (request, split) pairs, [B+1] offsets, launch order
+};
+DecodeWork decode_work(const outlets_ctx* c, const std::vector<int>& seq_len) {
+  DecodeWork w;
+  const int B = (int)seq_len.size();
+  long long total_keys = 0;
+  for (int b = 0; b < B; ++b) total_keys += seq_len[b];
+  const long long share = cdiv(total_keys * c->KVH, 3LL * kDecodeCtasPerSm * c->num_sms);
+  w.split_len = (int)std::max<long long>(kSplitLen, cdiv(share, kPageTokens) * kPageTokens);
+  w.work_off.assign(B + 1, 0);
+  for (int b = 0; b < B; ++b) {
+    const int ns = (int)cdiv(seq_len[b], w.split_len);
+    w.max_splits = std::max(w.max_splits, ns);
+    for (int sp = 0; sp < ns; ++sp) {
+      w.work.push_back(b);
+      w.work.push_back(sp);
+    }
+    w.work_off[b + 1] = (int)(w.work.size() / 2);
+  }
+  w.n_work = w.work_off[B];
+  std::vector<int> item_keys(w.n_work);
+  w.order.resize(w.n_work);
+  for (int i = 0; i < w.n_work; ++i) {
+    w.order[i] = i;
+    item_keys[i] = std::min(w.split_len, seq_len[w.work[2 * i]] - w.work[2 * i + 1] * w.split_len);
+  }
+  std::stable_sort(w.order.begin(), w.order.end(), [&](int x, int y) { return item_keys[x] > item_keys[y]; });
+  return w;
+}
+
 // Static prediction of the last rows only: x_hat (and the embedding half of
 // the layer input) of each sequence's last row, its q / k / v projection, and
 // RoPE of q at position L - 1 into rows 0 .. B-1 of c->q (the gate of gated
@@ -1657,7 +1701,24 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   const size_t off_pos_last = prune ? mb.put(pos_last) : 0;
   size_t off_items = 0, off_vstart = 0;
   int n_items = 0;
-  if (c->bf16) {
+  DecodeWork lw;  // pruned: decode attention of each prompt's last row over its head-major keys
+  size_t off_lsl = 0, off_lpl = 0, off_lpo = 0, off_lw = 0, off_lwo = 0, off_lord = 0;
+  if (prune) {
+    std::vector<int> lsl(B), lpl, lpo(B + 1, 0);
+    for (int b = 0; b < B; ++b) {
+      lsl[b] = cu[b + 1] - cu[b];
+      for (int p0 = 0; p0 < lsl[b]; p0 += kPageTokens) lpl.push_back(cu[b] + p0);  // page id = first row
+      lpo[b + 1] = (int)lpl.size();
+    }
+    lw = decode_work(c, lsl);
+    if ((size_t)lw.n_work > c->last_part_items) return c->fail(OUTLETS_ECAPACITY, "split-KV partial buffer too small");
+    off_lsl = mb.put(lsl);
+    off_lpl = mb.put(lpl);
+    off_lpo = mb.put(lpo);
+    off_lw = mb.put(lw.work);
+    off_lwo = mb.put(lw.work_off);
+    off_lord = mb.put(lw.order);
+  } else if (c->bf16) {
     // tcgen05 attention work items: 128-row query tiles x query heads, the
     // ones with the most key tiles first; V^T columns of each sequence start
     // at a multiple of 8
@@ -1673,8 +1734,7 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
     std::vector<int> tq;                    // per tile: b, tile index
     for (int b = 0; b < B; ++b) {
       const int L = cu[b + 1] - cu[b];
-      // pruned: one query row per sequence (its last), against all its keys
-      for (int i = prune ? (L - 1) / 128 : 0; i * 128 < L; ++i) {
+      for (int i = 0; i * 128 < L; ++i) {
         tiles.push_back({i + 1, (int)(tq.size() / 2)});
         tq.push_back(b);
         tq.push_back(i);
@@ -1687,9 +1747,7 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
       const int b = tq[2 * t.second], i = tq[2 * t.second + 1];
       const int L = cu[b + 1] - cu[b];
       for (int h = 0; h < c->H; ++h) {
-        // pruned: the query is row b of the compact q (position L - 1)
-        const int v[8] = {prune ? b : cu[b] + 128 * i, prune ? 1 : std::min(128, L - 128 * i), cu[b], L, vstart[b],
-                          h, i + 1, prune ? L - 1 : 128 * i};
+        const int v[8] = {cu[b] + 128 * i, std::min(128, L - 128 * i), cu[b], L, vstart[b], h, i + 1, 128 * i};
         items.insert(items.end(), v, v + 8);
       }
     }
@@ -1770,16 +1828,49 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
     }
   }
   if (prune) OUT_TRY(run_last_q(c, B, m + off_last, m + off_pos_last, s));
-  const int q_rows = prune ? B : T;
   // ---- attention
   c->stage_begin(OUTLETS_S_ATTN);
-  if (c->bf16) {
+  if (prune) {
+    // each prompt's last row against all its keys: the decode-attention
+    // kernels on the head-major K/V ("pages" of 64 rows from the prompt's first)
+    DecodeArgs da{};
+    da.B = B;
+    da.H = c->H;
+    da.KVH = c->KVH;
+    da.hd = c->hd;
+    da.q = c->q;
+    da.k_pool = c->kh;
+    da.v_pool = c->vh;
+    da.page_tokens = kPageTokens;
+    da.page_list = m + off_lpl;
+    da.page_off = m + off_lpo;
+    da.page_stride = 1;
+    da.head_stride = c->cfg.max_tokens;
+    da.seq_len = m + off_lsl;
+    da.work = m + off_lw;
+    da.work_off = m + off_lwo;
+    da.n_work = lw.n_work;
+    da.split_len = lw.split_len;
+    da.order = m + off_lord;
+    da.max_splits = lw.max_splits;
+    da.part_o = c->last_part_o;
+    da.part_ml = c->last_part_ml;
+    da.combine_count = c->dec_count;
+    da.out = c->attn;
+    da.gate = c->gate_act;  // null unless gated
+    da.err = c->err_dev;
+    CUtensorMap km, vm;
+    const uint64_t kv_rows = (uint64_t)c->KVH * c->cfg.max_tokens;
+    if (!cached_map(c, &km, c->kh, c->hd, kv_rows, c->hd, 64) || !cached_map(c, &vm, c->vh, c->hd, kv_rows, c->hd, 64))
+      return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for the head-major K/V");
+    OUT_CK(c, attn_decode_bf16_launch(km, vm, da, s));
+  } else if (c->bf16) {
     // V^T for the tcgen05 attention (keys contiguous), then the attention
     OUT_CK(c, v_transpose_launch(c->vh, cu_dev, m + off_vstart, B, T, c->cfg.max_tokens, c->KVH, c->hd, c->vt,
                                  c->vt_ld, s));
     CUtensorMap qm, km, vm;
     const uint64_t kv_rows = (uint64_t)c->KVH * c->cfg.max_tokens;
-    if (!cached_map(c, &qm, c->q, c->attn_w, q_rows, c->attn_w, 128) ||
+    if (!cached_map(c, &qm, c->q, c->attn_w, T, c->attn_w, 128) ||
         !cached_map(c, &km, c->kh, c->hd, kv_rows, c->hd, 128) ||
         !cached_map(c, &vm, c->vt, c->vt_ld, (uint64_t)c->KVH * c->hd, c->vt_ld, c->hd))
       return c->fail(OUTLETS_ECUDA, "cuTensorMapEncodeTiled failed for attention");
@@ -1849,15 +1940,7 @@ outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int
   if (!self_feed) OUT_TRY(prepare_taps(c, taps, B, tp, s));
 
   // ---- commit the append and build metadata
-  std::vector<int> pos(B), seq_len(B), po(B + 1, 0), pl, work, work_off(B + 1, 0);
-  // Keys per split-KV work item: about a third of one resident CTA's share of
-  // all keys (never below 512), so most requests need no split (and no merge)
-  // while the longest items still fit several times into the whole pass.
-  long long total_keys = 0;
-  for (int b = 0; b < B; ++b) total_keys += kv->len[slots[b]] + 1;
-  const long long share = cdiv(total_keys * c->KVH, 3LL * kDecodeCtasPerSm * c->num_sms);
-  const int split_len = (int)std::max<long long>(kSplitLen, cdiv(share, kPageTokens) * kPageTokens);
-  int max_splits = 1;
+  std::vector<int> pos(B), seq_len(B), po(B + 1, 0), pl;
   for (int b = 0; b < B; ++b) {
     const int sl = slots[b];
     if (kv->len[sl] % kPageTokens == 0) {
@@ -1869,30 +1952,17 @@ outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int
     seq_len[b] = kv->len[sl];
     pl.insert(pl.end(), kv->pages[sl].begin(), kv->pages[sl].end());
     po[b + 1] = (int)pl.size();
-    const int ns = (int)cdiv(seq_len[b], split_len);
-    max_splits = std::max(max_splits, ns);
-    for (int sp = 0; sp < ns; ++sp) {
-      work.push_back(b);
-      work.push_back(sp);
-    }
-    work_off[b + 1] = (int)(work.size() / 2);
   }
-  const int n_work = work_off[B];
-  // launch order: longest work items first (the short ones fill the tail)
-  std::vector<int> order(n_work), item_keys(n_work);
-  for (int w = 0; w < n_work; ++w) {
-    order[w] = w;
-    item_keys[w] = std::min(split_len, seq_len[work[2 * w]] - work[2 * w + 1] * split_len);
-  }
-  std::stable_sort(order.begin(), order.end(), [&](int x, int y) { return item_keys[x] > item_keys[y]; });
+  const DecodeWork dw = decode_work(c, seq_len);
+  const int n_work = dw.n_work, split_len = dw.split_len, max_splits = dw.max_splits;
   MetaBuilder mb;
   const size_t off_pos = mb.put(pos);
   const size_t off_sl = mb.put(seq_len);
   const size_t off_po = mb.put(po);
   const size_t off_pl = mb.put(pl);
-  const size_t off_w = mb.put(work);
-  const size_t off_wo = mb.put(work_off);
-  const size_t off_ord = mb.put(order);
+  const size_t off_w = mb.put(dw.work);
+  const size_t off_wo = mb.put(dw.work_off);
+  const size_t off_ord = mb.put(dw.order);
   const bool tok_host = tokens && !is_device_ptr(tokens);
   const size_t off_tok = tok_host ? mb.put(tokens, B) : 0;
   OUT_TRY(upload_meta(c, mb.v, s));
@@ -1938,6 +2008,8 @@ outlets_status predict_step(outlets_ctx* c, const void* const taps[3], const int
     da.page_tokens = kPageTokens;
     da.page_list = m + off_pl;
     da.page_off = m + off_po;
+    da.page_stride = (long long)c->KVH * kPageTokens;
+    da.head_stride = kPageTokens;
     da.seq_len = m + off_sl;
     da.work = m + off_w;
     da.work_off = m + off_wo;

@@ -31,7 +31,7 @@ using namespace outlets;
 namespace {
 
 constexpr int kPageTokens = 64;
-constexpr int kMaxTapChunks = 4;      // row chunks of host taps copied while earlier chunks compute
+constexpr int kMaxTapChunks = 8;      // row chunks of host taps copied while earlier chunks compute
 constexpr int kMinTapChunkRows = 2048;
 constexpr int kSplitLen = 512;        // shortest split-KV work item (keys)
 constexpr int kDecodeCtasPerSm = 3;   // resident decode-attention CTAs per SM

@@ -104,6 +104,43 @@ def test_pruned_prefill_writes_the_same_cache_as_the_whole_layer(name):
         check_z_len(out[keep][0], out[keep][1], ref["z"], ref["length"], shape.dtype, f"{name} keep_rows={keep}")
 
 
+def test_pruned_prefill_more_than_256_prompts():
+    """300 short prompts: the predicted rows take the large-M path (q / k / v
+    of the last rows by the tcgen05 GEMM, O / MLP / head on 300 rows)."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = MID64
+    pred, w = predictor("mid64", max_tokens=2048, max_batch=320)
+    rng = np.random.default_rng(7)
+    lengths = rng.integers(1, 7, size=300)
+    B = len(lengths)
+    cu = synth.cu_seqlens(lengths)
+    T = int(cu[-1])
+    assert pruned(shape.dtype, T) and B > 256
+    taps_np = _taps(shape, T, off=91)
+    taps = [to_device(t, shape.dtype) for t in taps_np]
+    st = [to_device(t, shape.dtype) for t in synth.make_taps(shape, B, 0, 92)]
+    slots = np.arange(B, dtype=np.int32)
+    out = {}
+    for keep in (True, False):
+        kv = OT.KVCache(pred, max_slots=B, max_tokens_total=T + 64 * B)
+        z, ln = pred.prefill(taps, cu, kv=kv, slots=slots, keep_rows=keep)
+        torch.cuda.synchronize()
+        pred.check()
+        h = to_np(pred.intermediate(OT.T_HDRAFT))
+        z2, ln2 = pred.step(st, kv, slots)
+        torch.cuda.synchronize()
+        pred.check()
+        out[keep] = (z.clone(), ln.clone(), h, z2.clone(), ln2.clone())
+        kv.close()
+    np.testing.assert_array_equal(to_np(out[False][3]), to_np(out[True][3]))
+    ref = OR.predict_prefill(w, shape, taps_np, cu)
+    for keep in (True, False):
+        check_z_len(out[keep][0], out[keep][1], ref["z"], ref["length"], shape.dtype, f"300 prompts keep_rows={keep}")
+        check_hidden(out[keep][2], ref["h_draft"], shape.dtype, f"300 prompts h_draft keep_rows={keep}")
+    ref2 = OR.predict_step(w, shape, synth.make_taps(shape, B, 0, 92), OR.caches_from_prefill(ref, cu))
+    check_z_len(out[False][3], out[False][4], ref2["z"], ref2["length"], shape.dtype, "300 prompts step")
+
+
 @pytest.mark.parametrize("name", ["tiny-f32", "mid128"])
 def test_all_tokens_mode_and_causal_prefix(name):
     shape = SHAPES[name]

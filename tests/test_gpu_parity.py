@@ -299,6 +299,14 @@ def test_argument_errors_change_nothing():
         pred.step([t[:2] for t in taps], kv, [0, 0])
     assert e.value.status == OT.EINVAL
     assert kv.slot_length(0) == 40
+    import ctypes
+    z = torch.empty(1, dtype=torch.float32, device="cuda")
+    tp = (ctypes.c_void_p * 3)(*[t.data_ptr() for t in taps])
+    cu = np.array([0, 40], np.int32)
+    for flags in (4, OT.ALL_TOKENS | OT.KEEP_ROWS | 8):  # unknown flag bits
+        st = pred.lib.outlets_predict_prefill(pred.h, tp, cu.ctypes.data, 1, 40, None, None, flags, z.data_ptr(),
+                                              None, None)
+        assert st == OT.EINVAL
     pred.check()
     kv.close()
 

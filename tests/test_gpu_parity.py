@@ -496,3 +496,45 @@ def test_nonunit_norm_gains(name, gated, embed):
     check_z_len(z2, ln2, ref2["z"], ref2["length"], shape.dtype, f"gains {name} step")
     kv.close()
     pred.close()
+
+
+_L2_KEEP_SCRIPT = r"""
+import sys, numpy as np, torch
+sys.path.insert(0, sys.argv[1]); sys.path.insert(0, sys.argv[1] + "/tests")
+from paper_2609_01068_gb300 import outlets, synth
+from _util import to_device
+shape = synth.ModelShape("mid-bf16-hd128", 1024, 8, 2, 128, 2816, (256,), 500000.0, 1e-5, "bf16")
+w = synth.make_weights(shape, 0)
+pred = outlets.Predictor(shape, w, max_tokens=2048, max_batch=8, max_position=4096)
+lengths = [70, 300, 5, 129]
+cu = synth.cu_seqlens(lengths)
+kv = outlets.KVCache(pred, max_slots=4, max_tokens_total=1024)
+taps = [to_device(t, "bf16") for t in synth.make_taps(shape, int(cu[-1]), 0, 95)]
+z0, _ = pred.prefill(taps, cu, kv=kv, slots=[0, 1, 2, 3])
+st = [to_device(t, "bf16") for t in synth.make_taps(shape, 4, 0, 96)]
+z1, _ = pred.step(st, kv, [0, 1, 2, 3])
+torch.cuda.synchronize()
+pred.check()
+np.save(sys.argv[2], np.concatenate([z0.cpu().numpy(), z1.cpu().numpy()]))
+"""
+
+
+def test_slice_discard_changes_no_value(tmp_path):
+    """Dropping the split-K slices from L2 after their last read
+    (OUTLETS_L2_DISCARD, default on) changes no output bit: the same static
+    prediction and step in two processes, with the discards and without."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    script = tmp_path / "run.py"
+    script.write_text(_L2_KEEP_SCRIPT)
+    out = {}
+    for v in ("1", "0"):
+        env = dict(os.environ, OUTLETS_L2_DISCARD=v)
+        f = tmp_path / f"z{v}.npy"
+        r = subprocess.run([sys.executable, str(script), root, str(f)], env=env, capture_output=True, text=True,
+                           timeout=600)
+        assert r.returncode == 0, r.stderr[-2000:]
+        out[v] = np.load(f)
+    np.testing.assert_array_equal(out["1"], out["0"])

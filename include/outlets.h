@@ -56,7 +56,7 @@ typedef enum outlets_status {
   OUTLETS_EINVAL = 1,        /* invalid argument; nothing was launched or changed */
   OUTLETS_ENOMEM = 2,        /* device or pinned-host allocation failed */
   OUTLETS_ECUDA = 3,         /* a CUDA runtime/driver call failed */
-  OUTLETS_EUNSUPPORTED = 4,  /* shape this build does not implement */
+  OUTLETS_EUNSUPPORTED = 4,  /* shape or feature the library does not implement */
   OUTLETS_ECAPACITY = 5,     /* KV cache or workspace too small; nothing changed */
   OUTLETS_ETIMEOUT = 6,      /* a kernel's bounded wait ran out (from outlets_check) */
   OUTLETS_EDEVICE = 7        /* a kernel refused an index (from outlets_check) */

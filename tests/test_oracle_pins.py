@@ -312,6 +312,30 @@ def test_prefill_equals_prefix_then_steps():
         caches = st["caches"]
 
 
+def test_static_prediction_reads_only_the_last_rows_past_the_keys_and_values():
+    """The evaluation order of the library's static prediction: keys and
+    values of every prompt row, then queries, attention, O, the MLP, the final
+    norm and the head for each prompt's last row only.  In the oracle that is
+    a step of the last row over the K/V cache of the rows before it; it gives
+    the whole-layer prediction (the prompt of length 1 has an empty cache)."""
+    w = _weights()
+    lengths = [6, 4, 1, 9]
+    full, taps, cu = _prefill(w, SMALL, lengths)
+    kpre = [L - 1 for L in lengths]
+    caches = []
+    for b, L in enumerate(lengths):
+        if L > 1:
+            sub = [t[cu[b]:cu[b] + L - 1] for t in taps]
+            caches += O.caches_from_prefill(O.predict_prefill(w, SMALL, sub, np.array([0, L - 1])), [0, L - 1])
+        else:
+            kh = np.zeros((0, SMALL.n_kv_heads, SMALL.head_dim))
+            caches.append((kh, kh.copy()))
+    last = [cu[b] + kpre[b] for b in range(len(lengths))]
+    st = O.predict_step(w, SMALL, [t[last] for t in taps], caches)
+    np.testing.assert_allclose(st["z"], full["z"], rtol=1e-11, atol=1e-11)
+    np.testing.assert_allclose(st["h_draft"], full["h_draft"], rtol=1e-11, atol=1e-11)
+
+
 def test_sampled_rows_equal_full_batch():
     w = _weights()
     lengths = [5, 2, 7, 1]

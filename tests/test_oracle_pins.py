@@ -35,6 +35,7 @@ def _taps(shape, T, seed=0, off=0):
 
 # ---------------------------------------------------------------- golden facts
 def test_tap_layer_indices_match_paper():
+    """Pins the input generator's tap selection (which target layers feed Eq. 1), not the oracle."""
     for c in _facts()["tap_layers"]["cases"]:
         assert list(synth.tap_layer_indices(c["n_layers"])) == c["layers"]
 
@@ -66,11 +67,6 @@ def test_head_parameter_count_consistent_with_paper():
     n_bad, _ = count(fact["widths_inconsistent"])
     assert abs(n_ok - fact["approx_params"]) / fact["approx_params"] < fact["rel_tol"]
     assert abs(n_bad - fact["approx_params"]) / fact["approx_params"] > fact["rel_tol"]
-
-
-def test_remaining_length_definition():
-    for c in _facts()["static_vs_dynamic"]["cases"]:
-        assert c["L"] - c["t"] == c["r"]
 
 
 # ---------------------------------------------------------------- head
@@ -256,6 +252,123 @@ def test_silu_against_library_sigmoid():
     x = np.linspace(-30, 30, 121)
     np.testing.assert_allclose(O.silu(x), x * scipy_special.expit(x), rtol=1e-13, atol=1e-300)
     assert O.silu(np.array([0.0]))[0] == 0.0
+
+
+def test_swiglu_mlp_brute_force():
+    """down(silu(x W_gate^T) * (x W_up^T)) (Sec. 4.1, the layer's MLP block read
+    as SwiGLU) in scalar loops; distinct gate and up weights, so a swap fails."""
+    rng = np.random.default_rng(31)
+    d, F = 5, 4
+    x = rng.standard_normal((3, d))
+    wg, wu, wd = rng.standard_normal((F, d)), rng.standard_normal((F, d)), rng.standard_normal((d, F))
+    got = O.swiglu_mlp(x, wg, wu, wd)
+    for r in range(3):
+        hid = []
+        for n in range(F):
+            g = sum(x[r, c] * wg[n, c] for c in range(d))
+            u = sum(x[r, c] * wu[n, c] for c in range(d))
+            hid.append(g / (1.0 + math.exp(-g)) * u)
+        for i in range(d):
+            assert got[r, i] == pytest.approx(sum(hid[n] * wd[i, n] for n in range(F)), rel=1e-12, abs=1e-12)
+    # the two inner projections are not interchangeable
+    assert np.max(np.abs(O.swiglu_mlp(x, wu, wg, wd) - got)) > 1e-3
+
+
+def _scalar_layer(w, shape, taps, lengths):
+    """One whole draft decoder layer and the length head in scalar Python loops,
+    written from the definitions (Eq. 1; Sec. 4.1 pre-norm layer: RMSNorm,
+    RoPE causal GQA attention, residual, RMSNorm, SwiGLU MLP, residual; final
+    RMSNorm and MLP_len of Sec. 4.2 at each sequence's last row)."""
+    d, H, KVH, hd, F = shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
+    eps, theta = shape.rms_eps, shape.rope_theta
+    T = sum(lengths)
+
+    def rms(vec, gain):
+        ms = sum(v * v for v in vec) / len(vec)
+        return [v / math.sqrt(ms + eps) * gn for v, gn in zip(vec, gain)]
+
+    def matvec(W, vec):
+        return [sum(W[o][c] * vec[c] for c in range(len(vec))) for o in range(len(W))]
+
+    start, pos = [], []
+    for b, L in enumerate(lengths):
+        for p in range(L):
+            start.append(sum(lengths[:b]))
+            pos.append(p)
+    f = []
+    for t in range(T):
+        f.append([sum(w["w_proj"][i][j * d + c] * taps[j][t][c] for j in range(3) for c in range(d))
+                  for i in range(d)])
+    x = [rms(f[t], w["g_in"]) for t in range(T)]
+
+    def rope(vec, p):
+        out = list(vec)
+        half = hd // 2
+        for i in range(half):
+            ang = p * theta ** (-2.0 * i / hd)
+            out[i] = vec[i] * math.cos(ang) - vec[i + half] * math.sin(ang)
+            out[i + half] = vec[i + half] * math.cos(ang) + vec[i] * math.sin(ang)
+        return out
+
+    q = [[rope(matvec(w["w_q"], x[t])[h * hd:(h + 1) * hd], pos[t]) for h in range(H)] for t in range(T)]
+    k = [[rope(matvec(w["w_k"], x[t])[g * hd:(g + 1) * hd], pos[t]) for g in range(KVH)] for t in range(T)]
+    v = [[matvec(w["w_v"], x[t])[g * hd:(g + 1) * hd] for g in range(KVH)] for t in range(T)]
+    a, y = [], []
+    for t in range(T):
+        o = []
+        for h in range(H):
+            g = h * KVH // H
+            keys = range(start[t], t + 1)
+            s = [sum(q[t][h][e] * k[j][g][e] for e in range(hd)) / math.sqrt(hd) for j in keys]
+            m = max(s)
+            p = [math.exp(si - m) for si in s]
+            z = sum(p)
+            o += [sum(p[n] * v[j][g][e] for n, j in enumerate(keys)) / z for e in range(hd)]
+        at = [f[t][i] + sum(w["w_o"][i][c] * o[c] for c in range(H * hd)) for i in range(d)]
+        ah = rms(at, w["g_post"])
+        gate, up = matvec(w["w_gate"], ah), matvec(w["w_up"], ah)
+        hid = [gate[n] / (1.0 + math.exp(-gate[n])) * up[n] for n in range(F)]
+        a.append(at)
+        y.append([at[i] + sum(w["w_down"][i][n] * hid[n] for n in range(F)) for i in range(d)])
+    last = [sum(lengths[:b + 1]) - 1 for b in range(len(lengths))]
+    hdraft = [rms(y[t], w["g_final"]) for t in last]
+    zs = []
+    for hrow in hdraft:
+        cur = hrow
+        n = len(shape.head_widths) + 1
+        for i in range(n):
+            nxt = [sum(w[f"head_w{i}"][o][c] * cur[c] for c in range(len(cur))) + w[f"head_b{i}"][o]
+                   for o in range(len(w[f"head_w{i}"]))]
+            cur = [max(0.0, u) for u in nxt] if i < n - 1 else nxt
+        zs.append(cur[0])
+    return dict(a=np.array(a), y=np.array(y), h_draft=np.array(hdraft), z=np.array(zs))
+
+
+def test_whole_layer_scalar_brute_force():
+    """The oracle's prefill against the scalar layer above on a tiny shape, with
+    distinct random gate and up weights and distinct non-unit gains g_in,
+    g_post and g_final, so a swapped projection, a norm of the wrong tensor or
+    a gain used in the wrong place changes a, y, h_draft or z."""
+    shape = synth.ModelShape("pin-layer", 8, 2, 1, 4, 6, (5,), 10000.0, 1e-5, "f32")
+    rng = np.random.default_rng(41)
+    w = {k: v.astype(np.float64) for k, v in synth.make_weights(shape, 3, std=0.4).items()}
+    w["w_up"] = rng.standard_normal(w["w_up"].shape) * 0.5
+    w["g_in"] = 1.0 + 0.5 * rng.standard_normal(shape.d)
+    w["g_post"] = 1.0 + 0.5 * rng.standard_normal(shape.d)
+    w["g_final"] = 1.0 + 0.5 * rng.standard_normal(shape.d)
+    w["head_b1"] = np.array([0.3])
+    lengths = [3, 2]
+    taps = [rng.standard_normal((sum(lengths), shape.d)) for _ in range(3)]
+    ref = _scalar_layer({k: np.asarray(v).tolist() for k, v in w.items()}, shape,
+                        [t.tolist() for t in taps], lengths)
+    out = O.predict_prefill(w, shape, taps, synth.cu_seqlens(lengths))
+    for key in ("a", "y"):
+        np.testing.assert_allclose(out[key], ref[key], rtol=1e-12, atol=1e-12, err_msg=key)
+    np.testing.assert_allclose(out["h_draft"], ref["h_draft"], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(out["z"], ref["z"], rtol=1e-12, atol=1e-12)
+    # the test is sensitive: the MLP and the attention both move y at this scale
+    assert np.max(np.abs(ref["y"] - ref["a"])) > 1e-2
+    assert np.max(np.abs(ref["a"] - out["f"])) > 1e-2
 
 
 # ---------------------------------------------------------------- whole forward

@@ -1,16 +1,22 @@
 #!/usr/bin/env python
 """Benchmark of OUTLETS length prediction on GB300.
 
-Workload (the headline): static prediction (Sec. 3.2) with a Llama-3.1-8B-shaped
-EAGLE-3 draft backbone (d=4096, 32/8 heads, hd 128, SwiGLU 14336, head
-4096->1024->1), bf16, over 64 ragged prompts (lognormal median 256, clipped to
-[16, 2048], packed varlen).  One step = one outlets_predict_prefill call: tap
-fusion, the draft decoder layer over every token, and the length head.
+Headline (the default line): static prediction (Sec. 3.2) with a
+Llama-3.3-70B-shaped EAGLE-3 draft backbone (d=8192, 64/8 heads, hd 128,
+SwiGLU 28672, head 8192->1024->1), bf16, over 32 ragged prompts (lognormal
+median 1024, clipped to [64, 4096], packed varlen): the largest single-GPU
+configuration.  One step = one outlets_predict_prefill call: tap fusion
+(Eq. 1), the keys and values of every prompt row, and the rest of the draft
+layer, the final norm and the length head for each prompt's last row (the
+outputs the static prediction reads; the same prediction with the whole layer
+on every row is reported beside it as "whole_layer").
 
-Also reported: dynamic prediction (one outlets_predict_step over 256 live
-requests with lognormal cache lengths, median 512, <= 4096), the CPU oracle on
-a bounded sample, and the end-to-end number through the C ABI with host
-buffers.  `--impl reference` times the CPU oracle alone (the reference arm).
+Sub-records of the same line: the Llama-3.1-8B-shaped static prediction
+(64 prompts, lognormal median 256, clipped to [16, 2048]), dynamic prediction
+(one outlets_predict_step over 256 live requests with lognormal cache lengths,
+median 512, <= 4096) and the saturated-serving sweep.  Also reported: the CPU
+oracle on a bounded sample, and the end-to-end number through the C ABI with
+host buffers.  `--impl reference` times the CPU oracle alone (the reference arm).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 Under torchrun each rank runs an independent replica (weak scaling).
@@ -62,9 +68,10 @@ def parse():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--mode", default="both", choices=["both", "prefill", "step", "sweep", "sched"],
-                    help="static prediction (headline), dynamic prediction, both, the serving sweep, or the "
-                         "length-aware scheduling model (host code, Sec. 5.5)")
+    ap.add_argument("--mode", default="all", choices=["all", "both", "prefill", "step", "sweep", "sched"],
+                    help="all (default): the 70B static prediction as the headline with the 8B static, step and "
+                         "sweep records beside it; or one of: static prediction of --model, dynamic prediction, "
+                         "both (8B), the serving sweep, the length-aware scheduling model (host code, Sec. 5.3)")
     ap.add_argument("--prompts", type=int, default=None,
                     help="first N prompts of the workload (profiling cases; default: all)")
     ap.add_argument("--gated", action="store_true",
@@ -80,12 +87,17 @@ def parse():
                          "keys/values are projected for every row and the rest runs on each prompt's last row)")
     ap.add_argument("--no-whole-layer", action="store_true",
                     help="skip the extra whole-layer timing that the default static-prediction line carries")
-    ap.add_argument("--model", default="8b", choices=["8b", "70b"],
-                    help="draft-layer shape; 70b (Llama-3.3-70B-shaped, 32 prompts) runs the static mode only")
+    ap.add_argument("--model", default=None, choices=["8b", "70b"],
+                    help="draft-layer shape of --mode prefill (default 8b) and of the reference arm (default 70b, "
+                         "the headline's); 70b (Llama-3.3-70B-shaped, 32 prompts) runs the static mode only")
     ap.add_argument("--step-requests", type=int, default=256, help="live requests of the dynamic-prediction run")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    return ap.parse_args()
+    ap.add_argument("--no-sweep", action="store_true", help="--mode all: leave out the serving-sweep record")
+    a = ap.parse_args()
+    if a.model is None:
+        a.model = "70b" if (a.impl == "reference" or a.mode == "all") else "8b"
+    return a
 
 
 TRAFFIC_SOURCES = {  # files whose content decides the kernel's DRAM traffic (incl. the tile raster)
@@ -117,6 +129,16 @@ def measured_traffic(kernel, workload):
     if not e or e.get("workload") != workload or e.get("sources_sha256") != sources_sha(kernel):
         return None
     return e["dram_bytes_per_launch"]
+
+
+def tensor_peak(peaks, region_ms, clocks):
+    """The bf16 denominator for a contraction timed over region_ms: the burst
+    figure for a region under a second without a power cap, else the sustained
+    one (measured over a seconds-long loop under the power cap)."""
+    capped = "sw_power_cap" in ((clocks or {}).get("reasons") or [])
+    if region_ms < 1000.0 and not capped:
+        return peaks["bf16"], f"bf16 burst {peaks['src']}"
+    return peaks["bf16_sus"], f"bf16 sustained {peaks['src']}"
 
 
 def load_peaks():
@@ -266,33 +288,49 @@ class ReplicaGroup:
 
 
 def run_reference(args):
+    """The reference arm: the CPU oracle (the plain definition of the forward,
+    fp64 numpy) on the host cores, on the workload of the default line (the
+    70B-shaped static prediction unless --model says otherwise).  Each step is
+    one whole prompt, taken in turn from the four shortest of the workload, so
+    that the whole run ends within a few minutes."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
+    from oracle import outlets_oracle as OR
     from paper_2609_01068_gb300 import synth
     shape, lengths, workload, _ = model_setup(args)
     w = synth.make_weights(shape, 0, gated=args.gated, embed_vocab=synth.LLAMA3_VOCAB if args.embed else 0)
     if args.dual:
         w["w_lm"] = synth.make_lm_head(shape, synth.LLAMA3_VOCAB, 0)
+    w = f64_weights(w)
     cu = synth.cu_seqlens(lengths)
     taps = synth.make_taps(shape, int(cu[-1]), 0)
     tok = synth.make_tokens(int(cu[-1]), synth.LLAMA3_VOCAB, 0, 0) if args.embed else None
-    budget = 400
     dk = args.dual or None
-    for _ in range(args.warmup):
-        oracle_sample(shape, w, taps, cu, lengths, budget, dk, tok)
-    n_pred, n_tok, secs = 0, 0, 0.0
-    for _ in range(args.steps):
-        p, t, dt = oracle_sample(shape, w, taps, cu, lengths, budget, dk, tok)
-        n_pred, n_tok, secs = n_pred + p, n_tok + t, secs + dt
-    value = n_pred / secs
+    pool = [int(b) for b in np.argsort(lengths, kind="stable")[:4]]
+
+    def one(i):
+        b = pool[i % len(pool)]
+        t0 = time.perf_counter()
+        OR.sample_prefill_rows(w, shape, taps, cu, [b], draft_k=dk, tokens=tok)
+        return int(lengths[b]), time.perf_counter() - t0
+
+    for i in range(args.warmup):
+        one(i)
+    n_tok, secs = 0, 0.0
+    for i in range(args.steps):
+        t, dt = one(i)
+        n_tok, secs = n_tok + t, secs + dt
+    value = args.steps / secs
+    sample = (f"one whole prompt per step, in turn from the 4 shortest of the workload "
+              f"({', '.join(str(int(lengths[b])) for b in pool)} tokens); weights held in f64 before timing")
     out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "predictions/s", "n_gpus": args.gpus,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * secs / args.steps,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "draft_tokens_per_s": n_tok / secs,
-           "config": {"workload": workload, "sample": f"~{budget} prompt tokens per step (whole prompts)"},
+           "config": {"workload": workload, "sample": sample},
            "cpu_baseline": {"value": value, "unit": "predictions/s", "cores": cpu_threads(), "kind": "oracle",
-                            "sample": f"{n_pred} prompts / {n_tok} tokens over {args.steps} steps"},
+                            "sample": f"{args.steps} prompts / {n_tok} tokens over {args.steps} steps; {sample}"},
            "e2e": {"value": value, "unit": "predictions/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
 
@@ -304,7 +342,7 @@ SCHED_TRACE = dict(n=6000, qps=13.0)
 
 def serving_metrics(arrival, output, finish):
     """Throughput (output tokens / makespan), mean latency, P99 latency (nearest rank) of
-    short (< 800), medium and long (>= 1300 tokens) requests: the categories of Sec. 5.5."""
+    short (< 800), medium and long (>= 1300 tokens) requests: the categories of Sec. 5.3 and its appendix "System-Level Evaluation Details"."""
     lat = finish - arrival
     out = {"throughput_tok_s": float(output.sum() / (finish.max() - arrival.min())),
            "mean_latency_s": float(lat.mean())}
@@ -370,25 +408,11 @@ def run_sched(args):
     print(json.dumps(out))
 
 
-def run_ours(args):
+def setup_static(args, local, rank, max_batch=0):
+    """Weights, taps and a predictor for the static prediction of args.model."""
     import torch
-    import torch.distributed as dist
 
-    from paper_2609_01068_gb300 import build as B
     from paper_2609_01068_gb300 import outlets, synth
-
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    if world > 1:
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    B.build()
-    peaks = load_peaks()
-    if args.model == "70b" and args.mode != "prefill":
-        raise SystemExit("--model 70b runs the static (prefill) mode only")
-    if args.embed and args.mode == "sweep":
-        raise SystemExit("--embed runs the static and dynamic modes (the sweep uses the plain layer input)")
     shape, lengths, workload, tkey = model_setup(args)
     args.workload, args.traffic_key = workload, tkey
     w = synth.make_weights(shape, 0, gated=args.gated, embed_vocab=synth.LLAMA3_VOCAB if args.embed else 0)
@@ -398,46 +422,92 @@ def run_ours(args):
     T, Bq = int(cu[-1]), len(lengths)
     taps = synth.make_taps(shape, T, 0, rank)
     args.tokens = synth.make_tokens(T, synth.LLAMA3_VOCAB, 0, rank) if args.embed else None
-
-    def dev(a):
-        return torch.from_numpy(synth.bf16_bits(a).view(np.int16)).view(torch.bfloat16).cuda()
-
-    taps_d = [dev(t) for t in taps]
-    step_B = args.step_requests
+    taps_d = [torch.from_numpy(synth.bf16_bits(t).view(np.int16)).view(torch.bfloat16).cuda() for t in taps]
     max_tokens = max(8192, (T + 1023) // 1024 * 1024)
-    pred = outlets.Predictor(shape, w, max_tokens=max_tokens, max_batch=max(step_B, Bq), max_position=8192,
+    pred = outlets.Predictor(shape, w, max_tokens=max_tokens, max_batch=max(max_batch, Bq), max_position=8192,
                              device=local)
-    stream = torch.cuda.current_stream()
+    return shape, lengths, cu, w, taps, taps_d, pred, max_tokens
 
+
+def run_ours(args):
+    import copy
+
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_01068_gb300 import build as B
+    from paper_2609_01068_gb300 import synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    B.build()
+    peaks = load_peaks()
+    if args.model == "70b" and args.mode not in ("prefill", "all"):
+        raise SystemExit("--model 70b runs the static (prefill) mode only")
+    if args.embed and args.mode == "sweep":
+        raise SystemExit("--embed runs the static and dynamic modes (the sweep uses the plain layer input)")
+    stream = torch.cuda.current_stream()
     group = ReplicaGroup(world, rank, "cuda", sync=torch.cuda.synchronize)
     barrier, max_over_ranks = group.barrier, group.max
 
     out = {"metric": METRIC, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic"}
-    if args.mode in ("both", "prefill"):
-        out.update(run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, world, rank, local,
-                                    barrier, max_over_ranks, stream))
-    if args.mode in ("both", "step"):
-        sm = run_step_mode(args, pred, shape, peaks, step_B, world, barrier, max_over_ranks, stream, max_tokens)
-        if args.mode == "step":
-            out.update({k: sm[k] for k in ("value", "unit", "ms_per_step", "e2e", "gpu_launches", "clocks",
-                                           "roofline")})
-            out["config"] = {"workload": sm["workload"], "parallelism": f"replicas x{world}"}
-        out["step_mode"] = sm
     if args.mode == "sweep":
-        pred.close()
+        a8 = copy.copy(args)
+        a8.model = "8b"
+        shape, _, _, _ = model_setup(a8)
+        w = synth.make_weights(shape, 0, gated=args.gated)
         sw = run_sweep(args, shape, w, world, local, barrier, max_over_ranks, stream)
         best = max(sw["points"], key=lambda x: x["predictions_per_s"])
         out.update({"value": best["predictions_per_s"], "unit": "predictions/s", "ms_per_step": best["ms_total"],
                     "config": {"workload": sw["workload"], "parallelism": f"replicas x{world}"}, "sweep": sw})
-        if rank == 0:
-            print(json.dumps(out))
-        if world > 1:
-            dist.destroy_process_group()
-        return
+    else:
+        if args.mode == "all":
+            # headline: the largest single-GPU configuration (70B-shaped static prediction)
+            a70 = copy.copy(args)
+            a70.model = "70b"
+            shape, lengths, cu, w, taps, taps_d, pred, _ = setup_static(a70, local, rank)
+            out.update(run_prefill_mode(a70, pred, shape, w, taps, taps_d, lengths, cu, peaks, world, rank, local,
+                                        barrier, max_over_ranks, stream))
+            pred.close()
+            del taps_d, taps, w
+            torch.cuda.empty_cache()
+            args.model = "8b"
+        if args.mode in ("all", "both", "prefill", "step"):
+            a = copy.copy(args)
+            if args.mode == "all":
+                a.no_cpu_baseline = True  # the headline's oracle sample is the one reported
+            shape, lengths, cu, w, taps, taps_d, pred, max_tokens = setup_static(a, local, rank, args.step_requests)
+            if args.mode in ("all", "both", "prefill"):
+                r = run_prefill_mode(a, pred, shape, w, taps, taps_d, lengths, cu, peaks, world, rank, local, barrier,
+                                     max_over_ranks, stream)
+                if args.mode == "all":
+                    out["llama8b_static"] = r
+                else:
+                    out.update(r)
+            if args.mode in ("all", "both", "step"):
+                sm = run_step_mode(args, pred, shape, peaks, args.step_requests, world, barrier, max_over_ranks,
+                                   stream, max_tokens)
+                if args.mode == "step":
+                    out.update({k: sm[k] for k in ("value", "unit", "ms_per_step", "e2e", "gpu_launches", "clocks",
+                                                   "roofline")})
+                    out["config"] = {"workload": sm["workload"], "parallelism": f"replicas x{world}"}
+                out["step_mode"] = sm
+            pred.close()
+            if args.mode == "all" and not args.no_sweep:
+                del taps_d
+                torch.cuda.empty_cache()
+                sw = run_sweep(args, shape, w, world, local, barrier, max_over_ranks, stream)
+                out["sweep"] = {"workload": sw["workload"],
+                                "points": [{k: p[k] for k in ("batch_tokens_cap", "ms_total", "predictions_per_s",
+                                                              "tokens_per_s", "prefill_ms", "step_ms")}
+                                           for p in sw["points"]]}
     if rank == 0:
         print(json.dumps(out))
-    pred.close()
     if world > 1:
         dist.destroy_process_group()
 
@@ -496,8 +566,11 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
             k_flops = 2.0 * T * (2 * shape.ffn) * shape.d
             name, alg = "gateup_swiglu_gemm (k_gemm_tc<256, SWIGLU>)", f"2*T*(2F)*d, T={T}"
         k_tflops = k_flops / (k_ms / k_n / 1e3) / 1e12
-        roof = {"bound": "tensor", "kernel": name, "achieved": k_tflops, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
-                "frac": k_tflops / peaks["bf16_sus"], "peak_kind": f"bf16 sustained {peaks['src']}",
+        peak, kind = tensor_peak(peaks, ms, clocks)
+        roof = {"bound": "tensor", "kernel": name, "achieved": k_tflops, "peak": peak, "unit": "TFLOP/s",
+                "frac": k_tflops / peak, "peak_kind": kind,
+                "frac_of_burst": k_tflops / peaks["bf16"], "frac_of_sustained": k_tflops / peaks["bf16_sus"],
+                "kernel_ms_per_launch": k_ms / k_n,
                 "traffic": measured_traffic(kern, f"{args.traffic_key}-static-{Bq}p-T{T}"),
                 "algorithmic_per_launch": f"{k_flops:.4g} FLOP = {alg}"}
         flops = (prefill_flops(shape, lengths, Bq, args.gated, args.embed, whole_layer=keep or not pruned_rows)
@@ -508,9 +581,10 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     whole = None
     if pruned_rows and not args.no_whole_layer:
         w_ms, _, w_clocks, w_roof, w_flops = timed(True)
+        w_tf = w_flops * args.steps / (w_ms / 1e3) / 1e12
         whole = {"ms_per_step": w_ms / args.steps, "value": world * Bq * args.steps / (w_ms / 1e3),
-                 "tensor_peak_frac_step": w_flops * args.steps / (w_ms / 1e3) / 1e12 / peaks["bf16_sus"],
-                 "roofline": w_roof, "clocks": w_clocks,
+                 "tflops_per_s": w_tf, "tensor_peak_frac_step": w_tf / w_roof["peak"],
+                 "peak_kind": w_roof["peak_kind"], "roofline": w_roof, "clocks": w_clocks,
                  "note": "the same prediction with the whole layer run on every prompt row (OUTLETS_KEEP_ROWS)"}
     # per-stage breakdown in a separate (untimed) pass: stage events serialize the kernels
     pred.profile(True)
@@ -540,10 +614,17 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
             run(host_taps, zh, lh, dh, tok_host)
             stream.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - t0)
+        h2d = int(sum(t.numel() * t.element_size() for t in host_taps)) + (int(tok_host.nbytes) if tok_host is not None
+                                                                            else 0)
+        ceil_gbs = h2d_ceiling(host_taps, taps_d, stream)
+        bound = Bq / max(ms_step / 1e3, h2d / (ceil_gbs * 1e9))  # copies fully overlapped with compute
         e2e = {"value": world * Bq * args.steps / e2e_s, "unit": "predictions/s",
-               "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_taps))
-               + (int(tok_host.nbytes) if tok_host is not None else 0),
-               "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4 + buffer_bytes(dh))}
+               "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": int(zh.numel() * 4 + lh.numel() * 4 + buffer_bytes(dh)),
+               "h2d_ceiling_gbs": ceil_gbs, "overlap_bound": world * bound,
+               "frac_of_overlap_bound": (Bq * args.steps / e2e_s) / bound,
+               "note": "h2d_ceiling_gbs: one cudaMemcpyAsync per pinned tap buffer, CUDA events; overlap_bound: "
+                       "predictions/s if the tap copies fully overlapped the device pass"}
 
     out = {"value": value, "unit": "predictions/s", "ms_per_step": ms_step,
            "config": {"workload": args.workload, "prompts_per_gpu": Bq, "tokens_per_gpu": T,
@@ -552,7 +633,7 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
                       "parallelism": f"replicas x{world}"},
            "draft_tokens_per_s": world * T * args.steps / (ms / 1e3),
            "tflops_per_s": flops * args.steps / (ms / 1e3) / 1e12,
-           "tensor_peak_frac_step": flops * args.steps / (ms / 1e3) / 1e12 / peaks["bf16_sus"],
+           "tensor_peak_frac_step": flops * args.steps / (ms / 1e3) / 1e12 / roofline["peak"],
            "roofline": roofline, "stages": stages, "clocks": clocks, "e2e": e2e,
            "gpu_launches": launches}
     out["config"]["layer_rows"] = ("keys/values for every prompt row; queries, attention, O, MLP, final norm and "
@@ -560,12 +641,43 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
     if whole:
         out["whole_layer"] = whole
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        # ~10 s of oracle work on the machine's host cores (~1.3 ms per prompt token there)
-        n_pred, n_tok, secs = oracle_sample(shape, w, taps, cu, lengths, 8000, args.dual or None, args.tokens)
+        # ~10 s of oracle work on the machine's host cores: whole prompts nearest the
+        # median length (8B: ~1.3 ms per prompt token there; 70B: one prompt)
+        budget = 8000 if shape.d <= 4096 else 1200
+        w64 = f64_weights(w)
+        n_pred, n_tok, secs = oracle_sample(shape, w64, taps, cu, lengths, budget, args.dual or None, args.tokens)
+        del w64
         out["cpu_baseline"] = {"value": n_pred / secs, "unit": "predictions/s", "cores": cpu_threads(),
                                "kind": "oracle",
-                               "sample": f"{n_pred} whole prompts ({n_tok} tokens) of the same workload, {secs:.1f} s"}
+                               "sample": f"{n_pred} whole prompt(s) ({n_tok} tokens) of the same workload, nearest "
+                                         f"the median length, {secs:.1f} s (weights held in f64 before timing)"}
     return out
+
+
+def f64_weights(w):
+    """The weights in the oracle's precision (float64), converted once before timing."""
+    return {k: (np.asarray(v, dtype=np.float64) if isinstance(v, np.ndarray) and v.dtype != np.int32 else v)
+            for k, v in w.items()}
+
+
+def h2d_ceiling(host, dev, stream):
+    """Host-to-device copy rate of the pinned tap buffers: one cudaMemcpyAsync
+    per buffer (the same bytes the device already holds), timed with CUDA events."""
+    import torch
+    nbytes = sum(t.numel() * t.element_size() for t in host)
+    for h, d in zip(host, dev):  # warm-up
+        d.copy_(h, non_blocking=True)
+    best = None
+    for _ in range(3):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for h, d in zip(host, dev):
+            d.copy_(h, non_blocking=True)
+        e1.record(stream)
+        e1.synchronize()
+        t = e0.elapsed_time(e1)
+        best = t if best is None else min(best, t)
+    return nbytes / (best / 1e3) / 1e9
 
 
 def run_step_mode(args, pred, shape, peaks, B, world, barrier, max_over_ranks, stream, max_tokens):

@@ -368,14 +368,16 @@ uint64_t outlets_launch_count(const outlets_ctx* ctx);
  *            final-normed draft states (OUTLETS_T_HDRAFT of a prediction call).
  *   z_out, len_out  device f32 [rows]: z_hat and max(0, expm1(z_hat));
  *            len_out may be NULL.
- * Same arithmetic as the head stage of the prediction calls.  The hidden
- * activations live in a 16 MiB array inside the library image (held by every
- * GPU that loads the library until the process exits) instead of allocated
- * memory; rows x (widest hidden layer) x (2 if the head has more than one
- * hidden layer) must fit in 4 Mi floats, else OUTLETS_ECAPACITY with a message
- * in outlets_last_error.  The first call on a device looks up the array's
- * device address; make that first call before any stream capture.  All calls
- * on a device share the array: calls that overlap on the GPU race.  Allocates
+ * The same length head as the prediction calls, agreeing with their z_hat
+ * within the bf16 / f32 tolerances (the prediction calls may split the first
+ * layer's sum over K for small batches, so the rounding order can differ).
+ * The hidden activations live in a 16 MiB array inside the library image
+ * instead of allocated memory; the array is reserved on a device when
+ * outlets_create makes a context there (it looks up the array's address) and
+ * stays until the process exits.  rows x (widest hidden layer) x (2 if the
+ * head has more than one hidden layer) must fit in 4 Mi floats, else
+ * OUTLETS_ECAPACITY with a message in outlets_last_error.  All calls on a
+ * device share the array: calls that overlap on the GPU race.  Allocates
  * nothing (no cudaMalloc, cudaFree or allocating library routine). */
 outlets_status outlets_length_head_noalloc(outlets_ctx* ctx, const void* h_draft, int32_t rows, float* z_out,
                                            float* len_out, void* stream);

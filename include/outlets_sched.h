@@ -1,6 +1,6 @@
 /*
- * Serving-side use of the static length prediction (Sec. 5.5 and its appendix
- * on the system evaluation): a discrete-event model of a disaggregated
+ * Serving-side use of the static length prediction (Sec. 5.3 and the appendix
+ * "System-Level Evaluation Details"): a discrete-event model of a disaggregated
  * deployment (one prefill instance, n decode instances) in which the static
  * prediction r_hat_0 of every request steers
  *   instance routing   RR (fixed cyclic order) or LB (the decode instance with

@@ -3,7 +3,7 @@
 Only the tests and bench.py's reference leg may import this module; the
 library never calls it and shares no code with it.
 
-Sec. 5.5 (and its appendix on the system evaluation) compares, on a
+Sec. 5.3 (and the appendix "System-Level Evaluation Details") compares, on a
 disaggregated deployment with one prefill and three decode instances, two
 decisions taken with the static prediction r_hat_0 as a proxy for decode cost:
 
@@ -140,7 +140,7 @@ def simulate(cfg, arrival, prompt, output, predicted):
 
 
 def summarize(arrival, output, finish, short_below=800, long_from=1300):
-    """Serving metrics of Sec. 5.5: throughput (output tokens / makespan), mean
+    """Serving metrics of Sec. 5.3 and its appendix: throughput (output tokens / makespan), mean
     latency, and P99 latency of short / medium / long requests by true length
     (nearest-rank percentile)."""
     lat = [f - a for f, a in zip(finish, arrival)]

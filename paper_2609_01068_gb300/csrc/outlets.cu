@@ -554,7 +554,9 @@ outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k
                        const float* residual, long long ldr, const float* bias, cudaStream_t s,
                        NormFold* nf = nullptr) {
   int bn = 256;
-  if (epi != EPI_SWIGLU) {
+  if (epi == EPI_BIAS_RELU) {
+    bn = 64;  // the head's first layer (N <= a few thousand): the only width built for this epilogue
+  } else if (epi != EPI_SWIGLU) {
     auto tiles = [&](int bnv) { return cdiv(M, 128) * cdiv(N, bnv); };
     if (tiles(256) >= c->num_sms) bn = 256;
     else if (tiles(128) >= c->num_sms) bn = 128;
@@ -1097,6 +1099,13 @@ outlets_status end_call(outlets_ctx* c, int out_rows, float* z_out, float* len_o
   return OUTLETS_OK;
 }
 
+// Device address of outlets_length_head_noalloc's static scratch array
+// (defined with that entry point at the end of this file).
+cudaError_t head_scratch_ptr(int device, float** out);
+outlets_status head_noalloc_run(outlets_ctx* c, const void* h_draft, int rows, float* z_out, float* len_out,
+                                cudaStream_t s);
+constexpr int kMaxDevices = 64;
+
 }  // namespace
 
 extern "C" {
@@ -1152,6 +1161,16 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
     outlets_destroy(c);
     return st;
   };
+  // Resolve the no-allocation head's scratch array here, where allocating is
+  // allowed: the lookup loads the module that holds the array, which commits
+  // its device memory, so that outlets_length_head_noalloc itself never does.
+  if (cfg->device < kMaxDevices) {
+    float* scratch = nullptr;
+    if (head_scratch_ptr(cfg->device, &scratch) != cudaSuccess) {
+      cudaGetLastError();
+      return cleanup_fail(OUTLETS_ECUDA);
+    }
+  }
   const int d = c->d;
   const size_t es = c->esz;
   // ---- weights (bf16: k-block-major swizzled, rows padded to a multiple of 768 =
@@ -1350,6 +1369,14 @@ outlets_status outlets_create(const outlets_config* cfg, const outlets_weights* 
     h2d(c->rope_sin, sn.data(), sn.size() * 4);
   }
   if (st != OUTLETS_OK) return cleanup_fail(st);
+  // One no-allocation head call on a zero row: under lazy module loading this
+  // loads every kernel that entry point launches (loading commits device
+  // memory), so that its later calls allocate nothing.
+  if (cfg->device < kMaxDevices) {
+    if (cudaMemset(c->hn, 0, (size_t)d * es) != cudaSuccess) return cleanup_fail(OUTLETS_ECUDA);
+    st = head_noalloc_run(c, c->hn, 1, c->h1a, c->h1b, nullptr);
+    if (st != OUTLETS_OK) return cleanup_fail(st);
+  }
   if (cudaDeviceSynchronize() != cudaSuccess) {
     cudaGetLastError();
     return cleanup_fail(OUTLETS_ECUDA);
@@ -2178,16 +2205,17 @@ outlets_status outlets_get_intermediate(outlets_ctx* c, int32_t which, void* dst
 // them, outlets_length_head_noalloc runs the length head (Linear+ReLU layers
 // and the output row) with its hidden activations in the file-scope array
 // below instead of in memory it allocates.  The array is part of the library
-// image: every GPU that loads the library holds its 16 MiB until the process
-// exits.  All calls on a device share it, so calls that overlap on the GPU
-// race; nothing in it has to start at zero (every value read was written
-// earlier in the same call).
+// image.  Under lazy module loading its 16 MiB are committed on a device when
+// the module holding it is first used there; outlets_create looks up the
+// array's address, so the memory is reserved when the first context is
+// created on that device and stays until the process exits.  All calls on a
+// device share it, so calls that overlap on the GPU race; nothing in it has
+// to start at zero (every value read was written earlier in the same call).
 namespace {
 
 constexpr size_t kHeadScratchFloats = (size_t)4 << 20;  // 16 MiB
 static __device__ __align__(256) float g_head_scratch[kHeadScratchFloats];
 
-constexpr int kMaxDevices = 64;
 std::mutex g_head_scratch_mu;
 float* g_head_scratch_ptr[kMaxDevices] = {};
 
@@ -2227,9 +2255,20 @@ extern "C" outlets_status outlets_length_head_noalloc(outlets_ctx* c, const void
                                           std::to_string(need) + " > " + std::to_string(kHeadScratchFloats) +
                                           " floats)");
   OUT_CK(c, cudaSetDevice(c->cfg.device));
+  return head_noalloc_run(c, h_draft, rows, z_out, len_out, (cudaStream_t)stream);
+}
+
+namespace {
+
+// The head on rows of draft states with its hidden activations in the static
+// scratch array (argument checks are the caller's).
+outlets_status head_noalloc_run(outlets_ctx* c, const void* h_draft, int rows, float* z_out, float* len_out,
+                                cudaStream_t s) {
   float* scratch = nullptr;
   OUT_CK(c, head_scratch_ptr(c->cfg.device, &scratch));
-  cudaStream_t s = (cudaStream_t)stream;
+  const int nl = (int)c->head_dims.size() - 1;
+  int wmax = 1;
+  for (int i = 1; i < nl; ++i) wmax = std::max(wmax, c->head_dims[i]);
   const int d = c->d;
   float* buf[2] = {scratch, scratch + (size_t)rows * wmax};
   float* cur = buf[0];
@@ -2250,3 +2289,5 @@ extern "C" outlets_status outlets_length_head_noalloc(outlets_ctx* c, const void
                              z_out, len_out, s));
   return OUTLETS_OK;
 }
+
+}  // namespace

@@ -1,4 +1,4 @@
-// Discrete-event model of length-aware serving (Sec. 5.5): RR / LB routing to
+// Discrete-event model of length-aware serving (Sec. 5.3 and the appendix "System-Level Evaluation Details"): RR / LB routing to
 // decode instances and FCFS / SJF admission, driven by the static prediction.
 // The model and its tie rules are stated in include/outlets_sched.h.  Built
 // without contracted multiply-adds (-ffp-contract=off) so that times are the

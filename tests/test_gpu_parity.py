@@ -312,20 +312,32 @@ def test_argument_errors_change_nothing():
 
 
 # ---------------------------------------------------------------- full-size configurations
-def _sampled_prefill(shape, lengths, max_tokens, sample, seed_off):
+def _sampled_prefill(shape, lengths, max_tokens, sample, seed_off, rows_too=False):
+    """Full-size static prediction, sampled prompts against the oracle; with
+    rows_too also the last rows of q, attention, a and y (the pruned order
+    keeps them for each prompt's last row, in prompt order)."""
     from paper_2609_01068_gb300 import outlets as OT
     w = synth.make_weights(shape, 0)
     pred = OT.Predictor(shape, w, max_tokens=max_tokens, max_batch=len(lengths), max_position=8192)
     cu = synth.cu_seqlens(lengths)
-    taps = synth.make_taps(shape, int(cu[-1]), 0, seed_off)
+    T = int(cu[-1])
+    taps = synth.make_taps(shape, T, 0, seed_off)
     z, ln = pred.prefill([to_device(t, "bf16") for t in taps], cu)
     torch.cuda.synchronize()
     pred.check()
     hd = to_np(pred.intermediate(OT.T_HDRAFT))
     ref = OR.sample_prefill_rows(w, shape, taps, cu, sample)
-    check_z_len(z[sample], ln[sample], ref["z"], ref["length"], "bf16", shape.name)
-    check_hidden(hd[sample], ref["h_draft"], "bf16", f"{shape.name} h_draft")
+    errs = {"z": check_z_len(z[sample], ln[sample], ref["z"], ref["length"], "bf16", shape.name)[0],
+            "h_draft": check_hidden(hd[sample], ref["h_draft"], "bf16", f"{shape.name} h_draft")}
+    if rows_too:
+        assert pruned("bf16", T)
+        sub_last = np.cumsum([lengths[b] for b in sample]) - 1
+        for which, key in ((OT.T_Q, "q"), (OT.T_ATTN, "attn"), (OT.T_A, "a"), (OT.T_Y, "y")):
+            g = to_np(pred.intermediate(which))[sample]
+            r = np.asarray(ref[key]).reshape(len(ref[key]), -1)[sub_last]
+            errs[key] = check_hidden(g, r, "bf16", f"{shape.name} {key}")
     pred.close()
+    return errs
 
 
 def test_llama8b_prefill_full_size_sampled():
@@ -336,10 +348,68 @@ def test_llama8b_prefill_full_size_sampled():
 
 
 def test_llama70b_prefill_sampled():
+    """The shortest, the median and the longest (4096-token) prompt of the
+    70B-shaped workload: z, h_draft and the last rows of q, attention, a, y."""
     lengths = synth.lengths_70b_prefill(0)
-    order = np.argsort(lengths)
-    sample = [int(order[0]), int(order[len(order) // 2])]
-    _sampled_prefill(synth.LLAMA70B, lengths, 65536, sample, 0)
+    order = np.argsort(lengths, kind="stable")
+    sample = [int(order[0]), int(order[len(order) // 2]), int(order[-1])]
+    assert lengths[sample[-1]] == 4096
+    errs = _sampled_prefill(synth.LLAMA70B, lengths, 65536, sample, 0, rows_too=True)
+    print("70B sampled errors:", errs)
+
+
+def test_long_prompt_positions_to_8191_match_oracle():
+    """A prompt of 8192 tokens (the largest position the sweep reaches) with
+    short ones: RoPE and attention at positions up to 8191, in both orders of
+    the static prediction (whole layer on every row, last rows only)."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = MID128
+    pred, w = predictor("mid128", max_tokens=9216)
+    lengths = [3, 8192, 700, 64]
+    cu = synth.cu_seqlens(lengths)
+    T = int(cu[-1])
+    taps = _taps(shape, T, off=71)
+    ref = OR.predict_prefill(w, shape, taps, cu)
+    taps_d = [to_device(t, shape.dtype) for t in taps]
+    for keep in (True, False):
+        z, ln = pred.prefill(taps_d, cu, keep_rows=keep)
+        torch.cuda.synchronize()
+        pred.check()
+        pr = pruned(shape.dtype, T, keep)
+        for which, r, what in [(OT.T_Q, ref["q"].reshape(T, -1), "q"), (OT.T_ATTN, ref["attn"], "attn"),
+                               (OT.T_A, ref["a"], "a"), (OT.T_Y, ref["y"], "y")]:
+            check_rows(pred.intermediate(which), r, cu, shape.dtype, f"8192-token prompt keep_rows={keep} {what}",
+                       pr)
+        check_z_len(z, ln, ref["z"], ref["length"], shape.dtype, f"8192-token prompt keep_rows={keep}")
+
+
+def test_steps_at_long_cache_lengths():
+    """Steps whose cache lengths cross a 64-position page boundary far out
+    (4095 -> 4096 -> 4097) and reach the last position (8190 -> 8191)."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = MID128
+    pred, w = predictor("mid128", max_tokens=16896)
+    pref = [8190, 4095, 4096, 5]
+    B = len(pref)
+    kv = OT.KVCache(pred, max_slots=B, max_tokens_total=sum(pref) + 64 * B)
+    slots = np.arange(B, dtype=np.int32)
+    cu = synth.cu_seqlens(pref)
+    taps = _taps(shape, int(cu[-1]), off=72)
+    pred.prefill([to_device(t, shape.dtype) for t in taps], cu, kv=kv, slots=slots)
+    caches = OR.caches_from_prefill(OR.predict_prefill(w, shape, taps, cu), cu)
+    for step in range(2):
+        st_taps = _taps(shape, B, off=73 + step)
+        z, ln = pred.step([to_device(t, shape.dtype) for t in st_taps], kv, slots)
+        torch.cuda.synchronize()
+        pred.check()
+        ref = OR.predict_step(w, shape, st_taps, caches)
+        caches = ref["caches"]
+        check_hidden(pred.intermediate(OT.T_Q), ref["q"].reshape(B, -1), shape.dtype, f"long step {step} q")
+        check_hidden(pred.intermediate(OT.T_ATTN), ref["attn"], shape.dtype, f"long step {step} attn")
+        check_hidden(pred.intermediate(OT.T_Y), ref["y"], shape.dtype, f"long step {step} y")
+        check_z_len(z, ln, ref["z"], ref["length"], shape.dtype, f"long step {step}")
+    assert [kv.slot_length(int(s)) for s in slots] == [L + 2 for L in pref]
+    kv.close()
 
 
 def test_llama8b_step_full_size_sampled():

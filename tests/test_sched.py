@@ -1,4 +1,4 @@
-"""Length-aware serving model (Sec. 5.5): oracle pins and the C++ model
+"""Length-aware serving model (Sec. 5.3): oracle pins and the C++ model
 (include/outlets_sched.h) against the oracle.  Host code only: these run on
 the CPU.  The decisions (instance per request) and the event times are
 compared exactly: both sides take the same IEEE double operations in the same
@@ -118,7 +118,7 @@ def test_p99_is_the_nearest_rank_percentile():
 
 
 def test_sjf_with_exact_predictions_cuts_the_short_tail_under_load():
-    """The effect Sec. 5.5 reports, in the model: at saturation, SJF with
+    """The effect Sec. 5.3 reports, in the model: at saturation, SJF with
     exact predictions lowers the P99 latency of short requests vs FCFS."""
     w = _lists(synth.make_serving_requests(600, 40.0, 4, pred_sigma=0.0))
     base = S.summarize(w[0], w[2], S.simulate(dict(BASE, route=S.RR, order=S.FCFS), *w)[0])

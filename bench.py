@@ -586,6 +586,12 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
                  "tflops_per_s": w_tf, "tensor_peak_frac_step": w_tf / w_roof["peak"],
                  "peak_kind": w_roof["peak_kind"], "roofline": w_roof, "clocks": w_clocks,
                  "note": "the same prediction with the whole layer run on every prompt row (OUTLETS_KEEP_ROWS)"}
+        pred.profile(True)  # its per-stage breakdown (untimed pass; stage events serialize the kernels)
+        for _ in range(2):
+            run(taps_d, z, ln, keep=True)
+        wprof = pred.profile_read()
+        pred.profile(False)
+        whole["stages"] = {k: v[0] / 2 for k, v in wprof.items() if v[1]}
     # per-stage breakdown in a separate (untimed) pass: stage events serialize the kernels
     pred.profile(True)
     for _ in range(3):

@@ -141,14 +141,17 @@ __global__ void __launch_bounds__(128, 3)
   }
   __syncthreads();
 
+  // K/V pages are read once per call and the cache is far larger than L2:
+  // evict them first, so the weights the next kernels prefetched stay in L2
+  const uint64_t kv_policy = l2_evict_first_policy();
   auto issue = [&](int pi, int stage) {
     const int row = (int)((long long)pages[page_begin + pi] * a.page_stride + (long long)g * a.head_stride);
     uint8_t* dk = sKV + stage * 2 * C::PAGE_BYTES;
     mbar_arrive_expect_tx(&full[stage], 2 * C::PAGE_BYTES);
 #pragma unroll
     for (int bx = 0; bx < NB; ++bx) {
-      tma_load_2d(dk + bx * 8192, &k_map, &full[stage], bx * 64, row);
-      tma_load_2d(dk + C::PAGE_BYTES + bx * 8192, &v_map, &full[stage], bx * 64, row);
+      tma_load_2d_hint(dk + bx * 8192, &k_map, &full[stage], bx * 64, row, kv_policy);
+      tma_load_2d_hint(dk + C::PAGE_BYTES + bx * 8192, &v_map, &full[stage], bx * 64, row, kv_policy);
     }
   };
   if (threadIdx.x == 0) {

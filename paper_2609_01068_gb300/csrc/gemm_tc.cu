@@ -84,6 +84,7 @@ __device__ __forceinline__ float fold_row_scale(const GemmArgs& p, int m) {
   if (!p.row_ss || m >= p.M) return 1.0f;
   const float* ss = p.row_ss + (long long)m * p.nrm_tiles;
   float t = 0.f;
+#pragma unroll 8
   for (int i = 0; i < p.nrm_tiles; ++i) t += ss[i];
   return rsqrtf(t / (float)p.nrm_d + p.nrm_eps);
 }
@@ -288,6 +289,12 @@ __global__ void __launch_bounds__(192, 1)
     uint32_t acc_phase = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
       const Tile tl = decode_tile(t, num_m, num_n, p.group_m, kb_total, kb_per);
+      // folded RMSNorm: this thread's row scales, read while the main loop runs
+      float rs_rows[MT];
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt)
+        rs_rows[mt] = (EPI == EPI_SWIGLU || EPI == EPI_ACT) ? fold_row_scale(p, tl.m_blk * TM + mt * BM + row_in_tile)
+                                                            : 1.0f;
       if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err)) break;
       tc_fence_after();
 #pragma unroll 1
@@ -300,7 +307,7 @@ __global__ void __launch_bounds__(192, 1)
         // B rows are interleaved in blocks of 32: tile columns [64j, 64j+32) are
         // gate and [64j+32, 64j+64) up for the same 32 outputs
         const int n_out = p.N / 2;
-        const float rs = fold_row_scale(p, m);  // 1 unless the norm is folded in
+        const float rs = rs_rows[mt];  // 1 unless the norm is folded in
         for (int c = 0; c < BN; c += 64) {
           uint32_t g[32], u[32];
           tmem_ld_32x32b_x32(tbase + c, g);
@@ -374,7 +381,7 @@ __global__ void __launch_bounds__(192, 1)
         }
       } else {
         float ssr[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // EPI_F32 producer of a folded norm
-        const float rs_mine = EPI == EPI_ACT ? fold_row_scale(p, m) : 1.0f;  // EPI_ACT consumer
+        const float rs_mine = rs_rows[mt];  // EPI_ACT consumer of a folded norm (else 1)
         for (int c = 0; c < BN; c += 32) {
           uint32_t r[32];
           tmem_ld_32x32b_x32(tbase + c, r);
@@ -1030,6 +1037,9 @@ cudaError_t gemm_tc_launch(const CUtensorMap a_maps[3], int bn, int epi, int mt,
   OUTLETS_TC_CASE(256, EPI_F32, 1)
   OUTLETS_TC_CASE(256, EPI_ACT, 1)
   OUTLETS_TC_CASE(256, EPI_SWIGLU, 1)
+  // large M, 256 x 256 tiles (two 128-row MMAs per staged weight tile)
+  OUTLETS_TC_CASE(256, EPI_F32, 2)
+  OUTLETS_TC_CASE(256, EPI_ACT, 2)
   OUTLETS_TC_CASE(128, EPI_F32, 1)
   OUTLETS_TC_CASE(128, EPI_ACT, 1)
   OUTLETS_TC_CASE(64, EPI_F32, 1)

@@ -562,7 +562,16 @@ outlets_status gemm_tc(outlets_ctx* c, const void* const* a, int n_pieces, int k
     else if (tiles(128) >= c->num_sms) bn = 128;
     else bn = 64;
   }
-  return gemm_tc_ex(c, a, n_pieces, k_piece, lda, M, b, b_np, N, K, epi, bn, 1, 1, out, ldo, residual, ldr, bias, s, nf);
+  // 256 x 256 tiles (two 128-row MMAs per staged weight tile, one TMEM
+  // accumulator) where a wave of them fills the SMs: a third fewer operand
+  // bytes per MMA and more of them in flight per ring stage, at the price of
+  // an epilogue that no longer overlaps the next tile's main loop.  That
+  // price outweighs the gain only for the f32 + residual epilogue after a
+  // short K loop (the O projection at K = 4096).
+  const bool wide_epi = !(epi == EPI_F32 && residual && K < 8192);
+  const int mt = (wide_epi && bn == 256 && cdiv(M, 256) * cdiv(N, 256) >= c->num_sms) ? 2 : 1;
+  return gemm_tc_ex(c, a, n_pieces, k_piece, lda, M, b, b_np, N, K, epi, bn, mt, 1, out, ldo, residual, ldr, bias, s,
+                    nf);
 }
 
 // Small-M GEMM (M <= 256): every weight tile is streamed once.  K is split so

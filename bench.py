@@ -118,17 +118,22 @@ def sources_sha(kernel):
 
 
 def measured_traffic(kernel, workload):
-    """DRAM bytes per launch from the committed ncu capture, or None if the kernel's
-    sources changed since (profiles/traffic.json records their hash)."""
+    """DRAM bytes per launch from the committed ncu capture of this kernel on this
+    workload, or None if there is none or the kernel's sources changed since
+    (profiles/traffic.json: kernel -> list of captures, each with its sources' hash)."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
     with open(p) as fh:
         j = json.load(fh)
-    e = j.get(kernel)
-    if not e or e.get("workload") != workload or e.get("sources_sha256") != sources_sha(kernel):
-        return None
-    return e["dram_bytes_per_launch"]
+    entries = j.get(kernel) or []
+    if isinstance(entries, dict):
+        entries = [entries]
+    sha = sources_sha(kernel)
+    for e in entries:
+        if e.get("workload") == workload and e.get("sources_sha256") == sha:
+            return e["dram_bytes_per_launch"]
+    return None
 
 
 def tensor_peak(peaks, region_ms, clocks):
@@ -561,10 +566,10 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
         k_ms, k_n = prof_live[kern]
         if kern == "fc_gemm":
             k_flops = 2.0 * T * shape.d * 3 * shape.d
-            name, alg = "fc_gemm (k_gemm_tc<256, F32>, folded input norm)", f"2*T*d*3d, T={T}"
+            name, alg = "fc_gemm (k_gemm_tc<256, F32, 2>: 256 x 256 tiles, folded input norm)", f"2*T*d*3d, T={T}"
         else:
             k_flops = 2.0 * T * (2 * shape.ffn) * shape.d
-            name, alg = "gateup_swiglu_gemm (k_gemm_tc<256, SWIGLU>)", f"2*T*(2F)*d, T={T}"
+            name, alg = "gateup_swiglu_gemm (k_gemm_tc<256, SWIGLU, 2>: 256 x 256 tiles)", f"2*T*(2F)*d, T={T}"
         k_tflops = k_flops / (k_ms / k_n / 1e3) / 1e12
         peak, kind = tensor_peak(peaks, ms, clocks)
         roof = {"bound": "tensor", "kernel": name, "achieved": k_tflops, "peak": peak, "unit": "TFLOP/s",

@@ -522,9 +522,16 @@ outlets_status gemm_tc_ex(outlets_ctx* c, const void* const* a, int n_pieces, in
   g.k_per_map = k_piece;
   g.splits = splits;
   g.prefetch = M <= 256 ? prefetch_blocks() : 0;  // small M streams every weight tile once
-  // tile raster: groups of M blocks whose activation panel (128 x K bf16 each)
-  // fills about 48 MB of L2, so each weight tile is fetched once per group
-  g.group_m = (int)std::max<long long>(8, std::min<long long>(cdiv(M, 128), (48ll << 20) / (128ll * K * 2)));
+  // Tile raster: groups of M blocks (tm rows each), N-major inside a group.
+  // A group's activation panel fills about 48 MB of L2, so its weight tiles
+  // are fetched once per group; and it is never narrower than a square wave
+  // (about sqrt(SMs * bn / tm) blocks), since the panels one wave of tiles
+  // touches are what it reads from DRAM when the panels do not stay in L2
+  // across waves (long K).
+  const long long tm = 128LL * mt;
+  const long long sq = (long long)std::lround(std::sqrt((double)c->num_sms * bn / (double)tm));
+  g.group_m = (int)std::max<long long>(std::max<long long>(1, sq),
+                                       std::min<long long>(cdiv(M, tm), (48ll << 20) / (tm * K * 2)));
   g.out = out;
   g.ldo = ldo;
   g.residual = residual;

@@ -138,11 +138,17 @@ def measured_traffic(kernel, workload):
 
 def tensor_peak(peaks, region_ms, clocks):
     """The bf16 denominator for a contraction timed over region_ms: the burst
-    figure for a region under a second without a power cap, else the sustained
-    one (measured over a seconds-long loop under the power cap)."""
-    capped = "sw_power_cap" in ((clocks or {}).get("reasons") or [])
-    if region_ms < 1000.0 and not capped:
-        return peaks["bf16"], f"bf16 burst {peaks['src']}"
+    figure for a region under a second whose SM clock stayed at its maximum
+    (no power cap pulled it down: median >= 97% of max), else the sustained
+    one (measured over a seconds-long loop with the clock held down by the
+    power cap)."""
+    clocks = clocks or {}
+    sm, smax = clocks.get("sm_mhz"), clocks.get("sm_max_mhz")
+    capped = "sw_power_cap" in (clocks.get("reasons") or [])
+    held = sm is not None and smax and sm >= 0.97 * smax
+    if region_ms < 1000.0 and (held or not capped):
+        why = " (power cap flagged, clock at its maximum)" if capped else ""
+        return peaks["bf16"], f"bf16 burst {peaks['src']}{why}"
     return peaks["bf16_sus"], f"bf16 sustained {peaks['src']}"
 
 

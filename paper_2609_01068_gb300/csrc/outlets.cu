@@ -15,6 +15,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <numeric>
 #include <cstdlib>
 #include <cstdio>
 #include <cstring>
@@ -31,8 +32,8 @@ using namespace outlets;
 namespace {
 
 constexpr int kPageTokens = 64;
-constexpr int kMaxTapChunks = 8;      // row chunks of host taps copied while earlier chunks compute
-constexpr int kMinTapChunkRows = 2048;
+constexpr int kMaxTapChunks = 16;     // row chunks of host taps copied while earlier chunks compute
+constexpr int kMinTapChunkRows = 1024;
 constexpr int kSplitLen = 512;        // shortest split-KV work item (keys)
 constexpr int kDecodeCtasPerSm = 3;   // resident decode-attention CTAs per SM
 constexpr int kRing = 4;
@@ -1724,11 +1725,26 @@ outlets_status predict_prefill(outlets_ctx* c, const void* const taps[3], const 
   // Large calls with host taps overlap the copy with the front of the pipeline
   // (FC, input norm, QKV, RoPE are row-wise): rows run in chunks of whole
   // 128-row tiles as their taps land.
+  // A chunk's FC tiles (256 x 256; d / 256 of them per 256 rows) are a whole
+  // number of waves over the SMs where such a chunk is small enough (at most
+  // kMaxTapChunks of them); else the chunks are equal, in whole 128-row tiles.
   int n_chunks = 1, chunk_rows = T;
   if (c->bf16 && !small_path(c, T) && !is_device_ptr(taps[0]) && !is_device_ptr(taps[1]) && !is_device_ptr(taps[2])) {
-    n_chunks = std::max(1, std::min(kMaxTapChunks, T / kMinTapChunkRows));
-    chunk_rows = (int)(cdiv(cdiv(T, n_chunks), 128) * 128);
+    const long long ntn = cdiv(c->d, 256);
+    const long long unit = 256LL * (c->num_sms / std::gcd((long long)c->num_sms, ntn));  // rows of whole waves
+    const long long per = cdiv(T, kMaxTapChunks);
+    const long long aligned = cdiv(per, unit) * unit;
+    if (aligned * 2 <= T) {
+      chunk_rows = (int)aligned;
+    } else {
+      const int n = std::max(1, std::min(8, T / kMinTapChunkRows));
+      chunk_rows = (int)(cdiv(cdiv(T, n), 128) * 128);
+    }
     n_chunks = (int)cdiv(T, chunk_rows);
+    if (n_chunks < 2) {
+      n_chunks = 1;
+      chunk_rows = T;
+    }
   }
 
   // ---- host metadata

@@ -36,6 +36,8 @@ constexpr int kBQ = 128;                         // query rows per work item
 constexpr int kBK = 128;                         // keys per K/V tile
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;              // tolerated growth of a row max before O is rescaled
+constexpr unsigned kPollSleepNs = 32;            // back-off of the polling roles when nothing is ready
+constexpr int kMaxLanes = 8;                     // independent partial maxima of a score row
 
 // 2^x with the hardware approximation (ex2.approx.ftz: -inf -> 0); the result
 // is rounded to bf16 or divided out by the row sum, far coarser than its error.
@@ -54,16 +56,21 @@ struct TcAttnCfg {
   // Q buffers and K/V stages share the 227 KB: K/V latency wants stages, and a
   // second Q buffer only hides the Q load between items
   static constexpr int NQ = HD >= 128 ? 1 : 2;
-  static constexpr int NS_FIT = (int)((232448u - 1024u - 512u - NQ * Q_BYTES) / (K_BYTES + V_BYTES));
+  static constexpr uint32_t BAR_BYTES = 512;          // mbarriers, TMEM address, abort flag
+  static constexpr uint32_t L_BYTES = 2 * kBQ * 4;     // row sums of the two O buffers
+  static constexpr int NS_FIT =
+      (int)((232448u - 1024u - BAR_BYTES - L_BYTES - NQ * Q_BYTES) / (K_BYTES + V_BYTES));
   static constexpr int NS = NS_FIT > 6 ? 6 : NS_FIT;
-  static constexpr size_t SMEM = 1024 + NQ * Q_BYTES + NS * (K_BYTES + V_BYTES) + 512;
+  static constexpr size_t SMEM = 1024 + NQ * Q_BYTES + NS * (K_BYTES + V_BYTES) + BAR_BYTES + L_BYTES;
   static_assert(NS >= 3, "K/V stages");
-  static constexpr uint32_t O_COL = 2 * kBK;           // TMEM: S0 [0,128), S1 [128,256), O [256, 256+hd)
+  // TMEM: S0 [0,128), S1 [128,256), O0 [256, 256+hd), O1 [256+hd, 256+2hd)
+  static constexpr uint32_t O_COL = 2 * kBK;
+  static_assert(O_COL + 2 * HD <= 512, "TMEM columns");
   static_assert(SMEM <= 232448, "shared memory");
 };
 
 template <int HD>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(320, 1)
     k_attn_prefill_tc(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap k_map,
                       const __grid_constant__ CUtensorMap vt_map, const TcAttnItem* __restrict__ items,
                       int n_items, int kv_ld, int H, int KVH, bf16* __restrict__ out, const bf16* __restrict__ gate,
@@ -77,13 +84,24 @@ __global__ void __launch_bounds__(192, 1)
   uint8_t* sV = sK + NS * C::K_BYTES;     // NS stages
   uint64_t* q_full = reinterpret_cast<uint64_t*>(sV + NS * C::V_BYTES);
   uint64_t* q_empty = q_full + NQ;
-  uint64_t* kv_full = q_empty + NQ;
-  uint64_t* kv_empty = kv_full + NS;
-  uint64_t* s_full = kv_empty + NS;
+  // K and V^T stages have their own rings: a K stage is free once its S is
+  // computed, a V stage once its PV is (long before, in the K case)
+  uint64_t* k_full = q_empty + NQ;
+  uint64_t* k_empty = k_full + NS;
+  uint64_t* v_full = k_empty + NS;
+  uint64_t* v_empty = v_full + NS;
+  uint64_t* s_full = v_empty + NS;
   uint64_t* p_full = s_full + 2;
   uint64_t* pv_done = p_full + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pv_done + 1);
+  // O is double-buffered in TMEM: item k accumulates into O[k & 1] while the
+  // epilogue warps store item k - 1 from the other buffer
+  uint64_t* o_full = pv_done + 1;   // [2] last PV of the item complete
+  uint64_t* o_empty = o_full + 2;   // [2] the epilogue has read O and l
+  uint64_t* l_full = o_empty + 2;   // [2] the softmax has written the row sums
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(l_full + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* l_buf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(q_full) + C::BAR_BYTES);  // [2][128]
+  static_assert((2 * NQ + 4 * NS + 10) * 8 + 8 <= (int)C::BAR_BYTES, "barrier area");
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
@@ -93,10 +111,17 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(&q_empty[i], 1);
     }
     for (int i = 0; i < NS; ++i) {
-      mbar_init(&kv_full[i], 1);
-      mbar_init(&kv_empty[i], 1);
+      mbar_init(&k_full[i], 1);
+      mbar_init(&k_empty[i], 1);
+      mbar_init(&v_full[i], 1);
+      mbar_init(&v_empty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) mbar_init(&s_full[i], 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&o_full[i], 1);
+      mbar_init(&o_empty[i], 4 * 32);
+      mbar_init(&l_full[i], 4 * 32);
+    }
     mbar_init(p_full, 4 * 32);
     mbar_init(pv_done, 1);
     *abort_flag = 0;
@@ -120,109 +145,183 @@ __global__ void __launch_bounds__(192, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      int g = 0;  // K/V tiles loaded by this CTA
-      int k = 0;  // items of this CTA
-      for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
-        const TcAttnItem w = items[it];
-        const int kvh = (w.head * KVH) / H;
-        const int qb = k % NQ;
-        if (k >= NQ && !mbar_wait(&q_empty[qb], ((k - NQ) / NQ) & 1, abort_flag, err)) break;
-        mbar_arrive_expect_tx(&q_full[qb], C::Q_BYTES);
+      // Producer, three cursors issued as their slots free up: Q of an item
+      // (with the item's first K tile), K tiles, V^T tiles.  K may run up to
+      // NS tiles ahead of V.
+      int k_it = blockIdx.x, k_k = 0, k_j = 0, k_g = 0;  // K cursor: item, item count, tile in item, tile count
+      int v_it = blockIdx.x, v_j = 0, v_g = 0;           // V cursor
+      unsigned long long t_idle = 0;
+      uint32_t spin = 0;
+      while (v_it < n_items) {
+        bool progressed = false;
+        if (k_it < n_items) {
+          const TcAttnItem w = items[k_it];
+          const int qb = k_k % NQ;
+          const int st = k_g % NS;
+          const bool q_ok = k_j > 0 || k_k < NQ || mbar_test_wait(&q_empty[qb], ((k_k - NQ) / NQ) & 1);
+          if (q_ok && (k_g < NS || mbar_test_wait(&k_empty[st], ((k_g - NS) / NS) & 1))) {
+            const int kvh = (w.head * KVH) / H;
+            if (k_j == 0) {
+              mbar_arrive_expect_tx(&q_full[qb], C::Q_BYTES);
 #pragma unroll
-        for (int b = 0; b < C::NB; ++b)
-          tma_load_2d(sQ + qb * C::Q_BYTES + b * (kBQ * 128), &q_map, &q_full[qb], w.head * HD + 64 * b, w.q_start);
-        bool ok = true;
-        for (int j = 0; j < w.n_kv; ++j, ++g) {
-          const int st = g % NS;
-          if (g >= NS && !mbar_wait(&kv_empty[st], ((g - NS) / NS) & 1, abort_flag, err)) {
-            ok = false;
+              for (int b = 0; b < C::NB; ++b)
+                tma_load_2d(sQ + qb * C::Q_BYTES + b * (kBQ * 128), &q_map, &q_full[qb], w.head * HD + 64 * b,
+                            w.q_start);
+            }
+            mbar_arrive_expect_tx(&k_full[st], C::K_BYTES);
+#pragma unroll
+            for (int b = 0; b < C::NB; ++b)
+              tma_load_2d(sK + st * C::K_BYTES + b * (kBK * 128), &k_map, &k_full[st], 64 * b,
+                          kvh * kv_ld + w.seq_start + kBK * k_j);
+            ++k_g;
+            if (++k_j == w.n_kv) {
+              k_j = 0;
+              ++k_k;
+              k_it += gridDim.x;
+            }
+            progressed = true;
+          }
+        }
+        {
+          const int st = v_g % NS;
+          if (v_g < k_g && (v_g < NS || mbar_test_wait(&v_empty[st], ((v_g - NS) / NS) & 1))) {
+            const TcAttnItem w = items[v_it];
+            const int kvh = (w.head * KVH) / H;
+            mbar_arrive_expect_tx(&v_full[st], C::V_BYTES);
+#pragma unroll
+            for (int b = 0; b < 2; ++b)
+              tma_load_2d(sV + st * C::V_BYTES + b * (HD * 128), &vt_map, &v_full[st], w.v_start + kBK * v_j + 64 * b,
+                          kvh * HD);
+            ++v_g;
+            if (++v_j == w.n_kv) {
+              v_j = 0;
+              v_it += gridDim.x;
+            }
+            progressed = true;
+          }
+        }
+        if (progressed) {
+          spin = 0;
+          t_idle = 0;
+          continue;
+        }
+        __nanosleep(kPollSleepNs);  // leave the issue slots to the softmax warps sharing this SM sub-partition
+        if ((++spin & 31u) == 0) {  // bounded, like every other wait
+          if (*abort_flag) break;
+          const unsigned long long now = global_timer_ns();
+          if (t_idle == 0) {
+            t_idle = now;
+          } else if (now - t_idle > kWaitTimeoutNs) {
+            *abort_flag = 1;
+            if (err) atomicOr(err, ERR_TIMEOUT);
             break;
           }
-          mbar_arrive_expect_tx(&kv_full[st], C::K_BYTES + C::V_BYTES);
-#pragma unroll
-          for (int b = 0; b < C::NB; ++b)
-            tma_load_2d(sK + st * C::K_BYTES + b * (kBK * 128), &k_map, &kv_full[st], 64 * b,
-                        kvh * kv_ld + w.seq_start + kBK * j);
-#pragma unroll
-          for (int b = 0; b < 2; ++b)
-            tma_load_2d(sV + st * C::V_BYTES + b * (HD * 128), &vt_map, &kv_full[st], w.v_start + kBK * j + 64 * b,
-                        kvh * HD);
         }
-        if (!ok) break;
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
+      // MMA issuer, two cursors issued as their inputs arrive: S_n = Q K_n^T
+      // (needs the item's Q, K tile n, and TMEM buffer n & 1 free: PV_{n-2}
+      // issued, since the tensor pipe runs in order) and PV_n = P_n V_n (needs
+      // the softmax's P_n and V tile n).  Neither waits for the other's inputs.
       constexpr uint32_t id_s = idesc_bf16_f32(kBQ, kBK);
       constexpr uint32_t id_o = idesc_bf16_f32(kBQ, HD);
-      // issue cursor of S (runs one tile ahead of the PV cursor)
       int s_it = blockIdx.x, s_k = 0, s_j = 0, s_g = 0;
       int s_nkv = s_it < n_items ? items[s_it].n_kv : 0;
-      auto issue_s = [&]() -> bool {
-        if (s_it >= n_items) return true;
-        const int qb = s_k % NQ;
-        if (s_j == 0 && !mbar_wait(&q_full[qb], (s_k / NQ) & 1, abort_flag, err)) return false;
-        const int st = s_g % NS;  // K/V stage
-        const int sb = s_g & 1;   // TMEM S buffer
-        if (!mbar_wait(&kv_full[st], (s_g / NS) & 1, abort_flag, err)) return false;
-        tc_fence_after();
-        const uint32_t qa = smem_u32(sQ + qb * C::Q_BYTES);
-        const uint32_t ka = smem_u32(sK + st * C::K_BYTES);
+      int p_it = blockIdx.x, p_k = 0, p_j = 0, p_g = 0;
+      int p_nkv = p_it < n_items ? items[p_it].n_kv : 0;
+      unsigned long long t_idle = 0;
+      uint32_t spin = 0;
+      while (p_it < n_items) {
+        bool progressed = false;
+        if (s_it < n_items && s_g < p_g + 2) {
+          const int qb = s_k % NQ;
+          const int st = s_g % NS;
+          if ((s_j > 0 || mbar_test_wait(&q_full[qb], (s_k / NQ) & 1)) &&
+              mbar_test_wait(&k_full[st], (s_g / NS) & 1)) {
+            tc_fence_after();
+            const int sb = s_g & 1;  // TMEM S buffer
+            const uint32_t qa = smem_u32(sQ + qb * C::Q_BYTES);
+            const uint32_t ka = smem_u32(sK + st * C::K_BYTES);
 #pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * (128 * 128);
-          tc_mma_bf16(tmem_base + sb * kBK, sw128_kmajor_desc(qa + off) + 2u * (kk & 3),
-                      sw128_kmajor_desc(ka + off) + 2u * (kk & 3), id_s, kk > 0 ? 1u : 0u);
+            for (int kk = 0; kk < HD / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * (128 * 128);
+              tc_mma_bf16(tmem_base + sb * kBK, sw128_kmajor_desc(qa + off) + 2u * (kk & 3),
+                          sw128_kmajor_desc(ka + off) + 2u * (kk & 3), id_s, kk > 0 ? 1u : 0u);
+            }
+            tc_commit(&s_full[sb]);
+            tc_commit(&k_empty[st]);                          // S_n has read its K tile
+            if (s_j == s_nkv - 1) tc_commit(&q_empty[qb]);  // last S of the item: its Q buffer is free
+            ++s_g;
+            if (++s_j == s_nkv) {
+              s_j = 0;
+              ++s_k;
+              s_it += gridDim.x;
+              s_nkv = s_it < n_items ? items[s_it].n_kv : 0;
+            }
+            progressed = true;
+          }
         }
-        tc_commit(&s_full[sb]);
-        if (s_j == s_nkv - 1) tc_commit(&q_empty[qb]);  // last S of the item: its Q buffer is free
-        ++s_g;
-        if (++s_j == s_nkv) {
-          s_j = 0;
-          ++s_k;
-          s_it += gridDim.x;
-          s_nkv = s_it < n_items ? items[s_it].n_kv : 0;
+        if (p_g < s_g) {
+          const int st = p_g % NS;
+          const int ob = p_k & 1;  // O buffer of this item
+          // the first PV of an item overwrites O[ob]: the epilogue must have read item p_k - 2 from it
+          if (mbar_test_wait(p_full, p_g & 1) && mbar_test_wait(&v_full[st], (p_g / NS) & 1) &&
+              (p_j > 0 || p_k < 2 || mbar_test_wait(&o_empty[ob], ((p_k - 2) >> 1) & 1))) {
+            tc_fence_after();
+            const int sb = p_g & 1;  // TMEM buffer holding P
+            const uint32_t va = smem_u32(sV + st * C::V_BYTES);
+            // A = P in TMEM (the S buffer it was computed in: 16 keys = 8 columns per MMA)
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk)
+              tc_mma_bf16_ta(tmem_base + C::O_COL + ob * HD, tmem_base + sb * kBK + 8 * kk,
+                             sw128_kmajor_desc(va + (kk >> 2) * (HD * 128)) + 2u * (kk & 3), id_o,
+                             (p_j > 0 || kk > 0) ? 1u : 0u);
+            tc_commit(pv_done);
+            tc_commit(&v_empty[st]);  // PV_n has read its V tile
+            if (p_j == p_nkv - 1) tc_commit(&o_full[ob]);  // the item's O is complete
+            ++p_g;
+            if (++p_j == p_nkv) {
+              p_j = 0;
+              ++p_k;
+              p_it += gridDim.x;
+              p_nkv = p_it < n_items ? items[p_it].n_kv : 0;
+            }
+            progressed = true;
+          }
         }
-        return true;
-      };
-      bool ok = issue_s();
-      int p_g = 0;
-      for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
-        const int nkv = items[it].n_kv;
-        for (int j = 0; j < nkv; ++j, ++p_g) {
-          if (!issue_s()) {
-            ok = false;
+        if (progressed) {
+          spin = 0;
+          t_idle = 0;
+          continue;
+        }
+        __nanosleep(kPollSleepNs);  // leave the issue slots to the softmax warps sharing this SM sub-partition
+        if ((++spin & 31u) == 0) {  // bounded, like every other wait
+          if (*abort_flag) break;
+          const unsigned long long now = global_timer_ns();
+          if (t_idle == 0) {
+            t_idle = now;
+          } else if (now - t_idle > kWaitTimeoutNs) {
+            *abort_flag = 1;
+            if (err) atomicOr(err, ERR_TIMEOUT);
             break;
           }
-          if (!mbar_wait(p_full, p_g & 1, abort_flag, err)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const int st = p_g % NS;  // K/V stage
-          const int sb = p_g & 1;   // TMEM buffer holding P_j
-          const uint32_t va = smem_u32(sV + st * C::V_BYTES);
-          // A = P_j in TMEM (the S buffer it was computed in: 16 keys = 8 columns per MMA)
-#pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk)
-            tc_mma_bf16_ta(tmem_base + C::O_COL, tmem_base + sb * kBK + 8 * kk,
-                           sw128_kmajor_desc(va + (kk >> 2) * (HD * 128)) + 2u * (kk & 3), id_o,
-                           (j > 0 || kk > 0) ? 1u : 0u);
-          tc_commit(pv_done);
-          tc_commit(&kv_empty[st]);  // S_j and PV_j have read this stage's K and V
         }
       }
     }
-  } else {
-    // softmax warps: thread = query row = TMEM lane
+  } else if (warp < 6) {
+    // softmax warps (2..5): thread = query row = TMEM lane
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
     const float sl2 = rsqrtf((float)HD) * kLog2e;
-    int g = 0;
+    int g = 0;  // key tiles of this CTA
+    int k = 0;  // items of this CTA
     bool ok = true;
-    for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x) {
+    for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ++k) {
       const TcAttnItem w = items[it];
+      const int ob = k & 1;         // O buffer of this item
       const int qp = w.q_pos0 + r;  // position of this row in its sequence
       float m_used = -INFINITY, l = 0.f;
       for (int j = 0; j < w.n_kv; ++j, ++g) {
@@ -241,19 +340,26 @@ __global__ void __launch_bounds__(192, 1)
         for (int c = 0; c < kBK / 32; ++c) tmem_ld_32x32b_x32(s_addr + 32 * c, v + 32 * c);
         tmem_ld_wait();
         // row max on the raw scores (the scale is positive); the causal mask
-        // only applies on the diagonal tile (key > query position)
-        float mx = -INFINITY;
+        // only applies on the diagonal tile (key > query position).  Eight
+        // independent partial maxima: one chain of 128 dependent max
+        // operations would sit in front of every exponential of the tile.
         if (diag) {
 #pragma unroll
-          for (int e = 0; e < kBK; ++e) {
+          for (int e = 0; e < kBK; ++e)
             if (key0 + e > qp) v[e] = __float_as_uint(-INFINITY);
-            mx = fmaxf(mx, __uint_as_float(v[e]));
-          }
-        } else {
-#pragma unroll
-          for (int e = 0; e < kBK; ++e) mx = fmaxf(mx, __uint_as_float(v[e]));
         }
-        mx *= sl2;  // in the log2 domain of the exponentials
+        float mp[kMaxLanes];
+#pragma unroll
+        for (int i = 0; i < kMaxLanes; ++i) mp[i] = __uint_as_float(v[i]);
+#pragma unroll
+        for (int e = kMaxLanes; e < kBK; e += kMaxLanes)
+#pragma unroll
+          for (int i = 0; i < kMaxLanes; ++i) mp[i] = fmaxf(mp[i], __uint_as_float(v[e + i]));
+#pragma unroll
+        for (int w2 = kMaxLanes / 2; w2 > 0; w2 >>= 1)
+#pragma unroll
+          for (int i = 0; i < w2; ++i) mp[i] = fmaxf(mp[i], mp[i + w2]);
+        const float mx = mp[0] * sl2;  // in the log2 domain of the exponentials
         float alpha = 1.f;
         bool resc = false;
         if (mx > m_used + kRescaleLog2) {
@@ -263,18 +369,20 @@ __global__ void __launch_bounds__(192, 1)
           resc = j > 0;
         }
         // P = exp2(s - m) as bf16 pairs, written back over the scores of this
-        // buffer (columns 0..63); the row sum takes the bf16 values the PV
-        // product uses (O / l stays a convex combination of the value rows)
+        // buffer (columns 0..63).  The row sum adds the f32 values before
+        // rounding: the bf16 weights the PV product uses then sum to l within
+        // a relative 2^-9 / sqrt(keys), below the bf16 rounding of the output,
+        // and the softmax saves a widening of every weight.
         uint32_t pk[kBK / 2];
-        float ps = 0.f;
+        float psum[4] = {0.f, 0.f, 0.f, 0.f};  // four partial sums, for the same reason
 #pragma unroll
         for (int e = 0; e < kBK; e += 2) {
           const float p0 = ex2_approx(fmaf(__uint_as_float(v[e]), sl2, -m_used));
           const float p1 = ex2_approx(fmaf(__uint_as_float(v[e + 1]), sl2, -m_used));
           pk[e >> 1] = pack_bf16x2(p0, p1);
-          const float2 pr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&pk[e >> 1]));
-          ps += pr.x + pr.y;
+          psum[(e >> 1) & 3] += p0 + p1;
         }
+        const float ps = (psum[0] + psum[1]) + (psum[2] + psum[3]);
         tmem_st_32x32b_x32(s_addr, pk);
         tmem_st_32x32b_x32(s_addr + 32, pk + 32);
         // the previous PV must be complete before this tile's P is released (the
@@ -291,7 +399,7 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll 1
           for (int c = 0; c < HD / 32; ++c) {
             uint32_t o[32];
-            const uint32_t o_addr = tmem_base + lane_off + C::O_COL + 32 * c;
+            const uint32_t o_addr = tmem_base + lane_off + C::O_COL + ob * HD + 32 * c;
             tmem_ld_32x32b_x32(o_addr, o);
             tmem_ld_wait();
 #pragma unroll
@@ -305,43 +413,57 @@ __global__ void __launch_bounds__(192, 1)
         mbar_arrive(p_full);
       }
       if (!ok) break;
-      // end of the item: O / l (x gate) as bf16
-      if (!mbar_wait(pv_done, (g - 1) & 1, abort_flag, err)) break;
+      // end of the item: the row sums go to the epilogue warps once they have
+      // taken item k - 2's from this buffer
+      if (k >= 2 && !mbar_wait(&o_empty[ob], ((k - 2) >> 1) & 1, abort_flag, err)) break;
+      l_buf[ob * kBQ + r] = l;
+      mbar_arrive(&l_full[ob]);
+    }
+  } else {
+    // epilogue warps (6..9): O[k & 1] / l (x gate) as bf16, one query row per thread,
+    // while the softmax warps run the next item
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    int k = 0;
+    for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
+      const int ob = k & 1;
+      if (!mbar_wait(&o_full[ob], (k >> 1) & 1, abort_flag, err)) break;
+      if (!mbar_wait(&l_full[ob], (k >> 1) & 1, abort_flag, err)) break;
       tc_fence_after();
-      const float inv = 1.f / l;
-      const bool row_ok = r < w.q_len;
-      bf16* orow = out + (long long)(w.q_start + r) * H * HD + w.head * HD;
-      const bf16* grow = gate ? gate + (long long)(w.q_start + r) * H * HD + w.head * HD : nullptr;
+      const TcAttnItem w = items[it];
+      const float inv = 1.f / l_buf[ob * kBQ + r];
       uint32_t ov[HD];
 #pragma unroll
-      for (int c = 0; c < HD / 32; ++c) tmem_ld_32x32b_x32(tmem_base + lane_off + C::O_COL + 32 * c, ov + 32 * c);
+      for (int c = 0; c < HD / 32; ++c)
+        tmem_ld_32x32b_x32(tmem_base + lane_off + C::O_COL + ob * HD + 32 * c, ov + 32 * c);
       tmem_ld_wait();
+      tc_fence_before();
+      mbar_arrive(&o_empty[ob]);
+      if (r < w.q_len) {
+        bf16* orow = out + (long long)(w.q_start + r) * H * HD + w.head * HD;
+        const bf16* grow = gate ? gate + (long long)(w.q_start + r) * H * HD + w.head * HD : nullptr;
 #pragma unroll
-      for (int c = 0; c < HD / 32; ++c) {
-        const uint32_t* v = ov + 32 * c;
-        if (row_ok) {
+        for (int c = 0; c < HD / 8; ++c) {
+          const uint32_t* v = ov + 8 * c;
+          float f[8];
 #pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            float f[8];
+          for (int e = 0; e < 8; ++e) f[e] = __uint_as_float(v[e]) * inv;
+          if (grow) {
+            const uint4 gq = *reinterpret_cast<const uint4*>(grow + 8 * c);
+            const __nv_bfloat162* gh = reinterpret_cast<const __nv_bfloat162*>(&gq);
 #pragma unroll
-            for (int e = 0; e < 8; ++e) f[e] = __uint_as_float(v[8 * t + e]) * inv;
-            if (grow) {
-              const uint4 gq = *reinterpret_cast<const uint4*>(grow + 32 * c + 8 * t);
-              const __nv_bfloat162* gh = reinterpret_cast<const __nv_bfloat162*>(&gq);
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const float2 gf = __bfloat1622float2(gh[e]);
-                f[2 * e] *= gf.x;
-                f[2 * e + 1] *= gf.y;
-              }
+            for (int e = 0; e < 4; ++e) {
+              const float2 gf = __bfloat1622float2(gh[e]);
+              f[2 * e] *= gf.x;
+              f[2 * e + 1] *= gf.y;
             }
-            *reinterpret_cast<uint4*>(orow + 32 * c + 8 * t) =
-                make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]), pack_bf16x2(f[4], f[5]),
-                           pack_bf16x2(f[6], f[7]));
           }
+          *reinterpret_cast<uint4*>(orow + 8 * c) =
+              make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]), pack_bf16x2(f[4], f[5]),
+                         pack_bf16x2(f[6], f[7]));
         }
       }
-      tc_fence_before();
     }
   }
 
@@ -419,7 +541,7 @@ cudaError_t launch_tc(const CUtensorMap& q_map, const CUtensorMap& k_map, const 
     attr = true;
   }
   const int grid = n_items < num_sms ? n_items : num_sms;
-  OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_tc<HD>, dim3(grid), dim3(192), C::SMEM, stream, q_map, k_map, vt_map,
+  OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_tc<HD>, dim3(grid), dim3(320), C::SMEM, stream, q_map, k_map, vt_map,
                               items, n_items, kv_ld, H, KVH, reinterpret_cast<bf16*>(out),
                               reinterpret_cast<const bf16*>(gate), err));
   return cudaGetLastError();

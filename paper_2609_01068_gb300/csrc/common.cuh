@@ -60,6 +60,19 @@ OUTLETS_DEV bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// Non-blocking test of the same condition (try_wait may suspend the thread for
+// a while; a role that polls several barriers must not stall on one of them).
+OUTLETS_DEV bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 
 // Waits for the phase with the given parity to complete.  Gives up (returns
 // false) when the CTA-wide abort flag is raised or after kWaitTimeoutNs, in

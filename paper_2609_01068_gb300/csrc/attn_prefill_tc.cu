@@ -3,26 +3,29 @@
 // o = softmax(q k^T / sqrt(hd) + causal mask) v per packed sequence, q-head h
 // reading kv-head floor(h * KVH / H), optionally gated (o * gate).
 //
-// Persistent kernel, one CTA per SM, 6 warps.  A work item is one 128-row
+// Persistent kernel, one CTA per SM, 16 warps.  A work item is one 128-row
 // query tile of one sequence x one query head; items are taken longest first
 // (most key tiles) with a grid stride.
-//   warp 0      TMA producer: Q tile (one or two buffers), then K and V^T
-//               tiles of 128 keys (three or more stages), continuously across
-//               items
-//   warp 1      TMEM owner and single-thread MMA issuer:
-//                 S_j = Q K_j^T     M=128 N=128 K=hd, into one of two TMEM S buffers
-//                 O  += P_j V_j     M=128 N=hd K=128, into the TMEM O accumulator
-//               S_{j+1} is issued before waiting for P_j, so the next scores
-//               are computed while the softmax of the current tile runs
-//   warps 2..5  softmax, one query row per thread (TMEM lane): the score row
-//               is read from TMEM once into registers; row max of the masked,
-//               scaled scores; P = exp2(s - m) written as bf16 pairs back
-//               into the S buffer it came from (the PV MMA reads its A
-//               operand from TMEM, so P is double-buffered with S and PV_j
-//               overlaps the softmax of the next tile),
-//               O and l rescaled in place only when a row max grows by more
-//               than 2^8 over the one in use (the result is exact either way);
-//               at the end of an item O / l (x gate) is stored as bf16
+//   warp 0       TMA producer: Q tile (one or two buffers), K tiles and V^T
+//                tiles of 128 keys in rings of their own (a K stage is freed
+//                by its S, a V stage by its PV), continuously across items
+//   warp 1       TMEM owner and single-thread MMA issuer, polling two streams:
+//                  S_j = Q K_j^T     M=128 N=128 K=hd, into one of two TMEM S buffers
+//                  O  += P_j V_j     M=128 N=hd K=128, into O[item & 1] in TMEM
+//                S_{j+1} is issued as soon as its inputs are there, so the
+//                next scores are computed while the softmax of this tile runs
+//   warps 4..11  softmax, two threads per query row (TMEM lane), each over
+//                half of the tile's keys: the scores are read from TMEM once
+//                into registers; the two halves exchange their maxima of the
+//                masked raw scores through shared memory; P = exp2(s - m) is
+//                written as bf16 pairs back into the S buffer it came from
+//                (the PV MMA reads its A operand from TMEM, so P is
+//                double-buffered with S and PV_j overlaps the softmax of the
+//                next tile); O and l are rescaled in place only when a row max
+//                grows by more than 2^8 over the one in use (the result is
+//                exact either way)
+//   warps 12..15 epilogue: O / l (x gate) of item k as bf16 from O[k & 1],
+//                while the softmax and the MMAs run item k + 1
 // V is read through a transposed copy V^T [KVH*hd, columns] (keys contiguous)
 // so both MMAs take K-major operands; each sequence starts at a column that is
 // a multiple of 8 (TMA coordinates in 16-byte units).  Every wait is bounded.
@@ -38,6 +41,8 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;              // tolerated growth of a row max before O is rescaled
 constexpr unsigned kPollSleepNs = 32;            // back-off of the polling roles when nothing is ready
 constexpr int kMaxLanes = 8;                     // independent partial maxima of a score row
+constexpr int kThreads = 512;                    // producer, MMA, 2 idle, 8 softmax, 4 epilogue warps
+constexpr int kSoftmaxThreads = 8 * 32;
 
 // 2^x with the hardware approximation (ex2.approx.ftz: -inf -> 0); the result
 // is rounded to bf16 or divided out by the row sum, far coarser than its error.
@@ -57,12 +62,18 @@ struct TcAttnCfg {
   // second Q buffer only hides the Q load between items
   static constexpr int NQ = HD >= 128 ? 1 : 2;
   static constexpr uint32_t BAR_BYTES = 512;          // mbarriers, TMEM address, abort flag
-  static constexpr uint32_t L_BYTES = 2 * kBQ * 4;     // row sums of the two O buffers
-  static constexpr int NS_FIT =
-      (int)((232448u - 1024u - BAR_BYTES - L_BYTES - NQ * Q_BYTES) / (K_BYTES + V_BYTES));
-  static constexpr int NS = NS_FIT > 6 ? 6 : NS_FIT;
-  static constexpr size_t SMEM = 1024 + NQ * Q_BYTES + NS * (K_BYTES + V_BYTES) + BAR_BYTES + L_BYTES;
-  static_assert(NS >= 3, "K/V stages");
+  static constexpr uint32_t L_BYTES = 2 * 2 * kBQ * 4;  // row sums: [O buffer][half of the keys][row]
+  static constexpr uint32_t X_BYTES = 2 * kBQ * 8;      // row max exchange: [half of the keys][row] x (max, ok)
+  // K and V^T stages in what is left: as many of each as fit, one more K
+  // stage where it fits (a K stage is held from its load to its S, a V
+  // stage from its load to its PV, later)
+  static constexpr uint32_t KV_BUDGET = 232448u - 1024u - BAR_BYTES - L_BYTES - X_BYTES - NQ * Q_BYTES;
+  static constexpr int NV_FIT = (int)(KV_BUDGET / (K_BYTES + V_BYTES));
+  static constexpr int NV = NV_FIT > 6 ? 6 : NV_FIT;
+  static constexpr int NK = (NV < 6 && KV_BUDGET - NV * (K_BYTES + V_BYTES) >= K_BYTES) ? NV + 1 : NV;
+  static constexpr size_t SMEM =
+      1024 + NQ * Q_BYTES + NK * K_BYTES + NV * V_BYTES + BAR_BYTES + L_BYTES + X_BYTES;
+  static_assert(NV >= 2 && NK >= 3, "K/V stages");
   // TMEM: S0 [0,128), S1 [128,256), O0 [256, 256+hd), O1 [256+hd, 256+2hd)
   static constexpr uint32_t O_COL = 2 * kBK;
   static_assert(O_COL + 2 * HD <= 512, "TMEM columns");
@@ -70,7 +81,7 @@ struct TcAttnCfg {
 };
 
 template <int HD>
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     k_attn_prefill_tc(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap k_map,
                       const __grid_constant__ CUtensorMap vt_map, const TcAttnItem* __restrict__ items,
                       int n_items, int kv_ld, int H, int KVH, bf16* __restrict__ out, const bf16* __restrict__ gate,
@@ -78,19 +89,19 @@ __global__ void __launch_bounds__(320, 1)
   using C = TcAttnCfg<HD>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  constexpr int NQ = C::NQ, NS = C::NS;
+  constexpr int NQ = C::NQ, NK = C::NK, NV = C::NV;
   uint8_t* sQ = smem;                     // NQ buffers
-  uint8_t* sK = sQ + NQ * C::Q_BYTES;     // NS stages
-  uint8_t* sV = sK + NS * C::K_BYTES;     // NS stages
-  uint64_t* q_full = reinterpret_cast<uint64_t*>(sV + NS * C::V_BYTES);
+  uint8_t* sK = sQ + NQ * C::Q_BYTES;     // NK stages
+  uint8_t* sV = sK + NK * C::K_BYTES;     // NV stages
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(sV + NV * C::V_BYTES);
   uint64_t* q_empty = q_full + NQ;
   // K and V^T stages have their own rings: a K stage is free once its S is
   // computed, a V stage once its PV is (long before, in the K case)
   uint64_t* k_full = q_empty + NQ;
-  uint64_t* k_empty = k_full + NS;
-  uint64_t* v_full = k_empty + NS;
-  uint64_t* v_empty = v_full + NS;
-  uint64_t* s_full = v_empty + NS;
+  uint64_t* k_empty = k_full + NK;
+  uint64_t* v_full = k_empty + NK;
+  uint64_t* v_empty = v_full + NV;
+  uint64_t* s_full = v_empty + NV;
   uint64_t* p_full = s_full + 2;
   uint64_t* pv_done = p_full + 1;
   // O is double-buffered in TMEM: item k accumulates into O[k & 1] while the
@@ -100,8 +111,9 @@ __global__ void __launch_bounds__(320, 1)
   uint64_t* l_full = o_empty + 2;   // [2] the softmax has written the row sums
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(l_full + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float* l_buf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(q_full) + C::BAR_BYTES);  // [2][128]
-  static_assert((2 * NQ + 4 * NS + 10) * 8 + 8 <= (int)C::BAR_BYTES, "barrier area");
+  float* l_buf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(q_full) + C::BAR_BYTES);  // [2][2][128]
+  float2* m_xchg = reinterpret_cast<float2*>(l_buf + 2 * 2 * kBQ);  // [2][128]: partial max, wait status
+  static_assert((2 * NQ + 2 * NK + 2 * NV + 10) * 8 + 8 <= (int)C::BAR_BYTES, "barrier area");
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
@@ -110,9 +122,11 @@ __global__ void __launch_bounds__(320, 1)
       mbar_init(&q_full[i], 1);
       mbar_init(&q_empty[i], 1);
     }
-    for (int i = 0; i < NS; ++i) {
+    for (int i = 0; i < NK; ++i) {
       mbar_init(&k_full[i], 1);
       mbar_init(&k_empty[i], 1);
+    }
+    for (int i = 0; i < NV; ++i) {
       mbar_init(&v_full[i], 1);
       mbar_init(&v_empty[i], 1);
     }
@@ -120,9 +134,9 @@ __global__ void __launch_bounds__(320, 1)
       mbar_init(&s_full[i], 1);
       mbar_init(&o_full[i], 1);
       mbar_init(&o_empty[i], 4 * 32);
-      mbar_init(&l_full[i], 4 * 32);
+      mbar_init(&l_full[i], kSoftmaxThreads);
     }
-    mbar_init(p_full, 4 * 32);
+    mbar_init(p_full, kSoftmaxThreads);
     mbar_init(pv_done, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -147,7 +161,7 @@ __global__ void __launch_bounds__(320, 1)
     if (lane == 0) {
       // Producer, three cursors issued as their slots free up: Q of an item
       // (with the item's first K tile), K tiles, V^T tiles.  K may run up to
-      // NS tiles ahead of V.
+      // NK tiles ahead of V.
       int k_it = blockIdx.x, k_k = 0, k_j = 0, k_g = 0;  // K cursor: item, item count, tile in item, tile count
       int v_it = blockIdx.x, v_j = 0, v_g = 0;           // V cursor
       unsigned long long t_idle = 0;
@@ -157,9 +171,9 @@ __global__ void __launch_bounds__(320, 1)
         if (k_it < n_items) {
           const TcAttnItem w = items[k_it];
           const int qb = k_k % NQ;
-          const int st = k_g % NS;
+          const int st = k_g % NK;
           const bool q_ok = k_j > 0 || k_k < NQ || mbar_test_wait(&q_empty[qb], ((k_k - NQ) / NQ) & 1);
-          if (q_ok && (k_g < NS || mbar_test_wait(&k_empty[st], ((k_g - NS) / NS) & 1))) {
+          if (q_ok && (k_g < NK || mbar_test_wait(&k_empty[st], ((k_g - NK) / NK) & 1))) {
             const int kvh = (w.head * KVH) / H;
             if (k_j == 0) {
               mbar_arrive_expect_tx(&q_full[qb], C::Q_BYTES);
@@ -183,8 +197,8 @@ __global__ void __launch_bounds__(320, 1)
           }
         }
         {
-          const int st = v_g % NS;
-          if (v_g < k_g && (v_g < NS || mbar_test_wait(&v_empty[st], ((v_g - NS) / NS) & 1))) {
+          const int st = v_g % NV;
+          if (v_g < k_g && (v_g < NV || mbar_test_wait(&v_empty[st], ((v_g - NV) / NV) & 1))) {
             const TcAttnItem w = items[v_it];
             const int kvh = (w.head * KVH) / H;
             mbar_arrive_expect_tx(&v_full[st], C::V_BYTES);
@@ -237,9 +251,9 @@ __global__ void __launch_bounds__(320, 1)
         bool progressed = false;
         if (s_it < n_items && s_g < p_g + 2) {
           const int qb = s_k % NQ;
-          const int st = s_g % NS;
+          const int st = s_g % NK;
           if ((s_j > 0 || mbar_test_wait(&q_full[qb], (s_k / NQ) & 1)) &&
-              mbar_test_wait(&k_full[st], (s_g / NS) & 1)) {
+              mbar_test_wait(&k_full[st], (s_g / NK) & 1)) {
             tc_fence_after();
             const int sb = s_g & 1;  // TMEM S buffer
             const uint32_t qa = smem_u32(sQ + qb * C::Q_BYTES);
@@ -264,10 +278,10 @@ __global__ void __launch_bounds__(320, 1)
           }
         }
         if (p_g < s_g) {
-          const int st = p_g % NS;
+          const int st = p_g % NV;
           const int ob = p_k & 1;  // O buffer of this item
           // the first PV of an item overwrites O[ob]: the epilogue must have read item p_k - 2 from it
-          if (mbar_test_wait(p_full, p_g & 1) && mbar_test_wait(&v_full[st], (p_g / NS) & 1) &&
+          if (mbar_test_wait(p_full, p_g & 1) && mbar_test_wait(&v_full[st], (p_g / NV) & 1) &&
               (p_j > 0 || p_k < 2 || mbar_test_wait(&o_empty[ob], ((p_k - 2) >> 1) & 1))) {
             tc_fence_after();
             const int sb = p_g & 1;  // TMEM buffer holding P
@@ -310,158 +324,199 @@ __global__ void __launch_bounds__(320, 1)
         }
       }
     }
-  } else if (warp < 6) {
-    // softmax warps (2..5): thread = query row = TMEM lane
+  } else if (warp >= 4 && warp < 12) {
+    // softmax warps 4..11: two per TMEM lane quarter (a warp reaches lanes
+    // 32 * (warp % 4) ..); thread = one query row x one half of the tile's
+    // 128 keys (half 0: warps 4..7, half 1: warps 8..11).  The two threads of
+    // a row exchange their partial maxima, so both scale P by the same m,
+    // and keep their own parts of the row sum.
     const int quarter = warp & 3;
+    const int half = (warp - 4) >> 2;
     const int r = quarter * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
     const float sl2 = rsqrtf((float)HD) * kLog2e;
+    constexpr int KH = kBK / 2;  // keys of a tile per thread
+    // Exchange with the row's other thread (named barrier 1 + quarter, the
+    // 64 threads of the two warps).  A failed bounded wait travels with the
+    // value; both threads of every row of both warps then leave together, so
+    // that no thread waits at a barrier its partner has left.  good is kept
+    // uniform over the warp (the tcgen05 loads and stores are warp-wide).
+    auto exchange = [&](float mine, bool& good) -> float {
+      tc_fence_before();
+      m_xchg[half * kBQ + r] = make_float2(mine, good ? 1.f : 0.f);
+      asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory");
+      tc_fence_after();
+      const float2 other = m_xchg[(half ^ 1) * kBQ + r];
+      asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory");  // both have read before either writes again
+      good = __all_sync(0xffffffffu, good && other.y != 0.f);
+      return other.x;
+    };
     int g = 0;  // key tiles of this CTA
     int k = 0;  // items of this CTA
-    bool ok = true;
-    for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ++k) {
+    bool good = true;
+    for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
       const TcAttnItem w = items[it];
       const int ob = k & 1;         // O buffer of this item
       const int qp = w.q_pos0 + r;  // position of this row in its sequence
       float m_used = -INFINITY, l = 0.f;
+      bool stop = false;
       for (int j = 0; j < w.n_kv; ++j, ++g) {
         const int sb = g & 1;
-        if (!mbar_wait(&s_full[sb], (g >> 1) & 1, abort_flag, err)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
+        if (good) good = mbar_wait(&s_full[sb], (g >> 1) & 1, abort_flag, err);
+        good = __all_sync(0xffffffffu, good);
         const uint32_t s_addr = tmem_base + lane_off + static_cast<uint32_t>(sb * kBK);
         const bool diag = j == w.n_kv - 1;
-        const int key0 = kBK * j;
-        // the row's 128 scores into registers: four loads, one wait
-        uint32_t v[kBK];
+        const int key0 = kBK * j + KH * half;
+        uint32_t v[KH];
+        float mx = -INFINITY;
+        if (good) {
+          tc_fence_after();
+          // this half of the row's scores into registers: two loads, one wait
 #pragma unroll
-        for (int c = 0; c < kBK / 32; ++c) tmem_ld_32x32b_x32(s_addr + 32 * c, v + 32 * c);
-        tmem_ld_wait();
-        // row max on the raw scores (the scale is positive); the causal mask
-        // only applies on the diagonal tile (key > query position).  Eight
-        // independent partial maxima: one chain of 128 dependent max
-        // operations would sit in front of every exponential of the tile.
-        if (diag) {
+          for (int c = 0; c < KH / 32; ++c) tmem_ld_32x32b_x32(s_addr + KH * half + 32 * c, v + 32 * c);
+          tmem_ld_wait();
+          // row max on the raw scores (the scale is positive); the causal
+          // mask only applies on the diagonal tile (key > query position).
+          // Independent partial maxima: one chain of dependent max operations
+          // would sit in front of every exponential of the tile.
+          if (diag) {
 #pragma unroll
-          for (int e = 0; e < kBK; ++e)
-            if (key0 + e > qp) v[e] = __float_as_uint(-INFINITY);
+            for (int e = 0; e < KH; ++e)
+              if (key0 + e > qp) v[e] = __float_as_uint(-INFINITY);
+          }
+          float mp[kMaxLanes];
+#pragma unroll
+          for (int i = 0; i < kMaxLanes; ++i) mp[i] = __uint_as_float(v[i]);
+#pragma unroll
+          for (int e = kMaxLanes; e < KH; e += kMaxLanes)
+#pragma unroll
+            for (int i = 0; i < kMaxLanes; ++i) mp[i] = fmaxf(mp[i], __uint_as_float(v[e + i]));
+#pragma unroll
+          for (int w2 = kMaxLanes / 2; w2 > 0; w2 >>= 1)
+#pragma unroll
+            for (int i = 0; i < w2; ++i) mp[i] = fmaxf(mp[i], mp[i + w2]);
+          mx = mp[0];
         }
-        float mp[kMaxLanes];
-#pragma unroll
-        for (int i = 0; i < kMaxLanes; ++i) mp[i] = __uint_as_float(v[i]);
-#pragma unroll
-        for (int e = kMaxLanes; e < kBK; e += kMaxLanes)
-#pragma unroll
-          for (int i = 0; i < kMaxLanes; ++i) mp[i] = fmaxf(mp[i], __uint_as_float(v[e + i]));
-#pragma unroll
-        for (int w2 = kMaxLanes / 2; w2 > 0; w2 >>= 1)
-#pragma unroll
-          for (int i = 0; i < w2; ++i) mp[i] = fmaxf(mp[i], mp[i + w2]);
-        const float mx = mp[0] * sl2;  // in the log2 domain of the exponentials
+        // the other half's maximum; both halves have read their scores
+        // before either writes P over them below
+        const float mo = exchange(mx, good);
+        if (!good) {
+          stop = true;
+          break;
+        }
+        const float mrow = fmaxf(mx, mo) * sl2;  // in the log2 domain of the exponentials
         float alpha = 1.f;
         bool resc = false;
-        if (mx > m_used + kRescaleLog2) {
-          alpha = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - mx);
+        if (mrow > m_used + kRescaleLog2) {
+          alpha = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - mrow);
           l *= alpha;
-          m_used = mx;
+          m_used = mrow;
           resc = j > 0;
         }
-        // P = exp2(s - m) as bf16 pairs, written back over the scores of this
-        // buffer (columns 0..63).  The row sum adds the f32 values before
-        // rounding: the bf16 weights the PV product uses then sum to l within
-        // a relative 2^-9 / sqrt(keys), below the bf16 rounding of the output,
-        // and the softmax saves a widening of every weight.
-        uint32_t pk[kBK / 2];
-        float psum[4] = {0.f, 0.f, 0.f, 0.f};  // four partial sums, for the same reason
+        // P = exp2(s - m) as bf16 pairs, this half's 32 columns of the first
+        // 64 of the buffer.  The row sum adds the f32 values before rounding:
+        // the bf16 weights the PV product uses then sum to l within a relative
+        // 2^-9 / sqrt(keys), below the bf16 rounding of the output.
+        uint32_t pk[KH / 2];
+        float psum[4] = {0.f, 0.f, 0.f, 0.f};  // partial sums, for the same reason as the maxima
 #pragma unroll
-        for (int e = 0; e < kBK; e += 2) {
+        for (int e = 0; e < KH; e += 2) {
           const float p0 = ex2_approx(fmaf(__uint_as_float(v[e]), sl2, -m_used));
           const float p1 = ex2_approx(fmaf(__uint_as_float(v[e + 1]), sl2, -m_used));
           pk[e >> 1] = pack_bf16x2(p0, p1);
           psum[(e >> 1) & 3] += p0 + p1;
         }
         const float ps = (psum[0] + psum[1]) + (psum[2] + psum[3]);
-        tmem_st_32x32b_x32(s_addr, pk);
-        tmem_st_32x32b_x32(s_addr + 32, pk + 32);
-        // the previous PV must be complete before this tile's P is released (the
-        // PV barrier then never runs two phases ahead of this thread) and
-        // before O is rescaled
-        if (j > 0 && !mbar_wait(pv_done, (g - 1) & 1, abort_flag, err)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, resc)) {
-          // rare: 32 columns at a time
-          const float a = resc ? alpha : 1.f;
+        tmem_st_32x32b_x32(s_addr + (KH / 2) * half, pk);
+        // The previous PV (of this item, or the last of the previous one) must
+        // be complete before this tile's P is released, and before O is
+        // rescaled.  Every release waits for it, the first tile of an item
+        // too: no thread's arrival for tile g can then reach the P barrier
+        // before every thread's arrival for tile g - 1 (which the PV of g - 1
+        // needs), and the PV barrier never runs two phases ahead of a thread.
+        if (g > 0) good = __all_sync(0xffffffffu, mbar_wait(pv_done, (g - 1) & 1, abort_flag, err));
+        if (good) {
+          tc_fence_after();
+          if (__any_sync(0xffffffffu, resc)) {
+            // rare: this half's hd / 2 columns of O, 32 at a time
+            const float a = resc ? alpha : 1.f;
 #pragma unroll 1
-          for (int c = 0; c < HD / 32; ++c) {
-            uint32_t o[32];
-            const uint32_t o_addr = tmem_base + lane_off + C::O_COL + ob * HD + 32 * c;
-            tmem_ld_32x32b_x32(o_addr, o);
-            tmem_ld_wait();
+            for (int c = 0; c < HD / 64; ++c) {
+              uint32_t o[32];
+              const uint32_t o_addr = tmem_base + lane_off + C::O_COL + ob * HD + (HD / 2) * half + 32 * c;
+              tmem_ld_32x32b_x32(o_addr, o);
+              tmem_ld_wait();
 #pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * a);
-            tmem_st_32x32b_x32(o_addr, o);
+              for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * a);
+              tmem_st_32x32b_x32(o_addr, o);
+            }
           }
+          tmem_st_wait();
+          l += ps;
+          tc_fence_before();
+          mbar_arrive(p_full);
         }
-        tmem_st_wait();
-        l += ps;
-        tc_fence_before();
-        mbar_arrive(p_full);
       }
-      if (!ok) break;
-      // end of the item: the row sums go to the epilogue warps once they have
-      // taken item k - 2's from this buffer
-      if (k >= 2 && !mbar_wait(&o_empty[ob], ((k - 2) >> 1) & 1, abort_flag, err)) break;
-      l_buf[ob * kBQ + r] = l;
-      mbar_arrive(&l_full[ob]);
+      if (stop) break;  // both halves, at the same exchange
+      // end of the item: this half's row sum goes to the epilogue warps once
+      // they have taken item k - 2's from this buffer (a failed wait reaches
+      // the partner with the next item's first exchange)
+      if (good && k >= 2) good = __all_sync(0xffffffffu, mbar_wait(&o_empty[ob], ((k - 2) >> 1) & 1, abort_flag, err));
+      if (good) {
+        l_buf[(ob * 2 + half) * kBQ + r] = l;
+        mbar_arrive(&l_full[ob]);
+      }
     }
-  } else {
-    // epilogue warps (6..9): O[k & 1] / l (x gate) as bf16, one query row per thread,
-    // while the softmax warps run the next item
+  } else if (warp >= 12) {
+    // epilogue warps 12..15: O[k & 1] / l (x gate) as bf16, one query row per
+    // thread, while the softmax warps run the next item
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    constexpr int CP = HD < 64 ? HD : 64;  // columns per pass
     int k = 0;
     for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
       const int ob = k & 1;
-      if (!mbar_wait(&o_full[ob], (k >> 1) & 1, abort_flag, err)) break;
-      if (!mbar_wait(&l_full[ob], (k >> 1) & 1, abort_flag, err)) break;
+      bool good = mbar_wait(&o_full[ob], (k >> 1) & 1, abort_flag, err);
+      good = good && mbar_wait(&l_full[ob], (k >> 1) & 1, abort_flag, err);
+      if (!__all_sync(0xffffffffu, good)) break;
       tc_fence_after();
       const TcAttnItem w = items[it];
-      const float inv = 1.f / l_buf[ob * kBQ + r];
-      uint32_t ov[HD];
+      const float inv = 1.f / (l_buf[(ob * 2) * kBQ + r] + l_buf[(ob * 2 + 1) * kBQ + r]);
+      bf16* orow = out + (long long)(w.q_start + r) * H * HD + w.head * HD;
+      const bf16* grow = gate ? gate + (long long)(w.q_start + r) * H * HD + w.head * HD : nullptr;
+#pragma unroll 1
+      for (int c0 = 0; c0 < HD; c0 += CP) {
+        uint32_t ov[CP];
 #pragma unroll
-      for (int c = 0; c < HD / 32; ++c)
-        tmem_ld_32x32b_x32(tmem_base + lane_off + C::O_COL + ob * HD + 32 * c, ov + 32 * c);
-      tmem_ld_wait();
-      tc_fence_before();
-      mbar_arrive(&o_empty[ob]);
-      if (r < w.q_len) {
-        bf16* orow = out + (long long)(w.q_start + r) * H * HD + w.head * HD;
-        const bf16* grow = gate ? gate + (long long)(w.q_start + r) * H * HD + w.head * HD : nullptr;
+        for (int c = 0; c < CP / 32; ++c)
+          tmem_ld_32x32b_x32(tmem_base + lane_off + C::O_COL + ob * HD + c0 + 32 * c, ov + 32 * c);
+        tmem_ld_wait();
+        if (c0 + CP == HD) {  // all of O (and l) read: the buffer is free
+          tc_fence_before();
+          mbar_arrive(&o_empty[ob]);
+        }
+        if (r < w.q_len) {
 #pragma unroll
-        for (int c = 0; c < HD / 8; ++c) {
-          const uint32_t* v = ov + 8 * c;
-          float f[8];
+          for (int c = 0; c < CP / 8; ++c) {
+            const uint32_t* v = ov + 8 * c;
+            float f[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) f[e] = __uint_as_float(v[e]) * inv;
-          if (grow) {
-            const uint4 gq = *reinterpret_cast<const uint4*>(grow + 8 * c);
-            const __nv_bfloat162* gh = reinterpret_cast<const __nv_bfloat162*>(&gq);
+            for (int e = 0; e < 8; ++e) f[e] = __uint_as_float(v[e]) * inv;
+            if (grow) {
+              const uint4 gq = *reinterpret_cast<const uint4*>(grow + c0 + 8 * c);
+              const __nv_bfloat162* gh = reinterpret_cast<const __nv_bfloat162*>(&gq);
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 gf = __bfloat1622float2(gh[e]);
-              f[2 * e] *= gf.x;
-              f[2 * e + 1] *= gf.y;
+              for (int e = 0; e < 4; ++e) {
+                const float2 gf = __bfloat1622float2(gh[e]);
+                f[2 * e] *= gf.x;
+                f[2 * e + 1] *= gf.y;
+              }
             }
+            *reinterpret_cast<uint4*>(orow + c0 + 8 * c) =
+                make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]), pack_bf16x2(f[4], f[5]),
+                           pack_bf16x2(f[6], f[7]));
           }
-          *reinterpret_cast<uint4*>(orow + 8 * c) =
-              make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]), pack_bf16x2(f[4], f[5]),
-                         pack_bf16x2(f[6], f[7]));
         }
       }
     }
@@ -541,7 +596,7 @@ cudaError_t launch_tc(const CUtensorMap& q_map, const CUtensorMap& k_map, const 
     attr = true;
   }
   const int grid = n_items < num_sms ? n_items : num_sms;
-  OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_tc<HD>, dim3(grid), dim3(320), C::SMEM, stream, q_map, k_map, vt_map,
+  OUTLETS_TRY_LAUNCH(launch_k(k_attn_prefill_tc<HD>, dim3(grid), dim3(kThreads), C::SMEM, stream, q_map, k_map, vt_map,
                               items, n_items, kv_ld, H, KVH, reinterpret_cast<bf16*>(out),
                               reinterpret_cast<const bf16*>(gate), err));
   return cudaGetLastError();

@@ -41,7 +41,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;              // tolerated growth of a row max before O is rescaled
 constexpr unsigned kPollSleepNs = 32;            // back-off of the polling roles when nothing is ready
 constexpr int kMaxLanes = 8;                     // independent partial maxima of a score row
-constexpr int kThreads = 512;                    // producer, MMA, 2 idle, 8 softmax, 4 epilogue warps
+constexpr int kThreads = 512;                    // producer, S issuer, idle, PV issuer, 8 softmax, 4 epilogue warps
 constexpr int kSoftmaxThreads = 8 * 32;
 
 // 2^x with the hardware approximation (ex2.approx.ftz: -inf -> 0); the result
@@ -109,11 +109,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* o_full = pv_done + 1;   // [2] last PV of the item complete
   uint64_t* o_empty = o_full + 2;   // [2] the epilogue has read O and l
   uint64_t* l_full = o_empty + 2;   // [2] the softmax has written the row sums
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(l_full + 2);
+  // PV_n complete, for the S issuer (S_{n+2} overwrites the buffer P_n is read
+  // from): two barriers, n & 1, so that neither runs two phases ahead of it
+  uint64_t* pv_free = l_full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pv_free + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* l_buf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(q_full) + C::BAR_BYTES);  // [2][2][128]
   float2* m_xchg = reinterpret_cast<float2*>(l_buf + 2 * 2 * kBQ);  // [2][128]: partial max, wait status
-  static_assert((2 * NQ + 2 * NK + 2 * NV + 10) * 8 + 8 <= (int)C::BAR_BYTES, "barrier area");
+  static_assert((2 * NQ + 2 * NK + 2 * NV + 12) * 8 + 8 <= (int)C::BAR_BYTES, "barrier area");
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
@@ -135,6 +138,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&o_full[i], 1);
       mbar_init(&o_empty[i], 4 * 32);
       mbar_init(&l_full[i], kSoftmaxThreads);
+      mbar_init(&pv_free[i], 1);
     }
     mbar_init(p_full, kSoftmaxThreads);
     mbar_init(pv_done, 1);
@@ -235,93 +239,72 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      // MMA issuer, two cursors issued as their inputs arrive: S_n = Q K_n^T
-      // (needs the item's Q, K tile n, and TMEM buffer n & 1 free: PV_{n-2}
-      // issued, since the tensor pipe runs in order) and PV_n = P_n V_n (needs
-      // the softmax's P_n and V tile n).  Neither waits for the other's inputs.
+      // S issuer: S_n = Q K_n^T (M=128 N=128 K=hd) into TMEM buffer n & 1, as
+      // soon as the item's Q, K tile n and the buffer are there (the PV that
+      // read P_{n-2} from it complete).  The PV issuer is another thread: the
+      // issue of an MMA blocks while the pipe's short queue is full, and a PV
+      // the softmax waits for does not queue behind the issue of an S.
       constexpr uint32_t id_s = idesc_bf16_f32(kBQ, kBK);
+      int g = 0;  // key tiles of this CTA
+      int k = 0;  // items of this CTA
+      for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
+        const int nkv = items[it].n_kv;
+        const int qb = k % NQ;
+        bool ok = mbar_wait(&q_full[qb], (k / NQ) & 1, abort_flag, err);
+        for (int j = 0; ok && j < nkv; ++j, ++g) {
+          const int st = g % NK;
+          const int sb = g & 1;
+          ok = mbar_wait(&k_full[st], (g / NK) & 1, abort_flag, err) &&
+               (g < 2 || mbar_wait(&pv_free[sb], ((g - 2) >> 1) & 1, abort_flag, err));
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t qa = smem_u32(sQ + qb * C::Q_BYTES);
+          const uint32_t ka = smem_u32(sK + st * C::K_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * (128 * 128);
+            tc_mma_bf16(tmem_base + sb * kBK, sw128_kmajor_desc(qa + off) + 2u * (kk & 3),
+                        sw128_kmajor_desc(ka + off) + 2u * (kk & 3), id_s, kk > 0 ? 1u : 0u);
+          }
+          tc_commit(&s_full[sb]);
+          tc_commit(&k_empty[st]);                      // S_n has read its K tile
+          if (j == nkv - 1) tc_commit(&q_empty[qb]);  // last S of the item: its Q buffer is free
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (warp == 3) {
+    if (lane == 0) {
+      // PV issuer: O[item & 1] += P_n V_n (M=128 N=hd K=128, A = P in TMEM)
+      // once the softmax has released P_n and V tile n is there; the first PV
+      // of an item overwrites O[k & 1], which the epilogue must have read
+      // (item k - 2)
       constexpr uint32_t id_o = idesc_bf16_f32(kBQ, HD);
-      int s_it = blockIdx.x, s_k = 0, s_j = 0, s_g = 0;
-      int s_nkv = s_it < n_items ? items[s_it].n_kv : 0;
-      int p_it = blockIdx.x, p_k = 0, p_j = 0, p_g = 0;
-      int p_nkv = p_it < n_items ? items[p_it].n_kv : 0;
-      unsigned long long t_idle = 0;
-      uint32_t spin = 0;
-      while (p_it < n_items) {
-        bool progressed = false;
-        if (s_it < n_items && s_g < p_g + 2) {
-          const int qb = s_k % NQ;
-          const int st = s_g % NK;
-          if ((s_j > 0 || mbar_test_wait(&q_full[qb], (s_k / NQ) & 1)) &&
-              mbar_test_wait(&k_full[st], (s_g / NK) & 1)) {
-            tc_fence_after();
-            const int sb = s_g & 1;  // TMEM S buffer
-            const uint32_t qa = smem_u32(sQ + qb * C::Q_BYTES);
-            const uint32_t ka = smem_u32(sK + st * C::K_BYTES);
+      int g = 0;
+      int k = 0;
+      for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
+        const int nkv = items[it].n_kv;
+        const int ob = k & 1;
+        bool ok = k < 2 || mbar_wait(&o_empty[ob], ((k - 2) >> 1) & 1, abort_flag, err);
+        for (int j = 0; ok && j < nkv; ++j, ++g) {
+          const int st = g % NV;
+          const int sb = g & 1;  // TMEM buffer holding P
+          ok = mbar_wait(p_full, g & 1, abort_flag, err) && mbar_wait(&v_full[st], (g / NV) & 1, abort_flag, err);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t va = smem_u32(sV + st * C::V_BYTES);
+          // A = P in TMEM (the S buffer it was computed in: 16 keys = 8 columns per MMA)
 #pragma unroll
-            for (int kk = 0; kk < HD / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * (128 * 128);
-              tc_mma_bf16(tmem_base + sb * kBK, sw128_kmajor_desc(qa + off) + 2u * (kk & 3),
-                          sw128_kmajor_desc(ka + off) + 2u * (kk & 3), id_s, kk > 0 ? 1u : 0u);
-            }
-            tc_commit(&s_full[sb]);
-            tc_commit(&k_empty[st]);                          // S_n has read its K tile
-            if (s_j == s_nkv - 1) tc_commit(&q_empty[qb]);  // last S of the item: its Q buffer is free
-            ++s_g;
-            if (++s_j == s_nkv) {
-              s_j = 0;
-              ++s_k;
-              s_it += gridDim.x;
-              s_nkv = s_it < n_items ? items[s_it].n_kv : 0;
-            }
-            progressed = true;
-          }
+          for (int kk = 0; kk < kBK / 16; ++kk)
+            tc_mma_bf16_ta(tmem_base + C::O_COL + ob * HD, tmem_base + sb * kBK + 8 * kk,
+                           sw128_kmajor_desc(va + (kk >> 2) * (HD * 128)) + 2u * (kk & 3), id_o,
+                           (j > 0 || kk > 0) ? 1u : 0u);
+          tc_commit(pv_done);
+          tc_commit(&pv_free[sb]);
+          tc_commit(&v_empty[st]);                   // PV_n has read its V tile
+          if (j == nkv - 1) tc_commit(&o_full[ob]);  // the item's O is complete
         }
-        if (p_g < s_g) {
-          const int st = p_g % NV;
-          const int ob = p_k & 1;  // O buffer of this item
-          // the first PV of an item overwrites O[ob]: the epilogue must have read item p_k - 2 from it
-          if (mbar_test_wait(p_full, p_g & 1) && mbar_test_wait(&v_full[st], (p_g / NV) & 1) &&
-              (p_j > 0 || p_k < 2 || mbar_test_wait(&o_empty[ob], ((p_k - 2) >> 1) & 1))) {
-            tc_fence_after();
-            const int sb = p_g & 1;  // TMEM buffer holding P
-            const uint32_t va = smem_u32(sV + st * C::V_BYTES);
-            // A = P in TMEM (the S buffer it was computed in: 16 keys = 8 columns per MMA)
-#pragma unroll
-            for (int kk = 0; kk < kBK / 16; ++kk)
-              tc_mma_bf16_ta(tmem_base + C::O_COL + ob * HD, tmem_base + sb * kBK + 8 * kk,
-                             sw128_kmajor_desc(va + (kk >> 2) * (HD * 128)) + 2u * (kk & 3), id_o,
-                             (p_j > 0 || kk > 0) ? 1u : 0u);
-            tc_commit(pv_done);
-            tc_commit(&v_empty[st]);  // PV_n has read its V tile
-            if (p_j == p_nkv - 1) tc_commit(&o_full[ob]);  // the item's O is complete
-            ++p_g;
-            if (++p_j == p_nkv) {
-              p_j = 0;
-              ++p_k;
-              p_it += gridDim.x;
-              p_nkv = p_it < n_items ? items[p_it].n_kv : 0;
-            }
-            progressed = true;
-          }
-        }
-        if (progressed) {
-          spin = 0;
-          t_idle = 0;
-          continue;
-        }
-        __nanosleep(kPollSleepNs);  // leave the issue slots to the softmax warps sharing this SM sub-partition
-        if ((++spin & 31u) == 0) {  // bounded, like every other wait
-          if (*abort_flag) break;
-          const unsigned long long now = global_timer_ns();
-          if (t_idle == 0) {
-            t_idle = now;
-          } else if (now - t_idle > kWaitTimeoutNs) {
-            *abort_flag = 1;
-            if (err) atomicOr(err, ERR_TIMEOUT);
-            break;
-          }
-        }
+        if (!ok) break;
       }
     }
   } else if (warp >= 4 && warp < 12) {

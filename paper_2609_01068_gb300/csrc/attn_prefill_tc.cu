@@ -58,9 +58,9 @@ struct TcAttnCfg {
   static constexpr uint32_t Q_BYTES = kBQ * HD * 2;    // [NB][128 rows][64]
   static constexpr uint32_t K_BYTES = kBK * HD * 2;    // [NB][128 keys][64]
   static constexpr uint32_t V_BYTES = HD * kBK * 2;    // V^T: [2][hd rows][64 keys]
-  // Q buffers and K/V stages share the 227 KB: K/V latency wants stages, and a
-  // second Q buffer only hides the Q load between items
-  static constexpr int NQ = HD >= 128 ? 1 : 2;
+  // Q buffers and K/V stages share the 227 KB; a second Q buffer lets the
+  // first S of an item start while the previous item's last S runs
+  static constexpr int NQ = 2;
   static constexpr uint32_t BAR_BYTES = 512;          // mbarriers, TMEM address, abort flag
   static constexpr uint32_t L_BYTES = 2 * 2 * kBQ * 4;  // row sums: [O buffer][half of the keys][row]
   static constexpr uint32_t X_BYTES = 2 * kBQ * 8;      // row max exchange: [half of the keys][row] x (max, ok)
@@ -73,7 +73,7 @@ struct TcAttnCfg {
   static constexpr int NK = (NV < 6 && KV_BUDGET - NV * (K_BYTES + V_BYTES) >= K_BYTES) ? NV + 1 : NV;
   static constexpr size_t SMEM =
       1024 + NQ * Q_BYTES + NK * K_BYTES + NV * V_BYTES + BAR_BYTES + L_BYTES + X_BYTES;
-  static_assert(NV >= 2 && NK >= 3, "K/V stages");
+  static_assert(NV >= 2 && NK >= 2, "K/V stages");
   // TMEM: S0 [0,128), S1 [128,256), O0 [256, 256+hd), O1 [256+hd, 256+2hd)
   static constexpr uint32_t O_COL = 2 * kBK;
   static_assert(O_COL + 2 * HD <= 512, "TMEM columns");

@@ -243,6 +243,18 @@ def prefill_flops(shape, lengths, n_out, gated=False, embed=False, whole_layer=T
     return per_tok * T + per_row * n_out + attn + head
 
 
+def attention_roofline(shape, lengths, ms, peaks):
+    """Rate of the causal prefill attention over its stage (the V^T transpose
+    and k_attn_prefill_tc, CUDA events around them): 4 H hd sum L(L+1)/2 FLOP."""
+    flop = 4 * shape.n_heads * shape.head_dim * float(np.sum(np.asarray(lengths, dtype=np.float64)
+                                                             * (np.asarray(lengths, dtype=np.float64) + 1) / 2))
+    tf = flop / (ms / 1e3) / 1e12
+    return {"bound": "tensor", "kernel": "k_attn_prefill_tc (stage incl. the V^T transpose)",
+            "flop_per_pass": flop, "ms_per_pass": ms, "achieved": tf, "unit": "TFLOP/s",
+            "frac_of_burst": tf / peaks["bf16"], "frac_of_sustained": tf / peaks["bf16_sus"],
+            "peaks": f"bf16 burst {peaks['bf16']} / sustained {peaks['bf16_sus']} {peaks['src']}"}
+
+
 def cpu_threads():
     try:
         from threadpoolctl import threadpool_info
@@ -603,6 +615,8 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
         wprof = pred.profile_read()
         pred.profile(False)
         whole["stages"] = {k: v[0] / 2 for k, v in wprof.items() if v[1]}
+        if "attention" in whole["stages"]:
+            whole["attention_roofline"] = attention_roofline(shape, lengths, whole["stages"]["attention"], peaks)
     # per-stage breakdown in a separate (untimed) pass: stage events serialize the kernels
     pred.profile(True)
     for _ in range(3):
@@ -653,6 +667,8 @@ def run_prefill_mode(args, pred, shape, w, taps, taps_d, lengths, cu, peaks, wor
            "tensor_peak_frac_step": flops * args.steps / (ms / 1e3) / 1e12 / roofline["peak"],
            "roofline": roofline, "stages": stages, "clocks": clocks, "e2e": e2e,
            "gpu_launches": launches}
+    if not pruned_rows and "attention" in stages:
+        out["attention_roofline"] = attention_roofline(shape, lengths, stages["attention"]["ms_per_step"], peaks)
     out["config"]["layer_rows"] = ("keys/values for every prompt row; queries, attention, O, MLP, final norm and "
                                    "head for each prompt's last row" if pruned_rows else "whole layer on every row")
     if whole:

@@ -271,6 +271,32 @@ def test_chunked_host_taps_match_device_taps():
     check_z_len(z_h[last], l_h[last], ref["z"], ref["length"], "bf16", "chunked host taps")
 
 
+def test_wave_aligned_tap_chunks_match_device_taps():
+    """A large call's host taps in chunks of whole FC waves (9 728 rows at
+    d = 1024, 256 x 256 tiles over 152 SMs): T = 21 957 gives chunks starting
+    at 0, 9 728 and 19 456, the last one partial and boundaries inside
+    sequences. Every prediction and draft state must be identical to the same
+    call on device taps."""
+    from paper_2609_01068_gb300 import outlets as OT
+    shape = MID128
+    pred, w = predictor("mid128", max_tokens=24576)
+    lengths = [8000, 7000, 6000, 957]
+    cu = synth.cu_seqlens(lengths)
+    T = int(cu[-1])
+    taps = _taps(shape, T, off=17)
+    dev = [to_device(t, "bf16") for t in taps]
+    z_d, l_d = pred.prefill(dev, cu, all_tokens=True)
+    h_d = to_np(pred.intermediate(OT.T_HDRAFT)).copy()
+    host = [t.cpu().pin_memory() for t in dev]
+    z_h = torch.empty(T, dtype=torch.float32).pin_memory()
+    l_h = torch.empty(T, dtype=torch.float32).pin_memory()
+    pred.prefill(host, cu, all_tokens=True, z_out=z_h, len_out=l_h)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(z_h.numpy(), z_d.cpu().numpy())
+    np.testing.assert_array_equal(l_h.numpy(), l_d.cpu().numpy())
+    np.testing.assert_array_equal(to_np(pred.intermediate(OT.T_HDRAFT)), h_d)
+
+
 def test_argument_errors_change_nothing():
     from paper_2609_01068_gb300 import outlets as OT
     shape = MID128

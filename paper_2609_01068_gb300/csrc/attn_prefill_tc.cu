@@ -3,20 +3,23 @@
 // o = softmax(q k^T / sqrt(hd) + causal mask) v per packed sequence, q-head h
 // reading kv-head floor(h * KVH / H), optionally gated (o * gate).
 //
-// Persistent kernel, one CTA per SM, 16 warps.  A work item is one 128-row
+// Persistent kernel, one CTA per SM, 8 + 4 kParts warps.  A work item is one 128-row
 // query tile of one sequence x one query head; items are taken longest first
 // (most key tiles) with a grid stride.
 //   warp 0       TMA producer: Q tile (one or two buffers), K tiles and V^T
 //                tiles of 128 keys in rings of their own (a K stage is freed
 //                by its S, a V stage by its PV), continuously across items
-//   warp 1       TMEM owner and single-thread MMA issuer, polling two streams:
+//   warp 1       TMEM owner; one thread issues the S MMAs
 //                  S_j = Q K_j^T     M=128 N=128 K=hd, into one of two TMEM S buffers
+//                as soon as their inputs are there (S_{j+2} once PV_j has
+//                completed), so the next scores are computed while the
+//                softmax of this tile runs
+//   warp 3       one thread issues the PV MMAs
 //                  O  += P_j V_j     M=128 N=hd K=128, into O[item & 1] in TMEM
-//                S_{j+1} is issued as soon as its inputs are there, so the
-//                next scores are computed while the softmax of this tile runs
-//   warps 4..11  softmax, two threads per query row (TMEM lane), each over
-//                half of the tile's keys: the scores are read from TMEM once
-//                into registers; the two halves exchange their maxima of the
+//                as soon as the softmax releases P_j
+//   warps 4..    softmax, kParts threads per query row (TMEM lane), each
+//                over a part of the tile's keys: the scores are read from TMEM
+//                once into registers; the parts exchange their maxima of the
 //                masked raw scores through shared memory; P = exp2(s - m) is
 //                written as bf16 pairs back into the S buffer it came from
 //                (the PV MMA reads its A operand from TMEM, so P is
@@ -24,7 +27,7 @@
 //                next tile); O and l are rescaled in place only when a row max
 //                grows by more than 2^8 over the one in use (the result is
 //                exact either way)
-//   warps 12..15 epilogue: O / l (x gate) of item k as bf16 from O[k & 1],
+//   last 4 warps epilogue: O / l (x gate) of item k as bf16 from O[k & 1],
 //                while the softmax and the MMAs run item k + 1
 // V is read through a transposed copy V^T [KVH*hd, columns] (keys contiguous)
 // so both MMAs take K-major operands; each sequence starts at a column that is
@@ -41,8 +44,26 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;              // tolerated growth of a row max before O is rescaled
 constexpr unsigned kPollSleepNs = 32;            // back-off of the polling roles when nothing is ready
 constexpr int kMaxLanes = 8;                     // independent partial maxima of a score row
-constexpr int kThreads = 512;                    // producer, S issuer, idle, PV issuer, 8 softmax, 4 epilogue warps
-constexpr int kSoftmaxThreads = 8 * 32;
+// Threads of a query row in the softmax (each over kBK / kParts keys of a tile)
+#ifndef OUTLETS_ATTN_PARTS
+#define OUTLETS_ATTN_PARTS 2
+#endif
+constexpr int kParts = OUTLETS_ATTN_PARTS;
+static_assert(kParts == 2 || kParts == 4, "softmax parts of a row");
+constexpr int kSoftmaxWarps = 4 * kParts;
+constexpr int kEpiWarp0 = 4 + kSoftmaxWarps;    // first epilogue warp
+// producer, S issuer, idle, PV issuer, the softmax warps, 4 epilogue warps
+constexpr int kThreads = 32 * (4 + kSoftmaxWarps + 4);
+constexpr int kSoftmaxThreads = 32 * kSoftmaxWarps;
+
+__device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};"
+      ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
 
 // 2^x with the hardware approximation (ex2.approx.ftz: -inf -> 0); the result
 // is rounded to bf16 or divided out by the row sum, far coarser than its error.
@@ -62,8 +83,8 @@ struct TcAttnCfg {
   // first S of an item start while the previous item's last S runs
   static constexpr int NQ = 2;
   static constexpr uint32_t BAR_BYTES = 512;          // mbarriers, TMEM address, abort flag
-  static constexpr uint32_t L_BYTES = 2 * 2 * kBQ * 4;  // row sums: [O buffer][half of the keys][row]
-  static constexpr uint32_t X_BYTES = 2 * kBQ * 8;      // row max exchange: [half of the keys][row] x (max, ok)
+  static constexpr uint32_t L_BYTES = 2 * kParts * kBQ * 4;  // row sums: [O buffer][part of the keys][row]
+  static constexpr uint32_t X_BYTES = kParts * kBQ * 8;      // row max exchange: [part of the keys][row] x (max, ok)
   // K and V^T stages in what is left: as many of each as fit, one more K
   // stage where it fits (a K stage is held from its load to its S, a V
   // stage from its load to its PV, later)
@@ -114,8 +135,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* pv_free = l_full + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pv_free + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float* l_buf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(q_full) + C::BAR_BYTES);  // [2][2][128]
-  float2* m_xchg = reinterpret_cast<float2*>(l_buf + 2 * 2 * kBQ);  // [2][128]: partial max, wait status
+  float* l_buf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(q_full) + C::BAR_BYTES);  // [2][kParts][128]
+  float2* m_xchg = reinterpret_cast<float2*>(l_buf + 2 * kParts * kBQ);  // [kParts][128]: partial max, wait status
   static_assert((2 * NQ + 2 * NK + 2 * NV + 12) * 8 + 8 <= (int)C::BAR_BYTES, "barrier area");
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -307,32 +328,40 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
       }
     }
-  } else if (warp >= 4 && warp < 12) {
-    // softmax warps 4..11: two per TMEM lane quarter (a warp reaches lanes
-    // 32 * (warp % 4) ..); thread = one query row x one half of the tile's
-    // 128 keys (half 0: warps 4..7, half 1: warps 8..11).  The two threads of
-    // a row exchange their partial maxima, so both scale P by the same m,
-    // and keep their own parts of the row sum.
+  } else if (warp >= 4 && warp < kEpiWarp0) {
+    // softmax warps 4 .. 4 + 4 kParts - 1: kParts per TMEM lane quarter (a
+    // warp reaches lanes 32 * (warp % 4) ..); thread = one query row x one
+    // part of the tile's 128 keys (part p: warps 4 + 4p .. 7 + 4p).  The
+    // threads of a row exchange their partial maxima, so all scale P by the
+    // same m, and keep their own parts of the row sum.
     const int quarter = warp & 3;
-    const int half = (warp - 4) >> 2;
+    const int part = (warp - 4) >> 2;
     const int r = quarter * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
     const float sl2 = rsqrtf((float)HD) * kLog2e;
-    constexpr int KH = kBK / 2;  // keys of a tile per thread
-    // Exchange with the row's other thread (named barrier 1 + quarter, the
-    // 64 threads of the two warps).  A failed bounded wait travels with the
-    // value; both threads of every row of both warps then leave together, so
-    // that no thread waits at a barrier its partner has left.  good is kept
-    // uniform over the warp (the tcgen05 loads and stores are warp-wide).
+    constexpr int KH = kBK / kParts;  // keys of a tile per thread
+    // Exchange with the row's other threads (named barrier 1 + quarter, the
+    // 32 kParts threads of the quarter's warps): the row max over all parts.
+    // A failed bounded wait travels with the value; all threads of every row
+    // then leave together, so that no thread waits at a barrier a partner
+    // has left.  good is kept uniform over the warp (the tcgen05 loads and
+    // stores are warp-wide).
     auto exchange = [&](float mine, bool& good) -> float {
       tc_fence_before();
-      m_xchg[half * kBQ + r] = make_float2(mine, good ? 1.f : 0.f);
-      asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory");
+      m_xchg[part * kBQ + r] = make_float2(mine, good ? 1.f : 0.f);
+      asm volatile("bar.sync %0, %1;" ::"r"(1 + quarter), "r"(32 * kParts) : "memory");
       tc_fence_after();
-      const float2 other = m_xchg[(half ^ 1) * kBQ + r];
-      asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory");  // both have read before either writes again
-      good = __all_sync(0xffffffffu, good && other.y != 0.f);
-      return other.x;
+      float m = mine;
+      bool all_ok = good;
+#pragma unroll
+      for (int q = 0; q < kParts; ++q) {
+        const float2 other = m_xchg[q * kBQ + r];
+        m = fmaxf(m, other.x);
+        all_ok = all_ok && other.y != 0.f;
+      }
+      asm volatile("bar.sync %0, %1;" ::"r"(1 + quarter), "r"(32 * kParts) : "memory");  // all have read before any writes again
+      good = __all_sync(0xffffffffu, all_ok);
+      return m;
     };
     int g = 0;  // key tiles of this CTA
     int k = 0;  // items of this CTA
@@ -349,14 +378,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         good = __all_sync(0xffffffffu, good);
         const uint32_t s_addr = tmem_base + lane_off + static_cast<uint32_t>(sb * kBK);
         const bool diag = j == w.n_kv - 1;
-        const int key0 = kBK * j + KH * half;
+        const int key0 = kBK * j + KH * part;
         uint32_t v[KH];
         float mx = -INFINITY;
         if (good) {
           tc_fence_after();
-          // this half of the row's scores into registers: two loads, one wait
+          // this part of the row's scores into registers: KH / 32 loads, one wait
 #pragma unroll
-          for (int c = 0; c < KH / 32; ++c) tmem_ld_32x32b_x32(s_addr + KH * half + 32 * c, v + 32 * c);
+          for (int c = 0; c < KH / 32; ++c) tmem_ld_32x32b_x32(s_addr + KH * part + 32 * c, v + 32 * c);
           tmem_ld_wait();
           // row max on the raw scores (the scale is positive); the causal
           // mask only applies on the diagonal tile (key > query position).
@@ -380,14 +409,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < w2; ++i) mp[i] = fmaxf(mp[i], mp[i + w2]);
           mx = mp[0];
         }
-        // the other half's maximum; both halves have read their scores
-        // before either writes P over them below
+        // the row max over all parts; every part has read its scores before
+        // any writes P over them below
         const float mo = exchange(mx, good);
         if (!good) {
           stop = true;
           break;
         }
-        const float mrow = fmaxf(mx, mo) * sl2;  // in the log2 domain of the exponentials
+        const float mrow = mo * sl2;  // in the log2 domain of the exponentials
         float alpha = 1.f;
         bool resc = false;
         if (mrow > m_used + kRescaleLog2) {
@@ -396,8 +425,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           m_used = mrow;
           resc = j > 0;
         }
-        // P = exp2(s - m) as bf16 pairs, this half's 32 columns of the first
-        // 64 of the buffer.  The row sum adds the f32 values before rounding:
+        // P = exp2(s - m) as bf16 pairs, this part's KH / 2 columns of the
+        // first 64 of the buffer.  The row sum adds the f32 values before rounding:
         // the bf16 weights the PV product uses then sum to l within a relative
         // 2^-9 / sqrt(keys), below the bf16 rounding of the output.
         uint32_t pk[KH / 2];
@@ -410,7 +439,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           psum[(e >> 1) & 3] += p0 + p1;
         }
         const float ps = (psum[0] + psum[1]) + (psum[2] + psum[3]);
-        tmem_st_32x32b_x32(s_addr + (KH / 2) * half, pk);
+        if constexpr (KH / 2 == 32) {
+          tmem_st_32x32b_x32(s_addr + (KH / 2) * part, pk);
+        } else {
+          tmem_st_32x32b_x16(s_addr + (KH / 2) * part, pk);
+        }
         // The previous PV (of this item, or the last of the previous one) must
         // be complete before this tile's P is released, and before O is
         // rescaled.  Every release waits for it, the first tile of an item
@@ -421,12 +454,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (good) {
           tc_fence_after();
           if (__any_sync(0xffffffffu, resc)) {
-            // rare: this half's hd / 2 columns of O, 32 at a time
+            // rare: this part's hd / kParts columns of O (whole 32-column
+            // chunks, over the parts in turn)
             const float a = resc ? alpha : 1.f;
 #pragma unroll 1
-            for (int c = 0; c < HD / 64; ++c) {
+            for (int c = part; c < HD / 32; c += kParts) {
               uint32_t o[32];
-              const uint32_t o_addr = tmem_base + lane_off + C::O_COL + ob * HD + (HD / 2) * half + 32 * c;
+              const uint32_t o_addr = tmem_base + lane_off + C::O_COL + ob * HD + 32 * c;
               tmem_ld_32x32b_x32(o_addr, o);
               tmem_ld_wait();
 #pragma unroll
@@ -441,22 +475,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (stop) break;  // both halves, at the same exchange
-      // end of the item: this half's row sum goes to the epilogue warps once
+      // end of the item: this part's row sum goes to the epilogue warps once
       // they have taken item k - 2's from this buffer (a failed wait reaches
       // the partner with the next item's first exchange)
       if (good && k >= 2) good = __all_sync(0xffffffffu, mbar_wait(&o_empty[ob], ((k - 2) >> 1) & 1, abort_flag, err));
       if (good) {
-        l_buf[(ob * 2 + half) * kBQ + r] = l;
+        l_buf[(ob * kParts + part) * kBQ + r] = l;
         mbar_arrive(&l_full[ob]);
       }
     }
-  } else if (warp >= 12) {
-    // epilogue warps 12..15: O[k & 1] / l (x gate) as bf16, one query row per
-    // thread, while the softmax warps run the next item
+  } else if (warp >= kEpiWarp0) {
+    // epilogue warps (the last 4): O[k & 1] / l (x gate) as bf16, one query
+    // row per thread, while the softmax warps run the next item
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
-    constexpr int CP = HD < 64 ? HD : 64;  // columns per pass
+    constexpr int CP = kParts > 2 ? 32 : (HD < 64 ? HD : 64);  // columns per pass (registers)
     int k = 0;
     for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
       const int ob = k & 1;
@@ -465,7 +499,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!__all_sync(0xffffffffu, good)) break;
       tc_fence_after();
       const TcAttnItem w = items[it];
-      const float inv = 1.f / (l_buf[(ob * 2) * kBQ + r] + l_buf[(ob * 2 + 1) * kBQ + r]);
+      float lsum = 0.f;
+#pragma unroll
+      for (int q = 0; q < kParts; ++q) lsum += l_buf[(ob * kParts + q) * kBQ + r];
+      const float inv = 1.f / lsum;
       bf16* orow = out + (long long)(w.q_start + r) * H * HD + w.head * HD;
       const bf16* grow = gate ? gate + (long long)(w.q_start + r) * H * HD + w.head * HD : nullptr;
 #pragma unroll 1

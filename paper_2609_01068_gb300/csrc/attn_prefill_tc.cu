@@ -6,9 +6,10 @@
 // Persistent kernel, one CTA per SM, 8 + 4 kParts warps.  A work item is one 128-row
 // query tile of one sequence x one query head; items are taken longest first
 // (most key tiles) with a grid stride.
-//   warp 0       TMA producer: Q tile (one or two buffers), K tiles and V^T
-//                tiles of 128 keys in rings of their own (a K stage is freed
-//                by its S, a V stage by its PV), continuously across items
+//   warps 0, 2   TMA producers, one thread each: Q tiles (two buffers) and
+//                K tiles of 128 keys (warp 0), V^T tiles (warp 2), in rings of
+//                their own (a K stage is freed by its S, a V stage by its PV),
+//                continuously across items
 //   warp 1       TMEM owner; one thread issues the S MMAs
 //                  S_j = Q K_j^T     M=128 N=128 K=hd, into one of two TMEM S buffers
 //                as soon as their inputs are there (S_{j+2} once PV_j has
@@ -42,7 +43,6 @@ constexpr int kBQ = 128;                         // query rows per work item
 constexpr int kBK = 128;                         // keys per K/V tile
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleLog2 = 8.f;              // tolerated growth of a row max before O is rescaled
-constexpr unsigned kPollSleepNs = 32;            // back-off of the polling roles when nothing is ready
 constexpr int kMaxLanes = 8;                     // independent partial maxima of a score row
 // Threads of a query row in the softmax (each over kBK / kParts keys of a tile)
 #ifndef OUTLETS_ATTN_PARTS
@@ -52,7 +52,7 @@ constexpr int kParts = OUTLETS_ATTN_PARTS;
 static_assert(kParts == 2 || kParts == 4, "softmax parts of a row");
 constexpr int kSoftmaxWarps = 4 * kParts;
 constexpr int kEpiWarp0 = 4 + kSoftmaxWarps;    // first epilogue warp
-// producer, S issuer, idle, PV issuer, the softmax warps, 4 epilogue warps
+// Q/K producer, S issuer, V producer, PV issuer, the softmax warps, 4 epilogue warps
 constexpr int kThreads = 32 * (4 + kSoftmaxWarps + 4);
 constexpr int kSoftmaxThreads = 32 * kSoftmaxWarps;
 
@@ -184,78 +184,56 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      // Producer, three cursors issued as their slots free up: Q of an item
-      // (with the item's first K tile), K tiles, V^T tiles.  K may run up to
-      // NK tiles ahead of V.
-      int k_it = blockIdx.x, k_k = 0, k_j = 0, k_g = 0;  // K cursor: item, item count, tile in item, tile count
-      int v_it = blockIdx.x, v_j = 0, v_g = 0;           // V cursor
-      unsigned long long t_idle = 0;
-      uint32_t spin = 0;
-      while (v_it < n_items) {
-        bool progressed = false;
-        if (k_it < n_items) {
-          const TcAttnItem w = items[k_it];
-          const int qb = k_k % NQ;
-          const int st = k_g % NK;
-          const bool q_ok = k_j > 0 || k_k < NQ || mbar_test_wait(&q_empty[qb], ((k_k - NQ) / NQ) & 1);
-          if (q_ok && (k_g < NK || mbar_test_wait(&k_empty[st], ((k_g - NK) / NK) & 1))) {
-            const int kvh = (w.head * KVH) / H;
-            if (k_j == 0) {
-              mbar_arrive_expect_tx(&q_full[qb], C::Q_BYTES);
+      // Q and K producer: each item's Q (into buffer k % NQ, once the last S
+      // of item k - NQ has read it), then its K tiles into the K ring (a
+      // stage once the S that read it has completed).  It blocks in its
+      // waits, which leaves the issue slots to the softmax warps of this SM
+      // sub-partition (a polling producer delayed them).
+      int g = 0;  // key tiles of this CTA
+      int k = 0;  // items of this CTA
+      for (int it = blockIdx.x; it < n_items; it += gridDim.x, ++k) {
+        const TcAttnItem w = items[it];
+        const int kvh = (w.head * KVH) / H;
+        const int qb = k % NQ;
+        bool ok = k < NQ || mbar_wait(&q_empty[qb], ((k - NQ) / NQ) & 1, abort_flag, err);
+        if (!ok) break;
+        mbar_arrive_expect_tx(&q_full[qb], C::Q_BYTES);
 #pragma unroll
-              for (int b = 0; b < C::NB; ++b)
-                tma_load_2d(sQ + qb * C::Q_BYTES + b * (kBQ * 128), &q_map, &q_full[qb], w.head * HD + 64 * b,
-                            w.q_start);
-            }
-            mbar_arrive_expect_tx(&k_full[st], C::K_BYTES);
+        for (int b = 0; b < C::NB; ++b)
+          tma_load_2d(sQ + qb * C::Q_BYTES + b * (kBQ * 128), &q_map, &q_full[qb], w.head * HD + 64 * b, w.q_start);
+        for (int j = 0; j < w.n_kv; ++j, ++g) {
+          const int st = g % NK;
+          ok = g < NK || mbar_wait(&k_empty[st], ((g - NK) / NK) & 1, abort_flag, err);
+          if (!ok) break;
+          mbar_arrive_expect_tx(&k_full[st], C::K_BYTES);
 #pragma unroll
-            for (int b = 0; b < C::NB; ++b)
-              tma_load_2d(sK + st * C::K_BYTES + b * (kBK * 128), &k_map, &k_full[st], 64 * b,
-                          kvh * kv_ld + w.seq_start + kBK * k_j);
-            ++k_g;
-            if (++k_j == w.n_kv) {
-              k_j = 0;
-              ++k_k;
-              k_it += gridDim.x;
-            }
-            progressed = true;
-          }
+          for (int b = 0; b < C::NB; ++b)
+            tma_load_2d(sK + st * C::K_BYTES + b * (kBK * 128), &k_map, &k_full[st], 64 * b,
+                        kvh * kv_ld + w.seq_start + kBK * j);
         }
-        {
-          const int st = v_g % NV;
-          if (v_g < k_g && (v_g < NV || mbar_test_wait(&v_empty[st], ((v_g - NV) / NV) & 1))) {
-            const TcAttnItem w = items[v_it];
-            const int kvh = (w.head * KVH) / H;
-            mbar_arrive_expect_tx(&v_full[st], C::V_BYTES);
+        if (!ok) break;
+      }
+    }
+  } else if (warp == 2) {
+    if (lane == 0) {
+      // V^T producer: the V^T tiles into the V ring (a stage once the PV
+      // that read it has completed), blocking like the Q and K producer
+      int g = 0;
+      for (int it = blockIdx.x; it < n_items; it += gridDim.x) {
+        const TcAttnItem w = items[it];
+        const int kvh = (w.head * KVH) / H;
+        bool ok = true;
+        for (int j = 0; j < w.n_kv; ++j, ++g) {
+          const int st = g % NV;
+          ok = g < NV || mbar_wait(&v_empty[st], ((g - NV) / NV) & 1, abort_flag, err);
+          if (!ok) break;
+          mbar_arrive_expect_tx(&v_full[st], C::V_BYTES);
 #pragma unroll
-            for (int b = 0; b < 2; ++b)
-              tma_load_2d(sV + st * C::V_BYTES + b * (HD * 128), &vt_map, &v_full[st], w.v_start + kBK * v_j + 64 * b,
-                          kvh * HD);
-            ++v_g;
-            if (++v_j == w.n_kv) {
-              v_j = 0;
-              v_it += gridDim.x;
-            }
-            progressed = true;
-          }
+          for (int b = 0; b < 2; ++b)
+            tma_load_2d(sV + st * C::V_BYTES + b * (HD * 128), &vt_map, &v_full[st], w.v_start + kBK * j + 64 * b,
+                        kvh * HD);
         }
-        if (progressed) {
-          spin = 0;
-          t_idle = 0;
-          continue;
-        }
-        __nanosleep(kPollSleepNs);  // leave the issue slots to the softmax warps sharing this SM sub-partition
-        if ((++spin & 31u) == 0) {  // bounded, like every other wait
-          if (*abort_flag) break;
-          const unsigned long long now = global_timer_ns();
-          if (t_idle == 0) {
-            t_idle = now;
-          } else if (now - t_idle > kWaitTimeoutNs) {
-            *abort_flag = 1;
-            if (err) atomicOr(err, ERR_TIMEOUT);
-            break;
-          }
-        }
+        if (!ok) break;
       }
     }
   } else if (warp == 1) {
